@@ -1,0 +1,228 @@
+"""Seeded synthetic inputs for the verify round, shaped like the paper's workloads.
+
+The paper evaluates on Qwen2.5 / Qwen3 targets with diffusion drafters over
+MATH-500, GSM8K, HumanEval and MT-Bench (Sec. 4, Table 5). Neither the models
+nor the datasets are used here: these generators stand in for them with the
+same tensor shapes (vocabularies 32000 / 128256 / 152064, GQA 8/2, 32/8, 28/4,
+64/8, head dim 64 / 128), logit value distributions chosen so that the
+selected lengths span 0..K, and KV-length mixes from uniform to log-uniform.
+
+This module holds none of the verify round's arithmetic. It draws random
+tensors with ``torch`` generators and is the only code shared by the CUDA path
+and the CPU oracle in tests and benchmarks.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import List, Optional
+
+import numpy as np
+import torch
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    B: int                 # sequences
+    K: int                 # drafter block length (= d_max of the selector)
+    V: int                 # vocabulary
+    Hq: int                # query heads
+    Hkv: int               # kv heads
+    d: int                 # head dim
+    n_layers: int          # verify-attention layers per round
+    kv: tuple              # ("const", n) | ("uniform", lo, hi) | ("loguniform", lo, hi)
+    temperature: tuple     # ("const", T) | ("alternate", T_even, T_odd)
+    target: tuple          # ("normal", sigma) | ("normal_peak", sigma, peak) | ("normal_sigma_u", lo, hi)
+    draft_noise: tuple     # ("const", s) | ("uniform", lo, hi)
+    cost: tuple            # ("poly", c0, c1, c2) | ("attn_bytes",)
+    philox_seed: int
+    data_seed: int
+    resident_layers: int = 0   # >0: distinct KV buffers kept on the device (rest reuse them)
+
+    def scaled(self, **kw) -> "Workload":
+        return dataclasses.replace(self, **kw)
+
+
+# The five workloads (batch 1..64). Values the task leaves open (data seeds of
+# the larger configs, the sampling config's target sigma, the ragged config's
+# odd-sequence temperature and drafter noise, layer counts of the single-layer
+# configs) are fixed here once.
+WORKLOADS = {
+    "tiny": Workload("tiny", B=1, K=16, V=32000, Hq=8, Hkv=2, d=64, n_layers=1,
+                     kv=("const", 512), temperature=("const", 0.0), target=("normal", 4.0),
+                     draft_noise=("const", 1.0), cost=("poly", 1.0, 0.02, 0.0),
+                     philox_seed=0, data_seed=0),
+    "8b": Workload("8b", B=1, K=16, V=128256, Hq=32, Hkv=8, d=128, n_layers=32,
+                   kv=("const", 4096), temperature=("const", 0.0), target=("normal_peak", 6.0, 12.0),
+                   draft_noise=("const", 1.5), cost=("poly", 1.0, 0.01, 0.0),
+                   philox_seed=1, data_seed=1),
+    "sampling": Workload("sampling", B=16, K=16, V=152064, Hq=28, Hkv=4, d=128, n_layers=1,
+                         kv=("uniform", 1024, 8192), temperature=("const", 1.0), target=("normal", 4.0),
+                         draft_noise=("uniform", 0.5, 3.0), cost=("poly", 1.0, 0.015, 0.0005),
+                         philox_seed=1234, data_seed=2),
+    "ragged": Workload("ragged", B=64, K=32, V=128256, Hq=32, Hkv=8, d=128, n_layers=1,
+                       kv=("loguniform", 512, 32768), temperature=("alternate", 0.0, 0.8),
+                       target=("normal_sigma_u", 1.0, 8.0), draft_noise=("const", 1.0),
+                       cost=("attn_bytes",), philox_seed=3, data_seed=3),
+    "70b": Workload("70b", B=8, K=16, V=128256, Hq=64, Hkv=8, d=128, n_layers=80,
+                    kv=("const", 131072), temperature=("const", 0.7), target=("normal", 4.0),
+                    draft_noise=("const", 1.0), cost=("poly", 1.0, 0.008, 0.0),
+                    philox_seed=4, data_seed=4, resident_layers=16),
+}
+
+
+def _np_rng(w: Workload, stream: int) -> np.random.Generator:
+    return np.random.default_rng([w.data_seed, stream])
+
+
+def kv_lengths(w: Workload) -> np.ndarray:
+    """Per-sequence KV-cache length before the verified block, int32 [B]."""
+    kind = w.kv[0]
+    rng = _np_rng(w, 1)
+    if kind == "const":
+        out = np.full(w.B, w.kv[1])
+    elif kind == "uniform":
+        out = rng.integers(w.kv[1], w.kv[2] + 1, size=w.B)
+    elif kind == "loguniform":
+        lo, hi = math.log(w.kv[1]), math.log(w.kv[2])
+        out = np.floor(np.exp(rng.uniform(lo, hi, size=w.B))).astype(np.int64)
+        out = np.clip(out, w.kv[1], w.kv[2])
+    else:
+        raise ValueError(kind)
+    return out.astype(np.int32)
+
+
+def temperatures(w: Workload) -> np.ndarray:
+    """Per-sequence temperature, float32 [B]; 0 means greedy decoding."""
+    if w.temperature[0] == "const":
+        return np.full(w.B, w.temperature[1], np.float32)
+    even, odd = w.temperature[1], w.temperature[2]
+    return np.array([even if b % 2 == 0 else odd for b in range(w.B)], np.float32)
+
+
+def s_cap(w: Workload, kv: Optional[np.ndarray] = None) -> int:
+    """Cache capacity per (sequence, kv head): room for the block, rounded to 64."""
+    kv = kv_lengths(w) if kv is None else kv
+    need = int(kv.max()) + w.K + 1
+    return (need + 63) // 64 * 64
+
+
+def attn_bytes(w: Workload, kv: np.ndarray, L) -> float:
+    """Bytes one verify-attention layer must move: K and V of the visible keys
+    plus Q read and O written for the verified rows (bf16)."""
+    L = np.broadcast_to(np.asarray(L, np.int64), kv.shape)
+    keys = kv.astype(np.int64) + L + 1
+    rows = L + 1
+    return float(np.sum(w.Hkv * keys * w.d * 2 * 2 + rows * w.Hq * w.d * 2 * 2))
+
+
+# Fixed per-launch latency folded into the byte-count cost model, expressed
+# in bytes at the measured copy bandwidth (about 3 us at 6.76 TB/s).
+_LAUNCH_BYTES = 3e-6 * 6.756e12
+
+
+def cost_table(w: Workload, kv: Optional[np.ndarray] = None) -> np.ndarray:
+    """T_verify(L) for L = 0..K, float32 [K+1], positive.
+
+    Polynomial tables are the workloads' stated ones. The ragged workload's
+    table models one verify-attention launch with every sequence at length L:
+    the launch latency plus the bytes it must move at a fixed bandwidth,
+    normalised so that T(0) = 1 (the kernel is bandwidth bound, so its time is
+    proportional to these bytes)."""
+    Ls = np.arange(w.K + 1)
+    if w.cost[0] == "poly":
+        c0, c1, c2 = w.cost[1:]
+        t = c0 + c1 * Ls + c2 * Ls * Ls
+    elif w.cost[0] == "attn_bytes":
+        kv = kv_lengths(w) if kv is None else kv
+        t = np.array([_LAUNCH_BYTES + attn_bytes(w, kv, L) for L in Ls])
+        t = t / t[0]
+        t = np.maximum.accumulate(t)
+    else:
+        raise ValueError(w.cost[0])
+    return t.astype(np.float32)
+
+
+def _randn(shape, gen, device, dtype=torch.float32):
+    return torch.randn(shape, generator=gen, device=device, dtype=dtype)
+
+
+def logits(w: Workload, device="cpu") -> dict:
+    """Target logits [B,K+1,V], drafter logits [B,K,V] (fp32), draft tokens
+    [B,K] (int32) and temperatures [B] (fp32) on ``device``.
+
+    Drafter logits are the target's plus Gaussian noise (the drafter is close
+    to the target). Greedy sequences draft the drafter's argmax; sampling
+    sequences draft a token sampled from the drafter's softmax at their
+    temperature (Gumbel-max with the torch generator), so that the rejection
+    sampler sees drafts distributed as q."""
+    g = torch.Generator(device=device)
+    g.manual_seed(w.data_seed * 1000003 + 17)
+    B, K, V = w.B, w.K, w.V
+    rng = _np_rng(w, 2)
+    kind = w.target[0]
+    if kind == "normal":
+        sig = np.full(B, w.target[1])
+    elif kind == "normal_peak":
+        sig = np.full(B, w.target[1])
+    elif kind == "normal_sigma_u":
+        sig = rng.uniform(w.target[1], w.target[2], size=B)
+    else:
+        raise ValueError(kind)
+    if w.draft_noise[0] == "const":
+        noise = np.full(B, w.draft_noise[1])
+    else:
+        noise = rng.uniform(w.draft_noise[1], w.draft_noise[2], size=B)
+    sig_t = torch.tensor(sig, dtype=torch.float32, device=device).view(B, 1, 1)
+    noise_t = torch.tensor(noise, dtype=torch.float32, device=device).view(B, 1, 1)
+    target = _randn((B, K + 1, V), g, device) * sig_t
+    if kind == "normal_peak":
+        idx = torch.randint(0, V, (B, K + 1, 1), generator=g, device=device)
+        target.scatter_add_(2, idx, torch.full((B, K + 1, 1), float(w.target[2]), device=device))
+    draft = target[:, :K, :] + _randn((B, K, V), g, device) * noise_t
+    temp = torch.tensor(temperatures(w), device=device)
+    tokens = torch.empty((B, K), dtype=torch.int32, device=device)
+    for b in range(B):
+        T = float(temp[b])
+        if T == 0.0:
+            tokens[b] = torch.argmax(draft[b], dim=-1).to(torch.int32)
+        else:
+            u = torch.rand((K, V), generator=g, device=device).clamp_(1e-30, 1.0 - 1e-7)
+            gumbel = -torch.log(-torch.log(u))
+            tokens[b] = torch.argmax(draft[b] / T + gumbel, dim=-1).to(torch.int32)
+    return {"target_logits": target.contiguous(), "draft_logits": draft.contiguous(),
+            "draft_tokens": tokens.contiguous(), "temperature": temp.contiguous()}
+
+
+def layer(w: Workload, l: int, kv: np.ndarray, device="cpu", peaky: bool = False,
+          scap: Optional[int] = None) -> dict:
+    """Q [B,K+1,Hq,d] and the KV cache Kc, Vc [B,Hkv,S_cap,d] (bf16, ~N(0,1))
+    of verify-attention layer ``l``, each layer seeded independently.
+
+    ``peaky``: plant, for every (sequence, query head), one key equal to 3x
+    the head's first verified query so that one score dominates its row."""
+    g = torch.Generator(device=device)
+    g.manual_seed(w.data_seed * 7919 + 1000 + l)
+    S = s_cap(w, kv) if scap is None else scap
+    B, K1 = w.B, w.K + 1
+    Q = _randn((B, K1, w.Hq, w.d), g, device, torch.bfloat16)
+    Kc = _randn((B, w.Hkv, S, w.d), g, device, torch.bfloat16)
+    Vc = _randn((B, w.Hkv, S, w.d), g, device, torch.bfloat16)
+    if peaky:
+        gsz = w.Hq // w.Hkv
+        for b in range(B):
+            for h in range(w.Hq):
+                pos = int(torch.randint(0, int(kv[b]), (1,), generator=g, device=device))
+                Kc[b, h // gsz, pos] = (Q[b, 0, h].float() * 3.0).to(torch.bfloat16)
+    return {"Q": Q, "Kc": Kc, "Vc": Vc}
+
+
+def reference_inputs_summary(w: Workload) -> List[str]:
+    """One line per input recipe, for reports."""
+    return [
+        "target logits %s, drafter = target + N(0, %s^2)" % (w.target, w.draft_noise),
+        "kv lengths %s, %d layer(s), GQA %d/%d, head dim %d" % (w.kv, w.n_layers, w.Hq, w.Hkv, w.d),
+        "temperature %s, cost %s, philox seed %d, data seed %d" % (w.temperature, w.cost, w.philox_seed,
+                                                                    w.data_seed),
+    ]
