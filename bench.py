@@ -1,0 +1,449 @@
+"""Benchmark of the LibraSpec verify round on GB300.
+
+One step = one verify round over one batch: drafter confidence + length
+selection, every verify-attention layer, acceptance. Default workload: the
+8B-class greedy round (B=1, K=16, V=128256, 32 layers of GQA 32/8 attention
+over a 4096-token cache).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+
+N > 1 runs under torchrun, one process per GPU; every rank verifies its own
+batch (weak scaling, no data-path collective) and rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verify-round µs (select+attn+accept) and HBM TB/s vs ~8 TB/s, batch 1–64"
+NOMINAL_HBM_GBS = 8000.0
+L2_BYTES = 129e6
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=0, help="timed steps (0: enough for ~2 s)")
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--config", default="8b")
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--e2e-steps", type=int, default=50)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle sample")
+    return p.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+_REASONS = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+
+
+class ClockSampler:
+    def __init__(self, gpu_index: int):
+        self.path = tempfile.mktemp(suffix=".csv")
+        self.proc = None
+        self.gpu = gpu_index
+
+    def __enter__(self):
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + q,
+                                          "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        out = {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        try:
+            rows = [l.strip().split(",") for l in open(self.path) if l.strip()]
+        except OSError:
+            return out
+        sm, mx, reasons = [], [], set()
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except ValueError:
+                continue
+            for name, val in zip(_REASONS, r[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if sm:
+            out.update(sm_mhz=statistics.median(sm), sm_max_mhz=max(mx), samples=len(sm))
+        out["reasons"] = sorted(reasons)
+        return out
+
+
+def physical_gpu(local_rank):
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [x.strip() for x in vis.split(",") if x.strip()]
+        if local_rank < len(ids):
+            return ids[local_rank]
+    return str(local_rank)
+
+
+# ---------------------------------------------------------------------------
+# algorithmic bytes (what the method must move)
+# ---------------------------------------------------------------------------
+def round_bytes(w, kv, L, temperature, n_acc):
+    conf = w.B * w.K * w.V * 4
+    select = w.B * w.K * 4 + (w.K + 1) * 4
+    accept = float(np.sum((L + 1).astype(np.int64) * w.V * 4))
+    rejected_sampling = np.sum((n_acc < L) & (temperature > 0))
+    accept += float(rejected_sampling) * 2 * w.V * 4
+    from paper_2608_08721_gb300 import workloads
+
+    attn_launch = workloads.attn_bytes(w, kv, L)
+    return {"conf": conf, "select": select, "attn_per_launch": attn_launch, "attn": attn_launch * w.n_layers,
+            "accept": accept, "total": conf + select + accept + attn_launch * w.n_layers}
+
+
+# ---------------------------------------------------------------------------
+# the oracle on the host cores (CPU baseline / reference arm)
+# ---------------------------------------------------------------------------
+def oracle_round_time(w, inp_host, layers_host, kv, budget_s):
+    """Time the oracle's round on a bounded sample: the full logits steps and
+    one attention layer (scaled to all layers). Repeats the sample until the
+    budget is spent; returns (us per round, threads, sample text)."""
+    import oracle
+
+    oracle.build()
+    threads = os.cpu_count() or 1
+    oracle.set_threads(threads)
+    cost = np.asarray(inp_host["cost_table"], np.float64)
+    times_logits, times_attn = [], []
+    t_end = time.perf_counter() + budget_s
+    while True:
+        t0 = time.perf_counter()
+        q, _ = oracle.confidence(inp_host["draft_logits"], inp_host["draft_tokens"], inp_host["temperature"])
+        L, _ = oracle.select_lengths(q, cost)
+        oracle.accept(inp_host["target_logits"], inp_host["draft_logits"], inp_host["draft_tokens"], L,
+                      inp_host["temperature"], w.philox_seed)
+        t1 = time.perf_counter()
+        lay = layers_host[len(times_attn) % len(layers_host)]
+        oracle.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L)
+        t2 = time.perf_counter()
+        times_logits.append(t1 - t0)
+        times_attn.append(t2 - t1)
+        if time.perf_counter() > t_end or len(times_attn) >= 50:
+            break
+    per_round = statistics.median(times_logits) + statistics.median(times_attn) * w.n_layers
+    sample = ("%d repetition(s) of: confidence, selection and acceptance on the full batch plus ONE of the %d "
+              "attention layers (fp64 C oracle, %d threads); attention time scaled by %d layers" %
+              (len(times_attn), w.n_layers, threads, w.n_layers))
+    return per_round * 1e6, threads, sample
+
+
+def host_inputs(w, kv, n_layer_samples=1):
+    from paper_2608_08721_gb300 import workloads
+
+    inp = workloads.logits(w)
+    host = {k: v.numpy() for k, v in inp.items()}
+    host["cost_table"] = workloads.cost_table(w, kv)
+    layers = [workloads.layer(w, l, kv) for l in range(n_layer_samples)]
+    return host, layers
+
+
+def run_reference(args, rank, world):
+    """The reference arm: the oracle as it stands, on this host's cores."""
+    from paper_2608_08721_gb300 import workloads
+
+    if rank != 0:
+        return
+    w = workloads.WORKLOADS[args.config]
+    kv = workloads.kv_lengths(w)
+    host, layers = host_inputs(w, kv)
+    steps = max(1, args.steps if args.steps > 0 else 3)
+    budget = max(10.0, args.cpu_seconds)
+    per = []
+    cores, sample = 0, ""
+    for _ in range(max(0, min(args.warmup, 1))):
+        oracle_round_time(w, host, layers, kv, 0.0)
+    for _ in range(steps):
+        us, cores, sample = oracle_round_time(w, host, layers, kv, budget / steps)
+        per.append(us)
+    value = statistics.median(per)
+    line = {"metric": METRIC, "value": round(value, 3), "unit": "us", "n_gpus": args.gpus, "steps": steps,
+            "warmup": args.warmup, "ms_per_step": round(value / 1000, 6), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": w.name, "B": w.B, "K": w.K, "V": w.V, "layers": w.n_layers,
+                       "gqa": "%d/%d" % (w.Hq, w.Hkv), "head_dim": w.d, "parallelism": "replicas"},
+            "cpu_baseline": {"value": round(value, 3), "unit": "us", "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(value, 3), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def traffic_record(kernel_file):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu
+    summary, if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "verify_attn_traffic.json")
+    try:
+        rec = json.load(open(path))
+    except (OSError, ValueError):
+        return None
+    sha = hashlib.sha256(open(kernel_file, "rb").read()).hexdigest()
+    if rec.get("kernel_source_sha256") != sha:
+        return None
+    return rec
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+
+    from paper_2608_08721_gb300 import binding as lr
+    from paper_2608_08721_gb300 import build as cuda_build
+    from paper_2608_08721_gb300 import dist as pdist
+    from paper_2608_08721_gb300 import workloads
+    from paper_2608_08721_gb300.api import VerifyRound
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if rank == 0 or not os.path.exists(lr.LIB_PATH):
+        cuda_build.build()
+    pdist.barrier()
+    w = workloads.WORKLOADS[args.config]
+    kv = workloads.kv_lengths(w)
+    seq_offset = rank * w.B  # weak scaling: each rank verifies its own B sequences
+    inp = workloads.logits(w, device=dev)
+    n_res = w.resident_layers if w.resident_layers else w.n_layers
+    S = workloads.s_cap(w, kv)
+    caches = [workloads.layer(w, l, kv, device=dev) for l in range(n_res)]
+    g = torch.Generator(device=dev).manual_seed(w.data_seed * 31 + 5)
+    Qs = [torch.randn((w.B, w.K + 1, w.Hq, w.d), generator=g, device=dev).to(torch.bfloat16)
+          for _ in range(w.n_layers)]
+    Os = [torch.empty_like(q) for q in Qs]
+    layers = [{"Q": Qs[l], "Kc": caches[l % n_res]["Kc"], "Vc": caches[l % n_res]["Vc"], "O": Os[l]}
+              for l in range(w.n_layers)]
+    cost = torch.tensor(workloads.cost_table(w, kv), device=dev)
+    kv_t = torch.tensor(kv, device=dev)
+    ws = lr.Workspace(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, S, device=dev)
+    conf = torch.empty((w.B, w.K), device=dev)
+    dstat = torch.empty((w.B, w.K, 2), device=dev)
+    L = torch.empty((w.B,), dtype=torch.int32, device=dev)
+    n_acc = torch.empty((w.B,), dtype=torch.int32, device=dev)
+    bonus = torch.empty((w.B,), dtype=torch.int32, device=dev)
+
+    def seg_select():
+        lr.libraspec_confidence(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], ws, conf=conf,
+                                dstat=dstat)
+        lr.libraspec_select_lengths(conf, cost, ws, L=L)
+
+    def seg_attn():
+        for lay in layers:
+            lr.libraspec_verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv_t, L, ws, O=lay["O"])
+
+    def seg_accept():
+        lr.libraspec_accept(inp["target_logits"], inp["draft_logits"], inp["draft_tokens"], conf, dstat, L,
+                            inp["temperature"], w.philox_seed, ws, seq_offset=seq_offset, n_accepted=n_acc,
+                            bonus_token=bonus)
+
+    # eager warm-up (also configures kernels), then capture three graphs
+    for _ in range(3):
+        seg_select(); seg_attn(); seg_accept()
+    torch.cuda.synchronize()
+    if lr.libraspec_get_status(ws) != 0:
+        raise RuntimeError("device status set during warm-up")
+    graphs = []
+    side = torch.cuda.Stream(device=dev)
+    for seg in (seg_select, seg_attn, seg_accept):
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=side):
+            seg()
+        graphs.append(gr)
+    stream = torch.cuda.current_stream()
+
+    def step(ev_a=None, ev_b=None):
+        graphs[0].replay()
+        if ev_a is not None:
+            ev_a.record(stream)
+        graphs[1].replay()
+        if ev_b is not None:
+            ev_b.record(stream)
+        graphs[2].replay()
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    # steps: enough for ~2 s of timed work unless given
+    if args.steps > 0:
+        K_steps = args.steps
+    else:
+        t0 = time.perf_counter()
+        for _ in range(20):
+            step()
+        torch.cuda.synchronize()
+        per = (time.perf_counter() - t0) / 20
+        K_steps = int(min(20000, max(50, 2.0 / max(per, 1e-6))))
+    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
+    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    pdist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(physical_gpu(local_rank)) as clocks:
+        start.record(stream)
+        for i in range(K_steps):
+            step(ev_a[i], ev_b[i])
+        end.record(stream)
+        torch.cuda.synchronize()
+    pdist.barrier()
+    elapsed_ms = start.elapsed_time(end)
+    attn_ms = sum(a.elapsed_time(b) for a, b in zip(ev_a, ev_b))
+    elapsed_max = pdist.max_over_ranks(elapsed_ms, device=dev)
+    if lr.libraspec_get_status(ws) != 0:
+        raise RuntimeError("device status set during the timed steps")
+
+    Lh = L.cpu().numpy()
+    nh = n_acc.cpu().numpy()
+    temp = inp["temperature"].cpu().numpy()
+    by = round_bytes(w, kv, Lh, temp, nh)
+    us_per_round = elapsed_ms * 1000.0 / K_steps
+    attn_launch_s = attn_ms / 1000.0 / (K_steps * w.n_layers)
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks["hbm_gbs"])
+    achieved = by["attn_per_launch"] / attn_launch_s / 1e9
+    trec = traffic_record(os.path.join(ROOT, "paper_2608_08721_gb300", "csrc", "attn.cu"))
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if args.e2e_steps > 0:
+        e2e = run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        host = {k: v.cpu().numpy() for k, v in inp.items()}
+        host["cost_table"] = workloads.cost_table(w, kv)
+        lay_host = [{"Q": layers[0]["Q"].cpu(), "Kc": layers[0]["Kc"].cpu(), "Vc": layers[0]["Vc"].cpu()}]
+        us, cores, sample = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds)
+        cpu = {"value": round(us, 1), "unit": "us", "cores": cores, "kind": "oracle", "sample": sample}
+
+    if rank != 0:
+        return
+    clk = clocks.summary()
+    value = elapsed_max * 1000.0 / (K_steps * world)
+    launches = K_steps * (w.n_layers + 4)
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": "us", "n_gpus": world, "steps": K_steps,
+        "warmup": max(3, args.warmup), "ms_per_step": round(elapsed_max / K_steps, 6), "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16+f32",
+        "data": "synthetic (seeded; shapes of the paper's 8B-70B-class targets, random values)",
+        "config": {"workload": w.name, "B": w.B, "K": w.K, "V": w.V, "layers": w.n_layers,
+                   "resident_kv_layers": n_res, "gqa": "%d/%d" % (w.Hq, w.Hkv), "head_dim": w.d,
+                   "kv_len": [int(kv.min()), int(kv.max())], "selected_L": [int(Lh.min()), int(Lh.max())],
+                   "parallelism": "dp%d (independent sequences)" % world,
+                   "l2": "no flush: %.0f MB of distinct inputs per step > 129 MB L2" % (by["total"] / 1e6),
+                   "timing": "3 CUDA graphs per step (conf+select | attention layers | accept), events between"},
+        "hbm_tbs": round(by["total"] / (us_per_round * 1e-6) / 1e12, 3),
+        "hbm_frac_of_measured": round(by["total"] / (us_per_round * 1e-6) / 1e9 / hbm_peak, 4),
+        "hbm_frac_of_nominal_8tbs": round(by["total"] / (us_per_round * 1e-6) / 1e9 / NOMINAL_HBM_GBS, 4),
+        "roofline": {"kernel": "verify_attn", "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
+                     "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
+                     "traffic": None if trec is None else trec.get("traffic_bytes_per_launch"),
+                     "algorithmic_bytes_per_launch": by["attn_per_launch"],
+                     "launch_us": round(attn_launch_s * 1e6, 3), "peak_source": peak_src + " (MEASURED_PEAKS.json hbm_gbs)"},
+        "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
+                   "samples": clk["samples"]},
+        "gpu_launches": launches,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset):
+    """Same metric through the public host-buffer API: per round, the round's
+    inputs are copied in from pinned host memory and the results read back."""
+    import torch
+
+    from paper_2608_08721_gb300.api import VerifyRound
+
+    n_res = len({id(l["Kc"]) for l in layers})
+    caches = [{"Kc": l["Kc"], "Vc": l["Vc"]} for l in layers]
+    runner = VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, layers[0]["Kc"].shape[2], caches, torch.tensor(kv),
+                         device=dev)
+    K1 = w.K + 1
+    host = {k: v.cpu().pin_memory() for k, v in inp.items()}
+    host["cost_table"] = cost.cpu().pin_memory()
+    host["layers"] = []
+    for l in layers:
+        Kn = torch.stack([l["Kc"][b, :, int(kv[b]):int(kv[b]) + K1] for b in range(w.B)]).cpu().pin_memory()
+        Vn = torch.stack([l["Vc"][b, :, int(kv[b]):int(kv[b]) + K1] for b in range(w.B)]).cpu().pin_memory()
+        host["layers"].append({"Q": l["Q"].cpu().pin_memory(), "K_new": Kn, "V_new": Vn})
+    for _ in range(3):
+        runner.run_host(host, w.philox_seed, seq_offset=seq_offset)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        runner.run_host(host, w.philox_seed, seq_offset=seq_offset)
+    dt = time.perf_counter() - t0
+    return {"value": round(dt * 1e6 / args.e2e_steps, 3), "unit": "us", "h2d_bytes_per_step": runner.h2d_bytes(),
+            "d2h_bytes_per_step": runner.d2h_bytes(), "steps": args.e2e_steps,
+            "api": "paper_2608_08721_gb300.api.VerifyRound.run_host (libraspec_verify_round)"}
+
+
+def main():
+    args = parse()
+    from paper_2608_08721_gb300 import dist as pdist
+
+    rank, world, local_rank = pdist.env_world()
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    pdist.init("nccl" if world > 1 else "gloo")
+    try:
+        run_ours(args, rank, world, local_rank)
+    finally:
+        import torch.distributed as dist
+
+        if dist.is_initialized():
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

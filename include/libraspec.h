@@ -1,0 +1,205 @@
+/*
+ * libraspec — the LibraSpec verify round on NVIDIA GB300 (sm_103a).
+ *
+ * One decoding round of diffusion-drafted speculative decoding with the
+ * LibraSpec length controller (arxiv 2608.08721), as four device steps:
+ *
+ *   1. libraspec_confidence      drafter confidence q of every drafted token
+ *   2. libraspec_select_lengths  per-sequence speculative length L_b
+ *   3. libraspec_verify_attn     block-causal GQA verify attention (per layer)
+ *   4. libraspec_accept          greedy / rejection-sampling acceptance
+ *
+ * libraspec_verify_round runs all four on one stream.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Every tensor pointer is a DEVICE pointer owned by the caller, contiguous
+ *   and row-major in the layout stated (last index fastest). The library
+ *   never frees or keeps them.
+ * - bf16 tensors are passed as uint16_t bit patterns.
+ * - `stream` is a cudaStream_t (NULL = the legacy default stream). Calls only
+ *   enqueue work on it and return without synchronising, except
+ *   libraspec_get_status.
+ * - The library allocates no device memory. Calls that need scratch space
+ *   take a caller-provided `workspace` of at least libraspec_workspace_size()
+ *   bytes, 256-byte aligned and zero-filled once before first use
+ *   (libraspec_workspace_init). Every call leaves its counters at zero again,
+ *   so a workspace can be reused by any number of calls in stream order.
+ *   Calls sharing one workspace must not overlap on the GPU.
+ * - Return value: LIBRASPEC_OK, or a negative status (below). Arguments are
+ *   checked on the host before anything is enqueued. Conditions only the
+ *   device can see (a selected length out of range, a non-positive cost, a
+ *   KV cache too short for the block) set a status word in the workspace,
+ *   read by libraspec_get_status. Kernels never trap and never spin without
+ *   a bound.
+ * - Logits must be finite. Vocabulary sizes need not be multiples of 4, but
+ *   rows whose byte length is a multiple of 16 use the vectorised path.
+ *
+ * Batch sharding: `seq_offset` is added to the batch index b wherever a
+ * random number is drawn, so a batch split over several GPUs draws exactly
+ * the numbers the unsplit batch would.
+ */
+#ifndef LIBRASPEC_H
+#define LIBRASPEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define LIBRASPEC_OK 0
+#define LIBRASPEC_EINVAL (-1)       /* null pointer, bad shape or alignment     */
+#define LIBRASPEC_EUNSUPPORTED (-2) /* valid but not supported (e.g. head dim)  */
+#define LIBRASPEC_ECUDA (-3)        /* a CUDA runtime call or launch failed     */
+#define LIBRASPEC_EDEVICE (-4)      /* a kernel reported a violation (status)   */
+
+/* Device status bits (libraspec_get_status). */
+#define LIBRASPEC_ST_BAD_LENGTH 0x1  /* L_b outside [0, K]                       */
+#define LIBRASPEC_ST_BAD_COST 0x2    /* cost_table entry not positive and finite */
+#define LIBRASPEC_ST_KV_OVERFLOW 0x4 /* kv_len_b + L_b + 1 > S_cap or kv_len < 0 */
+#define LIBRASPEC_ST_BAD_TOKEN 0x8   /* draft token outside [0, V)               */
+#define LIBRASPEC_ST_TIMEOUT 0x10    /* a bounded wait for an async copy expired */
+#define LIBRASPEC_ST_MISSING_INPUT 0x20 /* sampling sequence but conf/dstat NULL  */
+
+/* Limits of this build. */
+#define LIBRASPEC_MAX_K 64           /* drafter block length / d_max             */
+#define LIBRASPEC_MAX_B 4096         /* sequences per call                       */
+
+/* Version string of the library. */
+const char* libraspec_version(void);
+
+/* Human-readable name of a status code returned by any call. */
+const char* libraspec_status_string(int status);
+
+/*
+ * Bytes of workspace a round with these shapes needs (all calls of the
+ * round may share it). B sequences, K drafter block length, V vocabulary,
+ * Hq / Hkv query / kv heads, head_dim, S_cap cache capacity per (b, kv head).
+ * Pure host function; returns 0 for invalid shapes.
+ */
+size_t libraspec_workspace_size(int B, int K, int V, int Hq, int Hkv, int head_dim, int S_cap);
+
+/* Zero-fill `bytes` of workspace on `stream` (cudaMemsetAsync). */
+int libraspec_workspace_init(void* workspace, size_t bytes, void* stream);
+
+/*
+ * Synchronise `stream`, copy the device status word of `workspace` into
+ * *host_status (0 = no violation, else LIBRASPEC_ST_* bits) and clear it.
+ * Returns LIBRASPEC_EDEVICE if the word was non-zero.
+ */
+int libraspec_get_status(void* workspace, void* stream, int32_t* host_status);
+
+/*
+ * Step 1 — drafter confidence (paper Sec. 3.4, Assumption 1: the drafter's
+ * confidence q_k stands in for the target's acceptance probability p_k in
+ * Algorithm 1).
+ *
+ * For every sequence b and draft position k:
+ *   T      = temperature[b] > 0 ? temperature[b] : 1   (greedy uses T = 1)
+ *   m      = max_v draft_logits[b,k,v]
+ *   Z      = sum_v exp((draft_logits[b,k,v] - m) / T)
+ *   conf[b,k]    = exp((draft_logits[b,k,draft_tokens[b,k]] - m) / T) / Z
+ *   dstat[b,k,:] = (m, Z)       (optional; libraspec_accept needs it for
+ *                                sampling sequences)
+ * draft_logits [B,K,V] f32, draft_tokens [B,K] i32 in [0,V),
+ * temperature [B] f32 >= 0, conf [B,K] f32 out, dstat [B,K,2] f32 out or NULL.
+ * One pass over the logits (B*K*V*4 bytes), split over CTAs per row.
+ */
+int libraspec_confidence(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                         int B, int K, int V, float* conf, float* dstat, void* workspace, size_t ws_bytes,
+                         void* stream);
+
+/*
+ * Step 2 — LibraSpec length selection (paper Thm. 4, from Thm. 1's
+ * ratio comparison; Eq. 2 with negligible drafting cost).
+ *
+ * With P_j = prod_{k<=j} conf[b,k-1] (prefix acceptance) and
+ * E_L = 1 + sum_{j<=L} P_j (expected tokens from verifying L drafts,
+ * counting the token verification always emits), extend L -> L+1 while
+ *     P_{L+1} * T(L) > (T(L+1) - T(L)) * E_L ,      T(L) = cost_table[L],
+ * i.e. while the marginal gain per unit of added verification cost beats
+ * the expected speedup E_L / T(L) already reached. L[b] is the first L
+ * where the test fails, or K. Computed in binary64; the strict comparison
+ * means a tie does not extend.
+ * conf [B,K] f32 in [0,1], cost_table [K+1] f32 (each > 0 and finite,
+ * else status LIBRASPEC_ST_BAD_COST and L = 0), L [B] i32 out.
+ * One warp per sequence; K <= LIBRASPEC_MAX_K.
+ */
+int libraspec_select_lengths(const float* conf, const float* cost_table, int B, int K, int32_t* L,
+                             void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Step 3 — block-causal GQA verify attention, one layer (paper Sec. 3.1:
+ * the target scores all drafted positions in one forward pass).
+ *
+ * For sequence b, query head h (kv head h / g, g = Hq / Hkv) and block row
+ * t in [0, L[b]]: the block's own keys are already in the cache at
+ * positions kv_len[b] .. kv_len[b] + L[b]; row t attends to keys
+ * 0 .. kv_len[b] + t:
+ *   O[b,t,h,:]  = softmax_s(softmax_scale * Q[b,t,h,:] . Kc[b,h/g,s,:]) Vc[b,h/g,s,:]
+ *   lse[b,t,h]  = log sum_s exp(softmax_scale * Q . K)     (natural log)
+ * Rows t > L[b] of O and lse are not written.
+ * Q, O [B,K+1,Hq,head_dim] bf16; Kc, Vc [B,Hkv,S_cap,head_dim] bf16
+ * (16-byte aligned base); kv_len [B] i32 >= 0 with kv_len + L + 1 <= S_cap
+ * (else status LIBRASPEC_ST_KV_OVERFLOW, sequence skipped);
+ * L [B] i32 in [0,K]; lse [B,K+1,Hq] f32 out or NULL.
+ * head_dim in {64, 128}; Hq % Hkv == 0; (K+1) * Hq / Hkv <= 512.
+ * Split-KV over a persistent grid with a deterministic in-kernel merge.
+ */
+int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc, const int32_t* kv_len,
+                          const int32_t* L, int B, int K, int Hq, int Hkv, int head_dim, int S_cap,
+                          float softmax_scale, uint16_t* O, float* lse, void* workspace, size_t ws_bytes,
+                          void* stream);
+
+/*
+ * Step 4 — acceptance (paper Sec. 3.1; the standard speculative-sampling
+ * rule of Leviathan et al. that the paper cites, lossless with respect to
+ * the target distribution).
+ *
+ * Row j of target_logits is the target distribution p_j for draft position
+ * j; row L[b] is the bonus row. For each sequence b:
+ * temperature[b] == 0 (greedy): accept draft j while argmax_v p_j = x_j
+ *   (lowest index wins ties); n = first mismatch or L[b];
+ *   bonus = argmax p_n.
+ * temperature[b] > 0 (sampling at T): p, q = softmax at T;
+ *   for j < L[b], u_j = Philox4x32-10 uniform (purpose 0) and accept iff
+ *   u_j < min(1, p_j(x_j) / q_j(x_j)); at the first rejection r the bonus is
+ *   drawn from norm(max(0, p_r - q_r)), else from p_{L[b]}, by an
+ *   exponential race argmin_v E_v / w_v over purpose-1 uniforms.
+ * Generator: key = (seed lo, seed hi); counter = (idx, position,
+ *   seq_offset + b, purpose + 4 * round_offset); u = ((w >> 9) + 1/2) 2^-23.
+ * target_logits [B,K+1,V] f32, draft_logits [B,K,V] f32, draft_tokens
+ * [B,K] i32, conf [B,K] f32 and dstat [B,K,2] f32 from libraspec_confidence
+ * (may be NULL when every temperature is 0), L [B] i32, temperature [B] f32;
+ * n_accepted [B] i32 out, bonus_token [B] i32 out.
+ * Reads target rows 0..L[b] once, plus one or two V-rows per sampling
+ * sequence for its draw.
+ */
+int libraspec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
+                     const float* conf, const float* dstat, const int32_t* L, const float* temperature, int B,
+                     int K, int V, uint64_t seed, uint64_t round_offset, uint32_t seq_offset,
+                     int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * The whole round on one stream: confidence -> selection -> n_layers verify
+ * attention layers -> acceptance. Q, Kc, Vc, O point to HOST arrays of
+ * n_layers DEVICE pointers (layer l uses Q[l], Kc[l], Vc[l], O[l]); lse is a
+ * host array of n_layers device pointers or NULL. conf, dstat, L are device
+ * outputs the round also returns. Same shapes and rules as the four calls.
+ */
+int libraspec_verify_round(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                           const float* cost_table, const float* target_logits, const uint16_t* const* Q,
+                           const uint16_t* const* Kc, const uint16_t* const* Vc, uint16_t* const* O,
+                           float* const* lse, int n_layers, const int32_t* kv_len, int B, int K, int V, int Hq,
+                           int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                           uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
+                           int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                           void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LIBRASPEC_H */

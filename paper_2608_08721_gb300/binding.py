@@ -1,0 +1,262 @@
+"""Thin ctypes binding of libraspec.so (include/libraspec.h).
+
+Functions carry the C names and take torch tensors; they only check and
+marshal arguments (dtype, device, contiguity, shapes) and pass the current
+CUDA stream. Every step of the verify round runs in the library's kernels.
+A missing or unloadable library raises; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence, Tuple
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libraspec.so")
+
+OK, EINVAL, EUNSUPPORTED, ECUDA, EDEVICE = 0, -1, -2, -3, -4
+ST_BAD_LENGTH, ST_BAD_COST, ST_KV_OVERFLOW, ST_BAD_TOKEN, ST_TIMEOUT, ST_MISSING_INPUT = 1, 2, 4, 8, 16, 32
+MAX_K = 64
+
+# Every entry point declared in include/libraspec.h, with its ctypes signature.
+_P, _I, _U32, _U64, _F, _SZ = (ctypes.c_void_p, ctypes.c_int, ctypes.c_uint32, ctypes.c_uint64, ctypes.c_float,
+                               ctypes.c_size_t)
+SIGNATURES = {
+    "libraspec_version": (ctypes.c_char_p, []),
+    "libraspec_status_string": (ctypes.c_char_p, [_I]),
+    "libraspec_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I, _I]),
+    "libraspec_workspace_init": (_I, [_P, _SZ, _P]),
+    "libraspec_get_status": (_I, [_P, _P, _P]),
+    "libraspec_confidence": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
+    "libraspec_select_lengths": (_I, [_P, _P, _I, _I, _P, _P, _SZ, _P]),
+    "libraspec_verify_attn": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
+    "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
+    "libraspec_verify_round": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _I,
+                                    _F, _U64, _U64, _U32, _P, _P, _P, _P, _P, _P, _SZ, _P]),
+}
+
+_lib = None
+
+
+class LibraspecError(RuntimeError):
+    def __init__(self, what: str, status: int):
+        super().__init__("%s failed: %s (%d)" % (what, _status_name(status), status))
+        self.status = status
+
+
+def _status_name(status: int) -> str:
+    return {OK: "ok", EINVAL: "invalid argument", EUNSUPPORTED: "unsupported shape", ECUDA: "CUDA error",
+            EDEVICE: "device-reported violation"}.get(status, "unknown")
+
+
+def load() -> ctypes.CDLL:
+    """Load libraspec.so (built by build.py); raises if it is missing."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError("libraspec.so is not built (%s); run `python -m paper_2608_08721_gb300.build` or "
+                           "__graft_entry__.build()" % LIB_PATH)
+    lib = ctypes.CDLL(LIB_PATH)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(rc: int, what: str) -> None:
+    if rc != OK:
+        raise LibraspecError(what, rc)
+
+
+def _stream(stream: Optional[torch.cuda.Stream]) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _req(t: torch.Tensor, dtype, name: str, shape=None) -> torch.Tensor:
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("%s must be a torch tensor" % name)
+    if t.dtype != dtype:
+        raise TypeError("%s must be %s, got %s" % (name, dtype, t.dtype))
+    if not t.is_cuda:
+        raise ValueError("%s must be on a CUDA device" % name)
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError("%s must have shape %s, got %s" % (name, tuple(shape), tuple(t.shape)))
+    return t
+
+
+class Workspace:
+    """Device scratch for one round's shapes (a zero-filled torch buffer)."""
+
+    def __init__(self, B, K, V, Hq=1, Hkv=1, head_dim=64, S_cap=1, device=None):
+        lib = load()
+        self.nbytes = int(lib.libraspec_workspace_size(B, K, V, Hq, Hkv, head_dim, S_cap))
+        if self.nbytes == 0:
+            raise ValueError("invalid workspace shapes")
+        dev = torch.device("cuda") if device is None else torch.device(device)
+        self.buf = torch.zeros(self.nbytes, dtype=torch.uint8, device=dev)
+        if self.buf.data_ptr() % 256:
+            raise RuntimeError("workspace allocation is not 256-byte aligned")
+        self.shapes = (B, K, V, Hq, Hkv, head_dim, S_cap)
+
+    @property
+    def ptr(self) -> int:
+        return self.buf.data_ptr()
+
+
+def libraspec_version() -> str:
+    return load().libraspec_version().decode()
+
+
+def libraspec_workspace_size(B, K, V, Hq, Hkv, head_dim, S_cap) -> int:
+    return int(load().libraspec_workspace_size(B, K, V, Hq, Hkv, head_dim, S_cap))
+
+
+def libraspec_get_status(ws: Workspace, stream=None) -> int:
+    out = ctypes.c_int32(0)
+    rc = load().libraspec_get_status(ctypes.c_void_p(ws.ptr), _stream(stream), ctypes.byref(out))
+    if rc not in (OK, EDEVICE):
+        _check(rc, "libraspec_get_status")
+    return int(out.value)
+
+
+def libraspec_confidence(draft_logits, draft_tokens, temperature, ws: Workspace, conf=None, dstat=None,
+                         stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    B, K, V = draft_logits.shape
+    _req(draft_logits, torch.float32, "draft_logits")
+    _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+    _req(temperature, torch.float32, "temperature", (B,))
+    dev = draft_logits.device
+    conf = torch.empty((B, K), dtype=torch.float32, device=dev) if conf is None else _req(conf, torch.float32,
+                                                                                          "conf", (B, K))
+    dstat = torch.empty((B, K, 2), dtype=torch.float32, device=dev) if dstat is None else _req(
+        dstat, torch.float32, "dstat", (B, K, 2))
+    rc = load().libraspec_confidence(_ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature), B, K, V,
+                                     _ptr(conf), _ptr(dstat), ws.ptr, ws.nbytes, _stream(stream))
+    _check(rc, "libraspec_confidence")
+    return conf, dstat
+
+
+def libraspec_select_lengths(conf, cost_table, ws: Workspace, L=None, stream=None) -> torch.Tensor:
+    B, K = conf.shape
+    _req(conf, torch.float32, "conf")
+    _req(cost_table, torch.float32, "cost_table", (K + 1,))
+    L = torch.empty((B,), dtype=torch.int32, device=conf.device) if L is None else _req(L, torch.int32, "L", (B,))
+    rc = load().libraspec_select_lengths(_ptr(conf), _ptr(cost_table), B, K, _ptr(L), ws.ptr, ws.nbytes,
+                                         _stream(stream))
+    _check(rc, "libraspec_select_lengths")
+    return L
+
+
+def libraspec_verify_attn(Q, Kc, Vc, kv_len, L, ws: Workspace, softmax_scale=None, O=None, lse=None,
+                          want_lse=False, stream=None):
+    B, K1, Hq, D = Q.shape
+    _, Hkv, S_cap, D2 = Kc.shape
+    _req(Q, torch.bfloat16, "Q")
+    _req(Kc, torch.bfloat16, "Kc", (B, Hkv, S_cap, D))
+    _req(Vc, torch.bfloat16, "Vc", (B, Hkv, S_cap, D))
+    _req(kv_len, torch.int32, "kv_len", (B,))
+    _req(L, torch.int32, "L", (B,))
+    if softmax_scale is None:
+        softmax_scale = D ** -0.5
+    O = torch.empty_like(Q) if O is None else _req(O, torch.bfloat16, "O", Q.shape)
+    if want_lse and lse is None:
+        lse = torch.empty((B, K1, Hq), dtype=torch.float32, device=Q.device)
+    rc = load().libraspec_verify_attn(_ptr(Q), _ptr(Kc), _ptr(Vc), _ptr(kv_len), _ptr(L), B, K1 - 1, Hq, Hkv, D,
+                                      S_cap, float(softmax_scale), _ptr(O), _ptr(lse), ws.ptr, ws.nbytes,
+                                      _stream(stream))
+    _check(rc, "libraspec_verify_attn")
+    return O, lse
+
+
+def libraspec_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, seed: int,
+                     ws: Workspace, round_offset: int = 0, seq_offset: int = 0, n_accepted=None, bonus_token=None,
+                     stream=None):
+    B, K1, V = target_logits.shape
+    K = K1 - 1
+    _req(target_logits, torch.float32, "target_logits")
+    _req(draft_logits, torch.float32, "draft_logits", (B, K, V))
+    _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+    if conf is not None:
+        _req(conf, torch.float32, "conf", (B, K))
+    if dstat is not None:
+        _req(dstat, torch.float32, "dstat", (B, K, 2))
+    _req(L, torch.int32, "L", (B,))
+    _req(temperature, torch.float32, "temperature", (B,))
+    dev = target_logits.device
+    n_accepted = torch.empty((B,), dtype=torch.int32, device=dev) if n_accepted is None else n_accepted
+    bonus_token = torch.empty((B,), dtype=torch.int32, device=dev) if bonus_token is None else bonus_token
+    rc = load().libraspec_accept(_ptr(target_logits), _ptr(draft_logits), _ptr(draft_tokens), _ptr(conf),
+                                 _ptr(dstat), _ptr(L), _ptr(temperature), B, K, V, int(seed) & (2**64 - 1),
+                                 int(round_offset), int(seq_offset), _ptr(n_accepted), _ptr(bonus_token), ws.ptr,
+                                 ws.nbytes, _stream(stream))
+    _check(rc, "libraspec_accept")
+    return n_accepted, bonus_token
+
+
+def _ptr_array(tensors: Sequence[Optional[torch.Tensor]]):
+    arr = (ctypes.c_void_p * max(1, len(tensors)))()
+    for i, t in enumerate(tensors):
+        arr[i] = None if t is None else t.data_ptr()
+    return arr
+
+
+class RoundOutputs:
+    def __init__(self, conf, dstat, L, n_accepted, bonus_token, O, lse):
+        self.conf, self.dstat, self.L = conf, dstat, L
+        self.n_accepted, self.bonus_token = n_accepted, bonus_token
+        self.O, self.lse = O, lse
+
+
+def libraspec_verify_round(draft_logits, draft_tokens, temperature, cost_table, target_logits, layers, kv_len,
+                           seed: int, ws: Workspace, round_offset: int = 0, seq_offset: int = 0,
+                           softmax_scale=None, outputs: Optional[RoundOutputs] = None, want_lse=False,
+                           stream=None) -> RoundOutputs:
+    """layers: sequence of dicts with Q, Kc, Vc (and optionally O)."""
+    B, K, V = draft_logits.shape
+    _req(draft_logits, torch.float32, "draft_logits")
+    _req(target_logits, torch.float32, "target_logits", (B, K + 1, V))
+    _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+    _req(temperature, torch.float32, "temperature", (B,))
+    _req(cost_table, torch.float32, "cost_table", (K + 1,))
+    _req(kv_len, torch.int32, "kv_len", (B,))
+    n_layers = len(layers)
+    Hq, D = (layers[0]["Q"].shape[2], layers[0]["Q"].shape[3]) if n_layers else (1, 64)
+    Hkv, S_cap = (layers[0]["Kc"].shape[1], layers[0]["Kc"].shape[2]) if n_layers else (1, 1)
+    for i, lay in enumerate(layers):
+        _req(lay["Q"], torch.bfloat16, "Q[%d]" % i, (B, K + 1, Hq, D))
+        _req(lay["Kc"], torch.bfloat16, "Kc[%d]" % i, (B, Hkv, S_cap, D))
+        _req(lay["Vc"], torch.bfloat16, "Vc[%d]" % i, (B, Hkv, S_cap, D))
+    dev = draft_logits.device
+    if outputs is None:
+        outputs = RoundOutputs(
+            torch.empty((B, K), dtype=torch.float32, device=dev), torch.empty((B, K, 2), dtype=torch.float32, device=dev),
+            torch.empty((B,), dtype=torch.int32, device=dev), torch.empty((B,), dtype=torch.int32, device=dev),
+            torch.empty((B,), dtype=torch.int32, device=dev),
+            [lay.get("O") if lay.get("O") is not None else torch.empty_like(lay["Q"]) for lay in layers],
+            [torch.empty((B, K + 1, Hq), dtype=torch.float32, device=dev) for _ in layers] if want_lse else None)
+    if softmax_scale is None:
+        softmax_scale = D ** -0.5
+    qa = _ptr_array([lay["Q"] for lay in layers])
+    ka = _ptr_array([lay["Kc"] for lay in layers])
+    va = _ptr_array([lay["Vc"] for lay in layers])
+    oa = _ptr_array(outputs.O)
+    la = _ptr_array(outputs.lse) if outputs.lse is not None else None
+    rc = load().libraspec_verify_round(
+        _ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature), _ptr(cost_table), _ptr(target_logits), qa, ka, va,
+        oa, la, n_layers, _ptr(kv_len), B, K, V, Hq, Hkv, D, S_cap, float(softmax_scale), int(seed) & (2**64 - 1),
+        int(round_offset), int(seq_offset), _ptr(outputs.conf), _ptr(outputs.dstat), _ptr(outputs.L),
+        _ptr(outputs.n_accepted), _ptr(outputs.bonus_token), ws.ptr, ws.nbytes, _stream(stream))
+    _check(rc, "libraspec_verify_round")
+    return outputs

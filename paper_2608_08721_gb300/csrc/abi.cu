@@ -1,0 +1,203 @@
+// The C ABI (include/libraspec.h): argument checks, workspace, status and
+// the whole-round entry point. Kernels live in conf_select.cu, attn.cu and
+// accept.cu.
+#include <cstdio>
+#include <cstring>
+
+#include "common.cuh"
+
+namespace libraspec {
+
+cudaError_t launch_confidence(const float*, const int32_t*, const float*, int, int, int, float*, float*, char*,
+                              const WsLayout&, cudaStream_t);
+cudaError_t launch_select(const float*, const float*, int, int, int32_t*, char*, const WsLayout&, cudaStream_t);
+cudaError_t launch_verify_attn(const uint16_t*, const uint16_t*, const uint16_t*, const int32_t*, const int32_t*,
+                               int, int, int, int, int, int, float, uint16_t*, float*, char*, const WsLayout&,
+                               cudaStream_t);
+cudaError_t launch_accept(const float*, const float*, const int32_t*, const float*, const float*, const int32_t*,
+                          const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, char*,
+                          const WsLayout&, cudaStream_t);
+
+int num_sms_current() {
+  static int cached_dev = -1, cached_sms = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (dev != cached_dev) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 148;
+    cached_sms = sms;
+    cached_dev = dev;
+  }
+  return cached_sms;
+}
+
+}  // namespace libraspec
+
+using namespace libraspec;
+
+namespace {
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+bool shapes_ok(int B, int K, int V) {
+  return B >= 0 && B <= LIBRASPEC_MAX_B && K >= 0 && K <= LIBRASPEC_MAX_K && V >= 1;
+}
+
+bool attn_shapes_ok(int B, int K, int Hq, int Hkv, int D, int S_cap) {
+  if (B < 0 || B > LIBRASPEC_MAX_B || K < 0 || K > LIBRASPEC_MAX_K) return false;
+  if (Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || S_cap < 1) return false;
+  if ((long)(K + 1) * (Hq / Hkv) > 512) return false;
+  if ((long)B * Hkv > (1L << 30)) return false;
+  (void)D;
+  return true;
+}
+
+int from_cuda(cudaError_t e) { return e == cudaSuccess ? LIBRASPEC_OK : LIBRASPEC_ECUDA; }
+
+}  // namespace
+
+extern "C" {
+
+const char* libraspec_version(void) { return "libraspec 0.1 (sm_103a)"; }
+
+const char* libraspec_status_string(int status) {
+  switch (status) {
+    case LIBRASPEC_OK: return "ok";
+    case LIBRASPEC_EINVAL: return "invalid argument";
+    case LIBRASPEC_EUNSUPPORTED: return "unsupported shape";
+    case LIBRASPEC_ECUDA: return "CUDA error";
+    case LIBRASPEC_EDEVICE: return "device-reported violation";
+    default: return "unknown status";
+  }
+}
+
+size_t libraspec_workspace_size(int B, int K, int V, int Hq, int Hkv, int head_dim, int S_cap) {
+  if (!shapes_ok(B, K, V) || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || (head_dim != 64 && head_dim != 128) ||
+      S_cap < 1)
+    return 0;
+  return ws_layout(B, K, V, Hq, Hkv, head_dim, S_cap).total;
+}
+
+int libraspec_workspace_init(void* workspace, size_t bytes, void* stream) {
+  if (!workspace || !aligned(workspace, 256)) return LIBRASPEC_EINVAL;
+  return from_cuda(cudaMemsetAsync(workspace, 0, bytes, static_cast<cudaStream_t>(stream)));
+}
+
+int libraspec_get_status(void* workspace, void* stream, int32_t* host_status) {
+  if (!workspace || !host_status) return LIBRASPEC_EINVAL;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int32_t v = 0;
+  cudaError_t e = cudaMemcpyAsync(&v, workspace, sizeof(v), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess && v != 0) e = cudaMemsetAsync(workspace, 0, sizeof(v), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return LIBRASPEC_ECUDA;
+  *host_status = v;
+  return v == 0 ? LIBRASPEC_OK : LIBRASPEC_EDEVICE;
+}
+
+// The workspace must hold the regions of the layout computed from the call's
+// own shapes; the layout puts every region after the ones of smaller calls,
+// so we check the bytes the call touches.
+static bool ws_ok(const void* ws, size_t ws_bytes, const WsLayout& lay) {
+  return ws && aligned(ws, 256) && ws_bytes >= lay.total;
+}
+
+int libraspec_confidence(const float* draft_logits, const int32_t* draft_tokens, const float* temperature, int B,
+                         int K, int V, float* conf, float* dstat, void* workspace, size_t ws_bytes, void* stream) {
+  if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
+  if (B * K == 0) return LIBRASPEC_OK;
+  if (!draft_logits || !draft_tokens || !temperature || !conf) return LIBRASPEC_EINVAL;
+  if (!aligned(draft_logits, 4) || !aligned(conf, 4) || (dstat && !aligned(dstat, 4))) return LIBRASPEC_EINVAL;
+  const WsLayout lay = ws_layout(B, K, V, 1, 1, 64, 1);
+  if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_confidence(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat,
+                                     static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+}
+
+int libraspec_select_lengths(const float* conf, const float* cost_table, int B, int K, int32_t* L, void* workspace,
+                             size_t ws_bytes, void* stream) {
+  if (!shapes_ok(B, K, 1)) return LIBRASPEC_EINVAL;
+  if (B == 0) return LIBRASPEC_OK;
+  if ((!conf && K > 0) || !cost_table || !L) return LIBRASPEC_EINVAL;
+  const WsLayout lay = ws_layout(B, K, 1, 1, 1, 64, 1);
+  if (!workspace || !aligned(workspace, 256) || ws_bytes < 256) return LIBRASPEC_EINVAL;
+  return from_cuda(
+      launch_select(conf, cost_table, B, K, L, static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+}
+
+int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc, const int32_t* kv_len,
+                          const int32_t* L, int B, int K, int Hq, int Hkv, int head_dim, int S_cap, float softmax_scale,
+                          uint16_t* O, float* lse, void* workspace, size_t ws_bytes, void* stream) {
+  if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
+  if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap)) return LIBRASPEC_EINVAL;
+  if (B == 0) return LIBRASPEC_OK;
+  if (!Q || !Kc || !Vc || !kv_len || !L || !O) return LIBRASPEC_EINVAL;
+  if (!aligned(Q, 16) || !aligned(Kc, 16) || !aligned(Vc, 16) || !aligned(O, 16)) return LIBRASPEC_EINVAL;
+  if (lse && !aligned(lse, 4)) return LIBRASPEC_EINVAL;
+  if (!(softmax_scale > 0.f)) return LIBRASPEC_EINVAL;
+  const WsLayout lay = ws_layout(B, K, 1, Hq, Hkv, head_dim, S_cap);
+  if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_verify_attn(Q, Kc, Vc, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap, softmax_scale, O, lse,
+                                      static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+}
+
+int libraspec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
+                     const float* conf, const float* dstat, const int32_t* L, const float* temperature, int B, int K,
+                     int V, uint64_t seed, uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted,
+                     int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
+  if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
+  if (B == 0) return LIBRASPEC_OK;
+  if (!target_logits || (!draft_logits && K > 0) || (!draft_tokens && K > 0) || !L || !temperature ||
+      !n_accepted || !bonus_token)
+    return LIBRASPEC_EINVAL;
+  if (!aligned(target_logits, 4) || (draft_logits && !aligned(draft_logits, 4))) return LIBRASPEC_EINVAL;
+  const WsLayout lay = ws_layout(B, K, V, 1, 1, 64, 1);
+  if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V,
+                                 seed, round_offset, seq_offset, n_accepted, bonus_token,
+                                 static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+}
+
+int libraspec_verify_round(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                           const float* cost_table, const float* target_logits, const uint16_t* const* Q,
+                           const uint16_t* const* Kc, const uint16_t* const* Vc, uint16_t* const* O,
+                           float* const* lse, int n_layers, const int32_t* kv_len, int B, int K, int V, int Hq,
+                           int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                           uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
+                           int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                           void* stream) {
+  if (!shapes_ok(B, K, V) || n_layers < 0) return LIBRASPEC_EINVAL;
+  if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
+  if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap)) return LIBRASPEC_EINVAL;
+  if (B == 0) return LIBRASPEC_OK;
+  if (n_layers > 0 && (!Q || !Kc || !Vc || !O)) return LIBRASPEC_EINVAL;
+  if (!conf || !dstat || !L || !kv_len) return LIBRASPEC_EINVAL;
+  const WsLayout lay = ws_layout(B, K, V, Hq, Hkv, head_dim, S_cap);
+  if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!Q[l] || !Kc[l] || !Vc[l] || !O[l]) return LIBRASPEC_EINVAL;
+    if (!aligned(Q[l], 16) || !aligned(Kc[l], 16) || !aligned(Vc[l], 16) || !aligned(O[l], 16))
+      return LIBRASPEC_EINVAL;
+  }
+  if (!(softmax_scale > 0.f)) return LIBRASPEC_EINVAL;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  int rc = LIBRASPEC_OK;
+  if (K > 0) {
+    rc = libraspec_confidence(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes,
+                              stream);
+    if (rc != LIBRASPEC_OK) return rc;
+  }
+  rc = from_cuda(launch_select(conf, cost_table, B, K, L, ws, lay, s));
+  if (rc != LIBRASPEC_OK) return rc;
+  for (int l = 0; l < n_layers; ++l) {
+    rc = from_cuda(launch_verify_attn(Q[l], Kc[l], Vc[l], kv_len, L, B, K, Hq, Hkv, head_dim, S_cap, softmax_scale,
+                                      O[l], lse ? lse[l] : nullptr, ws, lay, s));
+    if (rc != LIBRASPEC_OK) return rc;
+  }
+  return libraspec_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed,
+                          round_offset, seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,391 @@
+// Step 4: acceptance (greedy argmax match / rejection sampling).
+#include "rowpass.cuh"
+
+namespace libraspec {
+
+// ---------------------------------------------------------------------------
+// Row statistics of the verified target rows. Grid (nsplit, K+1, B); rows
+// j > L_b exit at once. Greedy sequences need only max / argmax; sampling
+// sequences need (m, Z) at their temperature. Partials of a row are merged by
+// the last CTA to finish (atomic ticket) into row_stat[b, j].
+// ---------------------------------------------------------------------------
+template <bool VEC>
+__global__ void __launch_bounds__(kRowThreads) accept_rows_kernel(
+    const float* __restrict__ target, const int32_t* __restrict__ Ls, const float* __restrict__ temperature,
+    int K, int V, int nsplit, int chunk, RowPartial* __restrict__ part, uint32_t* __restrict__ cnt,
+    RowStat* __restrict__ stat, int* __restrict__ status) {
+  __shared__ float smf[64];
+  __shared__ int smi[32];
+  __shared__ int last;
+  const int split = blockIdx.x, j = blockIdx.y, b = blockIdx.z;
+  const int Lb = Ls[b];
+  if (Lb < 0 || Lb > K) {
+    if (split == 0 && j == 0 && threadIdx.x == 0) raise_status(status, LIBRASPEC_ST_BAD_LENGTH);
+    return;
+  }
+  if (j > Lb) return;
+  const int row = b * (K + 1) + j;
+  const float tb = temperature[b];
+  const bool sampling = tb > 0.f;
+  const float T = sampling ? tb : 1.f;
+  const float c = (float)(1.4426950408889634 / (double)T);
+  const float* xr = target + (size_t)row * V;
+  const int c0 = split * chunk, c1 = min(V, c0 + chunk);
+
+  SumAcc sa;
+  ArgAcc aa;
+  sa.init();
+  aa.init();
+  float m;
+  int arg = 0;
+  float s = 0.f;
+  if (sampling) {
+    row_slice_pass<true, false, VEC>(xr, c0, c1, c, sa, aa);
+    m = sa.m;
+    s = sa.value();
+    cta_reduce_sum(m, s, c, smf);
+  } else {
+    row_slice_pass<false, true, VEC>(xr, c0, c1, c, sa, aa);
+    m = aa.m;
+    arg = aa.arg;
+    cta_reduce_arg(m, arg, smf, smi);
+  }
+  if (nsplit == 1) {
+    if (threadIdx.x == 0) {
+      RowStat st;
+      st.m = m;
+      st.arg = arg;
+      st.Z = (double)s;
+      stat[row] = st;
+    }
+    return;
+  }
+  if (threadIdx.x == 0) {
+    RowPartial p;
+    p.m = m;
+    p.arg = arg;
+    p.s = (double)s;
+    part[(size_t)row * kRowMaxSplits + split] = p;
+    __threadfence();
+    const uint32_t ticket = atomicAdd(&cnt[row], 1u);
+    last = (ticket == (uint32_t)(nsplit - 1));
+  }
+  __syncthreads();
+  if (!last || threadIdx.x >= 32) return;
+  __threadfence();
+  float M;
+  int A;
+  double Z;
+  warp_merge_partials(part + (size_t)row * kRowMaxSplits, nsplit, (double)T, !sampling, M, A, Z);
+  if (threadIdx.x == 0) {
+    RowStat st;
+    st.m = M;
+    st.arg = sampling ? 0 : A;
+    st.Z = Z;
+    stat[row] = st;
+    cnt[row] = 0u;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Decision and draw. Grid (nsplit, B). Every CTA of sequence b first takes
+// the sequence's accept / reject decisions itself (they are cheap and
+// deterministic), then, for sampling sequences, streams its slice of the
+// vocabulary for the exponential race (argmin_v E_v / w_v, E_v = -ln u_v):
+// w = max(0, p_r - q_r) after a rejection at r, or w = p_{L_b} (unnormalised)
+// when all L_b drafts were accepted. The last CTA merges the slices.
+// ---------------------------------------------------------------------------
+struct Decision {
+  int n;       // accepted drafts (r)
+  int bonus;   // greedy: emitted token; sampling: -1 (drawn below)
+  bool ok;
+};
+
+__device__ Decision decide(int b, int K, int V, const float* __restrict__ target,
+                           const int32_t* __restrict__ tokens, const float* __restrict__ conf,
+                           const int32_t* __restrict__ Ls, const float* __restrict__ temperature,
+                           const RowStat* __restrict__ stat, uint64_t seed, uint64_t round_offset,
+                           uint32_t seq_offset, int* __restrict__ status) {
+  // executed by one full warp
+  const int lane = threadIdx.x & 31;
+  Decision d{0, -1, true};
+  const int Lb = Ls[b];
+  if (Lb < 0 || Lb > K) {
+    d.ok = false;
+    return d;
+  }
+  const float tb = temperature[b];
+  const RowStat* st = stat + (size_t)b * (K + 1);
+  int n = Lb;
+  for (int base = 0; base < Lb; base += 32) {
+    const int jj = base + lane;
+    bool reject = false;
+    if (jj < Lb) {
+      const int x = tokens[(size_t)b * K + jj];
+      if (x < 0 || x >= V) {
+        raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
+        reject = true;
+      } else if (tb == 0.f) {
+        reject = __ldcg(&st[jj].arg) != x;
+      } else if (conf == nullptr) {
+        reject = true;
+      } else {
+        const double T = (double)tb;
+        const double y = (double)target[((size_t)b * (K + 1) + jj) * V + x];
+        const double p = exp((y - (double)__ldcg(&st[jj].m)) / T) / __ldcg(&st[jj].Z);
+        const double q = (double)conf[(size_t)b * K + jj];
+        const double ratio = (q <= p) ? 1.0 : p / q;
+        const uint4 w = philox_block(seed, 0u, (uint32_t)jj, seq_offset + (uint32_t)b, 0u, round_offset);
+        const double u = (double)word_to_uniform(w.x);
+        reject = !(u < ratio);
+      }
+    }
+    const unsigned ball = __ballot_sync(0xffffffffu, reject);
+    if (ball) {
+      n = base + __ffs(ball) - 1;
+      break;
+    }
+  }
+  d.n = n;
+  if (tb == 0.f) d.bonus = __ldcg(&st[n].arg);
+  return d;
+}
+
+template <bool VEC>
+__global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
+    const float* __restrict__ target, const float* __restrict__ draft, const int32_t* __restrict__ tokens,
+    const float* __restrict__ conf, const float* __restrict__ dstat, const int32_t* __restrict__ Ls,
+    const float* __restrict__ temperature, int K, int V, int nsplit, int chunk, uint64_t seed,
+    uint64_t round_offset, uint32_t seq_offset, const RowStat* __restrict__ stat,
+    RacePartial* __restrict__ part, uint32_t* __restrict__ cnt, int32_t* __restrict__ n_accepted,
+    int32_t* __restrict__ bonus_token, int* __restrict__ status) {
+  __shared__ int sh_n, sh_bonus, sh_ok, last;
+  __shared__ float smk[32];
+  __shared__ int smi[32];
+  const int split = blockIdx.x, b = blockIdx.y;
+  if (threadIdx.x < 32) {
+    const Decision d = decide(b, K, V, target, tokens, conf, Ls, temperature, stat, seed, round_offset,
+                              seq_offset, status);
+    if (threadIdx.x == 0) {
+      sh_n = d.n;
+      sh_bonus = d.bonus;
+      sh_ok = d.ok;
+    }
+  }
+  __syncthreads();
+  const int n = sh_n;
+  if (!sh_ok) {
+    if (split == 0 && threadIdx.x == 0) {
+      n_accepted[b] = 0;
+      bonus_token[b] = 0;
+      raise_status(status, LIBRASPEC_ST_BAD_LENGTH);
+    }
+    return;
+  }
+  const float tb = temperature[b];
+  if (tb == 0.f) {
+    if (split == 0 && threadIdx.x == 0) {
+      n_accepted[b] = n;
+      bonus_token[b] = sh_bonus;
+    }
+    return;
+  }
+  if (conf == nullptr || dstat == nullptr) {  // sampling needs q and the drafter row statistics
+    if (split == 0 && threadIdx.x == 0) {
+      n_accepted[b] = 0;
+      bonus_token[b] = 0;
+      raise_status(status, LIBRASPEC_ST_MISSING_INPUT);
+    }
+    return;
+  }
+  // ---- sampling: exponential race over the vocabulary at position n ----
+  const int Lb = Ls[b];
+  const bool residual = n < Lb;
+  const float c = (float)(1.4426950408889634 / (double)tb);
+  const RowStat st = stat[(size_t)b * (K + 1) + n];
+  const float* yr = target + ((size_t)b * (K + 1) + n) * V;
+  const float* dr = residual ? draft + ((size_t)b * K + n) * V : nullptr;
+  const float mp = st.m;
+  const float invZp = (float)(1.0 / st.Z);
+  float mq = 0.f, invZq = 0.f;
+  if (residual) {
+    mq = dstat[2 * ((size_t)b * K + n)];
+    invZq = 1.0f / dstat[2 * ((size_t)b * K + n) + 1];
+  }
+  const uint32_t seq = seq_offset + (uint32_t)b;
+  const int c0 = split * chunk, c1 = min(V, c0 + chunk);
+  float best = INFINITY;
+  int besti = 0x7fffffff;
+  // groups of 4 consecutive tokens share one Philox block
+  for (int g = (c0 >> 2) + threadIdx.x; 4 * g < c1; g += kRowThreads) {
+    const uint4 w4 = philox_block(seed, (uint32_t)g, (uint32_t)n, seq, 1u, round_offset);
+    const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
+    float yv[4], dv[4];
+    if (VEC) {
+      const float4 a = ld_stream4(yr + 4 * g);
+      yv[0] = a.x; yv[1] = a.y; yv[2] = a.z; yv[3] = a.w;
+      if (residual) {
+        const float4 e = ld_stream4(dr + 4 * g);
+        dv[0] = e.x; dv[1] = e.y; dv[2] = e.z; dv[3] = e.w;
+      }
+    } else {
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int v = 4 * g + t;
+        yv[t] = v < V ? yr[v] : -INFINITY;
+        dv[t] = (residual && v < V) ? dr[v] : 0.f;
+      }
+    }
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int v = 4 * g + t;
+      if (v >= c1) break;
+      float wv = exp2f((yv[t] - mp) * c);
+      if (residual) {
+        const float pv = wv * invZp;
+        const float qv = exp2f((dv[t] - mq) * c) * invZq;
+        wv = pv - qv;
+      }
+      if (wv > 0.f) {
+        const float E = -logf(word_to_uniform(ws[t]));
+        const float key = E / wv;
+        argmin_combine(best, besti, key, v);
+      }
+    }
+  }
+  // CTA reduction of (key, index)
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float k2 = __shfl_xor_sync(0xffffffffu, best, off);
+    const int i2 = __shfl_xor_sync(0xffffffffu, besti, off);
+    argmin_combine(best, besti, k2, i2);
+  }
+  if (lane == 0) { smk[warp] = best; smi[warp] = besti; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    best = smk[0];
+    besti = smi[0];
+    for (int w = 1; w < kRowThreads / 32; ++w) argmin_combine(best, besti, smk[w], smi[w]);
+    RacePartial p;
+    p.key = best;
+    p.idx = besti;
+    part[(size_t)b * kRaceMaxSplits + split] = p;
+    __threadfence();
+    const uint32_t ticket = atomicAdd(&cnt[b], 1u);
+    last = (ticket == (uint32_t)(nsplit - 1));
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  if (threadIdx.x < 32) {
+    float kb = INFINITY;
+    int ib = 0x7fffffff;
+    for (int i = lane; i < nsplit; i += 32)
+      argmin_combine(kb, ib, __ldcg(&part[(size_t)b * kRaceMaxSplits + i].key),
+                     __ldcg(&part[(size_t)b * kRaceMaxSplits + i].idx));
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const float k2 = __shfl_xor_sync(0xffffffffu, kb, off);
+      const int i2 = __shfl_xor_sync(0xffffffffu, ib, off);
+      argmin_combine(kb, ib, k2, i2);
+    }
+    if (lane == 0) {
+      cnt[b] = 0u;
+      sh_bonus = ib;
+      sh_ok = (kb < INFINITY);
+    }
+  }
+  __syncthreads();
+  if (sh_ok) {
+    if (threadIdx.x == 0) {
+      n_accepted[b] = n;
+      bonus_token[b] = sh_bonus;
+    }
+    return;
+  }
+  // Residual identically zero (p_r == q_r to rounding): draw from p_r
+  // instead, in this CTA alone (rare).
+  best = INFINITY;
+  besti = 0x7fffffff;
+  for (int v = threadIdx.x; v < V; v += kRowThreads) {
+    const uint4 w4 = philox_block(seed, (uint32_t)(v >> 2), (uint32_t)n, seq, 1u, round_offset);
+    const uint32_t wsel = (v & 3) == 0 ? w4.x : (v & 3) == 1 ? w4.y : (v & 3) == 2 ? w4.z : w4.w;
+    const float wv = exp2f((yr[v] - mp) * c);
+    if (wv > 0.f) argmin_combine(best, besti, -logf(word_to_uniform(wsel)) / wv, v);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float k2 = __shfl_xor_sync(0xffffffffu, best, off);
+    const int i2 = __shfl_xor_sync(0xffffffffu, besti, off);
+    argmin_combine(best, besti, k2, i2);
+  }
+  if (lane == 0) { smk[warp] = best; smi[warp] = besti; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    best = smk[0];
+    besti = smi[0];
+    for (int w = 1; w < kRowThreads / 32; ++w) argmin_combine(best, besti, smk[w], smi[w]);
+    n_accepted[b] = n;
+    bonus_token[b] = besti == 0x7fffffff ? 0 : besti;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host launchers.
+// ---------------------------------------------------------------------------
+int num_sms_current();
+
+cudaError_t launch_accept(const float* target, const float* draft, const int32_t* tokens, const float* conf,
+                          const float* dstat, const int32_t* L, const float* temperature, int B, int K, int V,
+                          uint64_t seed, uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted,
+                          int32_t* bonus, char* ws, const WsLayout& lay, cudaStream_t stream) {
+  if (B == 0) return cudaSuccess;
+  const int sms = num_sms_current();
+  const bool vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(target) & 15) == 0) &&
+                   (draft == nullptr || (reinterpret_cast<uintptr_t>(draft) & 15) == 0);
+  auto* st = reinterpret_cast<int*>(ws + lay.status);
+  auto* rstat = reinterpret_cast<RowStat*>(ws + lay.row_stat);
+  {
+    const long rows = (long)B * (K + 1);
+    const int nsplit0 = row_splits(rows, V, sms, kRowMaxSplits, 2048);
+    const int chunk = row_chunk(V, nsplit0);
+    const int nsplit = (V + chunk - 1) / chunk;
+    dim3 grid(nsplit, K + 1, B);
+    auto* part = reinterpret_cast<RowPartial*>(ws + lay.row_part);
+    auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.row_cnt);
+    if (vec)
+      accept_rows_kernel<true><<<grid, kRowThreads, 0, stream>>>(target, L, temperature, K, V, nsplit, chunk,
+                                                                  part, cnt, rstat, st);
+    else
+      accept_rows_kernel<false><<<grid, kRowThreads, 0, stream>>>(target, L, temperature, K, V, nsplit, chunk,
+                                                                   part, cnt, rstat, st);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  {
+    // race slices: enough CTAs per sequence to stream one or two V-rows fast
+    long target_ctas = 2L * sms;
+    int nsplit = (int)((target_ctas + B - 1) / B);
+    const int cap = (V + 4095) / 4096;
+    if (nsplit > cap) nsplit = cap;
+    if (nsplit > kRaceMaxSplits) nsplit = kRaceMaxSplits;
+    if (nsplit < 1) nsplit = 1;
+    int chunk = row_chunk(V, nsplit);
+    nsplit = (V + chunk - 1) / chunk;
+    dim3 grid(nsplit, B);
+    auto* part = reinterpret_cast<RacePartial*>(ws + lay.race_part);
+    auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.race_cnt);
+    if (vec)
+      accept_decide_kernel<true><<<grid, kRowThreads, 0, stream>>>(
+          target, draft, tokens, conf, dstat, L, temperature, K, V, nsplit, chunk, seed, round_offset, seq_offset,
+          rstat, part, cnt, n_accepted, bonus, st);
+    else
+      accept_decide_kernel<false><<<grid, kRowThreads, 0, stream>>>(
+          target, draft, tokens, conf, dstat, L, temperature, K, V, nsplit, chunk, seed, round_offset, seq_offset,
+          rstat, part, cnt, n_accepted, bonus, st);
+    return cudaGetLastError();
+  }
+}
+
+}  // namespace libraspec

@@ -1,0 +1,161 @@
+// Shared device helpers of the libraspec kernels (sm_103a).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/libraspec.h"
+
+namespace libraspec {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+// ---------------------------------------------------------------------------
+// Workspace layout. Every region is 256-byte aligned; counters are reset to
+// zero by the kernel that uses them, so one zero-fill serves every call.
+// ---------------------------------------------------------------------------
+constexpr int kConfMaxSplits = 64;    // CTAs per drafter row
+constexpr int kRowMaxSplits = 64;     // CTAs per target row (acceptance)
+constexpr int kRaceMaxSplits = 128;   // CTAs per sequence for a vocabulary draw
+constexpr int kAttnMaxCtas = 1024;    // persistent attention grid cap
+constexpr int kAttnRows = 64;         // query rows per attention work item
+constexpr int kAttnTileKeys = 64;     // keys per KV tile
+
+struct RowPartial {      // one CTA's share of a logit row
+  float m;               // max
+  int arg;               // argmax (lowest index among maxima)
+  double s;              // sum of exp((x - m) / T)
+};
+
+struct RowStat {         // merged statistics of a target row
+  float m;
+  int arg;
+  double Z;
+};
+
+struct RacePartial {
+  float key;
+  int idx;
+};
+
+struct WsLayout {
+  size_t status, conf_part, conf_cnt, row_part, row_cnt, row_stat, race_part, race_cnt;
+  size_t attn_o, attn_ml, attn_cnt, total;
+  int max_items, max_groups;
+};
+
+inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap) {
+  (void)V; (void)S_cap;
+  WsLayout w{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) { size_t o = off; off = align256(off + bytes); return o; };
+  const size_t rows_d = size_t(B) * K, rows_t = size_t(B) * (K + 1);
+  const int g = Hkv > 0 ? Hq / Hkv : 1;
+  const int m_max = (K + 1) * g;
+  const int n_mg = (m_max + kAttnRows - 1) / kAttnRows;
+  w.max_groups = B * Hkv * n_mg;
+  w.max_items = kAttnMaxCtas + w.max_groups;
+  w.status = take(256);
+  w.conf_part = take(rows_d * kConfMaxSplits * sizeof(RowPartial));
+  w.conf_cnt = take(rows_d * sizeof(uint32_t));
+  w.row_part = take(rows_t * kRowMaxSplits * sizeof(RowPartial));
+  w.row_cnt = take(rows_t * sizeof(uint32_t));
+  w.row_stat = take(rows_t * sizeof(RowStat));
+  w.race_part = take(size_t(B) * kRaceMaxSplits * sizeof(RacePartial));
+  w.race_cnt = take(size_t(B) * sizeof(uint32_t));
+  w.attn_o = take(size_t(w.max_items) * kAttnRows * d * sizeof(float));
+  w.attn_ml = take(size_t(w.max_items) * kAttnRows * 2 * sizeof(float));
+  w.attn_cnt = take(size_t(w.max_groups) * sizeof(uint32_t));
+  w.total = off;
+  return w;
+}
+
+// ---------------------------------------------------------------------------
+// Status word (device side): bits are OR-ed in, never cleared by kernels.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void raise_status(int* status, int bits) {
+  if (status) atomicOr(status, bits);
+}
+
+// ---------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11), from its definition:
+// a round maps (x0,x1,x2,x3) with key (k0,k1) to
+// (hi(M1 x2) ^ x1 ^ k0, lo(M1 x2), hi(M0 x0) ^ x3 ^ k1, lo(M0 x0)); the key
+// advances by (W0, W1) between rounds.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+    k.x += 0x9E3779B9u;
+    k.y += 0xBB67AE85u;
+  }
+  return c;
+}
+
+// Counter of a draw: (idx, position j, global sequence, purpose + 4 * round).
+__device__ __forceinline__ uint4 philox_block(uint64_t seed, uint32_t idx, uint32_t j, uint32_t seq,
+                                              uint32_t purpose, uint64_t round_offset) {
+  return philox4x32_10(make_uint4(idx, j, seq, purpose + 4u * (uint32_t)round_offset),
+                       make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
+}
+
+// u = ((w >> 9) + 1/2) * 2^-23: strictly inside (0,1), exact in binary32.
+__device__ __forceinline__ float word_to_uniform(uint32_t w) {
+  return (__uint2float_rn(w >> 9) + 0.5f) * 1.1920928955078125e-07f;
+}
+
+// ---------------------------------------------------------------------------
+// Fast base-2 exponential (the MUFU instruction); used where the result only
+// needs relative accuracy of a few ulp.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Streaming 128-bit load that does not allocate in L1.
+__device__ __forceinline__ float4 ld_stream4(const float* p) {
+  float4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ float ld_stream(const float* p) {
+  float v;
+  asm volatile("ld.global.nc.L1::no_allocate.f32 %0, [%1];" : "=f"(v) : "l"(p));
+  return v;
+}
+
+// Combine two (m, s) pairs (binary64 sums); c = log2(e) / T.
+__device__ __forceinline__ void combine_ms(float& m, double& s, float m2, double s2, float c) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) { m = m2; s = s2; return; }
+  if (m2 > m) {
+    s = s * (double)exp2f((m - m2) * c) + s2;
+    m = m2;
+  } else {
+    s = s + s2 * (double)exp2f((m2 - m) * c);
+  }
+}
+
+// (value, index) max with the lowest index winning ties.
+__device__ __forceinline__ void argmax_combine(float& v, int& i, float v2, int i2) {
+  if (v2 > v || (v2 == v && i2 < i)) { v = v2; i = i2; }
+}
+
+// (key, index) min with the lowest index winning ties.
+__device__ __forceinline__ void argmin_combine(float& k, int& i, float k2, int i2) {
+  if (k2 < k || (k2 == k && i2 < i)) { k = k2; i = i2; }
+}
+
+}  // namespace libraspec

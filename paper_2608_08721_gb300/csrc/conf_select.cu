@@ -1,0 +1,178 @@
+// Step 1 (drafter confidence) and step 2 (LibraSpec length selection).
+#include "rowpass.cuh"
+
+namespace libraspec {
+
+// ---------------------------------------------------------------------------
+// Confidence: grid (nsplit, B*K), 256 threads. CTA `split` of row r streams
+// columns [split*chunk, (split+1)*chunk) once, keeping the running max and
+// sum of exp((x - m)/T). With several splits the last CTA to finish (atomic
+// ticket) merges the row's partials in binary64 and finalises
+// q = exp((x_tok - m)/T) / Z (Assumption 1: q_k, the drafter's probability
+// of its drafted token).
+// ---------------------------------------------------------------------------
+template <bool VEC>
+__global__ void __launch_bounds__(kRowThreads) conf_kernel(
+    const float* __restrict__ x, const int32_t* __restrict__ tokens, const float* __restrict__ temperature,
+    int K, int V, int nsplit, int chunk, float* __restrict__ conf, float* __restrict__ dstat,
+    RowPartial* __restrict__ part, uint32_t* __restrict__ cnt, int* __restrict__ status) {
+  __shared__ float sm[64];
+  __shared__ int last;
+  const int row = blockIdx.y, split = blockIdx.x;
+  const int b = row / K;
+  const float tb = temperature[b];
+  const float T = tb > 0.f ? tb : 1.f;
+  const float c = (float)(1.4426950408889634 / (double)T);
+  const float* xr = x + (size_t)row * V;
+  const int c0 = split * chunk, c1 = min(V, c0 + chunk);
+
+  SumAcc sa;
+  ArgAcc aa;
+  sa.init();
+  row_slice_pass<true, false, VEC>(xr, c0, c1, c, sa, aa);
+  float m = sa.m, s = sa.value();
+  cta_reduce_sum(m, s, c, sm);
+
+  double Z;
+  float M;
+  if (nsplit == 1) {
+    if (threadIdx.x != 0) return;
+    M = m;
+    Z = (double)s;
+  } else {
+    if (threadIdx.x == 0) {
+      RowPartial p;
+      p.m = m;
+      p.arg = 0;
+      p.s = (double)s;
+      part[(size_t)row * kConfMaxSplits + split] = p;
+      __threadfence();
+      const uint32_t ticket = atomicAdd(&cnt[row], 1u);
+      last = (ticket == (uint32_t)(nsplit - 1));
+    }
+    __syncthreads();
+    if (!last) return;
+    if (threadIdx.x >= 32) return;
+    __threadfence();
+    int dummy;
+    warp_merge_partials(part + (size_t)row * kConfMaxSplits, nsplit, (double)T, false, M, dummy, Z);
+    if (threadIdx.x != 0) return;
+    cnt[row] = 0u;  // ready for the next call
+  }
+  const int tok = tokens[row];
+  float q = 0.f;
+  if (tok < 0 || tok >= V) {
+    raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
+  } else {
+    q = (float)(exp(((double)xr[tok] - (double)M) / (double)T) / Z);
+  }
+  conf[row] = q;
+  if (dstat) {
+    dstat[2 * (size_t)row] = M;
+    dstat[2 * (size_t)row + 1] = (float)Z;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Selection (Thm. 4): one warp per sequence, binary64. Lane k of a 32-wide
+// chunk evaluates the step L = k -> k+1:
+//   P_{k+1} = prod_{i<=k} q_i          (multiplicative inclusive scan)
+//   E_k     = 1 + sum_{j<=k} P_j       (additive exclusive scan of P)
+//   extend  iff P_{k+1} * T(k) > (T(k+1) - T(k)) * E_k
+// L is the first lane (in chunk order) whose test fails, or K.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(128) select_kernel(const float* __restrict__ conf,
+                                                     const float* __restrict__ cost, int B, int K,
+                                                     int32_t* __restrict__ L, int* __restrict__ status) {
+  const int seq = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (seq >= B) return;
+  bool bad = false;
+  for (int l = lane; l <= K; l += 32) {
+    const float t = cost[l];
+    if (!(t > 0.f) || !isfinite(t)) bad = true;
+  }
+  if (__any_sync(0xffffffffu, bad)) {
+    if (lane == 0) {
+      L[seq] = 0;
+      raise_status(status, LIBRASPEC_ST_BAD_COST);
+    }
+    return;
+  }
+  double carryP = 1.0, carryE = 1.0;
+  int result = K;
+  for (int base = 0; base < K; base += 32) {
+    const int k = base + lane;
+    const bool live = k < K;
+    const double q = live ? (double)conf[(size_t)seq * K + k] : 1.0;
+    double P = q;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const double o = __shfl_up_sync(0xffffffffu, P, off);
+      if (lane >= off) P = __dmul_rn(P, o);
+    }
+    P = __dmul_rn(P, carryP);                 // P_{k+1}
+    double S = P;                             // inclusive sum of P over the chunk
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const double o = __shfl_up_sync(0xffffffffu, S, off);
+      if (lane >= off) S = __dadd_rn(S, o);
+    }
+    double Sx = __shfl_up_sync(0xffffffffu, S, 1);
+    if (lane == 0) Sx = 0.0;
+    const double E = __dadd_rn(carryE, Sx);   // E_k
+    bool fail = false;
+    if (live) {
+      const double Tk = (double)cost[k], Tk1 = (double)cost[k + 1];
+      const double lhs = __dmul_rn(P, Tk);
+      const double rhs = __dmul_rn(E, __dsub_rn(Tk1, Tk));
+      fail = !(lhs > rhs);
+    }
+    const unsigned ball = __ballot_sync(0xffffffffu, fail);
+    if (ball) {
+      result = base + __ffs(ball) - 1;
+      break;
+    }
+    carryP = __shfl_sync(0xffffffffu, P, 31);
+    carryE = __dadd_rn(carryE, __shfl_sync(0xffffffffu, S, 31));
+  }
+  if (lane == 0) L[seq] = result;
+}
+
+// ---------------------------------------------------------------------------
+// Host launchers (arguments already validated by the ABI layer).
+// ---------------------------------------------------------------------------
+int num_sms_current();
+
+cudaError_t launch_confidence(const float* x, const int32_t* tokens, const float* temperature, int B, int K,
+                              int V, float* conf, float* dstat, char* ws, const WsLayout& lay,
+                              cudaStream_t stream) {
+  const long rows = (long)B * K;
+  if (rows == 0) return cudaSuccess;
+  const int nsplit0 = row_splits(rows, V, num_sms_current(), kConfMaxSplits, 2048);
+  const int chunk = row_chunk(V, nsplit0);
+  const int nsplit = (V + chunk - 1) / chunk;
+  const bool vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
+  dim3 grid(nsplit, (unsigned)rows);
+  auto* part = reinterpret_cast<RowPartial*>(ws + lay.conf_part);
+  auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.conf_cnt);
+  auto* st = reinterpret_cast<int*>(ws + lay.status);
+  if (vec)
+    conf_kernel<true><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
+                                                        dstat, part, cnt, st);
+  else
+    conf_kernel<false><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
+                                                         dstat, part, cnt, st);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select(const float* conf, const float* cost, int B, int K, int32_t* L, char* ws,
+                          const WsLayout& lay, cudaStream_t stream) {
+  if (B == 0) return cudaSuccess;
+  const int threads = 128;
+  const int blocks = (B * 32 + threads - 1) / threads;
+  select_kernel<<<blocks, threads, 0, stream>>>(conf, cost, B, K, L, reinterpret_cast<int*>(ws + lay.status));
+  return cudaGetLastError();
+}
+
+}  // namespace libraspec

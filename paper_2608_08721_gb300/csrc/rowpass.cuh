@@ -1,0 +1,200 @@
+// One CTA's streaming pass over a slice of a logit row: max / argmax and the
+// sum of exponentials, in a single read of HBM with 128-bit loads.
+#pragma once
+
+#include "common.cuh"
+
+namespace libraspec {
+
+constexpr int kRowThreads = 256;
+
+// Per-thread running sum of 2^((x - m) * c), c = log2(e) / T, with the max
+// tracked online (the sum is rescaled when the max grows) and Kahan
+// compensation of the running sum.
+struct SumAcc {
+  float m, s, comp;
+  __device__ __forceinline__ void init() { m = -INFINITY; s = 0.f; comp = 0.f; }
+  __device__ __forceinline__ void add4(float4 v, float c) {
+    const float gm = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
+    if (gm > m) {
+      const float f = ex2_approx((m - gm) * c);
+      s *= f;
+      comp *= f;
+      m = gm;
+    }
+    const float t = (ex2_approx((v.x - m) * c) + ex2_approx((v.y - m) * c)) +
+                    (ex2_approx((v.z - m) * c) + ex2_approx((v.w - m) * c));
+    const float y = t - comp;
+    const float ts = s + y;
+    comp = (ts - s) - y;
+    s = ts;
+  }
+  __device__ __forceinline__ void add1(float x, float c) {
+    if (x > m) {
+      const float f = ex2_approx((m - x) * c);
+      s *= f;
+      comp *= f;
+      m = x;
+    }
+    const float y = ex2_approx((x - m) * c) - comp;
+    const float ts = s + y;
+    comp = (ts - s) - y;
+    s = ts;
+  }
+  __device__ __forceinline__ float value() const { return s - comp; }
+};
+
+// Per-thread running max with the lowest index among equal maxima
+// (elements are visited in increasing index order within a thread).
+struct ArgAcc {
+  float m;
+  int arg;
+  __device__ __forceinline__ void init() { m = -INFINITY; arg = 0x7fffffff; }
+  __device__ __forceinline__ void add4(float4 v, int i0) {
+    if (v.x > m) { m = v.x; arg = i0; }
+    if (v.y > m) { m = v.y; arg = i0 + 1; }
+    if (v.z > m) { m = v.z; arg = i0 + 2; }
+    if (v.w > m) { m = v.w; arg = i0 + 3; }
+  }
+  __device__ __forceinline__ void add1(float x, int i) {
+    if (x > m) { m = x; arg = i; }
+  }
+};
+
+// Stream x[c0, c1) (c0 a multiple of 4). VEC: x is 16-byte aligned and the
+// row length is a multiple of 4, so 128-bit loads cover the slice.
+template <bool SUM, bool ARG, bool VEC>
+__device__ __forceinline__ void row_slice_pass(const float* __restrict__ x, int c0, int c1, float c,
+                                               SumAcc& sa, ArgAcc& aa) {
+  const int tid = threadIdx.x;
+  if (VEC) {
+    const int g0 = c0 >> 2, g1 = c1 >> 2;  // groups of 4
+    int g = g0 + tid;
+    constexpr int U = 4;
+    for (; g + (U - 1) * kRowThreads < g1; g += U * kRowThreads) {
+      float4 v[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) v[u] = ld_stream4(x + 4 * (g + u * kRowThreads));
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (SUM) sa.add4(v[u], c);
+        if (ARG) aa.add4(v[u], 4 * (g + u * kRowThreads));
+      }
+    }
+    for (; g < g1; g += kRowThreads) {
+      const float4 v = ld_stream4(x + 4 * g);
+      if (SUM) sa.add4(v, c);
+      if (ARG) aa.add4(v, 4 * g);
+    }
+  } else {
+    for (int i = c0 + tid; i < c1; i += kRowThreads) {
+      const float v = ld_stream(x + i);
+      if (SUM) sa.add1(v, c);
+      if (ARG) aa.add1(v, i);
+    }
+  }
+}
+
+// Combine the (m, s) pairs of all threads of the CTA; result valid in thread 0.
+__device__ __forceinline__ void cta_reduce_sum(float& m, float& s, float c, float* sm /*[2*32]*/) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+    const float M = fmaxf(m, m2);
+    if (M != -INFINITY) {
+      s = s * ex2_approx((m - M) * c) + s2 * ex2_approx((m2 - M) * c);
+      m = M;
+    }
+  }
+  if (lane == 0) { sm[2 * warp] = m; sm[2 * warp + 1] = s; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    m = sm[0];
+    s = sm[1];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) {
+      const float m2 = sm[2 * w], s2 = sm[2 * w + 1];
+      const float M = fmaxf(m, m2);
+      if (M != -INFINITY) {
+        s = s * ex2_approx((m - M) * c) + s2 * ex2_approx((m2 - M) * c);
+        m = M;
+      }
+    }
+  }
+}
+
+// Combine (max, argmax) of all threads; result valid in thread 0.
+__device__ __forceinline__ void cta_reduce_arg(float& m, int& arg, float* smf /*[32]*/, int* smi /*[32]*/) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+    const int a2 = __shfl_xor_sync(0xffffffffu, arg, off);
+    argmax_combine(m, arg, m2, a2);
+  }
+  if (lane == 0) { smf[warp] = m; smi[warp] = arg; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    m = smf[0];
+    arg = smi[0];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) argmax_combine(m, arg, smf[w], smi[w]);
+  }
+}
+
+// Merge nsplit partials of one row in binary64 (one warp; result in lane 0).
+// T is the temperature: s_i * exp((m_i - M) / T) rescales each share.
+__device__ __forceinline__ void warp_merge_partials(const RowPartial* __restrict__ p, int nsplit, double T,
+                                                    bool want_arg, float& m_out, int& arg_out,
+                                                    double& s_out) {
+  const int lane = threadIdx.x & 31;
+  float m = -INFINITY;
+  int arg = 0x7fffffff;
+  for (int i = lane; i < nsplit; i += 32) {
+    const float mi = __ldcg(&p[i].m);
+    const int ai = __ldcg(&p[i].arg);
+    if (want_arg) argmax_combine(m, arg, mi, ai);
+    else m = fmaxf(m, mi);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+    const int a2 = __shfl_xor_sync(0xffffffffu, arg, off);
+    if (want_arg) argmax_combine(m, arg, m2, a2);
+    else m = fmaxf(m, m2);
+  }
+  double s = 0.0;
+  if (m != -INFINITY) {
+    for (int i = lane; i < nsplit; i += 32) {
+      const float mi = __ldcg(&p[i].m);
+      const double si = __ldcg(&p[i].s);
+      if (mi != -INFINITY) s += si * exp(((double)mi - (double)m) / T);
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  m_out = m;
+  arg_out = arg;
+  s_out = s;
+}
+
+// Choose how many CTAs share a row: enough CTAs in total to fill the GPU
+// several times over, each with at least min_elems elements.
+inline int row_splits(long rows, int V, int num_sms, int max_splits, int min_elems) {
+  if (rows <= 0) return 1;
+  const long target = 4L * 8 * num_sms;
+  long ns = (target + rows - 1) / rows;
+  const long cap = (V + min_elems - 1) / min_elems;
+  if (ns > cap) ns = cap;
+  if (ns > max_splits) ns = max_splits;
+  if (ns < 1) ns = 1;
+  return (int)ns;
+}
+
+// Split length: a multiple of 4 elements.
+inline int row_chunk(int V, int nsplit) {
+  int ch = (V + nsplit - 1) / nsplit;
+  return (ch + 3) & ~3;
+}
+
+}  // namespace libraspec

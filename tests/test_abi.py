@@ -1,0 +1,83 @@
+"""The C-ABI library: it loads, exports every symbol the header declares, and
+rejects bad arguments on the host (no GPU needed: nothing is enqueued)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_08721_gb300 import binding as lr
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "libraspec.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(libraspec_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_08721_gb300 import build
+
+    build.build()
+    return lr.load()
+
+
+def test_header_declares_the_round_entry_points():
+    names = _declared()
+    for n in ("libraspec_confidence", "libraspec_select_lengths", "libraspec_verify_attn", "libraspec_accept",
+              "libraspec_verify_round", "libraspec_workspace_size", "libraspec_get_status"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = _declared()
+    assert names
+    for n in names:
+        assert hasattr(lib, n), "libraspec.so does not export %s" % n
+    assert set(names) <= set(lr.SIGNATURES), "binding lacks a signature for %s" % (set(names) - set(lr.SIGNATURES))
+
+
+def test_version_and_status_strings(lib):
+    assert b"sm_103a" in lib.libraspec_version()
+    assert lib.libraspec_status_string(-1) == b"invalid argument"
+
+
+def test_workspace_size_is_host_only_and_validates(lib):
+    s = lib.libraspec_workspace_size(64, 32, 128256, 32, 8, 128, 32832)
+    assert s > 0 and s % 256 == 0
+    assert lib.libraspec_workspace_size(1, 16, 32000, 8, 2, 64, 576) < s
+    assert lib.libraspec_workspace_size(1, 16, 32000, 8, 3, 64, 576) == 0      # Hq % Hkv != 0
+    assert lib.libraspec_workspace_size(1, 65, 32000, 8, 2, 64, 576) == 0      # K > max
+    assert lib.libraspec_workspace_size(1, 16, 32000, 8, 2, 96, 576) == 0      # head dim
+
+
+def test_calls_reject_bad_arguments_before_any_launch(lib):
+    P = ctypes.c_void_p
+    fake = P(0x1000)  # never dereferenced: validation fails first
+    assert lib.libraspec_confidence(None, None, None, 1, 2, 8, None, None, None, 0, None) == lr.EINVAL
+    assert lib.libraspec_confidence(fake, fake, fake, -1, 2, 8, fake, None, fake, 1 << 20, None) == lr.EINVAL
+    assert lib.libraspec_select_lengths(fake, fake, 1, 65, fake, fake, 1 << 20, None) == lr.EINVAL
+    assert lib.libraspec_verify_attn(fake, fake, fake, fake, fake, 1, 4, 8, 2, 96, 64, 0.1, fake, None, fake,
+                                     1 << 30, None) == lr.EUNSUPPORTED
+    assert lib.libraspec_verify_attn(fake, fake, fake, fake, fake, 1, 4, 8, 3, 64, 64, 0.1, fake, None, fake,
+                                     1 << 30, None) == lr.EINVAL
+    # unaligned K cache pointer
+    assert lib.libraspec_verify_attn(fake, P(0x1008), fake, fake, fake, 1, 4, 8, 2, 64, 64, 0.1, fake, None,
+                                     fake, 1 << 30, None) == lr.EINVAL
+    # workspace too small
+    assert lib.libraspec_accept(fake, fake, fake, None, None, fake, fake, 2, 4, 64, 0, 0, 0, fake, fake, fake, 16,
+                                None) == lr.EINVAL
+    # empty batches are a no-op
+    assert lib.libraspec_accept(None, None, None, None, None, None, None, 0, 4, 64, 0, 0, 0, None, None, None, 0,
+                                None) == lr.OK
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(lr, "_lib", None)
+    monkeypatch.setattr(lr, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        lr.load()

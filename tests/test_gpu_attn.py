@@ -1,0 +1,138 @@
+"""GPU parity: block-causal GQA verify attention vs. the fp64 oracle."""
+import numpy as np
+import pytest
+import torch
+
+from helpers import check_attn, cuda
+from paper_2608_08721_gb300 import binding as lr
+from paper_2608_08721_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def _inputs(B, K, Hq, Hkv, d, kv, S_cap, seed, scale_k=1.0):
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    Q = torch.randn((B, K + 1, Hq, d), generator=g, device=cuda()).to(torch.bfloat16)
+    Kc = (torch.randn((B, Hkv, S_cap, d), generator=g, device=cuda()) * scale_k).to(torch.bfloat16)
+    Vc = torch.randn((B, Hkv, S_cap, d), generator=g, device=cuda()).to(torch.bfloat16)
+    return Q, Kc, Vc
+
+
+def _run(Q, Kc, Vc, kv, L, K):
+    B, _, Hq, d = Q.shape
+    Hkv, S_cap = Kc.shape[1], Kc.shape[2]
+    ws = lr.Workspace(B, K, 1, Hq, Hkv, d, S_cap, device=cuda())
+    kv_t = torch.tensor(kv, dtype=torch.int32, device=cuda())
+    L_t = torch.tensor(L, dtype=torch.int32, device=cuda())
+    O, lse = lr.libraspec_verify_attn(Q, Kc, Vc, kv_t, L_t, ws, want_lse=True)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) == 0
+    return O, lse
+
+
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("Hq,Hkv", [(8, 2), (28, 4), (32, 8), (64, 8), (4, 4)])
+def test_attn_small_ragged(orc, d, Hq, Hkv):
+    K = 9
+    kv = [0, 1, 63, 64, 200, 700]
+    L = [0, 9, 3, 1, 9, 5]
+    B = len(kv)
+    S_cap = max(k + l + 1 for k, l in zip(kv, L)) + 3
+    Q, Kc, Vc = _inputs(B, K, Hq, Hkv, d, kv, S_cap, seed=Hq * 7 + d, scale_k=2.0)
+    O, lse = _run(Q, Kc, Vc, kv, L, K)
+    O_ref, lse_ref = orc.verify_attn(Q, Kc, Vc, np.array(kv), np.array(L))
+    check_attn(O, lse, O_ref, lse_ref, L)
+
+
+def test_attn_rows_beyond_L_untouched():
+    K, B, Hq, Hkv, d = 6, 2, 8, 2, 64
+    kv, L = [30, 5], [2, 0]
+    Q, Kc, Vc = _inputs(B, K, Hq, Hkv, d, kv, 48, seed=1)
+    ws = lr.Workspace(B, K, 1, Hq, Hkv, d, 48, device=cuda())
+    O = torch.full_like(Q, 7.0)
+    lr.libraspec_verify_attn(Q, Kc, Vc, torch.tensor(kv, dtype=torch.int32, device=cuda()),
+                             torch.tensor(L, dtype=torch.int32, device=cuda()), ws, O=O)
+    torch.cuda.synchronize()
+    assert torch.all(O[0, 3:] == 7.0) and torch.all(O[1, 1:] == 7.0)
+    assert not torch.any(O[0, :3] == 7.0)
+
+
+@pytest.mark.parametrize("kv", [5000, 20000])
+def test_attn_long_split_kv_merge(orc, kv):
+    # one sequence, long cache: many work items per row group, merged in-kernel
+    K, Hq, Hkv, d = 16, 32, 8, 128
+    L = [11]
+    Q, Kc, Vc = _inputs(1, K, Hq, Hkv, d, [kv], kv + K + 1, seed=kv)
+    O, lse = _run(Q, Kc, Vc, [kv], L, K)
+    O_ref, lse_ref = orc.verify_attn(Q, Kc, Vc, np.array([kv]), np.array(L))
+    check_attn(O, lse, O_ref, lse_ref, L)
+
+
+def test_attn_peaky_scores(orc):
+    w = workloads.WORKLOADS["sampling"].scaled(B=4, kv=("uniform", 100, 3000))
+    kv = workloads.kv_lengths(w)
+    lay = workloads.layer(w, 0, kv, device=cuda(), peaky=True)
+    L = np.array([0, 16, 7, 3], np.int32)
+    O, lse = _run(lay["Q"], lay["Kc"], lay["Vc"], kv.tolist(), L.tolist(), w.K)
+    O_ref, lse_ref = orc.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L)
+    check_attn(O, lse, O_ref, lse_ref, L)
+
+
+def test_attn_equal_keys_closed_form():
+    # all keys equal: every row's output is the mean of its visible values
+    B, K, Hq, Hkv, d = 1, 4, 4, 1, 64
+    kv = [100]
+    L = [4]
+    S = 128
+    g = torch.Generator(device="cuda").manual_seed(3)
+    Q = torch.randn((B, K + 1, Hq, d), generator=g, device=cuda()).to(torch.bfloat16)
+    Kc = torch.full((B, Hkv, S, d), 0.25, device=cuda(), dtype=torch.bfloat16)
+    Vc = torch.randn((B, Hkv, S, d), generator=g, device=cuda()).to(torch.bfloat16)
+    O, _ = _run(Q, Kc, Vc, kv, L, K)
+    for t in range(5):
+        mean = Vc[0, 0, : kv[0] + t + 1].float().mean(0)
+        for h in range(Hq):
+            assert torch.allclose(O[0, t, h].float(), mean, atol=1e-2, rtol=1e-2)
+
+
+@pytest.mark.parametrize("name", ["tiny", "8b", "sampling", "ragged", "70b"])
+def test_attn_full_size_sampled_rows(orc, name):
+    """One layer at the workload's full size, in the launch configuration the
+    benchmark uses; the oracle checks a sample of rows one by one."""
+    w = workloads.WORKLOADS[name]
+    kv = workloads.kv_lengths(w)
+    rng = np.random.default_rng(len(name))
+    L = rng.integers(0, w.K + 1, size=w.B).astype(np.int32)
+    L[0] = w.K
+    if w.B > 1:
+        L[1] = 0
+    lay = workloads.layer(w, 3, kv, device=cuda())
+    O, lse = _run(lay["Q"], lay["Kc"], lay["Vc"], kv.tolist(), L.tolist(), w.K)
+    rows = []
+    for b in range(w.B):
+        for h in rng.choice(w.Hq, size=min(3, w.Hq), replace=False):
+            rows.append((b, int(h), int(L[b])))
+            rows.append((b, int(h), int(rng.integers(0, L[b] + 1))))
+    rows = np.array(rows, np.int32)
+    O_ref, lse_ref = orc.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L, rows=rows)
+    check_attn(O, lse, O_ref, lse_ref, L, rows=[tuple(r) for r in rows])
+
+
+def test_attn_kv_overflow_sets_status_and_skips():
+    B, K, Hq, Hkv, d, S = 2, 4, 4, 2, 64, 32
+    Q, Kc, Vc = _inputs(B, K, Hq, Hkv, d, None, S, seed=2)
+    ws = lr.Workspace(B, K, 1, Hq, Hkv, d, S, device=cuda())
+    O = torch.zeros_like(Q)
+    lr.libraspec_verify_attn(Q, Kc, Vc, torch.tensor([30, 5], dtype=torch.int32, device=cuda()),
+                             torch.tensor([4, 4], dtype=torch.int32, device=cuda()), ws, O=O)
+    assert lr.libraspec_get_status(ws) & lr.ST_KV_OVERFLOW
+    assert torch.all(O[0] == 0) and torch.any(O[1] != 0)
+
+
+def test_attn_deterministic():
+    B, K, Hq, Hkv, d = 3, 16, 32, 8, 128
+    kv = [9000, 300, 4000]
+    L = [16, 2, 9]
+    Q, Kc, Vc = _inputs(B, K, Hq, Hkv, d, kv, 9100, seed=11)
+    outs = [_run(Q, Kc, Vc, kv, L, K)[0] for _ in range(3)]
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[1], outs[2])

@@ -1,0 +1,72 @@
+"""GPU parity of the whole round (libraspec_verify_round and the host-buffer API)."""
+import numpy as np
+import pytest
+import torch
+
+from helpers import assert_exact_unless_flagged, check_attn, cuda
+from paper_2608_08721_gb300 import api
+from paper_2608_08721_gb300 import binding as lr
+from paper_2608_08721_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def _oracle_round(orc, w, inp, kv, layers, cost, rows_per_layer=None):
+    q, _ = orc.confidence(inp["draft_logits"].cpu().numpy(), inp["draft_tokens"].cpu().numpy(),
+                          inp["temperature"].cpu().numpy())
+    L, sflag = orc.select_lengths(q, cost.astype(np.float64))
+    n, bonus, aflag = orc.accept(inp["target_logits"].cpu().numpy(), inp["draft_logits"].cpu().numpy(),
+                                 inp["draft_tokens"].cpu().numpy(), L, inp["temperature"].cpu().numpy(),
+                                 w.philox_seed)
+    outs = [orc.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L, rows=rows_per_layer) for lay in layers]
+    return q, L, sflag, n, bonus, aflag, outs
+
+
+@pytest.mark.parametrize("name,n_layers", [("tiny", 1), ("8b", 2), ("sampling", 1)])
+def test_verify_round_matches_oracle(orc, name, n_layers):
+    w = workloads.WORKLOADS[name]
+    kv = workloads.kv_lengths(w)
+    inp = workloads.logits(w, device=cuda())
+    layers = [workloads.layer(w, l, kv, device=cuda()) for l in range(n_layers)]
+    cost = workloads.cost_table(w)
+    S = layers[0]["Kc"].shape[2]
+    ws = lr.Workspace(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, S, device=cuda())
+    out = lr.libraspec_verify_round(inp["draft_logits"], inp["draft_tokens"], inp["temperature"],
+                                    torch.tensor(cost, device=cuda()), inp["target_logits"], layers,
+                                    torch.tensor(kv, device=cuda()), w.philox_seed, ws, want_lse=True)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) == 0
+    q, L, sflag, n, bonus, aflag, outs = _oracle_round(orc, w, inp, kv, layers, cost)
+    L_gpu = out.L.cpu().numpy()
+    assert_exact_unless_flagged(L_gpu, L, sflag, "L")
+    if np.array_equal(L_gpu, L):
+        assert_exact_unless_flagged(out.n_accepted.cpu().numpy(), n, aflag, "n_accepted")
+        assert_exact_unless_flagged(out.bonus_token.cpu().numpy(), bonus, aflag, "bonus_token")
+        for l in range(n_layers):
+            check_attn(out.O[l], out.lse[l], outs[l][0], outs[l][1], L)
+
+
+def test_host_buffer_api_round_trip(orc):
+    w = workloads.WORKLOADS["tiny"]
+    kv = workloads.kv_lengths(w)
+    lay = workloads.layer(w, 0, kv, device=cuda())
+    inp = workloads.logits(w)
+    K1 = w.K + 1
+    caches = [{"Kc": lay["Kc"].clone(), "Vc": lay["Vc"].clone()}]
+    runner = api.VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, lay["Kc"].shape[2], caches, torch.tensor(kv))
+    host = {k: v.pin_memory() for k, v in inp.items()}
+    host["cost_table"] = torch.tensor(workloads.cost_table(w)).pin_memory()
+    kvb = int(kv[0])
+    host["layers"] = [{"Q": lay["Q"].cpu().pin_memory(),
+                       "K_new": lay["Kc"][:, :, kvb:kvb + K1].cpu().contiguous().pin_memory(),
+                       "V_new": lay["Vc"][:, :, kvb:kvb + K1].cpu().contiguous().pin_memory()}]
+    n, bonus = runner.run_host(host, seed=w.philox_seed)
+    q, _ = orc.confidence(inp["draft_logits"].numpy(), inp["draft_tokens"].numpy(), inp["temperature"].numpy())
+    L, sflag = orc.select_lengths(q, workloads.cost_table(w).astype(np.float64))
+    n_ref, b_ref, aflag = orc.accept(inp["target_logits"].numpy(), inp["draft_logits"].numpy(),
+                                     inp["draft_tokens"].numpy(), L, inp["temperature"].numpy(), w.philox_seed)
+    assert not sflag.any()
+    np.testing.assert_array_equal(n, n_ref)
+    np.testing.assert_array_equal(bonus, b_ref)
+    O_ref, lse_ref = orc.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L)
+    check_attn(runner.out.O[0], None, O_ref, lse_ref, L)
