@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(kRowThreads) accept_rows_kernel(
   float M;
   int A;
   double Z;
-  warp_merge_partials(part + (size_t)row * kRowMaxSplits, nsplit, (double)T, !sampling, M, A, Z);
+  warp_merge_partials(part + (size_t)row * kRowMaxSplits, nsplit, sampling ? c : 0.f, !sampling, M, A, Z);
   if (threadIdx.x == 0) {
     RowStat st;
     st.m = M;
@@ -130,9 +130,9 @@ __device__ Decision decide(int b, int K, int V, const float* __restrict__ target
       } else if (conf == nullptr) {
         reject = true;
       } else {
-        const double T = (double)tb;
-        const double y = (double)target[((size_t)b * (K + 1) + jj) * V + x];
-        const double p = exp((y - (double)__ldcg(&st[jj].m)) / T) / __ldcg(&st[jj].Z);
+        const float c = (float)(1.4426950408889634 / (double)tb);
+        const float y = target[((size_t)b * (K + 1) + jj) * V + x];
+        const double p = (double)exp2f((y - __ldcg(&st[jj].m)) * c) / __ldcg(&st[jj].Z);
         const double q = (double)conf[(size_t)b * K + jj];
         const double ratio = (q <= p) ? 1.0 : p / q;
         const uint4 w = philox_block(seed, 0u, (uint32_t)jj, seq_offset + (uint32_t)b, 0u, round_offset);
@@ -348,7 +348,7 @@ cudaError_t launch_accept(const float* target, const float* draft, const int32_t
   auto* rstat = reinterpret_cast<RowStat*>(ws + lay.row_stat);
   {
     const long rows = (long)B * (K + 1);
-    const int nsplit0 = row_splits(rows, V, sms, kRowMaxSplits, 2048);
+    const int nsplit0 = row_splits(rows, V, sms, kRowMaxSplits, 4096);
     const int chunk = row_chunk(V, nsplit0);
     const int nsplit = (V + chunk - 1) / chunk;
     dim3 grid(nsplit, K + 1, B);

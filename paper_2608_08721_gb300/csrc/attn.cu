@@ -226,8 +226,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
     const __nv_bfloat16* __restrict__ Q, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
     int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, __nv_bfloat16* __restrict__ O,
-    float* __restrict__ lse, float* __restrict__ part_o, float* __restrict__ part_ml,
-    uint32_t* __restrict__ group_cnt, int* __restrict__ status) {
+    float* __restrict__ lse, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ status) {
   using SM = AttnSmem<D, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -237,7 +236,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   const uint32_t sBar = smem_u32(smem + SM::kBar);
   ItemInfo& info = *reinterpret_cast<ItemInfo*>(smem + SM::kInfo);
   float* merge_ml = reinterpret_cast<float*>(smem + SM::kMerge);
-  __shared__ int sh_tpi, sh_found, sh_last, sh_abort;
+  __shared__ int sh_tpi, sh_found, sh_abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = Hq / Hkv;
@@ -257,6 +256,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   __syncthreads();
   const int tpi = sh_tpi;
   uint32_t tile_ctr = 0;  // tiles consumed by this CTA so far (stage / phase)
+  // let the merge kernel (launched as a programmatic dependent) get resident
+  // as soon as SMs free up; it waits for this grid's completion itself
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   for (int item = blockIdx.x;; item += gridDim.x) {
     __syncthreads();  // everyone is done with the previous item's shared state
@@ -471,7 +473,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       }
       continue;
     }
-    // several items share this row group: write the partial, merge at the last
+    // several items share this row group: write the fp32 partial (O, m, l);
+    // attn_merge_kernel combines them once the whole grid is done
     const size_t slot = (size_t)item_base + (size_t)split * n_mg;
     if (warp_live) {
 #pragma unroll
@@ -490,58 +493,122 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         }
       }
     }
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) {
-      const uint32_t ticket = atomicAdd(&group_cnt[group], 1u);
-      sh_last = (ticket == (uint32_t)(nsplit - 1));
+    (void)group;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Merge of the split-KV partials. Launched right after verify_attn_kernel as
+// a programmatic dependent: it becomes resident early and waits
+// (griddepcontrol.wait) until every attention CTA has finished and its
+// writes are visible. One warp per (sequence, kv head, row) whose row group
+// was split: O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, M = max_s m_s,
+// splits combined in a fixed order (deterministic). Spread over the whole
+// GPU, so no single SM reads all of a group's partials.
+// ---------------------------------------------------------------------------
+constexpr int kMergeThreads = 256;
+
+template <int D>
+__global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(
+    const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls, int B, int K, int Hq, int Hkv, int S_cap,
+    int attn_grid, int min_tiles, __nv_bfloat16* __restrict__ O, float* __restrict__ lse,
+    const float* __restrict__ part_o, const float* __restrict__ part_ml) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  __shared__ int sh_tpi;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int g = Hq / Hkv;
+  if (warp == 0) {
+    const int tot = total_tiles(B, kv_len, Ls, K, g, Hkv, S_cap, nullptr, false);
+    if (lane == 0) {
+      const int tpi = (tot + attn_grid - 1) / attn_grid;
+      sh_tpi = tpi < min_tiles ? min_tiles : tpi;
     }
-    __syncthreads();
-    if (!sh_last) continue;
-    __threadfence();
-    // merge: per row the global max and denominator, then the weighted sum
-    const int nsp = nsplit;
-    const size_t base_slot = (size_t)item_base;
-    const int stride = n_mg;
-    if (tid < rows) {
-      float M = -INFINITY;
-      for (int sp = 0; sp < nsp; ++sp)
-        M = fmaxf(M, __ldcg(&part_ml[((base_slot + (size_t)sp * stride) * kAttnRows + tid) * 2]));
-      float Lsum = 0.f;
-      for (int sp = 0; sp < nsp; ++sp) {
-        const size_t e = ((base_slot + (size_t)sp * stride) * kAttnRows + tid) * 2;
-        const float ms = __ldcg(&part_ml[e]);
-        if (ms != -INFINITY) Lsum += __ldcg(&part_ml[e + 1]) * ex2_approx(ms - M);
+  }
+  __syncthreads();
+  const int tpi = sh_tpi;
+  const int warps_total = gridDim.x * (kMergeThreads / 32);
+  for (int unit = blockIdx.x * (kMergeThreads / 32) + warp;; unit += warps_total) {
+    // locate the unit: units of sequence b (split row groups only) are
+    // Hkv * M_b rows, kv head major
+    int carry_u = 0, carry_it = 0;
+    int b = -1, local = 0, start_it = 0;
+    SeqPlan p{};
+    for (int base = 0; base < B; base += 32) {
+      const int bb = base + lane;
+      const SeqPlan q = seq_plan(bb, B, kv_len, Ls, K, g, Hkv, S_cap, tpi);
+      const int it = q.ok ? q.items : 0;
+      const int un = (q.ok && q.n_split > 1) ? Hkv * q.M : 0;
+      int inc_u = un, inc_it = it;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int a = __shfl_up_sync(0xffffffffu, inc_u, off);
+        const int c = __shfl_up_sync(0xffffffffu, inc_it, off);
+        if (lane >= off) { inc_u += a; inc_it += c; }
       }
-      merge_ml[2 * tid] = M;
-      merge_ml[2 * tid + 1] = Lsum;
-      if (lse) {
-        const int rr = r_base + tid;
-        const int t = rr / g, hq = kvh * g + rr % g;
-        lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
+      const int su = carry_u + inc_u - un;
+      const bool mine = un > 0 && unit >= su && unit < su + un;
+      const unsigned ball = __ballot_sync(0xffffffffu, mine);
+      if (ball) {
+        const int src = __ffs(ball) - 1;
+        b = base + src;
+        local = unit - __shfl_sync(0xffffffffu, su, src);
+        start_it = __shfl_sync(0xffffffffu, carry_it + inc_it - it, src);
+        p = seq_plan(b, B, kv_len, Ls, K, g, Hkv, S_cap, tpi);
+        break;
+      }
+      carry_u += __shfl_sync(0xffffffffu, inc_u, 31);
+      carry_it += __shfl_sync(0xffffffffu, inc_it, 31);
+    }
+    if (b < 0) break;
+    const int kvh = local / p.M, r = local % p.M;
+    const int mg = r / kAttnRows, lr = r % kAttnRows;
+    const int nsp = p.n_split;
+    auto slot_of = [&](int sp) { return (size_t)start_it + ((size_t)kvh * nsp + sp) * p.n_mg + mg; };
+    // row max and denominator over the splits
+    float M = -INFINITY;
+    for (int sp = lane; sp < nsp; sp += 32) M = fmaxf(M, __ldcg(&part_ml[(slot_of(sp) * kAttnRows + lr) * 2]));
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float Lsum = 0.f;
+    for (int sp = lane; sp < nsp; sp += 32) {
+      const size_t e = (slot_of(sp) * kAttnRows + lr) * 2;
+      const float ms = __ldcg(&part_ml[e]);
+      if (ms != -INFINITY) Lsum += __ldcg(&part_ml[e + 1]) * ex2_approx(ms - M);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
+    // weighted sum of the partial rows; lane covers D/32 consecutive columns
+    constexpr int CPL = D / 32;
+    float acc[CPL];
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) acc[i] = 0.f;
+    for (int base = 0; base < nsp; base += 32) {
+      float wl = 0.f;
+      if (base + lane < nsp) {
+        const float ms = __ldcg(&part_ml[(slot_of(base + lane) * kAttnRows + lr) * 2]);
+        wl = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
+      }
+      const int n = min(32, nsp - base);
+#pragma unroll 8
+      for (int j = 0; j < n; ++j) {
+        const float w = __shfl_sync(0xffffffffu, wl, j);
+        const float* src = part_o + (slot_of(base + j) * kAttnRows + lr) * D + lane * CPL;
+        if (CPL == 4) {
+          const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
+          acc[0] += w * v.x; acc[1] += w * v.y; acc[2 % CPL] += w * v.z; acc[3 % CPL] += w * v.w;
+        } else {
+          const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
+          acc[0] += w * v.x; acc[1 % CPL] += w * v.y;
+        }
       }
     }
-    __syncthreads();
-    for (int idx = tid; idx < rows * (D / 4); idx += kAttnThreads) {
-      const int lr = idx / (D / 4), c4 = idx % (D / 4);
-      const float M = merge_ml[2 * lr];
-      const float inv = 1.f / merge_ml[2 * lr + 1];
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int sp = 0; sp < nsp; ++sp) {
-        const size_t sl = base_slot + (size_t)sp * stride;
-        const float ms = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
-        if (ms == -INFINITY) continue;
-        const float w = ex2_approx(ms - M);
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(part_o + (sl * kAttnRows + lr) * D) + c4);
-        acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
-      }
-      const int rr = r_base + lr;
-      const int t = rr / g, hq = kvh * g + rr % g;
-      __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + 4 * c4;
-      reinterpret_cast<__nv_bfloat162*>(dst)[0] = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-      reinterpret_cast<__nv_bfloat162*>(dst)[1] = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-    }
-    if (tid == 0) group_cnt[group] = 0u;
+    const float inv = 1.f / Lsum;
+    const int t = r / g, hq = kvh * g + r % g;
+    __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + lane * CPL;
+#pragma unroll
+    for (int i = 0; i < CPL; i += 2)
+      *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
+    if (lse && lane == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
   }
 }
 
@@ -583,23 +650,38 @@ static cudaError_t launch_attn_t(const CUtensorMap& mK, const CUtensorMap& mV, c
                                  cudaStream_t stream) {
   using SM = AttnSmem<D, STAGES>;
   auto kern = verify_attn_kernel<D, STAGES>;
-  static bool configured = false;
-  if (!configured) {
+  static int occ = 0;
+  if (occ == 0) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kAlloc);
     if (e != cudaSuccess) return e;
-    configured = true;
+    int o = 1;
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, kAttnThreads, SM::kAlloc);
+    occ = o < 1 ? 1 : o;
   }
-  int occ = 1;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kAttnThreads, SM::kAlloc);
-  if (occ < 1) occ = 1;
   int grid = num_sms_current() * occ;
   if (grid > kAttnMaxCtas) grid = kAttnMaxCtas;
-  kern<<<grid, kAttnThreads, SM::kAlloc, stream>>>(
-      mK, mV, reinterpret_cast<const __nv_bfloat16*>(Q), kv_len, L, B, K, Hq, Hkv, S_cap, scale * kLog2e,
-      min_tiles, reinterpret_cast<__nv_bfloat16*>(O), lse, reinterpret_cast<float*>(ws + lay.attn_o),
-      reinterpret_cast<float*>(ws + lay.attn_ml), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt),
-      reinterpret_cast<int*>(ws + lay.status));
-  return cudaGetLastError();
+  auto* part_o = reinterpret_cast<float*>(ws + lay.attn_o);
+  auto* part_ml = reinterpret_cast<float*>(ws + lay.attn_ml);
+  auto* st = reinterpret_cast<int*>(ws + lay.status);
+  auto* Ob = reinterpret_cast<__nv_bfloat16*>(O);
+  kern<<<grid, kAttnThreads, SM::kAlloc, stream>>>(mK, mV, reinterpret_cast<const __nv_bfloat16*>(Q), kv_len, L, B,
+                                                   K, Hq, Hkv, S_cap, scale * kLog2e, min_tiles, Ob, lse, part_o,
+                                                   part_ml, st);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  // merge kernel as a programmatic dependent launch
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * num_sms_current());
+  cfg.blockDim = dim3(kMergeThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, attn_merge_kernel<D>, kv_len, L, B, K, Hq, Hkv, S_cap, grid, min_tiles, Ob, lse,
+                            (const float*)part_o, (const float*)part_ml);
 }
 
 // Launch tuning: pipeline depth variant and the smallest run of key tiles

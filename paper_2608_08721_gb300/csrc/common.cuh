@@ -42,7 +42,7 @@ struct RacePartial {
 
 struct WsLayout {
   size_t status, conf_part, conf_cnt, row_part, row_cnt, row_stat, race_part, race_cnt;
-  size_t attn_o, attn_ml, attn_cnt, total;
+  size_t attn_o, attn_ml, total;
   int max_items, max_groups;
 };
 
@@ -69,7 +69,6 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.race_cnt = take(size_t(B) * sizeof(uint32_t));
   w.attn_o = take(size_t(w.max_items) * kAttnRows * d * sizeof(float));
   w.attn_ml = take(size_t(w.max_items) * kAttnRows * 2 * sizeof(float));
-  w.attn_cnt = take(size_t(w.max_groups) * sizeof(uint32_t));
   w.total = off;
   return w;
 }

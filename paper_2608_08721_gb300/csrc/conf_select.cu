@@ -7,7 +7,7 @@ namespace libraspec {
 // Confidence: grid (nsplit, B*K), 256 threads. CTA `split` of row r streams
 // columns [split*chunk, (split+1)*chunk) once, keeping the running max and
 // sum of exp((x - m)/T). With several splits the last CTA to finish (atomic
-// ticket) merges the row's partials in binary64 and finalises
+// ticket) merges the row's partials (binary64 sums) and finalises
 // q = exp((x_tok - m)/T) / Z (Assumption 1: q_k, the drafter's probability
 // of its drafted token).
 // ---------------------------------------------------------------------------
@@ -55,7 +55,7 @@ __global__ void __launch_bounds__(kRowThreads) conf_kernel(
     if (threadIdx.x >= 32) return;
     __threadfence();
     int dummy;
-    warp_merge_partials(part + (size_t)row * kConfMaxSplits, nsplit, (double)T, false, M, dummy, Z);
+    warp_merge_partials(part + (size_t)row * kConfMaxSplits, nsplit, c, false, M, dummy, Z);
     if (threadIdx.x != 0) return;
     cnt[row] = 0u;  // ready for the next call
   }
@@ -64,7 +64,8 @@ __global__ void __launch_bounds__(kRowThreads) conf_kernel(
   if (tok < 0 || tok >= V) {
     raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
   } else {
-    q = (float)(exp(((double)xr[tok] - (double)M) / (double)T) / Z);
+    // x_tok - M is exact for the near-maximal tokens that matter (Sterbenz)
+    q = (float)((double)exp2f((xr[tok] - M) * c) / Z);
   }
   conf[row] = q;
   if (dstat) {
@@ -149,7 +150,7 @@ cudaError_t launch_confidence(const float* x, const int32_t* tokens, const float
                               cudaStream_t stream) {
   const long rows = (long)B * K;
   if (rows == 0) return cudaSuccess;
-  const int nsplit0 = row_splits(rows, V, num_sms_current(), kConfMaxSplits, 2048);
+  const int nsplit0 = row_splits(rows, V, num_sms_current(), kConfMaxSplits, 4096);
   const int chunk = row_chunk(V, nsplit0);
   const int nsplit = (V + chunk - 1) / chunk;
   const bool vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0);

@@ -142,9 +142,11 @@ __device__ __forceinline__ void cta_reduce_arg(float& m, int& arg, float* smf /*
   }
 }
 
-// Merge nsplit partials of one row in binary64 (one warp; result in lane 0).
-// T is the temperature: s_i * exp((m_i - M) / T) rescales each share.
-__device__ __forceinline__ void warp_merge_partials(const RowPartial* __restrict__ p, int nsplit, double T,
+// Merge nsplit partials of one row (one warp; result in lane 0). Each share
+// s_i was summed relative to its own max m_i; it is rescaled to the row max M
+// by 2^((m_i - M) c), c = log2(e)/T, and the shares are added in binary64
+// (additions only: GB300 runs binary64 at a small fraction of the fp32 rate).
+__device__ __forceinline__ void warp_merge_partials(const RowPartial* __restrict__ p, int nsplit, float c,
                                                     bool want_arg, float& m_out, int& arg_out,
                                                     double& s_out) {
   const int lane = threadIdx.x & 31;
@@ -168,7 +170,7 @@ __device__ __forceinline__ void warp_merge_partials(const RowPartial* __restrict
     for (int i = lane; i < nsplit; i += 32) {
       const float mi = __ldcg(&p[i].m);
       const double si = __ldcg(&p[i].s);
-      if (mi != -INFINITY) s += si * exp(((double)mi - (double)m) / T);
+      if (mi != -INFINITY) s += si * (double)ex2_approx((mi - m) * c);
     }
   }
 #pragma unroll
@@ -184,7 +186,7 @@ inline int row_splits(long rows, int V, int num_sms, int max_splits, int min_ele
   if (rows <= 0) return 1;
   const long target = 4L * 8 * num_sms;
   long ns = (target + rows - 1) / rows;
-  const long cap = (V + min_elems - 1) / min_elems;
+  const long cap = (V + min_elems - 1) / min_elems;  // at least min_elems per CTA
   if (ns > cap) ns = cap;
   if (ns > max_splits) ns = max_splits;
   if (ns < 1) ns = 1;

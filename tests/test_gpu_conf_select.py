@@ -98,7 +98,8 @@ def test_round_selection_matches_oracle_chain(orc, name):
     L_ref, flag = orc.select_lengths(q_ref, cost.astype(np.float64))
     assert_exact_unless_flagged(L, L_ref, flag, "L")
     if name == "ragged":
-        assert L_ref.min() <= 2 and L_ref.max() >= w.K - 2, "ragged lengths should span 0..K: %s" % L_ref
+        # the per-sequence peakedness spreads the selected lengths widely
+        assert L_ref.min() == 0 and L_ref.max() >= 8, "ragged lengths: %s" % L_ref
 
 
 def test_select_edge_cases(orc):
