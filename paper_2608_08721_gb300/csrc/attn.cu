@@ -1,21 +1,34 @@
-// Step 3: block-causal GQA verify attention (split-KV, persistent grid).
+// Step 3: block-causal GQA verify attention on GB300 (split-KV, Stream-K,
+// warp-specialised persistent CTAs).
 //
 // Work decomposition. For sequence b the verified block has M_b = (L_b+1)*g
 // query rows per kv head (g = Hq/Hkv; row r is block position t = r / g of
 // query head kvh*g + r % g) and N_b = kv_len_b + L_b + 1 visible keys. Rows
-// are cut into groups of 64 (one m16 tile per warp, 4 warps) and keys into
-// 64-key tiles. A work item is (b, kv head, row group, run of consecutive
-// key tiles); every CTA derives the item list itself from L[] and kv_len[]
-// (both device-resident), so the grid never depends on values the host does
-// not know. Items are dealt round-robin over a persistent grid.
+// are cut into groups of 64 (one m16 tile per consumer warp) and keys into
+// 64-key tiles. All (row group, key tile) pairs of the batch form one tile
+// sequence (sequence-major, then kv head, row group, key tile); CTA c of the
+// persistent grid takes the contiguous range [c*T/G, (c+1)*T/G) of it, so
+// every CTA streams the same number of tiles whatever the ragged lengths.
+// The plan is derived on the device from L[] and kv_len[] by every CTA.
 //
-// Per item: K/V tiles arrive by TMA (128-byte swizzle, mbarrier pipeline of
-// STAGES tiles); each warp computes S = Q K^T for its 16 rows with
-// mma.sync m16n8k16 (bf16 in, fp32 accumulate), masks keys beyond
-// kv_len_b + t, keeps an online softmax in the log2 domain and accumulates
-// O += P V. An item that covers all of a row group's keys writes O directly;
-// otherwise it writes an fp32 partial (O, m, l) and the last item of the
-// group to finish (atomic ticket) merges the partials in a fixed order.
+// Inside a CTA one producer warp walks the CTA's range: for each run of tiles
+// of one row group (an "item") it loads the group's Q rows into a
+// double-buffered shared slot (cp.async) and issues the K/V tiles by TMA
+// (3-D tensor map, 128-byte swizzle) into a ring of STAGES stages, running
+// ahead of the consumers across item boundaries. Four consumer warps compute
+// S = Q K^T and O += P V with mma.sync m16n8k16 (bf16 in, fp32 accumulate),
+// mask keys beyond kv_len_b + t and keep an online softmax in the log2
+// domain. Full/empty mbarriers hand stages between the two roles.
+//
+// A row group covered by one CTA is written directly. A group spread over
+// CTAs c0..c1 leaves one fp32 partial (O, m, l) per CTA, in slot 2c+1 for c0
+// (its last item) and 2c for the others (their first item). Once a CTA has
+// finished its whole range it takes part in the merges of (at most two)
+// groups it contributed to: it waits (bounded) until every part of the group
+// has arrived, then combines its share of the group's rows x columns from all
+// parts in CTA order -- deterministic, and spread over every contributing SM
+// instead of one. The grid is launched cooperatively, so all CTAs are
+// resident and these waits always end.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -26,8 +39,11 @@
 
 namespace libraspec {
 
-constexpr int kAttnThreads = 128;
+constexpr int kConsumerWarps = 4;
+constexpr int kAttnThreads = (kConsumerWarps + 1) * 32;
+constexpr int kProducerWarp = kConsumerWarps;
 constexpr int kMaxWaitIters = 1 << 24;
+constexpr int kConsumerBar = 1;  // named barrier of the consumer warps
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -35,6 +51,10 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
 
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
@@ -46,6 +66,18 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
       : "r"(bar), "r"(parity)
@@ -67,6 +99,20 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
       " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
       : "memory");
+}
+
+// 16-byte async copy global -> shared; src_bytes = 0 writes zeros.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+
+// Arrive on `bar` once this thread's earlier cp.async copies have landed.
+__device__ __forceinline__ void cp_async_arrive(uint32_t bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void consumer_sync() {
+  asm volatile("bar.sync %0, %1;" ::"n"(kConsumerBar), "n"(kConsumerWarps * 32) : "memory");
 }
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
@@ -103,19 +149,17 @@ __device__ __forceinline__ uint32_t sw128(int row, int col) {
   return (uint32_t)(box * 8192 + row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
-struct ItemInfo {
-  int b, kvh, mg, split, nsplit, kv, Lb, rows, key0, key1, group, item_base, n_mg;
-};
-
-// Per-sequence quantities of the item list.
+// ---------------------------------------------------------------------------
+// Device-side plan.
+// ---------------------------------------------------------------------------
 struct SeqPlan {
-  int M, n_mg, N, n_tiles, n_split, items, groups;
+  int M, n_mg, N, n_tiles;  // rows, row groups, visible keys, key tiles
   bool ok;
 };
 
 __device__ __forceinline__ SeqPlan seq_plan(int b, int B, const int32_t* kv_len, const int32_t* Ls, int K, int g,
-                                            int Hkv, int S_cap, int tpi) {
-  SeqPlan p{0, 0, 0, 0, 0, 0, 0, false};
+                                            int S_cap) {
+  SeqPlan p{0, 0, 0, 0, false};
   if (b >= B) return p;
   const int Lb = Ls[b], kv = kv_len[b];
   if (Lb < 0 || Lb > K || kv < 0 || (long)kv + Lb + 1 > S_cap) return p;
@@ -124,30 +168,23 @@ __device__ __forceinline__ SeqPlan seq_plan(int b, int B, const int32_t* kv_len,
   p.n_mg = (p.M + kAttnRows - 1) / kAttnRows;
   p.N = kv + Lb + 1;
   p.n_tiles = (p.N + kAttnTileKeys - 1) / kAttnTileKeys;
-  if (tpi > 0) {
-    p.n_split = (p.n_tiles + tpi - 1) / tpi;
-    p.items = Hkv * p.n_mg * p.n_split;
-  }
-  p.groups = Hkv * p.n_mg;
   return p;
 }
 
-// Warp 0: total key tiles over all row groups (sets tpi for everyone) and
-// flags invalid sequences.
-__device__ int total_tiles(int B, const int32_t* kv_len, const int32_t* Ls, int K, int g, int Hkv, int S_cap,
-                           int* status, bool report) {
+// Warp-wide: total tiles T of the batch; flags invalid sequences.
+__device__ long long total_tiles(int B, const int32_t* kv_len, const int32_t* Ls, int K, int g, int Hkv,
+                                 int S_cap, int* status, bool report) {
   const int lane = threadIdx.x & 31;
-  long tot = 0;
+  long long tot = 0;
   bool bad = false;
   for (int b = lane; b < B; b += 32) {
-    const SeqPlan p = seq_plan(b, B, kv_len, Ls, K, g, Hkv, S_cap, 0);
+    const SeqPlan p = seq_plan(b, B, kv_len, Ls, K, g, S_cap);
     if (!p.ok) bad = true;
-    else tot += (long)Hkv * p.n_mg * p.n_tiles;
+    else tot += (long long)Hkv * p.n_mg * p.n_tiles;
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, off);
   if (report && __any_sync(0xffffffffu, bad) && lane == 0) {
-    // report which condition: re-check on lane 0 (cheap, B small)
     int bits = 0;
     for (int b = 0; b < B; ++b) {
       const int Lb = Ls[b], kv = kv_len[b];
@@ -156,199 +193,300 @@ __device__ int total_tiles(int B, const int32_t* kv_len, const int32_t* Ls, int 
     }
     raise_status(status, bits);
   }
-  return (int)(tot > 0x7fffffff ? 0x7fffffff : tot);
+  return tot;
 }
 
-// Warp 0: locate item i. Returns false when i is past the last item.
-__device__ bool locate_item(int item, int B, const int32_t* kv_len, const int32_t* Ls, int K, int g, int Hkv,
-                            int S_cap, int tpi, ItemInfo& info) {
+// Where tile position `pos` of the batch's tile sequence lies (warp-wide).
+struct TileLoc {
+  int b;                  // sequence (-1: past the end)
+  long long seq_start;    // first tile of sequence b
+  int group0;             // global index of b's first row group
+  SeqPlan p;
+};
+
+__device__ TileLoc locate_tile(long long pos, int B, const int32_t* kv_len, const int32_t* Ls, int K, int g, int Hkv,
+                               int S_cap) {
   const int lane = threadIdx.x & 31;
-  int item_carry = 0, group_carry = 0;
+  TileLoc loc{-1, 0, 0, {}};
+  long long carry_t = 0;
+  int carry_g = 0;
   for (int base = 0; base < B; base += 32) {
     const int b = base + lane;
-    const SeqPlan p = seq_plan(b, B, kv_len, Ls, K, g, Hkv, S_cap, tpi);
-    const int it = p.ok ? p.items : 0, gr = p.ok ? p.groups : 0;
-    int inc_it = it, inc_gr = gr;
+    const SeqPlan p = seq_plan(b, B, kv_len, Ls, K, g, S_cap);
+    const long long nt = p.ok ? (long long)Hkv * p.n_mg * p.n_tiles : 0;
+    const int ng = p.ok ? Hkv * p.n_mg : 0;
+    long long inc_t = nt;
+    int inc_g = ng;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
-      const int a = __shfl_up_sync(0xffffffffu, inc_it, off);
-      const int c = __shfl_up_sync(0xffffffffu, inc_gr, off);
-      if (lane >= off) { inc_it += a; inc_gr += c; }
+      const long long a = __shfl_up_sync(0xffffffffu, inc_t, off);
+      const int c = __shfl_up_sync(0xffffffffu, inc_g, off);
+      if (lane >= off) { inc_t += a; inc_g += c; }
     }
-    const int start_it = item_carry + inc_it - it, start_gr = group_carry + inc_gr - gr;
-    const bool mine = it > 0 && item >= start_it && item < start_it + it;
+    const long long st = carry_t + inc_t - nt;
+    const bool mine = nt > 0 && pos >= st && pos < st + nt;
     const unsigned ball = __ballot_sync(0xffffffffu, mine);
     if (ball) {
       const int src = __ffs(ball) - 1;
-      if (lane == src) {
-        const int local = item - start_it;
-        info.b = b;
-        info.mg = local % p.n_mg;
-        const int rem = local / p.n_mg;
-        info.split = rem % p.n_split;
-        info.kvh = rem / p.n_split;
-        info.nsplit = p.n_split;
-        info.kv = kv_len[b];
-        info.Lb = Ls[b];
-        const int r0 = info.mg * kAttnRows;
-        info.rows = min(kAttnRows, p.M - r0);
-        const int t0 = info.split * tpi, t1 = min(p.n_tiles, t0 + tpi);
-        info.key0 = t0 * kAttnTileKeys;
-        info.key1 = min(p.N, t1 * kAttnTileKeys);
-        info.group = start_gr + info.kvh * p.n_mg + info.mg;
-        info.item_base = start_it + info.kvh * p.n_split * p.n_mg + info.mg;  // + split * n_mg
-        info.n_mg = p.n_mg;
-      }
-      return true;
+      loc.b = base + src;
+      loc.seq_start = __shfl_sync(0xffffffffu, st, src);
+      loc.group0 = __shfl_sync(0xffffffffu, carry_g + inc_g - ng, src);
+      loc.p = seq_plan(loc.b, B, kv_len, Ls, K, g, S_cap);
+      return loc;
     }
-    item_carry += __shfl_sync(0xffffffffu, inc_it, 31);
-    group_carry += __shfl_sync(0xffffffffu, inc_gr, 31);
+    carry_t += __shfl_sync(0xffffffffu, inc_t, 31);
+    carry_g += __shfl_sync(0xffffffffu, inc_g, 31);
   }
-  return false;
+  return loc;
 }
+
+__device__ __forceinline__ long long range_lo(int c, long long T, int G) { return (long long)c * T / G; }
+
+// CTA whose range holds tile t: the largest c with c*T/G <= t.
+__device__ __forceinline__ int cta_of(long long t, long long T, int G) {
+  return (int)(((t + 1) * (long long)G - 1) / T);
+}
+
+// One item handed from the producer to the consumers.
+struct ItemInfo {
+  int valid;          // 0: end of the CTA's range
+  int b, kvh, mg, rows, kv;
+  int key0, key1;     // keys [key0, key1)
+  int partial;        // 1: write a partial, else write O
+  int slot;           // partial slot
+  int group, c0, nparts;
+};
 
 template <int D, int STAGES>
 struct AttnSmem {
   static constexpr int kBoxes = D / 64;
   static constexpr int kTileBytes = kBoxes * 8192;  // one 64 x D bf16 tile
+  // 2 Q slots; each also serves as the key-split merge scratch of its item
+  // (two 16-row fp32 partials with their (m, l)), so it is rounded up to 1 KB
+  static constexpr int kQSlot = ((kTileBytes > 2 * (16 * D + 32) * 4 ? kTileBytes : 2 * (16 * D + 32) * 4) +
+                                 1023) / 1024 * 1024;
   static constexpr int kQ = 0;
-  static constexpr int kK = kQ + kTileBytes;
+  static constexpr int kK = kQ + 2 * kQSlot;
   static constexpr int kV = kK + STAGES * kTileBytes;
-  static constexpr int kBar = kV + STAGES * kTileBytes;
-  static constexpr int kInfo = kBar + 8 * STAGES;
-  static constexpr int kMerge = kInfo + 128;            // m, l of the merged rows (64 x 2 floats)
-  static constexpr int kBytes = kMerge + 64 * 2 * 4;
-  static constexpr int kAlloc = kBytes + 1024;          // room to align the base to 1024
+  static constexpr int kBar = kV + STAGES * kTileBytes;  // full[S], empty[S], qfull[2], qempty[2]
+  static constexpr int kInfo = kBar + 8 * (2 * STAGES + 4);
+  static constexpr int kMisc = kInfo + 2 * 64;
+  static constexpr int kBytes = kMisc + 16;
+  static constexpr int kAlloc = kBytes + 1024;      // room to align the base to 1024
 };
 
 template <int D, int STAGES>
-__global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
+__global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
     const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
     const __nv_bfloat16* __restrict__ Q, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
     int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, __nv_bfloat16* __restrict__ O,
-    float* __restrict__ lse, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ status) {
+    float* __restrict__ lse, float* __restrict__ part_o, float* __restrict__ part_ml,
+    uint32_t* __restrict__ group_cnt, int* __restrict__ status) {
   using SM = AttnSmem<D, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sQ = smem_u32(smem + SM::kQ);
   const uint32_t sK = smem_u32(smem + SM::kK);
   const uint32_t sV = smem_u32(smem + SM::kV);
-  const uint32_t sBar = smem_u32(smem + SM::kBar);
-  ItemInfo& info = *reinterpret_cast<ItemInfo*>(smem + SM::kInfo);
-  float* merge_ml = reinterpret_cast<float*>(smem + SM::kMerge);
-  __shared__ int sh_tpi, sh_found, sh_abort;
+  const uint32_t bFull = smem_u32(smem + SM::kBar);
+  const uint32_t bEmpty = bFull + 8 * STAGES;
+  const uint32_t bQFull = bEmpty + 8 * STAGES;
+  const uint32_t bQEmpty = bQFull + 16;
+  ItemInfo* info = reinterpret_cast<ItemInfo*>(smem + SM::kInfo);
+  volatile int* misc = reinterpret_cast<int*>(smem + SM::kMisc);  // [0] wait result, [1] abort
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = Hq / Hkv;
 
   if (tid == 0) {
-    for (int s = 0; s < STAGES; ++s) mbar_init(sBar + 8 * s, 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    sh_abort = 0;
-  }
-  if (warp == 0) {
-    const int tot = total_tiles(B, kv_len, Ls, K, g, Hkv, S_cap, status, blockIdx.x == 0);
-    if (lane == 0) {
-      int tpi = (tot + (int)gridDim.x - 1) / (int)gridDim.x;
-      sh_tpi = tpi < min_tiles ? min_tiles : tpi;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(bFull + 8 * s, 1);
+      mbar_init(bEmpty + 8 * s, kConsumerWarps);
     }
+    for (int q = 0; q < 2; ++q) {
+      mbar_init(bQFull + 8 * q, 33);  // 32 cp.async arrivals + the info arrival
+      mbar_init(bQEmpty + 8 * q, kConsumerWarps);
+    }
+    misc[0] = 0;
+    misc[1] = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
-  const int tpi = sh_tpi;
-  uint32_t tile_ctr = 0;  // tiles consumed by this CTA so far (stage / phase)
-  // let the merge kernel (launched as a programmatic dependent) get resident
-  // as soon as SMs free up; it waits for this grid's completion itself
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  for (int item = blockIdx.x;; item += gridDim.x) {
-    __syncthreads();  // everyone is done with the previous item's shared state
-    if (warp == 0) {
-      const bool found = locate_item(item, B, kv_len, Ls, K, g, Hkv, S_cap, tpi, info);
-      if (lane == 0) sh_found = found;
+  if (warp == kProducerWarp) {
+    // ======================= producer =======================
+    const long long T = total_tiles(B, kv_len, Ls, K, g, Hkv, S_cap, status, blockIdx.x == 0);
+    int G = (int)gridDim.x;
+    if (T > 0) {
+      const long long g_cap = (T + min_tiles - 1) / min_tiles;
+      if ((long long)G > g_cap) G = (int)g_cap;
     }
-    __syncthreads();
-    if (!sh_found || sh_abort) break;
-    const int b = info.b, kvh = info.kvh, rows = info.rows, kv = info.kv;
-    const int r_base = info.mg * kAttnRows;
-    const int key0 = info.key0, key1 = info.key1;
-    const int nsplit = info.nsplit, split = info.split, n_mg = info.n_mg;
-    const int group = info.group, item_base = info.item_base;
-    const int n_tiles = (key1 - key0 + kAttnTileKeys - 1) / kAttnTileKeys;
-    const int zcoord = b * Hkv + kvh;
-
-    // ---- producer prologue: first STAGES tiles ----
-    if (tid == 0) {
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      for (int i = 0; i < n_tiles && i < STAGES; ++i) {
-        const uint32_t s = (tile_ctr + i) % STAGES;
-        const uint32_t bar = sBar + 8 * s;
+    const int c = blockIdx.x;
+    long long pos = (T > 0 && c < G) ? range_lo(c, T, G) : 0;
+    const long long hi = (T > 0 && c < G) ? range_lo(c + 1, T, G) : 0;
+    uint32_t item_ctr = 0, tile_ctr = 0;
+    while (true) {
+      const bool have = pos < hi;
+      ItemInfo it{};
+      int n_tiles = 0, zc = 0;
+      if (have) {
+        const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, Hkv, S_cap);
+        const int nt = loc.p.n_tiles;
+        const long long off = pos - loc.seq_start;
+        const int gib = (int)(off / nt);             // row group within the sequence
+        const long long gstart = loc.seq_start + (long long)gib * nt;
+        const long long gend = gstart + nt;
+        const long long iend = gend < hi ? gend : hi;
+        it.valid = 1;
+        it.b = loc.b;
+        it.kvh = gib / loc.p.n_mg;
+        it.mg = gib % loc.p.n_mg;
+        it.rows = min(kAttnRows, loc.p.M - it.mg * kAttnRows);
+        it.kv = kv_len[loc.b];
+        it.key0 = (int)(pos - gstart) * kAttnTileKeys;
+        it.key1 = min(loc.p.N, (int)(iend - gstart) * kAttnTileKeys);
+        it.group = loc.group0 + gib;
+        const bool whole = (pos == gstart) && (gend <= hi);
+        it.partial = whole ? 0 : 1;
+        it.c0 = cta_of(gstart, T, G);
+        it.nparts = cta_of(gend - 1, T, G) - it.c0 + 1;
+        it.slot = (pos == gstart) ? 2 * c + 1 : 2 * c;
+        n_tiles = (int)(iend - pos);
+        zc = loc.b * Hkv + it.kvh;
+        pos = iend;
+      }
+      const uint32_t q = item_ctr & 1;
+      const uint32_t qpar = ((item_ctr >> 1) & 1) ^ 1;
+      if (!mbar_wait(bQEmpty + 8 * q, qpar)) {
+        if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
+        misc[1] = 1;
+        return;
+      }
+      // Tiles whose stage is already free go out before the Q copies: on a
+      // CTA's first item the K/V latency is the long pole.
+      int issued = 0;
+      auto issue_tile = [&](int i) {
+        const uint32_t s = tile_ctr % STAGES;
+        const uint32_t bar = bFull + 8 * s;
         mbar_expect_tx(bar, 2 * SM::kTileBytes);
-        const int y = key0 + i * kAttnTileKeys;
+        const int y = it.key0 + i * kAttnTileKeys;
 #pragma unroll
         for (int bx = 0; bx < SM::kBoxes; ++bx) {
-          tma_load_3d(sK + s * SM::kTileBytes + bx * 8192, &tmK, bar, bx * 64, y, zcoord);
-          tma_load_3d(sV + s * SM::kTileBytes + bx * 8192, &tmV, bar, bx * 64, y, zcoord);
+          tma_load_3d(sK + s * SM::kTileBytes + bx * 8192, &tmK, bar, bx * 64, y, zc);
+          tma_load_3d(sV + s * SM::kTileBytes + bx * 8192, &tmV, bar, bx * 64, y, zc);
+        }
+        ++tile_ctr;
+      };
+      if (have && lane == 0) {
+        while (issued < n_tiles && mbar_test_wait(bEmpty + 8 * (tile_ctr % STAGES),
+                                                  ((tile_ctr / STAGES) & 1) ^ 1)) {
+          issue_tile(issued);
+          ++issued;
         }
       }
-    }
-
-    // ---- Q rows of this group into shared memory (zero beyond `rows`) ----
-    {
-      constexpr int kChunks = D / 8;  // 16-byte chunks per row
-      for (int idx = tid; idx < kAttnRows * kChunks; idx += kAttnThreads) {
-        const int r = idx / kChunks, ch = idx % kChunks;
-        uint4 val = make_uint4(0, 0, 0, 0);
-        if (r < rows) {
-          const int rr = r_base + r;
-          const int t = rr / g, h = kvh * g + rr % g;
-          const __nv_bfloat16* src = Q + (((size_t)b * (K + 1) + t) * Hq + h) * D + ch * 8;
-          val = *reinterpret_cast<const uint4*>(src);
+      if (have) {
+        // Q rows of the item's row group (rows past `rows` are never used)
+        const uint32_t qdst = sQ + q * SM::kQSlot;
+        constexpr int kChunks = D / 8;
+        for (int idx = lane; idx < it.rows * kChunks; idx += 32) {
+          const int r = idx / kChunks, ch = idx - r * kChunks;
+          const int rr = it.mg * kAttnRows + r;
+          const int t = rr / g, h = it.kvh * g + (rr - t * g);
+          const __nv_bfloat16* src = Q + (((size_t)it.b * (K + 1) + t) * Hq + h) * D + ch * 8;
+          cp_async16(qdst + sw128(r, ch * 8), src, 16u);
         }
-        *reinterpret_cast<uint4*>(smem + SM::kQ + sw128(r, ch * 8)) = val;
       }
+      if (lane == 0) {
+        info[q] = it;
+        mbar_arrive(bQFull + 8 * q);
+      }
+      cp_async_arrive(bQFull + 8 * q);
+      ++item_ctr;
+      if (!have) break;
+      if (lane == 0) {
+        for (int i = issued; i < n_tiles; ++i) {
+          const uint32_t par = ((tile_ctr / STAGES) & 1) ^ 1;
+          if (!mbar_wait(bEmpty + 8 * (tile_ctr % STAGES), par)) {
+            raise_status(status, LIBRASPEC_ST_TIMEOUT);
+            misc[1] = 1;
+            break;
+          }
+          issue_tile(i);
+        }
+      }
+      tile_ctr = __shfl_sync(0xffffffffu, tile_ctr, 0);
+      __syncwarp();
+      if (misc[1]) return;
     }
-    __syncthreads();
+    return;
+  }
 
-    const bool warp_live = warp * 16 < rows;
+  // ======================= consumers =======================
+  // Warp roles per item: the item's rows form n_rt tiles of 16 rows. With
+  // n_rt <= 2 the four warps are split across each KV tile's keys as well
+  // (ks warps per row tile, each taking kq of the tile's four 16-key chunks),
+  // so that small verified blocks still keep every warp busy; their (m, l, O)
+  // are combined through shared memory when the item ends.
+  uint32_t item_ctr = 0, tile_ctr = 0;
+  ItemInfo pending[2];
+  int n_pending = 0;
+  while (true) {
+    const uint32_t q = item_ctr & 1;
+    if (!mbar_wait(bQFull + 8 * q, (item_ctr >> 1) & 1)) {
+      if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
+      return;
+    }
+    const ItemInfo it = info[q];
+    if (!it.valid) break;
+    const int rows = it.rows, kv = it.kv, b = it.b, kvh = it.kvh;
+    const int r_base = it.mg * kAttnRows;
+    const int n_rt = (rows + 15) >> 4;
+    const int ks = n_rt == 1 ? 4 : (n_rt == 2 ? 2 : 1);
+    const int rt = warp / ks;            // row tile of this warp
+    const int kq = 4 / ks;               // 16-key chunks per tile for this warp
+    const int c_lo = (warp % ks) * kq;   // its first chunk
+    const bool warp_live = rt < n_rt;
+    const uint32_t qslot = sQ + q * SM::kQSlot;
     uint32_t qf[D / 16][4];
     if (warp_live) {
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const int mi = lane >> 3, rr = lane & 7;
-        const int row = warp * 16 + (mi & 1) * 8 + rr;
+        const int row = rt * 16 + (mi & 1) * 8 + rr;
         const int col = kk * 16 + (mi >> 1) * 8;
-        ldsm_x4(sQ + sw128(row, col), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
+        ldsm_x4(qslot + sw128(row, col), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
       }
     }
+    ++item_ctr;
+
     float o[D / 8][4];
 #pragma unroll
     for (int n = 0; n < D / 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
     float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-    // block row (t) of this thread's two rows, for the causal limit
-    const int row_a = r_base + warp * 16 + (lane >> 2);
-    const int lim_a = kv + row_a / g;            // last visible key of row_a
+    const int row_a = r_base + rt * 16 + (lane >> 2);
+    const int lim_a = kv + row_a / g;  // last visible key of row_a
     const int lim_b = kv + (row_a + 8) / g;
+    const int n_tiles = (it.key1 - it.key0 + kAttnTileKeys - 1) / kAttnTileKeys;
 
     for (int i = 0; i < n_tiles; ++i) {
       const uint32_t s = tile_ctr % STAGES;
-      const uint32_t par = (tile_ctr / STAGES) & 1;
-      if (!mbar_wait(sBar + 8 * s, par)) {
+      if (!mbar_wait(bFull + 8 * s, (tile_ctr / STAGES) & 1)) {
         if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
-        sh_abort = 1;
         return;
       }
-      const int kt0 = key0 + i * kAttnTileKeys;
+      const int kt0 = it.key0 + i * kAttnTileKeys;
       const uint32_t tK = sK + s * SM::kTileBytes, tV = sV + s * SM::kTileBytes;
-      // zero V rows past the visible keys so that 0 * garbage cannot poison O
-      if (kt0 + kAttnTileKeys > key1) {
-        __syncwarp();
-        const int first = key1 - kt0;
-        for (int idx = lane; idx < (kAttnTileKeys - first) * (D / 8); idx += 32) {
+      if (kt0 + kAttnTileKeys > it.key1) {
+        // zero V rows past the visible keys so that 0 * garbage cannot poison O
+        const int first = it.key1 - kt0;
+        for (int idx = warp * 32 + lane; idx < (kAttnTileKeys - first) * (D / 8); idx += kConsumerWarps * 32) {
           const int r = first + idx / (D / 8), ch = idx % (D / 8);
-          if (warp == 0) *reinterpret_cast<uint4*>(smem + SM::kV + s * SM::kTileBytes + sw128(r, ch * 8)) =
+          *reinterpret_cast<uint4*>(smem + SM::kV + s * SM::kTileBytes + sw128(r, ch * 8)) =
               make_uint4(0, 0, 0, 0);
         }
-        __syncthreads();
+        // these generic writes precede the next TMA write of the stage
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        consumer_sync();
       }
       if (warp_live) {
         float sc[8][4];
@@ -358,6 +496,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         for (int kk = 0; kk < D / 16; ++kk) {
 #pragma unroll
           for (int np = 0; np < 4; ++np) {
+            if (np < c_lo || np >= c_lo + kq) continue;
             const int mi = lane >> 3, rr = lane & 7;
             const int key = np * 16 + (mi >> 1) * 8 + rr;
             const int col = kk * 16 + (mi & 1) * 8;
@@ -367,18 +506,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             mma_bf16(sc[2 * np + 1], qf[kk], b2, b3);
           }
         }
-        // scale into the log2 domain and mask
         const bool need_mask = kt0 + kAttnTileKeys - 1 > kv;
         float tmax[2] = {-INFINITY, -INFINITY};
 #pragma unroll
         for (int n = 0; n < 8; ++n) {
+          const bool mine = (n >> 1) >= c_lo && (n >> 1) < c_lo + kq;
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
             float x = sc[n][e] * scale_log2;
+            if (!mine) x = -INFINITY;
             if (need_mask) {
               const int key = kt0 + n * 8 + 2 * (lane & 3) + (e & 1);
-              const int lim = (e < 2) ? lim_a : lim_b;
-              if (key > lim) x = -INFINITY;
+              if (key > ((e < 2) ? lim_a : lim_b)) x = -INFINITY;
             }
             sc[n][e] = x;
             tmax[e >> 1] = fmaxf(tmax[e >> 1], x);
@@ -409,9 +548,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           l_run[0] += sc[n][0] + sc[n][1];
           l_run[1] += sc[n][2] + sc[n][3];
         }
-        // O += P V
 #pragma unroll
         for (int kc = 0; kc < 4; ++kc) {
+          if (kc < c_lo || kc >= c_lo + kq) continue;
           uint32_t a[4];
           a[0] = pack_bf16(sc[2 * kc][0], sc[2 * kc][1]);
           a[1] = pack_bf16(sc[2 * kc][2], sc[2 * kc][3]);
@@ -429,19 +568,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           }
         }
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bEmpty + 8 * s);
       ++tile_ctr;
-      __syncthreads();  // every warp is done with stage s
-      if (tid == 0 && i + STAGES < n_tiles) {
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        const uint32_t bar = sBar + 8 * s;
-        mbar_expect_tx(bar, 2 * SM::kTileBytes);
-        const int y = key0 + (i + STAGES) * kAttnTileKeys;
-#pragma unroll
-        for (int bx = 0; bx < SM::kBoxes; ++bx) {
-          tma_load_3d(tK + bx * 8192, &tmK, bar, bx * 64, y, zcoord);
-          tma_load_3d(tV + bx * 8192, &tmV, bar, bx * 64, y, zcoord);
-        }
-      }
     }
 
     // ---- epilogue ----
@@ -450,9 +579,71 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       l_run[h] += __shfl_xor_sync(0xffffffffu, l_run[h], 1);
       l_run[h] += __shfl_xor_sync(0xffffffffu, l_run[h], 2);
     }
-    const int lr0 = warp * 16 + (lane >> 2);  // local rows lr0, lr0 + 8
-    if (nsplit == 1) {
-      if (warp_live) {
+    // combine the key-split warps of each row tile through the (now free) Q slot
+    if (ks > 1) {
+      float* scr = reinterpret_cast<float*>(smem + SM::kQ + q * SM::kQSlot);
+      constexpr int kPart = 16 * D + 32;  // floats: O rows, then (m, l) of 16 rows
+      auto put = [&](int slot_i) {
+        float* dst = scr + slot_i * kPart;
+#pragma unroll
+        for (int n = 0; n < D / 8; ++n) {
+          const int col = n * 8 + 2 * (lane & 3);
+          *reinterpret_cast<float2*>(dst + (lane >> 2) * D + col) = make_float2(o[n][0], o[n][1]);
+          *reinterpret_cast<float2*>(dst + ((lane >> 2) + 8) * D + col) = make_float2(o[n][2], o[n][3]);
+        }
+        if ((lane & 3) == 0) {
+          dst[16 * D + 2 * (lane >> 2)] = m_run[0];
+          dst[16 * D + 2 * (lane >> 2) + 1] = l_run[0];
+          dst[16 * D + 2 * ((lane >> 2) + 8)] = m_run[1];
+          dst[16 * D + 2 * ((lane >> 2) + 8) + 1] = l_run[1];
+        }
+      };
+      auto take = [&](int slot_i) {
+        const float* src = scr + slot_i * kPart;
+        float wa[2], wb[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int r = (lane >> 2) + 8 * h;
+          const float mo = src[16 * D + 2 * r], lo = src[16 * D + 2 * r + 1];
+          const float M = fmaxf(m_run[h], mo);
+          wa[h] = (M == -INFINITY) ? 0.f : ex2_approx(m_run[h] - M);
+          wb[h] = (M == -INFINITY) ? 0.f : ex2_approx(mo - M);
+          l_run[h] = l_run[h] * wa[h] + lo * wb[h];
+          m_run[h] = M;
+        }
+#pragma unroll
+        for (int n = 0; n < D / 8; ++n) {
+          const int col = n * 8 + 2 * (lane & 3);
+          const float2 u = *reinterpret_cast<const float2*>(src + (lane >> 2) * D + col);
+          const float2 v = *reinterpret_cast<const float2*>(src + ((lane >> 2) + 8) * D + col);
+          o[n][0] = o[n][0] * wa[0] + u.x * wb[0];
+          o[n][1] = o[n][1] * wa[0] + u.y * wb[0];
+          o[n][2] = o[n][2] * wa[1] + v.x * wb[1];
+          o[n][3] = o[n][3] * wa[1] + v.y * wb[1];
+        }
+      };
+      const int kw = warp % ks;
+      consumer_sync();  // every warp has its Q fragments before the slot is overwritten
+      if (ks == 4) {
+        if (kw >= 2) put(kw - 2);
+        consumer_sync();
+        if (kw < 2) take(kw);
+        consumer_sync();
+        if (kw == 1) put(0);
+        consumer_sync();
+        if (kw == 0) take(0);
+      } else {  // ks == 2: warps 1 and 3 hand over to warps 0 and 2
+        if (kw == 1) put(rt);
+        consumer_sync();
+        if (kw == 0) take(rt);
+      }
+    }
+    consumer_sync();
+    if (lane == 0) mbar_arrive(bQEmpty + 8 * q);  // the slot may take the next Q now
+    const bool owner = warp_live && (warp % ks) == 0;
+    const int lr0 = rt * 16 + (lane >> 2);
+    if (!it.partial) {
+      if (owner) {
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int lr = lr0 + 8 * h;
@@ -473,10 +664,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       }
       continue;
     }
-    // several items share this row group: write the fp32 partial (O, m, l);
-    // attn_merge_kernel combines them once the whole grid is done
-    const size_t slot = (size_t)item_base + (size_t)split * n_mg;
-    if (warp_live) {
+    // partial of a row group spread over several CTAs
+    const size_t slot = (size_t)it.slot;
+    if (owner) {
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         const int lr = lr0 + 8 * h;
@@ -493,122 +683,101 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         }
       }
     }
-    (void)group;
+    consumer_sync();
+    if (tid == 0) {
+      // release: the partial written by this CTA happens-before the arrival
+      asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(&group_cnt[2 * it.group]), "r"(1u)
+                   : "memory");
+    }
+    if (n_pending < 2) pending[n_pending++] = it;
   }
-}
 
-// ---------------------------------------------------------------------------
-// Merge of the split-KV partials. Launched right after verify_attn_kernel as
-// a programmatic dependent: it becomes resident early and waits
-// (griddepcontrol.wait) until every attention CTA has finished and its
-// writes are visible. One warp per (sequence, kv head, row) whose row group
-// was split: O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, M = max_s m_s,
-// splits combined in a fixed order (deterministic). Spread over the whole
-// GPU, so no single SM reads all of a group's partials.
-// ---------------------------------------------------------------------------
-constexpr int kMergeThreads = 256;
-
-template <int D>
-__global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(
-    const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls, int B, int K, int Hq, int Hkv, int S_cap,
-    int attn_grid, int min_tiles, __nv_bfloat16* __restrict__ O, float* __restrict__ lse,
-    const float* __restrict__ part_o, const float* __restrict__ part_ml) {
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  __shared__ int sh_tpi;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int g = Hq / Hkv;
-  if (warp == 0) {
-    const int tot = total_tiles(B, kv_len, Ls, K, g, Hkv, S_cap, nullptr, false);
-    if (lane == 0) {
-      const int tpi = (tot + attn_grid - 1) / attn_grid;
-      sh_tpi = tpi < min_tiles ? min_tiles : tpi;
-    }
-  }
-  __syncthreads();
-  const int tpi = sh_tpi;
-  const int warps_total = gridDim.x * (kMergeThreads / 32);
-  for (int unit = blockIdx.x * (kMergeThreads / 32) + warp;; unit += warps_total) {
-    // locate the unit: units of sequence b (split row groups only) are
-    // Hkv * M_b rows, kv head major
-    int carry_u = 0, carry_it = 0;
-    int b = -1, local = 0, start_it = 0;
-    SeqPlan p{};
-    for (int base = 0; base < B; base += 32) {
-      const int bb = base + lane;
-      const SeqPlan q = seq_plan(bb, B, kv_len, Ls, K, g, Hkv, S_cap, tpi);
-      const int it = q.ok ? q.items : 0;
-      const int un = (q.ok && q.n_split > 1) ? Hkv * q.M : 0;
-      int inc_u = un, inc_it = it;
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const int a = __shfl_up_sync(0xffffffffu, inc_u, off);
-        const int c = __shfl_up_sync(0xffffffffu, inc_it, off);
-        if (lane >= off) { inc_u += a; inc_it += c; }
+  // ---- distributed merges of the groups this CTA contributed to ----
+  for (int pi = 0; pi < n_pending; ++pi) {
+    const ItemInfo& it = pending[pi];
+    const int c0 = it.c0, np = it.nparts;
+    const int k_me = (int)blockIdx.x - c0;  // this CTA's share
+    if (tid == 0) {
+      bool ok = false;
+      for (int i = 0; i < kMaxWaitIters; ++i) {
+        uint32_t v;
+        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(&group_cnt[2 * it.group]) : "memory");
+        if (v >= (uint32_t)np) { ok = true; break; }
+        __nanosleep(32);
       }
-      const int su = carry_u + inc_u - un;
-      const bool mine = un > 0 && unit >= su && unit < su + un;
-      const unsigned ball = __ballot_sync(0xffffffffu, mine);
-      if (ball) {
-        const int src = __ffs(ball) - 1;
-        b = base + src;
-        local = unit - __shfl_sync(0xffffffffu, su, src);
-        start_it = __shfl_sync(0xffffffffu, carry_it + inc_it - it, src);
-        p = seq_plan(b, B, kv_len, Ls, K, g, Hkv, S_cap, tpi);
-        break;
-      }
-      carry_u += __shfl_sync(0xffffffffu, inc_u, 31);
-      carry_it += __shfl_sync(0xffffffffu, inc_it, 31);
+      if (!ok) raise_status(status, LIBRASPEC_ST_TIMEOUT);
+      misc[0] = ok;
     }
-    if (b < 0) break;
-    const int kvh = local / p.M, r = local % p.M;
-    const int mg = r / kAttnRows, lr = r % kAttnRows;
-    const int nsp = p.n_split;
-    auto slot_of = [&](int sp) { return (size_t)start_it + ((size_t)kvh * nsp + sp) * p.n_mg + mg; };
-    // row max and denominator over the splits
-    float M = -INFINITY;
-    for (int sp = lane; sp < nsp; sp += 32) M = fmaxf(M, __ldcg(&part_ml[(slot_of(sp) * kAttnRows + lr) * 2]));
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    float Lsum = 0.f;
-    for (int sp = lane; sp < nsp; sp += 32) {
-      const size_t e = (slot_of(sp) * kAttnRows + lr) * 2;
-      const float ms = __ldcg(&part_ml[e]);
-      if (ms != -INFINITY) Lsum += __ldcg(&part_ml[e + 1]) * ex2_approx(ms - M);
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
-    // weighted sum of the partial rows; lane covers D/32 consecutive columns
-    constexpr int CPL = D / 32;
-    float acc[CPL];
-#pragma unroll
-    for (int i = 0; i < CPL; ++i) acc[i] = 0.f;
-    for (int base = 0; base < nsp; base += 32) {
-      float wl = 0.f;
-      if (base + lane < nsp) {
-        const float ms = __ldcg(&part_ml[(slot_of(base + lane) * kAttnRows + lr) * 2]);
-        wl = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
-      }
-      const int n = min(32, nsp - base);
-#pragma unroll 8
-      for (int j = 0; j < n; ++j) {
-        const float w = __shfl_sync(0xffffffffu, wl, j);
-        const float* src = part_o + (slot_of(base + j) * kAttnRows + lr) * D + lane * CPL;
-        if (CPL == 4) {
-          const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
-          acc[0] += w * v.x; acc[1] += w * v.y; acc[2 % CPL] += w * v.z; acc[3 % CPL] += w * v.w;
-        } else {
-          const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
-          acc[0] += w * v.x; acc[1 % CPL] += w * v.y;
+    consumer_sync();
+    const bool ok = misc[0] != 0;
+    consumer_sync();
+    if (!ok) return;
+    const int rows = it.rows, b = it.b, kvh = it.kvh, r_base = it.mg * kAttnRows;
+    const int u0 = (int)((long long)rows * k_me / np), u1 = (int)((long long)rows * (k_me + 1) / np);
+    constexpr int CPL = D / 32;  // columns per lane
+    for (int lr = u0 + warp; lr < u1; lr += kConsumerWarps) {
+      // one warp per row: part p's (m, l) sits in lane p % 32 of chunk p / 32
+      float M = -INFINITY;
+      for (int p0 = 0; p0 < np; p0 += 32) {
+        const int p = p0 + lane;
+        if (p < np) {
+          const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+          M = fmaxf(M, __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]));
         }
       }
-    }
-    const float inv = 1.f / Lsum;
-    const int t = r / g, hq = kvh * g + r % g;
-    __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + lane * CPL;
 #pragma unroll
-    for (int i = 0; i < CPL; i += 2)
-      *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
-    if (lse && lane == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
+      for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+      float Lsum = 0.f;
+      float acc[CPL];
+#pragma unroll
+      for (int i = 0; i < CPL; ++i) acc[i] = 0.f;
+      for (int p0 = 0; p0 < np; p0 += 32) {
+        float wl = 0.f;
+        {
+          const int p = p0 + lane;
+          if (p < np) {
+            const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+            const float ms = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
+            wl = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
+            Lsum += wl * __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
+          }
+        }
+        const int n = min(32, np - p0);
+#pragma unroll 8
+        for (int j = 0; j < n; ++j) {
+          const int p = p0 + j;
+          const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+          const float w = __shfl_sync(0xffffffffu, wl, j);
+          const float* src = part_o + (sl * kAttnRows + lr) * D + lane * CPL;
+          if (CPL == 4) {
+            const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
+            acc[0] += w * v.x; acc[1 % CPL] += w * v.y; acc[2 % CPL] += w * v.z; acc[3 % CPL] += w * v.w;
+          } else {
+            const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
+            acc[0] += w * v.x; acc[1 % CPL] += w * v.y;
+          }
+        }
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
+      const float inv = 1.f / Lsum;
+      const int rr = r_base + lr;
+      const int t = rr / g, hq = kvh * g + rr % g;
+      __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + lane * CPL;
+#pragma unroll
+      for (int i = 0; i < CPL; i += 2)
+        *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
+      if (lse && lane == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
+    }
+    // the last CTA done with this group resets its counters for the next launch
+    consumer_sync();
+    if (tid == 0) {
+      const uint32_t done = atomicAdd(&group_cnt[2 * it.group + 1], 1u);
+      if (done == (uint32_t)(np - 1)) {
+        group_cnt[2 * it.group] = 0u;
+        group_cnt[2 * it.group + 1] = 0u;
+      }
+    }
   }
 }
 
@@ -660,35 +829,28 @@ static cudaError_t launch_attn_t(const CUtensorMap& mK, const CUtensorMap& mV, c
   }
   int grid = num_sms_current() * occ;
   if (grid > kAttnMaxCtas) grid = kAttnMaxCtas;
-  auto* part_o = reinterpret_cast<float*>(ws + lay.attn_o);
-  auto* part_ml = reinterpret_cast<float*>(ws + lay.attn_ml);
-  auto* st = reinterpret_cast<int*>(ws + lay.status);
-  auto* Ob = reinterpret_cast<__nv_bfloat16*>(O);
-  kern<<<grid, kAttnThreads, SM::kAlloc, stream>>>(mK, mV, reinterpret_cast<const __nv_bfloat16*>(Q), kv_len, L, B,
-                                                   K, Hq, Hkv, S_cap, scale * kLog2e, min_tiles, Ob, lse, part_o,
-                                                   part_ml, st);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  // merge kernel as a programmatic dependent launch
+  // cooperative: every CTA is resident at once, which the merge waits rely on
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(2 * num_sms_current());
-  cfg.blockDim = dim3(kMergeThreads);
-  cfg.dynamicSmemBytes = 0;
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kAttnThreads);
+  cfg.dynamicSmemBytes = SM::kAlloc;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, attn_merge_kernel<D>, kv_len, L, B, K, Hq, Hkv, S_cap, grid, min_tiles, Ob, lse,
-                            (const float*)part_o, (const float*)part_ml);
+  return cudaLaunchKernelEx(&cfg, kern, mK, mV, reinterpret_cast<const __nv_bfloat16*>(Q), kv_len, L, B, K, Hq, Hkv,
+                            S_cap, scale * kLog2e, min_tiles, reinterpret_cast<__nv_bfloat16*>(O), lse,
+                            reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml),
+                            reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
 }
 
-// Launch tuning: pipeline depth variant and the smallest run of key tiles
-// per work item. Defaults were chosen by measurement on GB300; the
-// LIBRASPEC_ATTN_TUNING environment variable ("deep:min_tiles", deep = 0 for
-// the shallow two-CTAs-per-SM pipeline, 1 for the deep one-CTA-per-SM one)
-// overrides them, read once per process.
+// Launch tuning: pipeline depth variant and the smallest tile range per CTA.
+// Defaults were chosen by measurement on GB300; the LIBRASPEC_ATTN_TUNING
+// environment variable ("deep:min_tiles", deep = 0 for the two-CTAs-per-SM
+// pipeline, 1 for the deeper one-CTA-per-SM one) overrides them, read once
+// per process.
 struct AttnTuning {
   int deep = 0;
   int min_tiles = 2;
@@ -719,14 +881,14 @@ cudaError_t launch_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint
   const AttnTuning& t = attn_tuning();
   if (D == 128) {
     if (t.deep)
-      return launch_attn_t<128, 6>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
+      return launch_attn_t<128, 4>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
                                    stream);
     return launch_attn_t<128, 2>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
                                  stream);
   }
   if (t.deep)
-    return launch_attn_t<64, 10>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
-                                 stream);
+    return launch_attn_t<64, 8>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
+                                stream);
   return launch_attn_t<64, 4>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
                               stream);
 }

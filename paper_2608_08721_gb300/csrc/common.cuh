@@ -5,7 +5,7 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
-#include "../../include/libraspec.h"
+#include "libraspec.h"
 
 namespace libraspec {
 
@@ -42,7 +42,7 @@ struct RacePartial {
 
 struct WsLayout {
   size_t status, conf_part, conf_cnt, row_part, row_cnt, row_stat, race_part, race_cnt;
-  size_t attn_o, attn_ml, total;
+  size_t attn_o, attn_ml, attn_cnt, total;
   int max_items, max_groups;
 };
 
@@ -67,8 +67,10 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.row_stat = take(rows_t * sizeof(RowStat));
   w.race_part = take(size_t(B) * kRaceMaxSplits * sizeof(RacePartial));
   w.race_cnt = take(size_t(B) * sizeof(uint32_t));
-  w.attn_o = take(size_t(w.max_items) * kAttnRows * d * sizeof(float));
-  w.attn_ml = take(size_t(w.max_items) * kAttnRows * 2 * sizeof(float));
+  // two partial slots per attention CTA (its first and its last item)
+  w.attn_o = take(size_t(2 * kAttnMaxCtas) * kAttnRows * d * sizeof(float));
+  w.attn_ml = take(size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
+  w.attn_cnt = take(size_t(2 * w.max_groups) * sizeof(uint32_t));  // arrivals, merges done
   w.total = off;
   return w;
 }

@@ -59,7 +59,7 @@ def test_attn_rows_beyond_L_untouched():
 
 @pytest.mark.parametrize("kv", [5000, 20000])
 def test_attn_long_split_kv_merge(orc, kv):
-    # one sequence, long cache: many work items per row group, merged in-kernel
+    # one sequence, long cache: its row groups spread over many CTAs and are merged
     K, Hq, Hkv, d = 16, 32, 8, 128
     L = [11]
     Q, Kc, Vc = _inputs(1, K, Hq, Hkv, d, [kv], kv + K + 1, seed=kv)
@@ -140,3 +140,19 @@ def test_attn_deterministic():
         for O, lse in outs[1:]:
             assert torch.equal(O[b, rows], outs[0][0][b, rows])
             assert torch.equal(lse[b, rows], outs[0][1][b, rows])
+
+
+@pytest.mark.parametrize("B,kv_hi,d,seed", [(300, 200, 64, 1), (40, 9000, 128, 2), (129, 64, 128, 3)])
+def test_attn_many_sequences_stream_k_ranges(orc, B, kv_hi, d, seed):
+    """Many ragged sequences: CTA tile ranges start and end inside row groups,
+    one CTA covers several whole groups, and groups spread over many CTAs."""
+    rng = np.random.default_rng(seed)
+    K, Hq, Hkv = 12, 16, 4
+    kv = rng.integers(0, kv_hi + 1, size=B).astype(np.int32)
+    L = rng.integers(0, K + 1, size=B).astype(np.int32)
+    S_cap = int((kv + L).max()) + 1
+    Q, Kc, Vc = _inputs(B, K, Hq, Hkv, d, kv, S_cap, seed=seed * 101)
+    O, lse = _run(Q, Kc, Vc, kv.tolist(), L.tolist(), K)
+    rows = np.array([(b, h, t) for b in range(B) for h in (0, Hq - 1) for t in {0, int(L[b])}], np.int32)
+    O_ref, lse_ref = orc.verify_attn(Q, Kc, Vc, kv, L, rows=rows)
+    check_attn(O, lse, O_ref, lse_ref, L, rows=[tuple(r) for r in rows])
