@@ -683,13 +683,15 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
         }
       }
     }
-    consumer_sync();
-    if (tid == 0) {
-      // release: the partial written by this CTA happens-before the arrival
-      asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(&group_cnt[2 * it.group]), "r"(1u)
-                   : "memory");
-    }
     if (n_pending < 2) pending[n_pending++] = it;
+  }
+  // Announce this CTA's partials (at most two) once its whole range is done:
+  // one release after all of them instead of a fence per item.
+  consumer_sync();
+  if (tid == 0) {
+    for (int pi = 0; pi < n_pending; ++pi)
+      asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(&group_cnt[2 * pending[pi].group]), "r"(1u)
+                   : "memory");
   }
 
   // ---- distributed merges of the groups this CTA contributed to ----
@@ -714,60 +716,135 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
     if (!ok) return;
     const int rows = it.rows, b = it.b, kvh = it.kvh, r_base = it.mg * kAttnRows;
     const int u0 = (int)((long long)rows * k_me / np), u1 = (int)((long long)rows * (k_me + 1) / np);
-    constexpr int CPL = D / 32;  // columns per lane
-    for (int lr = u0 + warp; lr < u1; lr += kConsumerWarps) {
-      // one warp per row: part p's (m, l) sits in lane p % 32 of chunk p / 32
-      float M = -INFINITY;
-      for (int p0 = 0; p0 < np; p0 += 32) {
-        const int p = p0 + lane;
-        if (p < np) {
+    // scratch in the (now idle) Q slot 0: part weights, then per-stripe sums
+    float* wsh = reinterpret_cast<float*>(smem + SM::kQ);             // [np] weights
+    float* lsh = wsh + np;                                              // [np] weighted l
+    float* acc_sh = reinterpret_cast<float*>(smem + SM::kQ + SM::kQSlot);  // [4][D]
+    constexpr int kStripes = 4;                      // parts handled by 4 thread stripes
+    constexpr int kColT = kConsumerWarps * 32 / kStripes;  // threads per stripe (32)
+    constexpr int CPT = D / kColT;                   // columns per thread (4 or 2)
+    const int stripe = tid / kColT, ct = tid % kColT;
+    if (u1 - u0 >= kConsumerWarps) {
+      // many rows: one warp per row, lanes over columns, parts in sequence
+      constexpr int CPL = D / 32;
+      for (int lr = u0 + warp; lr < u1; lr += kConsumerWarps) {
+        float M = -INFINITY;
+        for (int p = lane; p < np; p += 32) {
           const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
           M = fmaxf(M, __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]));
         }
-      }
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-      float Lsum = 0.f;
-      float acc[CPL];
+        for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+        float Lsum = 0.f, acc[CPL];
 #pragma unroll
-      for (int i = 0; i < CPL; ++i) acc[i] = 0.f;
-      for (int p0 = 0; p0 < np; p0 += 32) {
-        float wl = 0.f;
-        {
-          const int p = p0 + lane;
-          if (p < np) {
+        for (int i = 0; i < CPL; ++i) acc[i] = 0.f;
+        for (int p0 = 0; p0 < np; p0 += 32) {
+          float wl = 0.f;
+          if (p0 + lane < np) {
+            const int p = p0 + lane;
             const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
             const float ms = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
             wl = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
             Lsum += wl * __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
           }
-        }
-        const int n = min(32, np - p0);
+          const int n = min(32, np - p0);
 #pragma unroll 8
-        for (int j = 0; j < n; ++j) {
-          const int p = p0 + j;
-          const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-          const float w = __shfl_sync(0xffffffffu, wl, j);
-          const float* src = part_o + (sl * kAttnRows + lr) * D + lane * CPL;
-          if (CPL == 4) {
-            const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
-            acc[0] += w * v.x; acc[1 % CPL] += w * v.y; acc[2 % CPL] += w * v.z; acc[3 % CPL] += w * v.w;
-          } else {
-            const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
-            acc[0] += w * v.x; acc[1 % CPL] += w * v.y;
+          for (int j = 0; j < n; ++j) {
+            const int p = p0 + j;
+            const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+            const float w = __shfl_sync(0xffffffffu, wl, j);
+            const float* src = part_o + (sl * kAttnRows + lr) * D + lane * CPL;
+            if (CPL == 4) {
+              const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
+              acc[0] += w * v.x; acc[1 % CPL] += w * v.y; acc[2 % CPL] += w * v.z; acc[3 % CPL] += w * v.w;
+            } else {
+              const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
+              acc[0] += w * v.x; acc[1 % CPL] += w * v.y;
+            }
           }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
+        const float inv = 1.f / Lsum;
+        const int rr = r_base + lr;
+        const int t = rr / g, hq = kvh * g + rr % g;
+        __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + lane * CPL;
+#pragma unroll
+        for (int i = 0; i < CPL; i += 2)
+          *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
+        if (lse && lane == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
+      }
+    } else
+    for (int lr = u0; lr < u1; ++lr) {
+      // few rows: all consumer threads on one row, parts striped over threads
+      // 1) row max over the parts and the weights 2^(m_p - M)
+      float mloc = -INFINITY;
+      for (int p = tid; p < np; p += kConsumerWarps * 32) {
+        const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+        const float mp = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
+        wsh[p] = mp;
+        lsh[p] = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
+        mloc = fmaxf(mloc, mp);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, off));
+      if (lane == 0) acc_sh[warp] = mloc;
+      consumer_sync();
+      float M = acc_sh[0];
+      for (int w = 1; w < kConsumerWarps; ++w) M = fmaxf(M, acc_sh[w]);
+      consumer_sync();
+      float lpart = 0.f;
+      for (int p = tid; p < np; p += kConsumerWarps * 32) {
+        const float mp = wsh[p];
+        const float w = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
+        wsh[p] = w;
+        lpart += lsh[p] * w;
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) lpart += __shfl_xor_sync(0xffffffffu, lpart, off);
+      if (lane == 0) acc_sh[warp] = lpart;
+      consumer_sync();
+      float Lsum = 0.f;
+      for (int w = 0; w < kConsumerWarps; ++w) Lsum += acc_sh[w];
+      consumer_sync();
+      // 2) weighted sum of the part rows: stripe k takes parts k, k+4, ...
+      float acc[CPT];
+#pragma unroll
+      for (int i = 0; i < CPT; ++i) acc[i] = 0.f;
+#pragma unroll 8
+      for (int p = stripe; p < np; p += kStripes) {
+        const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+        const float w = wsh[p];
+        const float* src = part_o + (sl * kAttnRows + lr) * D + ct * CPT;
+        if (CPT == 4) {
+          const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
+          acc[0] += w * v.x; acc[1 % CPT] += w * v.y; acc[2 % CPT] += w * v.z; acc[3 % CPT] += w * v.w;
+        } else {
+          const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
+          acc[0] += w * v.x; acc[1 % CPT] += w * v.y;
         }
       }
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
-      const float inv = 1.f / Lsum;
-      const int rr = r_base + lr;
-      const int t = rr / g, hq = kvh * g + rr % g;
-      __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + lane * CPL;
+      for (int i = 0; i < CPT; ++i) acc_sh[stripe * D + ct * CPT + i] = acc[i];
+      consumer_sync();
+      if (stripe == 0) {
+        const float inv = 1.f / Lsum;
+        const int rr = r_base + lr;
+        const int t = rr / g, hq = kvh * g + rr % g;
+        __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + ct * CPT;
 #pragma unroll
-      for (int i = 0; i < CPL; i += 2)
-        *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
-      if (lse && lane == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
+        for (int i = 0; i < CPT; i += 2) {
+          float x0 = 0.f, x1 = 0.f;
+#pragma unroll
+          for (int k = 0; k < kStripes; ++k) {
+            x0 += acc_sh[k * D + ct * CPT + i];
+            x1 += acc_sh[k * D + ct * CPT + i + 1];
+          }
+          *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(x0 * inv, x1 * inv);
+        }
+        if (lse && ct == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
+      }
+      consumer_sync();
     }
     // the last CTA done with this group resets its counters for the next launch
     consumer_sync();
