@@ -276,8 +276,7 @@ def run_ours(args, rank, world, local_rank):
         lr.libraspec_select_lengths(conf, cost, ws, L=L)
 
     def seg_attn():
-        for lay in layers:
-            lr.libraspec_verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv_t, L, ws, O=lay["O"])
+        lr.libraspec_verify_attn_layers(layers, kv_t, L, ws)
 
     def seg_accept():
         lr.libraspec_accept(inp["target_logits"], inp["draft_logits"], inp["draft_tokens"], conf, dstat, L,
@@ -367,7 +366,7 @@ def run_ours(args, rank, world, local_rank):
         return
     clk = clocks.summary()
     value = elapsed_max * 1000.0 / (K_steps * world)
-    launches = K_steps * (w.n_layers + 4)
+    launches = K_steps * (w.n_layers + 1 + 4)  # layers + final merge, conf, select, 2 accept
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "us", "n_gpus": world, "steps": K_steps,
         "warmup": max(3, args.warmup), "ms_per_step": round(elapsed_max / K_steps, 6), "higher_is_better": False,

@@ -154,6 +154,25 @@ int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t*
                           void* stream);
 
 /*
+ * Step 3 over n_layers layers that share kv_len and L (the verified block of
+ * every layer of the target), with the same per-layer definition as
+ * libraspec_verify_attn. Q, Kc, Vc, O are HOST arrays of n_layers DEVICE
+ * pointers; lse is a host array of n_layers device pointers (entries may be
+ * NULL) or NULL. Layer l+1 is launched as a programmatic dependent of layer
+ * l: while layer l finishes, layer l+1 already plans its work and prefetches
+ * the tiles that lie wholly in the cache prefix (keys < kv_len[b], written in
+ * earlier rounds); it reads Q, the block's own keys and layer l's split-KV
+ * partials only once layer l is complete, and merges those partials itself.
+ * The caller must therefore not let one layer's Q, O or cache rows at or past
+ * kv_len[b] be produced by an earlier layer of the same call (they are
+ * inputs here), and must not modify the cache prefix during the call.
+ */
+int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
+                                 int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                                 int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,
+                                 void* workspace, size_t ws_bytes, void* stream);
+
+/*
  * Step 4 — acceptance (paper Sec. 3.1; the standard speculative-sampling
  * rule of Leviathan et al. that the paper cites, lossless with respect to
  * the target distribution).

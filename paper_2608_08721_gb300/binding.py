@@ -32,6 +32,7 @@ SIGNATURES = {
     "libraspec_confidence": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "libraspec_select_lengths": (_I, [_P, _P, _I, _I, _P, _P, _SZ, _P]),
     "libraspec_verify_attn": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
+    "libraspec_verify_attn_layers": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_round": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _I,
                                     _F, _U64, _U64, _U32, _P, _P, _P, _P, _P, _P, _SZ, _P]),
@@ -178,6 +179,36 @@ def libraspec_verify_attn(Q, Kc, Vc, kv_len, L, ws: Workspace, softmax_scale=Non
                                       _stream(stream))
     _check(rc, "libraspec_verify_attn")
     return O, lse
+
+
+def libraspec_verify_attn_layers(layers, kv_len, L, ws: Workspace, softmax_scale=None, want_lse=False,
+                                 stream=None):
+    """layers: sequence of dicts with Q, Kc, Vc (and optionally O, lse). Returns (O list, lse list or None)."""
+    n = len(layers)
+    if n == 0:
+        return [], None
+    B, K1, Hq, D = layers[0]["Q"].shape
+    _, Hkv, S_cap, _ = layers[0]["Kc"].shape
+    for i, lay in enumerate(layers):
+        _req(lay["Q"], torch.bfloat16, "Q[%d]" % i, (B, K1, Hq, D))
+        _req(lay["Kc"], torch.bfloat16, "Kc[%d]" % i, (B, Hkv, S_cap, D))
+        _req(lay["Vc"], torch.bfloat16, "Vc[%d]" % i, (B, Hkv, S_cap, D))
+    _req(kv_len, torch.int32, "kv_len", (B,))
+    _req(L, torch.int32, "L", (B,))
+    if softmax_scale is None:
+        softmax_scale = D ** -0.5
+    outs = [lay.get("O") if lay.get("O") is not None else torch.empty_like(lay["Q"]) for lay in layers]
+    lses = None
+    if want_lse:
+        lses = [lay.get("lse") if lay.get("lse") is not None else
+                torch.empty((B, K1, Hq), dtype=torch.float32, device=layers[0]["Q"].device) for lay in layers]
+    rc = load().libraspec_verify_attn_layers(
+        _ptr_array([l["Q"] for l in layers]), _ptr_array([l["Kc"] for l in layers]),
+        _ptr_array([l["Vc"] for l in layers]), n, _ptr(kv_len), _ptr(L), B, K1 - 1, Hq, Hkv, D, S_cap,
+        float(softmax_scale), _ptr_array(outs), _ptr_array(lses) if lses is not None else None, ws.ptr, ws.nbytes,
+        _stream(stream))
+    _check(rc, "libraspec_verify_attn_layers")
+    return outs, lses
 
 
 def libraspec_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, seed: int,

@@ -14,6 +14,9 @@ cudaError_t launch_select(const float*, const float*, int, int, int32_t*, char*,
 cudaError_t launch_verify_attn(const uint16_t*, const uint16_t*, const uint16_t*, const int32_t*, const int32_t*,
                                int, int, int, int, int, int, float, uint16_t*, float*, char*, const WsLayout&,
                                cudaStream_t);
+cudaError_t launch_verify_attn_layers(const uint16_t* const*, const uint16_t* const*, const uint16_t* const*, int,
+                                      const int32_t*, const int32_t*, int, int, int, int, int, int, float,
+                                      uint16_t* const*, float* const*, char*, const WsLayout&, cudaStream_t);
 cudaError_t launch_accept(const float*, const float*, const int32_t*, const float*, const float*, const int32_t*,
                           const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, char*,
                           const WsLayout&, cudaStream_t);
@@ -142,6 +145,28 @@ int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t*
                                       static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
 }
 
+int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
+                                 int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                                 int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,
+                                 void* workspace, size_t ws_bytes, void* stream) {
+  if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
+  if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap) || n_layers < 0) return LIBRASPEC_EINVAL;
+  if (B == 0 || n_layers == 0) return LIBRASPEC_OK;
+  if (!Q || !Kc || !Vc || !O || !kv_len || !L) return LIBRASPEC_EINVAL;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!Q[l] || !Kc[l] || !Vc[l] || !O[l]) return LIBRASPEC_EINVAL;
+    if (!aligned(Q[l], 16) || !aligned(Kc[l], 16) || !aligned(Vc[l], 16) || !aligned(O[l], 16))
+      return LIBRASPEC_EINVAL;
+    if (lse && lse[l] && !aligned(lse[l], 4)) return LIBRASPEC_EINVAL;
+  }
+  if (!(softmax_scale > 0.f)) return LIBRASPEC_EINVAL;
+  const WsLayout lay = ws_layout(B, K, 1, Hq, Hkv, head_dim, S_cap);
+  if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap,
+                                             softmax_scale, O, lse, static_cast<char*>(workspace), lay,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
 int libraspec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
                      const float* conf, const float* dstat, const int32_t* L, const float* temperature, int B, int K,
                      int V, uint64_t seed, uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted,
@@ -191,11 +216,9 @@ int libraspec_verify_round(const float* draft_logits, const int32_t* draft_token
   }
   rc = from_cuda(launch_select(conf, cost_table, B, K, L, ws, lay, s));
   if (rc != LIBRASPEC_OK) return rc;
-  for (int l = 0; l < n_layers; ++l) {
-    rc = from_cuda(launch_verify_attn(Q[l], Kc[l], Vc[l], kv_len, L, B, K, Hq, Hkv, head_dim, S_cap, softmax_scale,
-                                      O[l], lse ? lse[l] : nullptr, ws, lay, s));
-    if (rc != LIBRASPEC_OK) return rc;
-  }
+  rc = from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap,
+                                           softmax_scale, O, lse, ws, lay, s));
+  if (rc != LIBRASPEC_OK) return rc;
   return libraspec_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed,
                           round_offset, seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
 }

@@ -22,13 +22,19 @@
 //
 // A row group covered by one CTA is written directly. A group spread over
 // CTAs c0..c1 leaves one fp32 partial (O, m, l) per CTA, in slot 2c+1 for c0
-// (its last item) and 2c for the others (their first item). Once a CTA has
-// finished its whole range it takes part in the merges of (at most two)
-// groups it contributed to: it waits (bounded) until every part of the group
-// has arrived, then combines its share of the group's rows x columns from all
-// parts in CTA order -- deterministic, and spread over every contributing SM
-// instead of one. The grid is launched cooperatively, so all CTAs are
-// resident and these waits always end.
+// (its last item) and 2c for the others (their first item). Those partials
+// are merged by the NEXT launch of the kernel: every layer has the same plan
+// (same lengths, same grid), so CTA c of layer l+1 merges its share of the
+// rows of the (at most two) split groups it also contributed to in layer l,
+// in CTA order (deterministic), right after griddepcontrol.wait, while its
+// producer already streams layer l+1's tiles. Partial buffers alternate with
+// the layer parity; a merge-only launch finishes the last layer.
+//
+// Layers after the first are launched as programmatic dependents: before
+// griddepcontrol.wait a CTA only plans (from L and kv_len, which no layer
+// writes) and prefetches tiles that lie wholly in the cache prefix
+// (keys < kv_len_b, state from earlier rounds); Q, the block's own keys and
+// the previous layer's partials are read after it.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -44,6 +50,7 @@ constexpr int kAttnThreads = (kConsumerWarps + 1) * 32;
 constexpr int kProducerWarp = kConsumerWarps;
 constexpr int kMaxWaitIters = 1 << 24;
 constexpr int kConsumerBar = 1;  // named barrier of the consumer warps
+constexpr int kStartBar = 2;     // producer + consumers: previous-layer merge done
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -275,13 +282,216 @@ struct AttnSmem {
   static constexpr int kAlloc = kBytes + 1024;      // room to align the base to 1024
 };
 
+
+// ---------------------------------------------------------------------------
+// Merge of the previous layer's split row groups (consumer warps, after
+// griddepcontrol.wait). CTA c merges, for each split group whose tile range
+// it shares (its first and its last item), rows [rows*k/np, rows*(k+1)/np)
+// where k = c - c0: parts c0..c0+np-1 combined in order with weights
+// 2^(m_p - M), M = max_p m_p, O = sum_p w_p O_p / sum_p w_p l_p.
+// ---------------------------------------------------------------------------
+struct MergeTask {
+  int b, kvh, mg, rows, c0, np;
+};
+
+template <int D, int STAGES>
+__device__ void merge_previous_layer(uint8_t* smem, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
+                                     int B, int K, int Hq, int Hkv, int S_cap, int min_tiles,
+                                     const float* __restrict__ part_o, const float* __restrict__ part_ml,
+                                     __nv_bfloat16* __restrict__ O, float* __restrict__ lse, int* __restrict__ status) {
+  using SM = AttnSmem<D, STAGES>;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = Hq / Hkv;
+  MergeTask* tasks = reinterpret_cast<MergeTask*>(smem + SM::kInfo);  // 2 tasks; info is not in use yet
+  volatile int* ntask = reinterpret_cast<volatile int*>(smem + SM::kMisc) + 2;
+  if (warp == 0) {
+    const long long T = total_tiles(B, kv_len, Ls, K, g, Hkv, S_cap, status, false);
+    int G = (int)gridDim.x;
+    if (T > 0) {
+      const long long g_cap = (T + min_tiles - 1) / min_tiles;
+      if ((long long)G > g_cap) G = (int)g_cap;
+    }
+    const int c = blockIdx.x;
+    int n = 0;
+    if (T > 0 && c < G) {
+      const long long lo = range_lo(c, T, G), hi = range_lo(c + 1, T, G);
+      int first_group = -1;
+      for (int e = 0; e < 2; ++e) {
+        const long long pos = e == 0 ? lo : hi - 1;
+        const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, Hkv, S_cap);
+        const int nt = loc.p.n_tiles;
+        const int gib = (int)((pos - loc.seq_start) / nt);
+        const long long gstart = loc.seq_start + (long long)gib * nt, gend = gstart + nt;
+        const int group = loc.group0 + gib;
+        if ((gstart < lo || gend > hi) && group != first_group) {
+          if (lane == 0) {
+            MergeTask t;
+            t.b = loc.b;
+            t.kvh = gib / loc.p.n_mg;
+            t.mg = gib % loc.p.n_mg;
+            t.rows = min(kAttnRows, loc.p.M - t.mg * kAttnRows);
+            t.c0 = cta_of(gstart, T, G);
+            t.np = cta_of(gend - 1, T, G) - t.c0 + 1;
+            tasks[n] = t;
+          }
+          ++n;
+        }
+        if (e == 0) first_group = group;
+      }
+    }
+    if (lane == 0) *ntask = n;
+  }
+  consumer_sync();
+  const int n_tasks = *ntask;
+  for (int ti = 0; ti < n_tasks; ++ti) {
+    const MergeTask it = tasks[ti];
+    const int c0 = it.c0, np = it.np;
+    const int k_me = (int)blockIdx.x - c0;
+    const int rows = it.rows, b = it.b, kvh = it.kvh, r_base = it.mg * kAttnRows;
+    const int u0 = (int)((long long)rows * k_me / np), u1 = (int)((long long)rows * (k_me + 1) / np);
+    // scratch in the (now idle) Q slot 0: part weights, then per-stripe sums
+    float* wsh = reinterpret_cast<float*>(smem + SM::kQ);             // [np] weights
+    float* lsh = wsh + np;                                              // [np] weighted l
+    float* acc_sh = reinterpret_cast<float*>(smem + SM::kQ + SM::kQSlot);  // [4][D]
+    constexpr int kStripes = 4;                      // parts handled by 4 thread stripes
+    constexpr int kColT = kConsumerWarps * 32 / kStripes;  // threads per stripe (32)
+    constexpr int CPT = D / kColT;                   // columns per thread (4 or 2)
+    const int stripe = tid / kColT, ct = tid % kColT;
+    if (u1 - u0 >= kConsumerWarps) {
+      // many rows: one warp per row, lanes over columns, parts in sequence
+      constexpr int CPL = D / 32;
+      for (int lr = u0 + warp; lr < u1; lr += kConsumerWarps) {
+        float M = -INFINITY;
+        for (int p = lane; p < np; p += 32) {
+          const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+          M = fmaxf(M, __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]));
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+        float Lsum = 0.f, acc[CPL];
+#pragma unroll
+        for (int i = 0; i < CPL; ++i) acc[i] = 0.f;
+        for (int p0 = 0; p0 < np; p0 += 32) {
+          float wl = 0.f;
+          if (p0 + lane < np) {
+            const int p = p0 + lane;
+            const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+            const float ms = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
+            wl = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
+            Lsum += wl * __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
+          }
+          const int n = min(32, np - p0);
+#pragma unroll 8
+          for (int j = 0; j < n; ++j) {
+            const int p = p0 + j;
+            const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+            const float w = __shfl_sync(0xffffffffu, wl, j);
+            const float* src = part_o + (sl * kAttnRows + lr) * D + lane * CPL;
+            if (CPL == 4) {
+              const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
+              acc[0] += w * v.x; acc[1 % CPL] += w * v.y; acc[2 % CPL] += w * v.z; acc[3 % CPL] += w * v.w;
+            } else {
+              const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
+              acc[0] += w * v.x; acc[1 % CPL] += w * v.y;
+            }
+          }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
+        const float inv = 1.f / Lsum;
+        const int rr = r_base + lr;
+        const int t = rr / g, hq = kvh * g + rr % g;
+        __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + lane * CPL;
+#pragma unroll
+        for (int i = 0; i < CPL; i += 2)
+          *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
+        if (lse && lane == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
+      }
+    } else
+    for (int lr = u0; lr < u1; ++lr) {
+      // few rows: all consumer threads on one row, parts striped over threads
+      // 1) row max over the parts and the weights 2^(m_p - M)
+      float mloc = -INFINITY;
+      for (int p = tid; p < np; p += kConsumerWarps * 32) {
+        const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+        const float mp = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
+        wsh[p] = mp;
+        lsh[p] = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
+        mloc = fmaxf(mloc, mp);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, off));
+      if (lane == 0) acc_sh[warp] = mloc;
+      consumer_sync();
+      float M = acc_sh[0];
+      for (int w = 1; w < kConsumerWarps; ++w) M = fmaxf(M, acc_sh[w]);
+      consumer_sync();
+      float lpart = 0.f;
+      for (int p = tid; p < np; p += kConsumerWarps * 32) {
+        const float mp = wsh[p];
+        const float w = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
+        wsh[p] = w;
+        lpart += lsh[p] * w;
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) lpart += __shfl_xor_sync(0xffffffffu, lpart, off);
+      if (lane == 0) acc_sh[warp] = lpart;
+      consumer_sync();
+      float Lsum = 0.f;
+      for (int w = 0; w < kConsumerWarps; ++w) Lsum += acc_sh[w];
+      consumer_sync();
+      // 2) weighted sum of the part rows: stripe k takes parts k, k+4, ...
+      float acc[CPT];
+#pragma unroll
+      for (int i = 0; i < CPT; ++i) acc[i] = 0.f;
+#pragma unroll 8
+      for (int p = stripe; p < np; p += kStripes) {
+        const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
+        const float w = wsh[p];
+        const float* src = part_o + (sl * kAttnRows + lr) * D + ct * CPT;
+        if (CPT == 4) {
+          const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
+          acc[0] += w * v.x; acc[1 % CPT] += w * v.y; acc[2 % CPT] += w * v.z; acc[3 % CPT] += w * v.w;
+        } else {
+          const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
+          acc[0] += w * v.x; acc[1 % CPT] += w * v.y;
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < CPT; ++i) acc_sh[stripe * D + ct * CPT + i] = acc[i];
+      consumer_sync();
+      if (stripe == 0) {
+        const float inv = 1.f / Lsum;
+        const int rr = r_base + lr;
+        const int t = rr / g, hq = kvh * g + rr % g;
+        __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + ct * CPT;
+#pragma unroll
+        for (int i = 0; i < CPT; i += 2) {
+          float x0 = 0.f, x1 = 0.f;
+#pragma unroll
+          for (int k = 0; k < kStripes; ++k) {
+            x0 += acc_sh[k * D + ct * CPT + i];
+            x1 += acc_sh[k * D + ct * CPT + i + 1];
+          }
+          *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(x0 * inv, x1 * inv);
+        }
+        if (lse && ct == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
+      }
+      consumer_sync();
+    }
+  }
+  consumer_sync();  // the shared scratch is free again for the items
+}
+
 template <int D, int STAGES>
 __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
     const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
     const __nv_bfloat16* __restrict__ Q, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
     int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, __nv_bfloat16* __restrict__ O,
     float* __restrict__ lse, float* __restrict__ part_o, float* __restrict__ part_ml,
-    uint32_t* __restrict__ group_cnt, int* __restrict__ status) {
+    const float* __restrict__ prev_part_o, const float* __restrict__ prev_part_ml,
+    __nv_bfloat16* __restrict__ prev_O, float* __restrict__ prev_lse, int merge_prev, int own_work,
+    int* __restrict__ status) {
   using SM = AttnSmem<D, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -312,6 +522,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
+  // the next launch of the chain may get resident as SMs free up
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == kProducerWarp) {
     // ======================= producer =======================
@@ -322,9 +534,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
       if ((long long)G > g_cap) G = (int)g_cap;
     }
     const int c = blockIdx.x;
-    long long pos = (T > 0 && c < G) ? range_lo(c, T, G) : 0;
-    const long long hi = (T > 0 && c < G) ? range_lo(c + 1, T, G) : 0;
+    long long pos = (own_work && T > 0 && c < G) ? range_lo(c, T, G) : 0;
+    const long long hi = (own_work && T > 0 && c < G) ? range_lo(c + 1, T, G) : 0;
     uint32_t item_ctr = 0, tile_ctr = 0;
+    bool waited = false;
     while (true) {
       const bool have = pos < hi;
       ItemInfo it{};
@@ -377,6 +590,21 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
         }
         ++tile_ctr;
       };
+      if (!waited) {
+        // before the previous layer is known complete: cache-prefix tiles only
+        if (have && lane == 0) {
+          while (issued < n_tiles && it.key0 + (issued + 1) * kAttnTileKeys <= it.kv &&
+                 mbar_test_wait(bEmpty + 8 * (tile_ctr % STAGES), ((tile_ctr / STAGES) & 1) ^ 1)) {
+            issue_tile(issued);
+            ++issued;
+          }
+        }
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        waited = true;
+        // the consumers merge the previous layer through the Q slots and the
+        // info area first; Q copies and item hand-off start after that
+        if (merge_prev) asm volatile("bar.sync %0, %1;" ::"n"(kStartBar), "n"(kAttnThreads) : "memory");
+      }
       if (have && lane == 0) {
         while (issued < n_tiles && mbar_test_wait(bEmpty + 8 * (tile_ctr % STAGES),
                                                   ((tile_ctr / STAGES) & 1) ^ 1)) {
@@ -428,8 +656,12 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
   // so that small verified blocks still keep every warp busy; their (m, l, O)
   // are combined through shared memory when the item ends.
   uint32_t item_ctr = 0, tile_ctr = 0;
-  ItemInfo pending[2];
-  int n_pending = 0;
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (merge_prev) {
+    merge_previous_layer<D, STAGES>(smem, kv_len, Ls, B, K, Hq, Hkv, S_cap, min_tiles, prev_part_o, prev_part_ml,
+                                    prev_O, prev_lse, status);
+    asm volatile("bar.sync %0, %1;" ::"n"(kStartBar), "n"(kAttnThreads) : "memory");
+  }
   while (true) {
     const uint32_t q = item_ctr & 1;
     if (!mbar_wait(bQFull + 8 * q, (item_ctr >> 1) & 1)) {
@@ -683,178 +915,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
         }
       }
     }
-    if (n_pending < 2) pending[n_pending++] = it;
-  }
-  // Announce this CTA's partials (at most two) once its whole range is done:
-  // one release after all of them instead of a fence per item.
-  consumer_sync();
-  if (tid == 0) {
-    for (int pi = 0; pi < n_pending; ++pi)
-      asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(&group_cnt[2 * pending[pi].group]), "r"(1u)
-                   : "memory");
-  }
-
-  // ---- distributed merges of the groups this CTA contributed to ----
-  for (int pi = 0; pi < n_pending; ++pi) {
-    const ItemInfo& it = pending[pi];
-    const int c0 = it.c0, np = it.nparts;
-    const int k_me = (int)blockIdx.x - c0;  // this CTA's share
-    if (tid == 0) {
-      bool ok = false;
-      for (int i = 0; i < kMaxWaitIters; ++i) {
-        uint32_t v;
-        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(&group_cnt[2 * it.group]) : "memory");
-        if (v >= (uint32_t)np) { ok = true; break; }
-        __nanosleep(32);
-      }
-      if (!ok) raise_status(status, LIBRASPEC_ST_TIMEOUT);
-      misc[0] = ok;
-    }
-    consumer_sync();
-    const bool ok = misc[0] != 0;
-    consumer_sync();
-    if (!ok) return;
-    const int rows = it.rows, b = it.b, kvh = it.kvh, r_base = it.mg * kAttnRows;
-    const int u0 = (int)((long long)rows * k_me / np), u1 = (int)((long long)rows * (k_me + 1) / np);
-    // scratch in the (now idle) Q slot 0: part weights, then per-stripe sums
-    float* wsh = reinterpret_cast<float*>(smem + SM::kQ);             // [np] weights
-    float* lsh = wsh + np;                                              // [np] weighted l
-    float* acc_sh = reinterpret_cast<float*>(smem + SM::kQ + SM::kQSlot);  // [4][D]
-    constexpr int kStripes = 4;                      // parts handled by 4 thread stripes
-    constexpr int kColT = kConsumerWarps * 32 / kStripes;  // threads per stripe (32)
-    constexpr int CPT = D / kColT;                   // columns per thread (4 or 2)
-    const int stripe = tid / kColT, ct = tid % kColT;
-    if (u1 - u0 >= kConsumerWarps) {
-      // many rows: one warp per row, lanes over columns, parts in sequence
-      constexpr int CPL = D / 32;
-      for (int lr = u0 + warp; lr < u1; lr += kConsumerWarps) {
-        float M = -INFINITY;
-        for (int p = lane; p < np; p += 32) {
-          const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-          M = fmaxf(M, __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]));
-        }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-        float Lsum = 0.f, acc[CPL];
-#pragma unroll
-        for (int i = 0; i < CPL; ++i) acc[i] = 0.f;
-        for (int p0 = 0; p0 < np; p0 += 32) {
-          float wl = 0.f;
-          if (p0 + lane < np) {
-            const int p = p0 + lane;
-            const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-            const float ms = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
-            wl = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
-            Lsum += wl * __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
-          }
-          const int n = min(32, np - p0);
-#pragma unroll 8
-          for (int j = 0; j < n; ++j) {
-            const int p = p0 + j;
-            const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-            const float w = __shfl_sync(0xffffffffu, wl, j);
-            const float* src = part_o + (sl * kAttnRows + lr) * D + lane * CPL;
-            if (CPL == 4) {
-              const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
-              acc[0] += w * v.x; acc[1 % CPL] += w * v.y; acc[2 % CPL] += w * v.z; acc[3 % CPL] += w * v.w;
-            } else {
-              const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
-              acc[0] += w * v.x; acc[1 % CPL] += w * v.y;
-            }
-          }
-        }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
-        const float inv = 1.f / Lsum;
-        const int rr = r_base + lr;
-        const int t = rr / g, hq = kvh * g + rr % g;
-        __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + lane * CPL;
-#pragma unroll
-        for (int i = 0; i < CPL; i += 2)
-          *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
-        if (lse && lane == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
-      }
-    } else
-    for (int lr = u0; lr < u1; ++lr) {
-      // few rows: all consumer threads on one row, parts striped over threads
-      // 1) row max over the parts and the weights 2^(m_p - M)
-      float mloc = -INFINITY;
-      for (int p = tid; p < np; p += kConsumerWarps * 32) {
-        const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-        const float mp = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
-        wsh[p] = mp;
-        lsh[p] = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
-        mloc = fmaxf(mloc, mp);
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, off));
-      if (lane == 0) acc_sh[warp] = mloc;
-      consumer_sync();
-      float M = acc_sh[0];
-      for (int w = 1; w < kConsumerWarps; ++w) M = fmaxf(M, acc_sh[w]);
-      consumer_sync();
-      float lpart = 0.f;
-      for (int p = tid; p < np; p += kConsumerWarps * 32) {
-        const float mp = wsh[p];
-        const float w = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
-        wsh[p] = w;
-        lpart += lsh[p] * w;
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) lpart += __shfl_xor_sync(0xffffffffu, lpart, off);
-      if (lane == 0) acc_sh[warp] = lpart;
-      consumer_sync();
-      float Lsum = 0.f;
-      for (int w = 0; w < kConsumerWarps; ++w) Lsum += acc_sh[w];
-      consumer_sync();
-      // 2) weighted sum of the part rows: stripe k takes parts k, k+4, ...
-      float acc[CPT];
-#pragma unroll
-      for (int i = 0; i < CPT; ++i) acc[i] = 0.f;
-#pragma unroll 8
-      for (int p = stripe; p < np; p += kStripes) {
-        const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-        const float w = wsh[p];
-        const float* src = part_o + (sl * kAttnRows + lr) * D + ct * CPT;
-        if (CPT == 4) {
-          const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
-          acc[0] += w * v.x; acc[1 % CPT] += w * v.y; acc[2 % CPT] += w * v.z; acc[3 % CPT] += w * v.w;
-        } else {
-          const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
-          acc[0] += w * v.x; acc[1 % CPT] += w * v.y;
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < CPT; ++i) acc_sh[stripe * D + ct * CPT + i] = acc[i];
-      consumer_sync();
-      if (stripe == 0) {
-        const float inv = 1.f / Lsum;
-        const int rr = r_base + lr;
-        const int t = rr / g, hq = kvh * g + rr % g;
-        __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + ct * CPT;
-#pragma unroll
-        for (int i = 0; i < CPT; i += 2) {
-          float x0 = 0.f, x1 = 0.f;
-#pragma unroll
-          for (int k = 0; k < kStripes; ++k) {
-            x0 += acc_sh[k * D + ct * CPT + i];
-            x1 += acc_sh[k * D + ct * CPT + i + 1];
-          }
-          *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(x0 * inv, x1 * inv);
-        }
-        if (lse && ct == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
-      }
-      consumer_sync();
-    }
-    // the last CTA done with this group resets its counters for the next launch
-    consumer_sync();
-    if (tid == 0) {
-      const uint32_t done = atomicAdd(&group_cnt[2 * it.group + 1], 1u);
-      if (done == (uint32_t)(np - 1)) {
-        group_cnt[2 * it.group] = 0u;
-        group_cnt[2 * it.group + 1] = 0u;
-      }
-    }
   }
 }
 
@@ -889,11 +949,15 @@ static bool make_kv_map(CUtensorMap* map, const void* base, int D, int S_cap, in
   return r == CUDA_SUCCESS;
 }
 
+// One layer of the chain (own_work) and/or the merge of the previous layer's
+// partials (merge_prev). Partial buffers alternate with the layer parity.
+// pdl: launch as a programmatic dependent of the previous kernel in the stream.
 template <int D, int STAGES>
 static cudaError_t launch_attn_t(const CUtensorMap& mK, const CUtensorMap& mV, const uint16_t* Q,
                                  const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv, int S_cap,
-                                 float scale, int min_tiles, uint16_t* O, float* lse, char* ws, const WsLayout& lay,
-                                 cudaStream_t stream) {
+                                 float scale, int min_tiles, uint16_t* O, float* lse, uint16_t* prev_O,
+                                 float* prev_lse, int parity, int merge_prev, int own_work, bool pdl, char* ws,
+                                 const WsLayout& lay, cudaStream_t stream) {
   using SM = AttnSmem<D, STAGES>;
   auto kern = verify_attn_kernel<D, STAGES>;
   static int occ = 0;
@@ -906,21 +970,25 @@ static cudaError_t launch_attn_t(const CUtensorMap& mK, const CUtensorMap& mV, c
   }
   int grid = num_sms_current() * occ;
   if (grid > kAttnMaxCtas) grid = kAttnMaxCtas;
-  // cooperative: every CTA is resident at once, which the merge waits rely on
+  const size_t o_half = (lay.attn_ml - lay.attn_o) / 2, ml_half = (lay.attn_cnt - lay.attn_ml) / 2;
+  float* cur_o = reinterpret_cast<float*>(ws + lay.attn_o + parity * o_half);
+  float* cur_ml = reinterpret_cast<float*>(ws + lay.attn_ml + parity * ml_half);
+  const float* prv_o = reinterpret_cast<const float*>(ws + lay.attn_o + (parity ^ 1) * o_half);
+  const float* prv_ml = reinterpret_cast<const float*>(ws + lay.attn_ml + (parity ^ 1) * ml_half);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kAttnThreads);
   cfg.dynamicSmemBytes = SM::kAlloc;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kern, mK, mV, reinterpret_cast<const __nv_bfloat16*>(Q), kv_len, L, B, K, Hq, Hkv,
-                            S_cap, scale * kLog2e, min_tiles, reinterpret_cast<__nv_bfloat16*>(O), lse,
-                            reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml),
-                            reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
+                            S_cap, scale * kLog2e, min_tiles, reinterpret_cast<__nv_bfloat16*>(O), lse, cur_o, cur_ml,
+                            prv_o, prv_ml, reinterpret_cast<__nv_bfloat16*>(prev_O), prev_lse, merge_prev, own_work,
+                            reinterpret_cast<int*>(ws + lay.status));
 }
 
 // Launch tuning: pipeline depth variant and the smallest tile range per CTA.
@@ -948,26 +1016,55 @@ static const AttnTuning& attn_tuning() {
   return t;
 }
 
-cudaError_t launch_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc, const int32_t* kv_len,
-                               const int32_t* L, int B, int K, int Hq, int Hkv, int D, int S_cap, float scale,
-                               uint16_t* O, float* lse, char* ws, const WsLayout& lay, cudaStream_t stream) {
-  if (B == 0) return cudaSuccess;
+template <int D, int STAGES>
+static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
+                                   int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq,
+                                   int Hkv, int S_cap, float scale, int min_tiles, uint16_t* const* O,
+                                   float* const* lse, char* ws, const WsLayout& lay, cudaStream_t stream) {
   CUtensorMap mK, mV;
-  if (!make_kv_map(&mK, Kc, D, S_cap, B * Hkv) || !make_kv_map(&mV, Vc, D, S_cap, B * Hkv))
-    return cudaErrorInvalidValue;
+  for (int l = 0; l <= n_layers; ++l) {
+    const bool own = l < n_layers;
+    if (own) {
+      if (!make_kv_map(&mK, Kc[l], D, S_cap, B * Hkv) || !make_kv_map(&mV, Vc[l], D, S_cap, B * Hkv))
+        return cudaErrorInvalidValue;
+    }
+    // the final launch only merges the last layer (its maps are never used)
+    cudaError_t e = launch_attn_t<D, STAGES>(
+        mK, mV, own ? Q[l] : Q[l - 1], kv_len, L, B, K, Hq, Hkv, S_cap, scale, min_tiles, own ? O[l] : nullptr,
+        own ? (lse ? lse[l] : nullptr) : nullptr, l > 0 ? O[l - 1] : nullptr,
+        (l > 0 && lse) ? lse[l - 1] : nullptr, l & 1, l > 0 ? 1 : 0, own ? 1 : 0, l > 0, ws, lay, stream);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc,
+                                      const uint16_t* const* Vc, int n_layers, const int32_t* kv_len,
+                                      const int32_t* L, int B, int K, int Hq, int Hkv, int D, int S_cap, float scale,
+                                      uint16_t* const* O, float* const* lse, char* ws, const WsLayout& lay,
+                                      cudaStream_t stream) {
+  if (B == 0 || n_layers == 0) return cudaSuccess;
   const AttnTuning& t = attn_tuning();
   if (D == 128) {
     if (t.deep)
-      return launch_attn_t<128, 4>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
-                                   stream);
-    return launch_attn_t<128, 2>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
-                                 stream);
+      return launch_layers_t<128, 4>(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O,
+                                     lse, ws, lay, stream);
+    return launch_layers_t<128, 2>(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse,
+                                   ws, lay, stream);
   }
   if (t.deep)
-    return launch_attn_t<64, 8>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
-                                stream);
-  return launch_attn_t<64, 4>(mK, mV, Q, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse, ws, lay,
-                              stream);
+    return launch_layers_t<64, 8>(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse,
+                                  ws, lay, stream);
+  return launch_layers_t<64, 4>(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, S_cap, scale, t.min_tiles, O, lse,
+                                ws, lay, stream);
+}
+
+cudaError_t launch_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc, const int32_t* kv_len,
+                               const int32_t* L, int B, int K, int Hq, int Hkv, int D, int S_cap, float scale,
+                               uint16_t* O, float* lse, char* ws, const WsLayout& lay, cudaStream_t stream) {
+  float* lse_arr[1] = {lse};
+  return launch_verify_attn_layers(&Q, &Kc, &Vc, 1, kv_len, L, B, K, Hq, Hkv, D, S_cap, scale, &O,
+                                   lse ? lse_arr : nullptr, ws, lay, stream);
 }
 
 }  // namespace libraspec

@@ -67,10 +67,11 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.row_stat = take(rows_t * sizeof(RowStat));
   w.race_part = take(size_t(B) * kRaceMaxSplits * sizeof(RacePartial));
   w.race_cnt = take(size_t(B) * sizeof(uint32_t));
-  // two partial slots per attention CTA (its first and its last item)
-  w.attn_o = take(size_t(2 * kAttnMaxCtas) * kAttnRows * d * sizeof(float));
-  w.attn_ml = take(size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
-  w.attn_cnt = take(size_t(2 * w.max_groups) * sizeof(uint32_t));  // arrivals, merges done
+  // two partial slots per attention CTA (its first and its last item), in two
+  // buffers that alternate with the layer parity
+  w.attn_o = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * d * sizeof(float));
+  w.attn_ml = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
+  w.attn_cnt = take(256);  // end marker of the partial buffers
   w.total = off;
   return w;
 }

@@ -157,3 +157,29 @@ def test_attn_many_sequences_stream_k_ranges(orc, B, kv_hi, d, seed):
     for _ in range(4):  # repeated: warps of one item race on shared memory if unsynchronised
         O, lse = _run(Q, Kc, Vc, kv.tolist(), L.tolist(), K)
         check_attn(O, lse, O_ref, lse_ref, L, rows=[tuple(r) for r in rows])
+
+
+@pytest.mark.parametrize("name,n_layers", [("8b", 4), ("sampling", 3), ("tiny", 3)])
+def test_attn_layer_chain_matches_per_layer_oracle(orc, name, n_layers):
+    """libraspec_verify_attn_layers: each layer's split groups are merged by the
+    next launch of the chain (and the last by a merge-only launch)."""
+    w = workloads.WORKLOADS[name]
+    kv = workloads.kv_lengths(w)
+    rng = np.random.default_rng(7)
+    L = rng.integers(0, w.K + 1, size=w.B).astype(np.int32)
+    layers = [workloads.layer(w, l, kv, device=cuda()) for l in range(n_layers)]
+    S = layers[0]["Kc"].shape[2]
+    ws = lr.Workspace(w.B, w.K, 1, w.Hq, w.Hkv, w.d, S, device=cuda())
+    outs, lses = lr.libraspec_verify_attn_layers(layers, torch.tensor(kv, device=cuda()),
+                                                 torch.tensor(L, device=cuda()), ws, want_lse=True)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) == 0
+    rows = np.array([(b, h, t) for b in range(w.B) for h in (0, w.Hq - 1) for t in {0, int(L[b])}], np.int32)
+    for l in range(n_layers):
+        O_ref, lse_ref = orc.verify_attn(layers[l]["Q"], layers[l]["Kc"], layers[l]["Vc"], kv, L, rows=rows)
+        check_attn(outs[l], lses[l], O_ref, lse_ref, L, rows=[tuple(r) for r in rows])
+    # the chain equals one layer at a time
+    for l in range(n_layers):
+        O1, lse1 = _run(layers[l]["Q"], layers[l]["Kc"], layers[l]["Vc"], kv.tolist(), L.tolist(), w.K)
+        for b in range(w.B):
+            assert torch.equal(O1[b, : L[b] + 1], outs[l][b, : L[b] + 1])
