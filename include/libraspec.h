@@ -112,6 +112,30 @@ int libraspec_confidence(const float* draft_logits, const int32_t* draft_tokens,
                          void* stream);
 
 /*
+ * libraspec_confidence without a workspace, for callers that cannot allocate
+ * device memory. The paper has no counterpart: this is an integration
+ * variant of Step 1 with the same results (the same kernels run).
+ *
+ * Scratch is one file-scope __device__ array of the library, sized for
+ * B*K <= LIBRASPEC_NOALLOC_MAX_ROWS drafter rows (about 4.2 MB per device);
+ * larger calls return LIBRASPEC_EUNSUPPORTED and launch nothing. The call
+ * allocates nothing. The first call on a device looks the array's address up
+ * (cudaGetSymbolAddress, with that device current, which may load the
+ * module): make it before any stream capture. Each call clears the status
+ * word and its row tickets in the array (cudaMemsetAsync on `stream`).
+ * Calls share the one array per device, so calls whose executions overlap
+ * (other streams, other host threads) race and give undefined results: order
+ * them on one stream or synchronise between them.
+ *
+ * Arguments as for libraspec_confidence. status: device int32 or NULL; when
+ * given it receives, in stream order, this call's LIBRASPEC_ST_* bits
+ * (0 = no violation; e.g. LIBRASPEC_ST_BAD_TOKEN).
+ */
+#define LIBRASPEC_NOALLOC_MAX_ROWS 4096
+int libraspec_confidence_noalloc(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                                 int B, int K, int V, float* conf, float* dstat, int32_t* status, void* stream);
+
+/*
  * Step 2 — LibraSpec length selection (paper Thm. 4, from Thm. 1's
  * ratio comparison; Eq. 2 with negligible drafting cost).
  *

@@ -30,6 +30,7 @@ SIGNATURES = {
     "libraspec_workspace_init": (_I, [_P, _SZ, _P]),
     "libraspec_get_status": (_I, [_P, _P, _P]),
     "libraspec_confidence": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
+    "libraspec_confidence_noalloc": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P]),
     "libraspec_select_lengths": (_I, [_P, _P, _I, _I, _P, _P, _SZ, _P]),
     "libraspec_verify_attn": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_attn_layers": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
@@ -147,6 +148,31 @@ def libraspec_confidence(draft_logits, draft_tokens, temperature, ws: Workspace,
                                      _ptr(conf), _ptr(dstat), ws.ptr, ws.nbytes, _stream(stream))
     _check(rc, "libraspec_confidence")
     return conf, dstat
+
+
+NOALLOC_MAX_ROWS = 4096
+
+
+def libraspec_confidence_noalloc(draft_logits, draft_tokens, temperature, conf, dstat=None, status=None,
+                                 stream=None) -> None:
+    """libraspec_confidence with the library's static scratch instead of a
+    workspace. Allocates nothing: the outputs (conf [B,K], optional dstat
+    [B,K,2], optional status [1] int32) are caller tensors."""
+    B, K, V = draft_logits.shape
+    _req(draft_logits, torch.float32, "draft_logits")
+    _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+    _req(temperature, torch.float32, "temperature", (B,))
+    _req(conf, torch.float32, "conf", (B, K))
+    if dstat is not None:
+        _req(dstat, torch.float32, "dstat", (B, K, 2))
+    if status is not None:
+        _req(status, torch.int32, "status", (1,))
+    if B * K > NOALLOC_MAX_ROWS:
+        raise ValueError("libraspec_confidence_noalloc: B*K = %d drafter rows exceeds the static scratch limit "
+                         "of %d rows; use libraspec_confidence with a workspace" % (B * K, NOALLOC_MAX_ROWS))
+    rc = load().libraspec_confidence_noalloc(_ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature), B, K, V,
+                                             _ptr(conf), _ptr(dstat), _ptr(status), _stream(stream))
+    _check(rc, "libraspec_confidence_noalloc")
 
 
 def libraspec_select_lengths(conf, cost_table, ws: Workspace, L=None, stream=None) -> torch.Tensor:
