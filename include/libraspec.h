@@ -60,7 +60,7 @@ extern "C" {
 #define LIBRASPEC_ST_BAD_COST 0x2    /* cost_table entry not positive and finite */
 #define LIBRASPEC_ST_KV_OVERFLOW 0x4 /* kv_len_b + L_b + 1 > S_cap or kv_len < 0 */
 #define LIBRASPEC_ST_BAD_TOKEN 0x8   /* draft token outside [0, V)               */
-#define LIBRASPEC_ST_TIMEOUT 0x10    /* a bounded wait for an async copy expired */
+#define LIBRASPEC_ST_TIMEOUT 0x10    /* a bounded wait (async copy, grid barrier) expired */
 #define LIBRASPEC_ST_MISSING_INPUT 0x20 /* sampling sequence but conf/dstat NULL  */
 
 /* Limits of this build. */
@@ -170,7 +170,9 @@ int libraspec_select_lengths(const float* conf, const float* cost_table, int B, 
  * (else status LIBRASPEC_ST_KV_OVERFLOW, sequence skipped);
  * L [B] i32 in [0,K]; lse [B,K+1,Hq] f32 out or NULL.
  * head_dim in {64, 128}; Hq % Hkv == 0; (K+1) * Hq / Hkv <= 512.
- * Split-KV over a persistent grid with a deterministic in-kernel merge.
+ * Split-KV over a persistent grid with a deterministic in-kernel merge (one
+ * cooperative launch; the same kernel as libraspec_verify_attn_layers with
+ * one layer).
  */
 int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc, const int32_t* kv_len,
                           const int32_t* L, int B, int K, int Hq, int Hkv, int head_dim, int S_cap,
@@ -182,15 +184,23 @@ int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t*
  * every layer of the target), with the same per-layer definition as
  * libraspec_verify_attn. Q, Kc, Vc, O are HOST arrays of n_layers DEVICE
  * pointers; lse is a host array of n_layers device pointers (entries may be
- * NULL) or NULL. Layer l+1 is launched as a programmatic dependent of layer
- * l: while layer l finishes, layer l+1 already plans its work and prefetches
- * the tiles that lie wholly in the cache prefix (keys < kv_len[b], written in
- * earlier rounds); it reads Q, the block's own keys and layer l's split-KV
- * partials only once layer l is complete, and merges those partials itself.
- * The caller must therefore not let one layer's Q, O or cache rows at or past
+ * NULL) or NULL.
+ *
+ * Up to LIBRASPEC_ATTN_LAYERS_PER_LAUNCH layers run in one persistent,
+ * cooperative kernel launch (more layers take further launches). Layer l+1
+ * starts once every CTA has finished layer l (a grid-wide barrier), as it
+ * would in a model whose layer l+1 input depends on layer l. Before that
+ * barrier the kernel already streams layer l+1's tiles that lie wholly in the
+ * cache prefix (keys < kv_len[b], written in earlier rounds); after it, it
+ * reads Q, the block's own keys, and merges layer l's split-KV partials. The
+ * caller must therefore not let one layer's Q, O or cache rows at or past
  * kv_len[b] be produced by an earlier layer of the same call (they are
  * inputs here), and must not modify the cache prefix during the call.
+ * If a wait inside the kernel gives up (LIBRASPEC_ST_TIMEOUT in the status
+ * word), re-initialise the workspace (libraspec_workspace_init) before its
+ * next use: its barrier counters are then left mid-count.
  */
+#define LIBRASPEC_ATTN_LAYERS_PER_LAUNCH 96
 int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
                                  int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
                                  int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,

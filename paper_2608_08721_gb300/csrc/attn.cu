@@ -1,5 +1,5 @@
 // Step 3: block-causal GQA verify attention on GB300 (split-KV, Stream-K,
-// warp-specialised persistent CTAs).
+// warp-specialised persistent CTAs, all layers of a round in one launch).
 //
 // Work decomposition. For sequence b the verified block has M_b = (L_b+1)*g
 // query rows per kv head (g = Hq/Hkv; row r is block position t = r / g of
@@ -9,32 +9,33 @@
 // sequence (sequence-major, then kv head, row group, key tile); CTA c of the
 // persistent grid takes the contiguous range [c*T/G, (c+1)*T/G) of it, so
 // every CTA streams the same number of tiles whatever the ragged lengths.
-// The plan is derived on the device from L[] and kv_len[] by every CTA.
+// The plan is derived on the device from L[] and kv_len[] by every CTA, and
+// it is the same for every layer (all layers share L and kv_len).
 //
-// Inside a CTA one producer warp walks the CTA's range: for each run of tiles
-// of one row group (an "item") it loads the group's Q rows into a
-// double-buffered shared slot (cp.async) and issues the K/V tiles by TMA
-// (3-D tensor map, 128-byte swizzle) into a ring of STAGES stages, running
-// ahead of the consumers across item boundaries. Four consumer warps compute
-// S = Q K^T and O += P V with mma.sync m16n8k16 (bf16 in, fp32 accumulate),
-// mask keys beyond kv_len_b + t and keep an online softmax in the log2
-// domain. Full/empty mbarriers hand stages between the two roles.
+// Inside a CTA one producer warp walks the CTA's range layer after layer: for
+// each run of tiles of one row group (an "item") it loads the group's Q rows
+// into a double-buffered shared slot (cp.async) and issues the K/V tiles by
+// TMA (3-D tensor map per layer, 128-byte swizzle) into a ring of STAGES
+// stages. Four consumer warps compute S = Q K^T and O += P V with
+// mma.sync m16n8k16 (bf16 in, fp32 accumulate), mask keys beyond
+// kv_len_b + t and keep an online softmax in the log2 domain; with few rows
+// the warps also split each tile's keys. Full/empty mbarriers hand stages
+// between the two roles.
 //
-// A row group covered by one CTA is written directly. A group spread over
-// CTAs c0..c1 leaves one fp32 partial (O, m, l) per CTA, in slot 2c+1 for c0
-// (its last item) and 2c for the others (their first item). Those partials
-// are merged by the NEXT launch of the kernel: every layer has the same plan
-// (same lengths, same grid), so CTA c of layer l+1 merges its share of the
-// rows of the (at most two) split groups it also contributed to in layer l,
-// in CTA order (deterministic), right after griddepcontrol.wait, while its
-// producer already streams layer l+1's tiles. Partial buffers alternate with
-// the layer parity; a merge-only launch finishes the last layer.
+// Layers. Layer l+1 may read Q, the block's own keys (positions >= kv_len_b)
+// and the merged output of layer l only after every CTA has finished layer l:
+// a grid-wide barrier (one counter per layer; the launch is cooperative, so
+// all CTAs are resident and the bounded waits end). The cache prefix
+// (keys < kv_len_b) is state from earlier rounds, so the producer streams the
+// next layer's prefix tiles while the consumers still finish the current
+// layer: HBM stays busy across layer boundaries.
 //
-// Layers after the first are launched as programmatic dependents: before
-// griddepcontrol.wait a CTA only plans (from L and kv_len, which no layer
-// writes) and prefetches tiles that lie wholly in the cache prefix
-// (keys < kv_len_b, state from earlier rounds); Q, the block's own keys and
-// the previous layer's partials are read after it.
+// Split groups. A row group covered by one CTA is written directly. A group
+// spread over CTAs c0..c1 leaves one fp32 partial (O, m, l) per CTA, in slot
+// 2c+1 for c0 (its last item) and 2c for the others (their first item), in a
+// buffer chosen by the layer parity. After the barrier that ends layer l,
+// each of those CTAs merges its share of the group's rows from all parts in
+// CTA order (deterministic, spread over every contributing SM).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -50,7 +51,6 @@ constexpr int kAttnThreads = (kConsumerWarps + 1) * 32;
 constexpr int kProducerWarp = kConsumerWarps;
 constexpr int kMaxWaitIters = 1 << 24;
 constexpr int kConsumerBar = 1;  // named barrier of the consumer warps
-constexpr int kStartBar = 2;     // producer + consumers: previous-layer merge done
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -108,14 +108,12 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
-// 16-byte async copy global -> shared; src_bytes = 0 writes zeros.
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
-}
-
-// Arrive on `bar` once this thread's earlier cp.async copies have landed.
-__device__ __forceinline__ void cp_async_arrive(uint32_t bar) {
-  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+// Bulk async copy global -> shared of `bytes` (multiple of 16; both addresses
+// 16-byte aligned), completing as transaction bytes on `bar`.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
 }
 
 __device__ __forceinline__ void consumer_sync() {
@@ -254,21 +252,56 @@ __device__ __forceinline__ int cta_of(long long t, long long T, int G) {
   return (int)(((t + 1) * (long long)G - 1) / T);
 }
 
+
+// Bounded poll of a grid-barrier counter (acquire).
+__device__ __forceinline__ bool wait_counter(const uint32_t* ctr, uint32_t target) {
+  for (int i = 0; i < kMaxWaitIters; ++i) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+    if (v >= target) return true;
+    __nanosleep(32);
+  }
+  return false;
+}
+
 // One item handed from the producer to the consumers.
 struct ItemInfo {
-  int valid;          // 0: end of the CTA's range
+  int layer;
   int b, kvh, mg, rows, kv;
   int key0, key1;     // keys [key0, key1)
   int partial;        // 1: write a partial, else write O
   int slot;           // partial slot
-  int group, c0, nparts;
+  int pad[3];
+};
+
+// A split row group this CTA helps merge (the same for every layer).
+struct MergeTask {
+  int b, kvh, mg, rows, c0, np;
+};
+
+constexpr int kMaxLayers = kAttnMaxLayers;
+constexpr int kMaxParts = kAttnMaxCtas;  // parts of one split group <= grid size
+
+struct LayerPtrs {
+  const __nv_bfloat16* Q;
+  __nv_bfloat16* O;
+  float* lse;
+};
+
+// Everything a launch needs per layer, passed by value as one kernel
+// parameter (< 32 KB).
+struct LayerSet {
+  CUtensorMap K[kMaxLayers];
+  CUtensorMap V[kMaxLayers];
+  LayerPtrs p[kMaxLayers];
+  int n;
 };
 
 template <int D, int STAGES>
 struct AttnSmem {
   static constexpr int kBoxes = D / 64;
   static constexpr int kTileBytes = kBoxes * 8192;  // one 64 x D bf16 tile
-  // 2 Q slots; each also serves as the key-split merge scratch of its item
+  // 2 Q slots; each also serves as the key-split combine scratch of its item
   // (two 16-row fp32 partials with their (m, l)), so it is rounded up to 1 KB
   static constexpr int kQSlot = ((kTileBytes > 2 * (16 * D + 32) * 4 ? kTileBytes : 2 * (16 * D + 32) * 4) +
                                  1023) / 1024 * 1024;
@@ -277,82 +310,35 @@ struct AttnSmem {
   static constexpr int kV = kK + STAGES * kTileBytes;
   static constexpr int kBar = kV + STAGES * kTileBytes;  // full[S], empty[S], qfull[2], qempty[2]
   static constexpr int kInfo = kBar + 8 * (2 * STAGES + 4);
-  static constexpr int kMisc = kInfo + 2 * 64;
+  static constexpr int kTasks = kInfo + 2 * 64;
+  static constexpr int kMergeW = kTasks + 64;            // [kMaxParts] weights, [kMaxParts] weighted l
+  static constexpr int kMergeAcc = kMergeW + 2 * kMaxParts * 4;  // [4][D]
+  static constexpr int kMisc = kMergeAcc + 4 * D * 4;
   static constexpr int kBytes = kMisc + 16;
-  static constexpr int kAlloc = kBytes + 1024;      // room to align the base to 1024
+  static constexpr int kAlloc = kBytes + 1024;           // room to align the base to 1024
 };
 
-
-// ---------------------------------------------------------------------------
-// Merge of the previous layer's split row groups (consumer warps, after
-// griddepcontrol.wait). CTA c merges, for each split group whose tile range
-// it shares (its first and its last item), rows [rows*k/np, rows*(k+1)/np)
-// where k = c - c0: parts c0..c0+np-1 combined in order with weights
-// 2^(m_p - M), M = max_p m_p, O = sum_p w_p O_p / sum_p w_p l_p.
-// ---------------------------------------------------------------------------
-struct MergeTask {
-  int b, kvh, mg, rows, c0, np;
-};
-
+// Merge, for layer l's split groups this CTA contributed to, its share of
+// rows [rows*k/np, rows*(k+1)/np) (k = this CTA's index among the group's
+// CTAs): O = sum_p w_p O_p / sum_p w_p l_p, w_p = 2^(m_p - M), M = max m_p,
+// parts in CTA order. Consumer warps only.
 template <int D, int STAGES>
-__device__ void merge_previous_layer(uint8_t* smem, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
-                                     int B, int K, int Hq, int Hkv, int S_cap, int min_tiles,
-                                     const float* __restrict__ part_o, const float* __restrict__ part_ml,
-                                     __nv_bfloat16* __restrict__ O, float* __restrict__ lse, int* __restrict__ status) {
+__device__ void merge_layer(uint8_t* smem, const MergeTask* tasks, int n_tasks, int K, int Hq, int Hkv,
+                            const float* __restrict__ part_o, const float* __restrict__ part_ml,
+                            __nv_bfloat16* __restrict__ O, float* __restrict__ lse) {
   using SM = AttnSmem<D, STAGES>;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = Hq / Hkv;
-  MergeTask* tasks = reinterpret_cast<MergeTask*>(smem + SM::kInfo);  // 2 tasks; info is not in use yet
-  volatile int* ntask = reinterpret_cast<volatile int*>(smem + SM::kMisc) + 2;
-  if (warp == 0) {
-    const long long T = total_tiles(B, kv_len, Ls, K, g, Hkv, S_cap, status, false);
-    int G = (int)gridDim.x;
-    if (T > 0) {
-      const long long g_cap = (T + min_tiles - 1) / min_tiles;
-      if ((long long)G > g_cap) G = (int)g_cap;
-    }
-    const int c = blockIdx.x;
-    int n = 0;
-    if (T > 0 && c < G) {
-      const long long lo = range_lo(c, T, G), hi = range_lo(c + 1, T, G);
-      int first_group = -1;
-      for (int e = 0; e < 2; ++e) {
-        const long long pos = e == 0 ? lo : hi - 1;
-        const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, Hkv, S_cap);
-        const int nt = loc.p.n_tiles;
-        const int gib = (int)((pos - loc.seq_start) / nt);
-        const long long gstart = loc.seq_start + (long long)gib * nt, gend = gstart + nt;
-        const int group = loc.group0 + gib;
-        if ((gstart < lo || gend > hi) && group != first_group) {
-          if (lane == 0) {
-            MergeTask t;
-            t.b = loc.b;
-            t.kvh = gib / loc.p.n_mg;
-            t.mg = gib % loc.p.n_mg;
-            t.rows = min(kAttnRows, loc.p.M - t.mg * kAttnRows);
-            t.c0 = cta_of(gstart, T, G);
-            t.np = cta_of(gend - 1, T, G) - t.c0 + 1;
-            tasks[n] = t;
-          }
-          ++n;
-        }
-        if (e == 0) first_group = group;
-      }
-    }
-    if (lane == 0) *ntask = n;
-  }
-  consumer_sync();
-  const int n_tasks = *ntask;
   for (int ti = 0; ti < n_tasks; ++ti) {
     const MergeTask it = tasks[ti];
     const int c0 = it.c0, np = it.np;
     const int k_me = (int)blockIdx.x - c0;
     const int rows = it.rows, b = it.b, kvh = it.kvh, r_base = it.mg * kAttnRows;
     const int u0 = (int)((long long)rows * k_me / np), u1 = (int)((long long)rows * (k_me + 1) / np);
-    // scratch in the (now idle) Q slot 0: part weights, then per-stripe sums
-    float* wsh = reinterpret_cast<float*>(smem + SM::kQ);             // [np] weights
+    // merge scratch: part weights, weighted l, per-stripe sums
+    float* wsh = reinterpret_cast<float*>(smem + SM::kMergeW);        // [np] weights
     float* lsh = wsh + np;                                              // [np] weighted l
-    float* acc_sh = reinterpret_cast<float*>(smem + SM::kQ + SM::kQSlot);  // [4][D]
+    float* acc_sh = reinterpret_cast<float*>(smem + SM::kMergeAcc);   // [4][D]
     constexpr int kStripes = 4;                      // parts handled by 4 thread stripes
     constexpr int kColT = kConsumerWarps * 32 / kStripes;  // threads per stripe (32)
     constexpr int CPT = D / kColT;                   // columns per thread (4 or 2)
@@ -480,17 +466,13 @@ __device__ void merge_previous_layer(uint8_t* smem, const int32_t* __restrict__ 
       consumer_sync();
     }
   }
-  consumer_sync();  // the shared scratch is free again for the items
 }
 
 template <int D, int STAGES>
 __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
-    const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-    const __nv_bfloat16* __restrict__ Q, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
-    int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, __nv_bfloat16* __restrict__ O,
-    float* __restrict__ lse, float* __restrict__ part_o, float* __restrict__ part_ml,
-    const float* __restrict__ prev_part_o, const float* __restrict__ prev_part_ml,
-    __nv_bfloat16* __restrict__ prev_O, float* __restrict__ prev_lse, int merge_prev, int own_work,
+    const __grid_constant__ LayerSet set, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
+    int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, float* __restrict__ part_buf_o,
+    float* __restrict__ part_buf_ml, size_t part_o_stride, size_t part_ml_stride, uint32_t* __restrict__ bar_cnt,
     int* __restrict__ status) {
   using SM = AttnSmem<D, STAGES>;
   extern __shared__ uint8_t smem_raw[];
@@ -503,10 +485,14 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
   const uint32_t bQFull = bEmpty + 8 * STAGES;
   const uint32_t bQEmpty = bQFull + 16;
   ItemInfo* info = reinterpret_cast<ItemInfo*>(smem + SM::kInfo);
-  volatile int* misc = reinterpret_cast<int*>(smem + SM::kMisc);  // [0] wait result, [1] abort
+  MergeTask* tasks = reinterpret_cast<MergeTask*>(smem + SM::kTasks);
+  volatile int* misc = reinterpret_cast<int*>(smem + SM::kMisc);  // [0] abort, [1] n_tasks, [2] n_items
+  uint32_t* exit_cnt = bar_cnt + kMaxLayers;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = Hq / Hkv;
+  const int n_layers = set.n;
+  const uint32_t n_ctas = gridDim.x;
 
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -514,43 +500,83 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
       mbar_init(bEmpty + 8 * s, kConsumerWarps);
     }
     for (int q = 0; q < 2; ++q) {
-      mbar_init(bQFull + 8 * q, 33);  // 32 cp.async arrivals + the info arrival
+      mbar_init(bQFull + 8 * q, 1);  // the producer's arrive; the Q bytes complete as transactions
       mbar_init(bQEmpty + 8 * q, kConsumerWarps);
     }
     misc[0] = 0;
-    misc[1] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  __syncthreads();
-  // the next launch of the chain may get resident as SMs free up
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-
-  if (warp == kProducerWarp) {
-    // ======================= producer =======================
+  // The plan (identical for every layer): this CTA's tile range, its item
+  // count and the split groups it helps merge.
+  if (warp == 0) {
     const long long T = total_tiles(B, kv_len, Ls, K, g, Hkv, S_cap, status, blockIdx.x == 0);
-    int G = (int)gridDim.x;
+    int G = (int)n_ctas;
     if (T > 0) {
       const long long g_cap = (T + min_tiles - 1) / min_tiles;
       if ((long long)G > g_cap) G = (int)g_cap;
     }
     const int c = blockIdx.x;
-    long long pos = (own_work && T > 0 && c < G) ? range_lo(c, T, G) : 0;
-    const long long hi = (own_work && T > 0 && c < G) ? range_lo(c + 1, T, G) : 0;
-    uint32_t item_ctr = 0, tile_ctr = 0;
-    bool waited = false;
-    while (true) {
-      const bool have = pos < hi;
-      ItemInfo it{};
-      int n_tiles = 0, zc = 0;
-      if (have) {
+    int n_items = 0, n_tasks = 0;
+    if (T > 0 && c < G) {
+      const long long lo = range_lo(c, T, G), hi = range_lo(c + 1, T, G);
+      int group_lo = 0;
+      for (int e = 0; e < 2; ++e) {
+        const long long pos = e == 0 ? lo : hi - 1;
         const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, Hkv, S_cap);
         const int nt = loc.p.n_tiles;
-        const long long off = pos - loc.seq_start;
-        const int gib = (int)(off / nt);             // row group within the sequence
+        const int gib = (int)((pos - loc.seq_start) / nt);
+        const long long gstart = loc.seq_start + (long long)gib * nt, gend = gstart + nt;
+        const int group = loc.group0 + gib;
+        if (e == 0) group_lo = group;
+        else n_items = group - group_lo + 1;
+        if ((gstart < lo || gend > hi) && !(e == 1 && group == group_lo)) {
+          if (lane == 0) {
+            MergeTask t;
+            t.b = loc.b;
+            t.kvh = gib / loc.p.n_mg;
+            t.mg = gib % loc.p.n_mg;
+            t.rows = min(kAttnRows, loc.p.M - t.mg * kAttnRows);
+            t.c0 = cta_of(gstart, T, G);
+            t.np = cta_of(gend - 1, T, G) - t.c0 + 1;
+            tasks[n_tasks] = t;
+          }
+          ++n_tasks;
+        }
+      }
+    }
+    if (lane == 0) {
+      misc[1] = n_tasks;
+      misc[2] = n_items;
+    }
+  }
+  __syncthreads();
+  const int n_tasks = misc[1], n_items = misc[2];
+
+  if (warp == kProducerWarp) {
+    // ======================= producer =======================
+    const long long T = total_tiles(B, kv_len, Ls, K, g, Hkv, S_cap, status, false);
+    int G = (int)n_ctas;
+    if (T > 0) {
+      const long long g_cap = (T + min_tiles - 1) / min_tiles;
+      if ((long long)G > g_cap) G = (int)g_cap;
+    }
+    const int c = blockIdx.x;
+    const long long lo = (T > 0 && c < G) ? range_lo(c, T, G) : 0;
+    const long long hi = (T > 0 && c < G) ? range_lo(c + 1, T, G) : 0;
+    uint32_t item_ctr = 0, tile_ctr = 0;
+    for (int layer = 0; layer < n_layers; ++layer) {
+      // layer's dependent data (Q, the block's keys) is readable once every
+      // CTA has finished the previous layer
+      bool ready = layer == 0;
+      for (long long pos = lo; pos < hi;) {
+        ItemInfo it{};
+        const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, Hkv, S_cap);
+        const int nt = loc.p.n_tiles;
+        const int gib = (int)((pos - loc.seq_start) / nt);
         const long long gstart = loc.seq_start + (long long)gib * nt;
         const long long gend = gstart + nt;
         const long long iend = gend < hi ? gend : hi;
-        it.valid = 1;
+        it.layer = layer;
         it.b = loc.b;
         it.kvh = gib / loc.p.n_mg;
         it.mg = gib % loc.p.n_mg;
@@ -558,93 +584,86 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
         it.kv = kv_len[loc.b];
         it.key0 = (int)(pos - gstart) * kAttnTileKeys;
         it.key1 = min(loc.p.N, (int)(iend - gstart) * kAttnTileKeys);
-        it.group = loc.group0 + gib;
-        const bool whole = (pos == gstart) && (gend <= hi);
-        it.partial = whole ? 0 : 1;
-        it.c0 = cta_of(gstart, T, G);
-        it.nparts = cta_of(gend - 1, T, G) - it.c0 + 1;
+        it.partial = ((pos == gstart) && (gend <= hi)) ? 0 : 1;
         it.slot = (pos == gstart) ? 2 * c + 1 : 2 * c;
-        n_tiles = (int)(iend - pos);
-        zc = loc.b * Hkv + it.kvh;
+        const int n_tiles = (int)(iend - pos);
+        const int zc = loc.b * Hkv + it.kvh;
         pos = iend;
-      }
-      const uint32_t q = item_ctr & 1;
-      const uint32_t qpar = ((item_ctr >> 1) & 1) ^ 1;
-      if (!mbar_wait(bQEmpty + 8 * q, qpar)) {
-        if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
-        misc[1] = 1;
-        return;
-      }
-      // Tiles whose stage is already free go out before the Q copies: on a
-      // CTA's first item the K/V latency is the long pole.
-      int issued = 0;
-      auto issue_tile = [&](int i) {
-        const uint32_t s = tile_ctr % STAGES;
-        const uint32_t bar = bFull + 8 * s;
-        mbar_expect_tx(bar, 2 * SM::kTileBytes);
-        const int y = it.key0 + i * kAttnTileKeys;
-#pragma unroll
-        for (int bx = 0; bx < SM::kBoxes; ++bx) {
-          tma_load_3d(sK + s * SM::kTileBytes + bx * 8192, &tmK, bar, bx * 64, y, zc);
-          tma_load_3d(sV + s * SM::kTileBytes + bx * 8192, &tmV, bar, bx * 64, y, zc);
+        const uint32_t q = item_ctr & 1;
+        if (!mbar_wait(bQEmpty + 8 * q, ((item_ctr >> 1) & 1) ^ 1)) {
+          if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
+          misc[0] = 1;
+          return;
         }
-        ++tile_ctr;
-      };
-      if (!waited) {
-        // before the previous layer is known complete: cache-prefix tiles only
-        if (have && lane == 0) {
-          while (issued < n_tiles && it.key0 + (issued + 1) * kAttnTileKeys <= it.kv &&
+        int issued = 0;
+        auto issue_tile = [&](int i) {
+          const uint32_t s = tile_ctr % STAGES;
+          const uint32_t bar = bFull + 8 * s;
+          mbar_expect_tx(bar, 2 * SM::kTileBytes);
+          const int y = it.key0 + i * kAttnTileKeys;
+#pragma unroll
+          for (int bx = 0; bx < SM::kBoxes; ++bx) {
+            tma_load_3d(sK + s * SM::kTileBytes + bx * 8192, &set.K[layer], bar, bx * 64, y, zc);
+            tma_load_3d(sV + s * SM::kTileBytes + bx * 8192, &set.V[layer], bar, bx * 64, y, zc);
+          }
+          ++tile_ctr;
+        };
+        if (lane == 0) {
+          // tiles whose stage is free go out first; before the barrier only
+          // tiles that lie wholly in the cache prefix
+          while (issued < n_tiles && (ready || it.key0 + (issued + 1) * kAttnTileKeys <= it.kv) &&
                  mbar_test_wait(bEmpty + 8 * (tile_ctr % STAGES), ((tile_ctr / STAGES) & 1) ^ 1)) {
             issue_tile(issued);
             ++issued;
           }
-        }
-        asm volatile("griddepcontrol.wait;" ::: "memory");
-        waited = true;
-        // the consumers merge the previous layer through the Q slots and the
-        // info area first; Q copies and item hand-off start after that
-        if (merge_prev) asm volatile("bar.sync %0, %1;" ::"n"(kStartBar), "n"(kAttnThreads) : "memory");
-      }
-      if (have && lane == 0) {
-        while (issued < n_tiles && mbar_test_wait(bEmpty + 8 * (tile_ctr % STAGES),
-                                                  ((tile_ctr / STAGES) & 1) ^ 1)) {
-          issue_tile(issued);
-          ++issued;
-        }
-      }
-      if (have) {
-        // Q rows of the item's row group (rows past `rows` are never used)
-        const uint32_t qdst = sQ + q * SM::kQSlot;
-        constexpr int kChunks = D / 8;
-        for (int idx = lane; idx < it.rows * kChunks; idx += 32) {
-          const int r = idx / kChunks, ch = idx - r * kChunks;
-          const int rr = it.mg * kAttnRows + r;
-          const int t = rr / g, h = it.kvh * g + (rr - t * g);
-          const __nv_bfloat16* src = Q + (((size_t)it.b * (K + 1) + t) * Hq + h) * D + ch * 8;
-          cp_async16(qdst + sw128(r, ch * 8), src, 16u);
-        }
-      }
-      if (lane == 0) {
-        info[q] = it;
-        mbar_arrive(bQFull + 8 * q);
-      }
-      cp_async_arrive(bQFull + 8 * q);
-      ++item_ctr;
-      if (!have) break;
-      if (lane == 0) {
-        for (int i = issued; i < n_tiles; ++i) {
-          const uint32_t par = ((tile_ctr / STAGES) & 1) ^ 1;
-          if (!mbar_wait(bEmpty + 8 * (tile_ctr % STAGES), par)) {
-            raise_status(status, LIBRASPEC_ST_TIMEOUT);
-            misc[1] = 1;
-            break;
+          if (!ready) {
+            if (!wait_counter(bar_cnt + (layer - 1), n_ctas)) {
+              raise_status(status, LIBRASPEC_ST_TIMEOUT);
+              misc[0] = 1;
+            }
           }
-          issue_tile(i);
         }
+        __syncwarp();
+        if (misc[0]) return;
+        ready = true;
+        // Q rows of the item's row group (rows past `rows` are never used), one
+        // bulk copy per row and 64-column half, unswizzled: row r of half hb at
+        // hb * 8192 + r * 128. Bulk copies, like the K/V tiles, complete as
+        // transaction bytes on an mbarrier; non-bulk cp.async copies in flight
+        // in the warp that issues TMA loads were seen on GB300 to lose their
+        // mbarrier arrival, so the producer issues none.
+        if (lane == 0) {
+          info[q] = it;
+          mbar_expect_tx(bQFull + 8 * q, (uint32_t)it.rows * D * 2);
+        }
+        __syncwarp();
+        {
+          const uint32_t qdst = sQ + q * SM::kQSlot;
+          const __nv_bfloat16* Qb = set.p[layer].Q;
+          for (int idx = lane; idx < it.rows * SM::kBoxes; idx += 32) {
+            const int r = idx / SM::kBoxes, hb = idx - r * SM::kBoxes;
+            const int rr = it.mg * kAttnRows + r;
+            const int t = rr / g, h = it.kvh * g + (rr - t * g);
+            const __nv_bfloat16* src = Qb + (((size_t)it.b * (K + 1) + t) * Hq + h) * D + hb * 64;
+            bulk_load(qdst + hb * 8192 + r * 128, src, 128u, bQFull + 8 * q);
+          }
+        }
+        ++item_ctr;
+        if (lane == 0) {
+          for (int i = issued; i < n_tiles; ++i) {
+            const uint32_t par = ((tile_ctr / STAGES) & 1) ^ 1;
+            if (!mbar_wait(bEmpty + 8 * (tile_ctr % STAGES), par)) {
+              raise_status(status, LIBRASPEC_ST_TIMEOUT);
+              misc[0] = 1;
+              break;
+            }
+            issue_tile(i);
+          }
+        }
+        tile_ctr = __shfl_sync(0xffffffffu, tile_ctr, 0);
+        __syncwarp();
+        if (misc[0]) return;
       }
-      tile_ctr = __shfl_sync(0xffffffffu, tile_ctr, 0);
-      __syncwarp();
-      if (misc[1]) return;
     }
     return;
   }
@@ -656,20 +675,30 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
   // so that small verified blocks still keep every warp busy; their (m, l, O)
   // are combined through shared memory when the item ends.
   uint32_t item_ctr = 0, tile_ctr = 0;
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  if (merge_prev) {
-    merge_previous_layer<D, STAGES>(smem, kv_len, Ls, B, K, Hq, Hkv, S_cap, min_tiles, prev_part_o, prev_part_ml,
-                                    prev_O, prev_lse, status);
-    asm volatile("bar.sync %0, %1;" ::"n"(kStartBar), "n"(kAttnThreads) : "memory");
-  }
-  while (true) {
+  for (int layer = 0; layer < n_layers; ++layer) {
+    float* part_o = part_buf_o + (layer & 1) * part_o_stride;
+    float* part_ml = part_buf_ml + (layer & 1) * part_ml_stride;
+    if (layer > 0) {
+      // every CTA is done with the previous layer: merge its split groups
+      if (tid == 0 && !wait_counter(bar_cnt + (layer - 1), n_ctas)) {
+        raise_status(status, LIBRASPEC_ST_TIMEOUT);
+        misc[0] = 1;
+      }
+      consumer_sync();
+      if (misc[0]) return;
+      merge_layer<D, STAGES>(smem, tasks, n_tasks, K, Hq, Hkv, part_buf_o + ((layer - 1) & 1) * part_o_stride,
+                             part_buf_ml + ((layer - 1) & 1) * part_ml_stride, set.p[layer - 1].O,
+                             set.p[layer - 1].lse);
+    }
+    __nv_bfloat16* O = set.p[layer].O;
+    float* lse = set.p[layer].lse;
+    for (int item = 0; item < n_items; ++item) {
     const uint32_t q = item_ctr & 1;
     if (!mbar_wait(bQFull + 8 * q, (item_ctr >> 1) & 1)) {
       if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
       return;
     }
     const ItemInfo it = info[q];
-    if (!it.valid) break;
     const int rows = it.rows, kv = it.kv, b = it.b, kvh = it.kvh;
     const int r_base = it.mg * kAttnRows;
     const int n_rt = (rows + 15) >> 4;
@@ -686,7 +715,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
         const int mi = lane >> 3, rr = lane & 7;
         const int row = rt * 16 + (mi & 1) * 8 + rr;
         const int col = kk * 16 + (mi >> 1) * 8;
-        ldsm_x4(qslot + sw128(row, col), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
+        ldsm_x4(qslot + (col >> 6) * 8192 + row * 128 + (col & 63) * 2, qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
       }
     }
     ++item_ctr;
@@ -915,6 +944,31 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
         }
       }
     }
+    }
+    // this CTA is done with the layer
+    consumer_sync();
+    if (tid == 0) asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(bar_cnt + layer), "r"(1u) : "memory");
+  }
+  // merge the last layer, then the last CTA out resets the counters
+  if (n_layers > 0) {
+    if (tid == 0 && !wait_counter(bar_cnt + (n_layers - 1), n_ctas)) {
+      raise_status(status, LIBRASPEC_ST_TIMEOUT);
+      misc[0] = 1;
+    }
+    consumer_sync();
+    if (misc[0]) return;
+    merge_layer<D, STAGES>(smem, tasks, n_tasks, K, Hq, Hkv, part_buf_o + ((n_layers - 1) & 1) * part_o_stride,
+                           part_buf_ml + ((n_layers - 1) & 1) * part_ml_stride, set.p[n_layers - 1].O,
+                           set.p[n_layers - 1].lse);
+  }
+  consumer_sync();
+  if (tid == 0) {
+    const uint32_t done = atomicAdd(exit_cnt, 1u);
+    if (done == n_ctas - 1) {
+      for (int l = 0; l < n_layers; ++l) bar_cnt[l] = 0u;
+      *exit_cnt = 0u;
+      __threadfence();
+    }
   }
 }
 
@@ -949,48 +1003,6 @@ static bool make_kv_map(CUtensorMap* map, const void* base, int D, int S_cap, in
   return r == CUDA_SUCCESS;
 }
 
-// One layer of the chain (own_work) and/or the merge of the previous layer's
-// partials (merge_prev). Partial buffers alternate with the layer parity.
-// pdl: launch as a programmatic dependent of the previous kernel in the stream.
-template <int D, int STAGES>
-static cudaError_t launch_attn_t(const CUtensorMap& mK, const CUtensorMap& mV, const uint16_t* Q,
-                                 const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv, int S_cap,
-                                 float scale, int min_tiles, uint16_t* O, float* lse, uint16_t* prev_O,
-                                 float* prev_lse, int parity, int merge_prev, int own_work, bool pdl, char* ws,
-                                 const WsLayout& lay, cudaStream_t stream) {
-  using SM = AttnSmem<D, STAGES>;
-  auto kern = verify_attn_kernel<D, STAGES>;
-  static int occ = 0;
-  if (occ == 0) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kAlloc);
-    if (e != cudaSuccess) return e;
-    int o = 1;
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, kAttnThreads, SM::kAlloc);
-    occ = o < 1 ? 1 : o;
-  }
-  int grid = num_sms_current() * occ;
-  if (grid > kAttnMaxCtas) grid = kAttnMaxCtas;
-  const size_t o_half = (lay.attn_ml - lay.attn_o) / 2, ml_half = (lay.attn_cnt - lay.attn_ml) / 2;
-  float* cur_o = reinterpret_cast<float*>(ws + lay.attn_o + parity * o_half);
-  float* cur_ml = reinterpret_cast<float*>(ws + lay.attn_ml + parity * ml_half);
-  const float* prv_o = reinterpret_cast<const float*>(ws + lay.attn_o + (parity ^ 1) * o_half);
-  const float* prv_ml = reinterpret_cast<const float*>(ws + lay.attn_ml + (parity ^ 1) * ml_half);
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kAttnThreads);
-  cfg.dynamicSmemBytes = SM::kAlloc;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kern, mK, mV, reinterpret_cast<const __nv_bfloat16*>(Q), kv_len, L, B, K, Hq, Hkv,
-                            S_cap, scale * kLog2e, min_tiles, reinterpret_cast<__nv_bfloat16*>(O), lse, cur_o, cur_ml,
-                            prv_o, prv_ml, reinterpret_cast<__nv_bfloat16*>(prev_O), prev_lse, merge_prev, own_work,
-                            reinterpret_cast<int*>(ws + lay.status));
-}
-
 // Launch tuning: pipeline depth variant and the smallest tile range per CTA.
 // Defaults were chosen by measurement on GB300; the LIBRASPEC_ATTN_TUNING
 // environment variable ("deep:min_tiles", deep = 0 for the two-CTAs-per-SM
@@ -1021,18 +1033,47 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
                                    int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq,
                                    int Hkv, int S_cap, float scale, int min_tiles, uint16_t* const* O,
                                    float* const* lse, char* ws, const WsLayout& lay, cudaStream_t stream) {
-  CUtensorMap mK, mV;
-  for (int l = 0; l <= n_layers; ++l) {
-    const bool own = l < n_layers;
-    if (own) {
-      if (!make_kv_map(&mK, Kc[l], D, S_cap, B * Hkv) || !make_kv_map(&mV, Vc[l], D, S_cap, B * Hkv))
+  using SM = AttnSmem<D, STAGES>;
+  auto kern = verify_attn_kernel<D, STAGES>;
+  static int occ = 0;
+  if (occ == 0) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kAlloc);
+    if (e != cudaSuccess) return e;
+    int o = 1;
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, kAttnThreads, SM::kAlloc);
+    occ = o < 1 ? 1 : o;
+  }
+  int grid = num_sms_current() * occ;
+  if (grid > kAttnMaxCtas) grid = kAttnMaxCtas;
+  // layers beyond kMaxLayers go in further launches of the same kernel
+  for (int l0 = 0; l0 < n_layers; l0 += kMaxLayers) {
+    LayerSet set;  // ~27 KB: built on the host, copied into the launch parameters
+    const int n = n_layers - l0 < kMaxLayers ? n_layers - l0 : kMaxLayers;
+    set.n = n;
+    for (int i = 0; i < n; ++i) {
+      const int l = l0 + i;
+      if (!make_kv_map(&set.K[i], Kc[l], D, S_cap, B * Hkv) || !make_kv_map(&set.V[i], Vc[l], D, S_cap, B * Hkv))
         return cudaErrorInvalidValue;
+      set.p[i].Q = reinterpret_cast<const __nv_bfloat16*>(Q[l]);
+      set.p[i].O = reinterpret_cast<__nv_bfloat16*>(O[l]);
+      set.p[i].lse = lse ? lse[l] : nullptr;
     }
-    // the final launch only merges the last layer (its maps are never used)
-    cudaError_t e = launch_attn_t<D, STAGES>(
-        mK, mV, own ? Q[l] : Q[l - 1], kv_len, L, B, K, Hq, Hkv, S_cap, scale, min_tiles, own ? O[l] : nullptr,
-        own ? (lse ? lse[l] : nullptr) : nullptr, l > 0 ? O[l - 1] : nullptr,
-        (l > 0 && lse) ? lse[l - 1] : nullptr, l & 1, l > 0 ? 1 : 0, own ? 1 : 0, l > 0, ws, lay, stream);
+    const size_t o_half = (lay.attn_ml - lay.attn_o) / 2, ml_half = (lay.attn_cnt - lay.attn_ml) / 2;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kAttnThreads);
+    cfg.dynamicSmemBytes = SM::kAlloc;
+    cfg.stream = stream;
+    // cooperative: every CTA is resident at once, which the layer barriers rely on
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(
+        &cfg, kern, set, kv_len, L, B, K, Hq, Hkv, S_cap, scale * kLog2e, min_tiles,
+        reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_half / sizeof(float),
+        ml_half / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

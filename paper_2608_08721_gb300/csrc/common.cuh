@@ -19,9 +19,10 @@ constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kConfMaxSplits = 64;    // CTAs per drafter row
 constexpr int kRowMaxSplits = 64;     // CTAs per target row (acceptance)
 constexpr int kRaceMaxSplits = 128;   // CTAs per sequence for a vocabulary draw
-constexpr int kAttnMaxCtas = 1024;    // persistent attention grid cap
+constexpr int kAttnMaxCtas = 512;     // persistent attention grid cap (>= SMs x CTAs per SM)
 constexpr int kAttnRows = 64;         // query rows per attention work item
 constexpr int kAttnTileKeys = 64;     // keys per KV tile
+constexpr int kAttnMaxLayers = LIBRASPEC_ATTN_LAYERS_PER_LAUNCH;  // layers per attention launch
 
 struct RowPartial {      // one CTA's share of a logit row
   float m;               // max
@@ -71,7 +72,8 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   // buffers that alternate with the layer parity
   w.attn_o = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * d * sizeof(float));
   w.attn_ml = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
-  w.attn_cnt = take(256);  // end marker of the partial buffers
+  // grid-barrier counters, one per layer of a launch, then the exit counter
+  w.attn_cnt = take((kAttnMaxLayers + 1) * sizeof(uint32_t));
   w.total = off;
   return w;
 }

@@ -161,8 +161,8 @@ def test_attn_many_sequences_stream_k_ranges(orc, B, kv_hi, d, seed):
 
 @pytest.mark.parametrize("name,n_layers", [("8b", 4), ("sampling", 3), ("tiny", 3)])
 def test_attn_layer_chain_matches_per_layer_oracle(orc, name, n_layers):
-    """libraspec_verify_attn_layers: each layer's split groups are merged by the
-    next launch of the chain (and the last by a merge-only launch)."""
+    """libraspec_verify_attn_layers: all layers in one persistent launch; each
+    layer's split groups are merged after the grid barrier that ends it."""
     w = workloads.WORKLOADS[name]
     kv = workloads.kv_lengths(w)
     rng = np.random.default_rng(7)
