@@ -29,7 +29,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "verify-round µs (select+attn+accept) and HBM TB/s vs ~8 TB/s, batch 1–64"
 NOMINAL_HBM_GBS = 8000.0
-ATTN_LAYERS_PER_LAUNCH = 96  # LIBRASPEC_ATTN_LAYERS_PER_LAUNCH
+ATTN_LAYERS_PER_LAUNCH = 64  # LIBRASPEC_ATTN_LAYERS_PER_LAUNCH
 L2_BYTES = 129e6
 
 

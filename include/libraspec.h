@@ -200,7 +200,7 @@ int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t*
  * word), re-initialise the workspace (libraspec_workspace_init) before its
  * next use: its barrier counters are then left mid-count.
  */
-#define LIBRASPEC_ATTN_LAYERS_PER_LAUNCH 96
+#define LIBRASPEC_ATTN_LAYERS_PER_LAUNCH 64
 int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
                                  int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
                                  int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,

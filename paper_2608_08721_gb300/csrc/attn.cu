@@ -293,9 +293,12 @@ struct LayerPtrs {
 struct LayerSet {
   CUtensorMap K[kMaxLayers];
   CUtensorMap V[kMaxLayers];
+  CUtensorMap Q[kMaxLayers];  // used when g divides 64 (q_tma)
   LayerPtrs p[kMaxLayers];
   int n;
+  int q_tma;
 };
+static_assert(sizeof(LayerSet) <= 32000, "kernel parameters are limited to 32764 bytes");
 
 template <int D, int STAGES>
 struct AttnSmem {
@@ -311,160 +314,94 @@ struct AttnSmem {
   static constexpr int kBar = kV + STAGES * kTileBytes;  // full[S], empty[S], qfull[2], qempty[2]
   static constexpr int kInfo = kBar + 8 * (2 * STAGES + 4);
   static constexpr int kTasks = kInfo + 2 * 64;
-  static constexpr int kMergeW = kTasks + 64;            // [kMaxParts] weights, [kMaxParts] weighted l
-  static constexpr int kMergeAcc = kMergeW + 2 * kMaxParts * 4;  // [4][D]
-  static constexpr int kMisc = kMergeAcc + 4 * D * 4;
+  // merge scratch: (m or weight, l) for rows x parts of one share, whose
+  // product is at most kAttnRows + kMaxParts, then 1/L and lse of its rows
+  static constexpr int kMergeCap = kAttnRows + kMaxParts;
+  static constexpr int kMergeW = kTasks + 64;
+  static constexpr int kMisc = kMergeW + (2 * kMergeCap + 2 * kAttnRows) * 4;
   static constexpr int kBytes = kMisc + 16;
   static constexpr int kAlloc = kBytes + 1024;           // room to align the base to 1024
 };
 
 // Merge, for layer l's split groups this CTA contributed to, its share of
-// rows [rows*k/np, rows*(k+1)/np) (k = this CTA's index among the group's
+// rows [rows*k/np, rows*(k+1)/np) (k = this CTA's index among the group's np
 // CTAs): O = sum_p w_p O_p / sum_p w_p l_p, w_p = 2^(m_p - M), M = max m_p,
-// parts in CTA order. Consumer warps only.
+// parts in CTA order. Consumer warps only. Three batched phases (all (m, l)
+// of the share; weights and sums per row; the weighted O rows), so that each
+// phase issues all of its loads at once.
 template <int D, int STAGES>
 __device__ void merge_layer(uint8_t* smem, const MergeTask* tasks, int n_tasks, int K, int Hq, int Hkv,
                             const float* __restrict__ part_o, const float* __restrict__ part_ml,
                             __nv_bfloat16* __restrict__ O, float* __restrict__ lse) {
   using SM = AttnSmem<D, STAGES>;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  constexpr int kT = kConsumerWarps * 32;
+  constexpr int C4 = D / 4;  // float4 columns of a row
   const int g = Hq / Hkv;
+  float* m_sh = reinterpret_cast<float*>(smem + SM::kMergeW);  // [nr * np] m, then weights
+  float* l_sh = m_sh + SM::kMergeCap;                           // [nr * np] l
+  float* row_sh = l_sh + SM::kMergeCap;                         // [nr] 1/L, [nr] lse (log2)
   for (int ti = 0; ti < n_tasks; ++ti) {
     const MergeTask it = tasks[ti];
     const int c0 = it.c0, np = it.np;
     const int k_me = (int)blockIdx.x - c0;
-    const int rows = it.rows, b = it.b, kvh = it.kvh, r_base = it.mg * kAttnRows;
-    const int u0 = (int)((long long)rows * k_me / np), u1 = (int)((long long)rows * (k_me + 1) / np);
-    // merge scratch: part weights, weighted l, per-stripe sums
-    float* wsh = reinterpret_cast<float*>(smem + SM::kMergeW);        // [np] weights
-    float* lsh = wsh + np;                                              // [np] weighted l
-    float* acc_sh = reinterpret_cast<float*>(smem + SM::kMergeAcc);   // [4][D]
-    constexpr int kStripes = 4;                      // parts handled by 4 thread stripes
-    constexpr int kColT = kConsumerWarps * 32 / kStripes;  // threads per stripe (32)
-    constexpr int CPT = D / kColT;                   // columns per thread (4 or 2)
-    const int stripe = tid / kColT, ct = tid % kColT;
-    if (u1 - u0 >= kConsumerWarps) {
-      // many rows: one warp per row, lanes over columns, parts in sequence
-      constexpr int CPL = D / 32;
-      for (int lr = u0 + warp; lr < u1; lr += kConsumerWarps) {
-        float M = -INFINITY;
-        for (int p = lane; p < np; p += 32) {
-          const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-          M = fmaxf(M, __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]));
-        }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-        float Lsum = 0.f, acc[CPL];
-#pragma unroll
-        for (int i = 0; i < CPL; ++i) acc[i] = 0.f;
-        for (int p0 = 0; p0 < np; p0 += 32) {
-          float wl = 0.f;
-          if (p0 + lane < np) {
-            const int p = p0 + lane;
-            const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-            const float ms = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
-            wl = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
-            Lsum += wl * __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
-          }
-          const int n = min(32, np - p0);
-#pragma unroll 8
-          for (int j = 0; j < n; ++j) {
-            const int p = p0 + j;
-            const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-            const float w = __shfl_sync(0xffffffffu, wl, j);
-            const float* src = part_o + (sl * kAttnRows + lr) * D + lane * CPL;
-            if (CPL == 4) {
-              const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
-              acc[0] += w * v.x; acc[1 % CPL] += w * v.y; acc[2 % CPL] += w * v.z; acc[3 % CPL] += w * v.w;
-            } else {
-              const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
-              acc[0] += w * v.x; acc[1 % CPL] += w * v.y;
-            }
-          }
-        }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
-        const float inv = 1.f / Lsum;
-        const int rr = r_base + lr;
-        const int t = rr / g, hq = kvh * g + rr % g;
-        __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + lane * CPL;
-#pragma unroll
-        for (int i = 0; i < CPL; i += 2)
-          *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
-        if (lse && lane == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
-      }
-    } else
-    for (int lr = u0; lr < u1; ++lr) {
-      // few rows: all consumer threads on one row, parts striped over threads
-      // 1) row max over the parts and the weights 2^(m_p - M)
-      float mloc = -INFINITY;
-      for (int p = tid; p < np; p += kConsumerWarps * 32) {
-        const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-        const float mp = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2]);
-        wsh[p] = mp;
-        lsh[p] = __ldcg(&part_ml[(sl * kAttnRows + lr) * 2 + 1]);
-        mloc = fmaxf(mloc, mp);
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, off));
-      if (lane == 0) acc_sh[warp] = mloc;
-      consumer_sync();
-      float M = acc_sh[0];
-      for (int w = 1; w < kConsumerWarps; ++w) M = fmaxf(M, acc_sh[w]);
-      consumer_sync();
-      float lpart = 0.f;
-      for (int p = tid; p < np; p += kConsumerWarps * 32) {
-        const float mp = wsh[p];
-        const float w = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
-        wsh[p] = w;
-        lpart += lsh[p] * w;
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) lpart += __shfl_xor_sync(0xffffffffu, lpart, off);
-      if (lane == 0) acc_sh[warp] = lpart;
-      consumer_sync();
-      float Lsum = 0.f;
-      for (int w = 0; w < kConsumerWarps; ++w) Lsum += acc_sh[w];
-      consumer_sync();
-      // 2) weighted sum of the part rows: stripe k takes parts k, k+4, ...
-      float acc[CPT];
-#pragma unroll
-      for (int i = 0; i < CPT; ++i) acc[i] = 0.f;
-#pragma unroll 8
-      for (int p = stripe; p < np; p += kStripes) {
-        const size_t sl = (p == 0) ? (size_t)(2 * c0 + 1) : (size_t)(2 * (c0 + p));
-        const float w = wsh[p];
-        const float* src = part_o + (sl * kAttnRows + lr) * D + ct * CPT;
-        if (CPT == 4) {
-          const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
-          acc[0] += w * v.x; acc[1 % CPT] += w * v.y; acc[2 % CPT] += w * v.z; acc[3 % CPT] += w * v.w;
-        } else {
-          const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
-          acc[0] += w * v.x; acc[1 % CPT] += w * v.y;
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < CPT; ++i) acc_sh[stripe * D + ct * CPT + i] = acc[i];
-      consumer_sync();
-      if (stripe == 0) {
-        const float inv = 1.f / Lsum;
-        const int rr = r_base + lr;
-        const int t = rr / g, hq = kvh * g + rr % g;
-        __nv_bfloat16* dst = O + (((size_t)b * (K + 1) + t) * Hq + hq) * D + ct * CPT;
-#pragma unroll
-        for (int i = 0; i < CPT; i += 2) {
-          float x0 = 0.f, x1 = 0.f;
-#pragma unroll
-          for (int k = 0; k < kStripes; ++k) {
-            x0 += acc_sh[k * D + ct * CPT + i];
-            x1 += acc_sh[k * D + ct * CPT + i + 1];
-          }
-          *reinterpret_cast<__nv_bfloat162*>(dst + i) = __floats2bfloat162_rn(x0 * inv, x1 * inv);
-        }
-        if (lse && ct == 0) lse[((size_t)b * (K + 1) + t) * Hq + hq] = (M + __log2f(Lsum)) * kLn2;
-      }
-      consumer_sync();
+    const int u0 = (int)((long long)it.rows * k_me / np), u1 = (int)((long long)it.rows * (k_me + 1) / np);
+    const int nr = u1 - u0;
+    if (nr <= 0) continue;
+    auto slot_of = [&](int p) { return (size_t)(p == 0 ? 2 * c0 + 1 : 2 * (c0 + p)); };
+    // 1) (m, l) of every part of every row of the share
+    for (int idx = tid; idx < nr * np; idx += kT) {
+      const int r = idx / np, p = idx - r * np;
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(part_ml + (slot_of(p) * kAttnRows + u0 + r) * 2));
+      m_sh[idx] = ml.x;
+      l_sh[idx] = ml.y;
     }
+    consumer_sync();
+    // 2) per row (one warp): M, the weights, 1/L and lse
+    for (int r = warp; r < nr; r += kConsumerWarps) {
+      float M = -INFINITY;
+      for (int p = lane; p < np; p += 32) M = fmaxf(M, m_sh[r * np + p]);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+      float Ls = 0.f;
+      for (int p = lane; p < np; p += 32) {
+        const float mp = m_sh[r * np + p];
+        const float w = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
+        m_sh[r * np + p] = w;
+        Ls += w * l_sh[r * np + p];
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, off);
+      if (lane == 0) {
+        row_sh[r] = 1.f / Ls;
+        row_sh[kAttnRows + r] = M + __log2f(Ls);
+      }
+    }
+    consumer_sync();
+    // 3) the weighted sum of the part rows, one float4 column per thread
+    for (int idx = tid; idx < nr * C4; idx += kT) {
+      const int r = idx / C4, c = idx - r * C4;
+      const float* wr = m_sh + r * np;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+      for (int p = 0; p < np; ++p) {
+        const float4 v =
+            __ldcg(reinterpret_cast<const float4*>(part_o + (slot_of(p) * kAttnRows + u0 + r) * D) + c);
+        const float w = wr[p];
+        acc.x += w * v.x;
+        acc.y += w * v.y;
+        acc.z += w * v.z;
+        acc.w += w * v.w;
+      }
+      const float inv = row_sh[r];
+      const int rr = it.mg * kAttnRows + u0 + r;
+      const int t = rr / g, hq = it.kvh * g + rr % g;
+      __nv_bfloat16* dst = O + (((size_t)it.b * (K + 1) + t) * Hq + hq) * D + c * 4;
+      *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+      *reinterpret_cast<__nv_bfloat162*>(dst + 2) = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+      if (lse && c == 0) lse[((size_t)it.b * (K + 1) + t) * Hq + hq] = row_sh[kAttnRows + r] * kLn2;
+    }
+    consumer_sync();  // the scratch is reused by the next task
   }
 }
 
@@ -610,35 +547,54 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
         };
         if (lane == 0) {
           // tiles whose stage is free go out first; before the barrier only
-          // tiles that lie wholly in the cache prefix
-          while (issued < n_tiles && (ready || it.key0 + (issued + 1) * kAttnTileKeys <= it.kv) &&
-                 mbar_test_wait(bEmpty + 8 * (tile_ctr % STAGES), ((tile_ctr / STAGES) & 1) ^ 1)) {
-            issue_tile(issued);
-            ++issued;
-          }
-          if (!ready) {
-            if (!wait_counter(bar_cnt + (layer - 1), n_ctas)) {
+          // tiles that lie wholly in the cache prefix, issued as the consumers
+          // free stages while the barrier is polled
+          const int n_pre = ready ? n_tiles : min(n_tiles, max(0, (it.kv - it.key0) / kAttnTileKeys));
+          for (int spin = 0;; ++spin) {
+            while (issued < n_pre &&
+                   mbar_test_wait(bEmpty + 8 * (tile_ctr % STAGES), ((tile_ctr / STAGES) & 1) ^ 1)) {
+              issue_tile(issued);
+              ++issued;
+            }
+            if (ready) break;
+            uint32_t v;
+            asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(bar_cnt + (layer - 1)) : "memory");
+            if (v >= n_ctas) break;
+            if (spin >= kMaxWaitIters) {
               raise_status(status, LIBRASPEC_ST_TIMEOUT);
               misc[0] = 1;
+              break;
             }
+            __nanosleep(32);
           }
         }
         __syncwarp();
         if (misc[0]) return;
         ready = true;
-        // Q rows of the item's row group (rows past `rows` are never used), one
-        // bulk copy per row and 64-column half, unswizzled: row r of half hb at
-        // hb * 8192 + r * 128. Bulk copies, like the K/V tiles, complete as
-        // transaction bytes on an mbarrier; non-bulk cp.async copies in flight
-        // in the warp that issues TMA loads were seen on GB300 to lose their
-        // mbarrier arrival, so the producer issues none.
-        if (lane == 0) {
-          info[q] = it;
-          mbar_expect_tx(bQFull + 8 * q, (uint32_t)it.rows * D * 2);
-        }
-        __syncwarp();
-        {
-          const uint32_t qdst = sQ + q * SM::kQSlot;
+        // Q rows of the item's row group into the slot, unswizzled: row r of
+        // 64-column half hb at hb * 8192 + r * 128. When g divides 64 a group is
+        // 64/g whole positions of its kv head's g query heads: one TMA box per
+        // half (rows past `rows` are read but never used). Otherwise one bulk
+        // copy per row and half. Both complete as transaction bytes on the
+        // slot's mbarrier; the producer issues no non-bulk cp.async copies
+        // (on GB300, non-bulk copies in flight in the warp issuing TMA loads
+        // were seen to lose their mbarrier arrival).
+        const uint32_t qdst = sQ + q * SM::kQSlot;
+        if (set.q_tma) {
+          if (lane == 0) {
+            info[q] = it;
+            mbar_expect_tx(bQFull + 8 * q, (uint32_t)kAttnRows * D * 2);
+#pragma unroll
+            for (int hb = 0; hb < SM::kBoxes; ++hb)
+              tma_load_3d(qdst + hb * 8192, &set.Q[layer], bQFull + 8 * q, hb * 64, it.kvh * g,
+                          it.b * (K + 1) + it.mg * (kAttnRows / g));
+          }
+        } else {
+          if (lane == 0) {
+            info[q] = it;
+            mbar_expect_tx(bQFull + 8 * q, (uint32_t)it.rows * D * 2);
+          }
+          __syncwarp();
           const __nv_bfloat16* Qb = set.p[layer].Q;
           for (int idx = lane; idx < it.rows * SM::kBoxes; idx += 32) {
             const int r = idx / SM::kBoxes, hb = idx - r * SM::kBoxes;
@@ -679,16 +635,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
     float* part_o = part_buf_o + (layer & 1) * part_o_stride;
     float* part_ml = part_buf_ml + (layer & 1) * part_ml_stride;
     if (layer > 0) {
-      // every CTA is done with the previous layer: merge its split groups
+      // layer's inputs are ready once every CTA is done with the previous layer
       if (tid == 0 && !wait_counter(bar_cnt + (layer - 1), n_ctas)) {
         raise_status(status, LIBRASPEC_ST_TIMEOUT);
         misc[0] = 1;
       }
       consumer_sync();
       if (misc[0]) return;
-      merge_layer<D, STAGES>(smem, tasks, n_tasks, K, Hq, Hkv, part_buf_o + ((layer - 1) & 1) * part_o_stride,
-                             part_buf_ml + ((layer - 1) & 1) * part_ml_stride, set.p[layer - 1].O,
-                             set.p[layer - 1].lse);
     }
     __nv_bfloat16* O = set.p[layer].O;
     float* lse = set.p[layer].lse;
@@ -945,6 +898,15 @@ __global__ void __launch_bounds__(kAttnThreads, 2) verify_attn_kernel(
       }
     }
     }
+    // the previous layer's split groups: its partials (the other parity
+    // buffer) stay untouched until every CTA has passed this layer's barrier,
+    // and the producer already streams the next layer's first tiles meanwhile
+    if (layer > 0) {
+      consumer_sync();
+      merge_layer<D, STAGES>(smem, tasks, n_tasks, K, Hq, Hkv, part_buf_o + ((layer - 1) & 1) * part_o_stride,
+                             part_buf_ml + ((layer - 1) & 1) * part_ml_stride, set.p[layer - 1].O,
+                             set.p[layer - 1].lse);
+    }
     // this CTA is done with the layer
     consumer_sync();
     if (tid == 0) asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(bar_cnt + layer), "r"(1u) : "memory");
@@ -988,6 +950,21 @@ static PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
       fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
   }
   return fn;
+}
+
+// Q [B*(K+1), Hq, D] as 3-D; box = 64 columns x g heads x 64/g positions
+// (one 64-row group of one kv head), no swizzle.
+static bool make_q_map(CUtensorMap* map, const void* base, int D, int Hq, int BT, int g) {
+  auto enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hq, (cuuint64_t)BT};
+  cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hq * D * 2};
+  cuuint32_t box[3] = {64, (cuuint32_t)g, (cuuint32_t)(kAttnRows / g)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
 }
 
 static bool make_kv_map(CUtensorMap* map, const void* base, int D, int S_cap, int BH) {
@@ -1050,10 +1027,13 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     LayerSet set;  // ~27 KB: built on the host, copied into the launch parameters
     const int n = n_layers - l0 < kMaxLayers ? n_layers - l0 : kMaxLayers;
     set.n = n;
+    const int g = Hq / Hkv;
+    set.q_tma = (kAttnRows % g == 0) ? 1 : 0;
     for (int i = 0; i < n; ++i) {
       const int l = l0 + i;
       if (!make_kv_map(&set.K[i], Kc[l], D, S_cap, B * Hkv) || !make_kv_map(&set.V[i], Vc[l], D, S_cap, B * Hkv))
         return cudaErrorInvalidValue;
+      if (set.q_tma && !make_q_map(&set.Q[i], Q[l], D, Hq, B * (K + 1), g)) return cudaErrorInvalidValue;
       set.p[i].Q = reinterpret_cast<const __nv_bfloat16*>(Q[l]);
       set.p[i].O = reinterpret_cast<__nv_bfloat16*>(O[l]);
       set.p[i].lse = lse ? lse[l] : nullptr;
