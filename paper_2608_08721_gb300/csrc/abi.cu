@@ -50,6 +50,7 @@ bool attn_shapes_ok(int B, int K, int Hq, int Hkv, int D, int S_cap) {
   if (B < 0 || B > LIBRASPEC_MAX_B || K < 0 || K > LIBRASPEC_MAX_K) return false;
   if (Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || S_cap < 1) return false;
   if ((long)(K + 1) * (Hq / Hkv) > 512) return false;
+  if (Hq / Hkv > kAttnRows) return false;  // a row group holds at least one block position
   if ((long)B * Hkv > (1L << 30)) return false;
   (void)D;
   return true;

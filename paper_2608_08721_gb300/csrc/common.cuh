@@ -19,8 +19,8 @@ constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kConfMaxSplits = 64;    // CTAs per drafter row
 constexpr int kRowMaxSplits = 64;     // CTAs per target row (acceptance)
 constexpr int kRaceMaxSplits = 128;   // CTAs per sequence for a vocabulary draw
-constexpr int kAttnMaxCtas = 512;     // persistent attention grid cap (>= SMs x CTAs per SM)
-constexpr int kAttnRows = 64;         // query rows per attention work item
+constexpr int kAttnMaxCtas = 192;     // persistent attention grid cap (one CTA per SM)
+constexpr int kAttnRows = 128;        // query rows per attention row group (at most)
 constexpr int kAttnTileKeys = 64;     // keys per KV tile
 constexpr int kAttnMaxLayers = LIBRASPEC_ATTN_LAYERS_PER_LAUNCH;  // layers per attention launch
 
@@ -57,7 +57,8 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   const size_t rows_d = size_t(B) * K, rows_t = size_t(B) * (K + 1);
   const int g = Hkv > 0 ? Hq / Hkv : 1;
   const int m_max = (K + 1) * g;
-  const int n_mg = (m_max + kAttnRows - 1) / kAttnRows;
+  const int rows = g >= 1 && g <= kAttnRows ? g * (kAttnRows / g) : 1;
+  const int n_mg = (m_max + rows - 1) / rows;
   w.max_groups = B * Hkv * n_mg;
   w.max_items = kAttnMaxCtas + w.max_groups;
   w.status = take(256);
