@@ -60,7 +60,9 @@ namespace libraspec {
 constexpr int kSoftmaxWarps = 4;
 constexpr int kProducerWarp = 4;
 constexpr int kMmaWarp = 5;
-constexpr int kAttnThreads = 6 * 32;
+constexpr int kMergeWarp = 6;
+constexpr int kAttnThreads = 7 * 32;
+constexpr int kPBufs = 4;  // P buffers in tensor memory
 constexpr int kMaxWaitIters = 1 << 24;
 constexpr int kSoftmaxBar = 1;  // named barrier of the softmax warpgroup
 constexpr float kRescaleLog2 = 8.f;
@@ -82,17 +84,31 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 
+// try_wait with a suspend-time hint: a waiting thread is parked by the
+// hardware until the phase completes (or the hint, in ns, elapses) instead of
+// re-polling, so waiting warps leave the SM's shared-memory pipe to the
+// working ones.
+constexpr uint32_t kSuspendHintNs = 1000000;
+
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(kSuspendHintNs)
       : "memory");
   return ok != 0;
 }
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
+
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // a wait that lasts 2 s has failed
 
 __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
@@ -106,12 +122,24 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Bounded wait: false after kMaxWaitIters polls (each poll may suspend).
+// Bounded wait: false once kWaitLimitNs have passed.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-  for (int i = 0; i < kMaxWaitIters; ++i)
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
-  return false;
+    if (global_ns() - t0 > kWaitLimitNs) return false;
+  }
 }
+
+// Bounded wait of a whole (converged) warp, with one verdict for all lanes.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity));
+}
+
+// The MMA-issuing thread waits like the others (a parked thread is woken when
+// the phase completes).
+__device__ __forceinline__ bool mbar_spin(uint32_t bar, uint32_t parity) { return mbar_wait(bar, parity); }
 
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y,
                                             int z) {
@@ -359,105 +387,163 @@ struct AttnSmem {
   static constexpr int kK = kQ + 2 * kQSlot;
   static constexpr int kV = kK + STAGES * kTileBytes;
   // mbarriers: full[S], empty[S], qfull[2], qempty[2], sfull[2], sfree[2],
-  // pfull[2], pvdone[2], ofree[2], drain
+  // pfull[4], pvdone[4], ofree[2], drain, merged
   static constexpr int kBar = kV + STAGES * kTileBytes;
-  static constexpr int kNumBars = 2 * STAGES + 15;
+  static constexpr int kNumBars = 2 * STAGES + 2 * 4 + 2 * kPBufs + 2 + 2;
   static constexpr int kInfo = kBar + ((8 * kNumBars + 63) / 64) * 64;
   static constexpr int kTasks = kInfo + 2 * 64;
   static constexpr int kTmem = kTasks + 64;
-  // merge scratch: (m or weight, l) for rows x parts of one share (product at
-  // most kAttnRows + kMaxParts), then 1/L and lse of its rows
-  static constexpr int kMergeCap = kAttnRows + kMaxParts;
-  static constexpr int kMergeW = kTmem + 16;
-  static constexpr int kMisc = kMergeW + (2 * kMergeCap + 2 * kAttnRows) * 4;
-  static constexpr int kBytes = kMisc + 16;
+  // [0] abort, [1] merge tasks, [2] items per layer, [3] merge chunks per
+  // layer, [4] chunks claimed, [5] chunks done, [6] layers whose weights are ready
+  static constexpr int kMisc = kTmem + 16;
+  // merge scratch: weights and l for rows x parts of at most two tasks (each
+  // product at most kAttnRows + kMaxParts), then per task 1/L and lse per row
+  static constexpr int kMergeCap = 2 * (kAttnRows + kMaxParts);
+  static constexpr int kMergeW = kMisc + 32;
+  static constexpr int kBytes = kMergeW + (2 * kMergeCap + 4 * kAttnRows) * 4;
   static constexpr int kAlloc = kBytes + 1024;           // room to align the base to 1024
   // tensor-memory columns
   static constexpr int kColS = 0;                        // S[2]: 64 fp32 columns each
-  static constexpr int kColP = 128;                      // P[2]: 64 bf16 = 32 columns each
+  static constexpr int kColP = 128;                      // P[4]: 64 bf16 = 32 columns each
   static constexpr int kColO = 256;                      // O[2]: D fp32 columns each
-  static_assert(kColO + 2 * D <= kTmemCols, "tensor memory");
+  static_assert(kColP + 32 * kPBufs <= kColO && kColO + 2 * D <= kTmemCols, "tensor memory");
 };
 
-// Merge, for layer l's split groups this CTA contributed to, its share of
-// rows [rows*k/np, rows*(k+1)/np) (k = this CTA's index among the group's np
-// CTAs): O = sum_p w_p O_p / sum_p w_p l_p, w_p = 2^(m_p - M), M = max m_p,
-// parts in CTA order. Softmax warps only. Three batched phases (all (m, l)
-// of the share; weights and sums per row; the weighted O rows), so that each
-// phase issues all of its loads at once.
+// Merging a layer's split groups. This CTA merges its share of rows
+// [rows*k/np, rows*(k+1)/np) of each group it contributed to (k = its index
+// among the group's np CTAs): O = sum_p w_p O_p / sum_p w_p l_p,
+// w_p = 2^(m_p - M), M = max m_p, parts in CTA order. The merge warp computes
+// every weight and 1/L of the layer into shared memory (merge_weights, right
+// after the layer's grid barrier, beside the next layer's items); the
+// weighted sums are cut into chunks of 32 (row, 4-column) items that any warp
+// may claim (merge_chunks): the merge warp first, the softmax warps once
+// their own items of the next layer are done.
+struct MergeScratch {
+  float* w;    // per task t at w_off[t]: [nr][np] weights
+  float* l;    // same layout: l, then unused
+  float* row;  // per task t at 2 * kAttnRows * t: [nr] 1/L, then [nr] lse (log2)
+};
+
 template <int D, int STAGES>
-__device__ void merge_layer(uint8_t* smem, const MergeTask* tasks, int n_tasks, int K, int Hq, int Hkv, int R,
-                            const float* __restrict__ part_o, const float* __restrict__ part_ml,
-                            __nv_bfloat16* __restrict__ O, float* __restrict__ lse) {
+__device__ __forceinline__ MergeScratch merge_scratch(uint8_t* smem) {
   using SM = AttnSmem<D, STAGES>;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  constexpr int kT = kSoftmaxWarps * 32;
-  constexpr int C4 = D / 4;  // float4 columns of a row
-  const int g = Hq / Hkv;
-  float* m_sh = reinterpret_cast<float*>(smem + SM::kMergeW);  // [nr * np] m, then weights
-  float* l_sh = m_sh + SM::kMergeCap;                           // [nr * np] l
-  float* row_sh = l_sh + SM::kMergeCap;                         // [nr] 1/L, [nr] lse (log2)
+  float* base = reinterpret_cast<float*>(smem + SM::kMergeW);
+  return MergeScratch{base, base + SM::kMergeCap, base + 2 * SM::kMergeCap};
+}
+
+template <int D, int STAGES>
+__device__ void merge_weights(uint8_t* smem, const MergeTask* tasks, int n_tasks, const float* __restrict__ part_ml) {
+  const MergeScratch sc = merge_scratch<D, STAGES>(smem);
+  const int lane = threadIdx.x & 31;
+  int off = 0;
   for (int ti = 0; ti < n_tasks; ++ti) {
     const MergeTask it = tasks[ti];
     const int c0 = it.c0, np = it.np;
     const int k_me = (int)blockIdx.x - c0;
     const int u0 = (int)((long long)it.rows * k_me / np), u1 = (int)((long long)it.rows * (k_me + 1) / np);
     const int nr = u1 - u0;
-    if (nr <= 0) continue;
+    float* w = sc.w + off;
+    float* l = sc.l + off;
+    float* row = sc.row + 2 * kAttnRows * ti;
     auto slot_of = [&](int p) { return (size_t)(p == 0 ? 2 * c0 + 1 : 2 * (c0 + p)); };
-    // 1) (m, l) of every part of every row of the share
-    for (int idx = tid; idx < nr * np; idx += kT) {
+    for (int idx = lane; idx < nr * np; idx += 32) {
       const int r = idx / np, p = idx - r * np;
       const float2 ml = __ldcg(reinterpret_cast<const float2*>(part_ml + (slot_of(p) * kAttnRows + u0 + r) * 2));
-      m_sh[idx] = ml.x;
-      l_sh[idx] = ml.y;
+      w[idx] = ml.x;
+      l[idx] = ml.y;
     }
-    softmax_sync();
-    // 2) per row (one warp): M, the weights, 1/L and lse
-    for (int r = warp; r < nr; r += kSoftmaxWarps) {
+    __syncwarp();
+    for (int r = 0; r < nr; ++r) {
       float M = -INFINITY;
-      for (int p = lane; p < np; p += 32) M = fmaxf(M, m_sh[r * np + p]);
+      for (int p = lane; p < np; p += 32) M = fmaxf(M, w[r * np + p]);
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
       float Ls = 0.f;
       for (int p = lane; p < np; p += 32) {
-        const float mp = m_sh[r * np + p];
-        const float w = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
-        m_sh[r * np + p] = w;
-        Ls += w * l_sh[r * np + p];
+        const float mp = w[r * np + p];
+        const float wp = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
+        w[r * np + p] = wp;
+        Ls += wp * l[r * np + p];
       }
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, off);
+      for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
       if (lane == 0) {
-        row_sh[r] = 1.f / Ls;
-        row_sh[kAttnRows + r] = M + __log2f(Ls);
+        row[r] = 1.f / Ls;
+        row[kAttnRows + r] = M + __log2f(Ls);
       }
     }
-    softmax_sync();
-    // 3) the weighted sum of the part rows, one float4 column per thread
-    for (int idx = tid; idx < nr * C4; idx += kT) {
-      const int r = idx / C4, c = idx - r * C4;
-      const float* wr = m_sh + r * np;
+    __syncwarp();
+    off += nr * np;
+  }
+}
+
+// Claims and merges chunks of layer `layer` until none is left; the warp
+// that completes the layer's last chunk arrives on `merged`. Chunks are
+// numbered [layer * C, (layer + 1) * C) on the CTA's monotonic counters.
+template <int D, int STAGES>
+__device__ void merge_chunks(uint8_t* smem, int layer, const MergeTask* tasks, int n_tasks, int C, int* ctr_claim,
+                             int* ctr_done, uint32_t merged, int K, int Hq, int Hkv, int R,
+                             const float* __restrict__ part_o, __nv_bfloat16* __restrict__ O,
+                             float* __restrict__ lse) {
+  const MergeScratch sc = merge_scratch<D, STAGES>(smem);
+  const int lane = threadIdx.x & 31;
+  constexpr int C4 = D / 4;
+  const int g = Hq / Hkv;
+  const int hi = (layer + 1) * C;
+  for (;;) {
+    int u = 0;
+    if (lane == 0) {
+      u = *reinterpret_cast<volatile int*>(ctr_claim);
+      while (u < hi) {
+        const int prev = atomicCAS(ctr_claim, u, u + 1);
+        if (prev == u) break;
+        u = prev;
+      }
+    }
+    u = __shfl_sync(0xffffffffu, u, 0);
+    if (u >= hi) return;
+    // item of this lane: (task, row, float4 column), tasks' items back to back
+    int i = (u - layer * C) * 32 + lane, ti = 0, off = 0;
+    bool live = false;
+    int nr = 0, u0 = 0;
+    for (; ti < n_tasks; ++ti) {
+      const MergeTask& t = tasks[ti];
+      const int k_me = (int)blockIdx.x - t.c0;
+      u0 = (int)((long long)t.rows * k_me / t.np);
+      nr = (int)((long long)t.rows * (k_me + 1) / t.np) - u0;
+      if (i < nr * C4) {
+        live = true;
+        break;
+      }
+      i -= nr * C4;
+      off += nr * t.np;
+    }
+    if (live) {
+      const MergeTask& t = tasks[ti];
+      const int r = i / C4, c = i - r * C4, np = t.np, c0 = t.c0;
+      const float* wr = sc.w + off + r * np;
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 8
       for (int p = 0; p < np; ++p) {
-        const float4 v =
-            __ldcg(reinterpret_cast<const float4*>(part_o + (slot_of(p) * kAttnRows + u0 + r) * D) + c);
+        const size_t slot = (size_t)(p == 0 ? 2 * c0 + 1 : 2 * (c0 + p));
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(part_o + (slot * kAttnRows + u0 + r) * D) + c);
         const float w = wr[p];
         acc.x += w * v.x;
         acc.y += w * v.y;
         acc.z += w * v.z;
         acc.w += w * v.w;
       }
-      const float inv = row_sh[r];
-      const int rr = it.mg * R + u0 + r;
-      const int t = rr / g, hq = it.kvh * g + rr % g;
-      __nv_bfloat16* dst = O + (((size_t)it.b * (K + 1) + t) * Hq + hq) * D + c * 4;
+      const float* row = sc.row + 2 * kAttnRows * ti;
+      const float inv = row[r];
+      const int rr = t.mg * R + u0 + r;
+      const int tt = rr / g, hq = t.kvh * g + rr % g;
+      __nv_bfloat16* dst = O + (((size_t)t.b * (K + 1) + tt) * Hq + hq) * D + c * 4;
       *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
       *reinterpret_cast<__nv_bfloat162*>(dst + 2) = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-      if (lse && c == 0) lse[((size_t)it.b * (K + 1) + t) * Hq + hq] = row_sh[kAttnRows + r] * kLn2;
+      if (lse && c == 0) lse[((size_t)t.b * (K + 1) + tt) * Hq + hq] = row[kAttnRows + r] * kLn2;
     }
-    softmax_sync();  // the scratch is reused by the next task
+    __syncwarp();
+    if (lane == 0 && atomicAdd(ctr_done, 1) + 1 == hi) mbar_arrive(merged);
   }
 }
 
@@ -480,13 +566,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   const uint32_t bSFull = bQEmpty + 16;
   const uint32_t bSFree = bSFull + 16;
   const uint32_t bPFull = bSFree + 16;
-  const uint32_t bPVDone = bPFull + 16;
-  const uint32_t bOFree = bPVDone + 16;
+  const uint32_t bPVDone = bPFull + 8 * kPBufs;
+  const uint32_t bOFree = bPVDone + 8 * kPBufs;
   const uint32_t bDrain = bOFree + 16;
+  const uint32_t bMerged = bDrain + 8;  // the merge warp finished a layer's merge
   ItemInfo* info = reinterpret_cast<ItemInfo*>(smem + SM::kInfo);
   MergeTask* tasks = reinterpret_cast<MergeTask*>(smem + SM::kTasks);
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + SM::kTmem);
-  volatile int* misc = reinterpret_cast<int*>(smem + SM::kMisc);  // [0] abort, [1] n_tasks, [2] n_items
+  volatile int* misc = reinterpret_cast<int*>(smem + SM::kMisc);
   uint32_t* exit_cnt = bar_cnt + kMaxLayers;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -505,12 +592,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       mbar_init(bQEmpty + 8 * q, 1 + kSoftmaxWarps);  // MMA commit (Q read) + softmax warps (info read)
       mbar_init(bSFull + 8 * q, 1);
       mbar_init(bSFree + 8 * q, kSoftmaxWarps);
-      mbar_init(bPFull + 8 * q, kSoftmaxWarps);
-      mbar_init(bPVDone + 8 * q, 1);
       mbar_init(bOFree + 8 * q, kSoftmaxWarps);
     }
+    for (int p = 0; p < kPBufs; ++p) {
+      mbar_init(bPFull + 8 * p, kSoftmaxWarps);
+      mbar_init(bPVDone + 8 * p, 1);
+    }
     mbar_init(bDrain, 1);
+    mbar_init(bMerged, 1);
     misc[0] = 0;
+    misc[4] = 0;
+    misc[5] = 0;
+    misc[6] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == kMmaWarp) {
@@ -560,14 +653,37 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       }
     }
     if (lane == 0) {
+      int U = 0;  // this CTA's share of rows of its split groups
+      for (int ti = 0; ti < n_tasks; ++ti) {
+        const MergeTask& t = tasks[ti];
+        const int k_me = (int)blockIdx.x - t.c0;
+        U += (int)((long long)t.rows * (k_me + 1) / t.np) - (int)((long long)t.rows * k_me / t.np);
+      }
       misc[1] = n_tasks;
       misc[2] = n_items;
+      misc[3] = (U * (D / 4) + 31) / 32;  // merge chunks of 32 (row, 4-column) items
     }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const int n_tasks = misc[1], n_items = misc[2];
+  const int n_tasks = misc[1], n_items = misc[2], merge_n = misc[3];
+  int* merge_claimed = const_cast<int*>(misc) + 4;
+  int* merge_done = const_cast<int*>(misc) + 5;
+  // bounded wait until the merge warp has the weights of `layers` layers ready
+  auto weights_ready = [&](int layers) {
+    bool ok = true;
+    if ((threadIdx.x & 31) == 0) {
+      int i = 0;
+      while (misc[6] < layers && i < kMaxWaitIters) {
+        __nanosleep(32);
+        ++i;
+      }
+      ok = misc[6] >= layers;
+      __threadfence_block();  // the weights written before the flag are read after it
+    }
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+  };
   const uint32_t tmem = *tmem_slot;
 
   if (warp == kProducerWarp) {
@@ -686,23 +802,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       bool ok = true;
       // O[ob] += P(gt) V(gt); the first PV of an item overwrites O
       auto issue_pv = [&](uint32_t gt, uint32_t item, bool first) {
-        const uint32_t sb = gt & 1, s = gt % STAGES, ob = item & 1;
-        ok = ok && mbar_wait(bPFull + 8 * sb, (gt >> 1) & 1);
-        if (first) ok = ok && mbar_wait(bOFree + 8 * ob, ((item >> 1) & 1) ^ 1);
+        const uint32_t pb = gt % kPBufs, s = gt % STAGES, ob = item & 1;
+        ok = ok && mbar_spin(bPFull + 8 * pb, (gt / kPBufs) & 1);
+        if (first) ok = ok && mbar_spin(bOFree + 8 * ob, ((item >> 1) & 1) ^ 1);
         if (!ok) return;
         tc_fence_after();
         const uint32_t vtile = sV + s * SM::kTileBytes;
 #pragma unroll
         for (int kc = 0; kc < kAttnTileKeys / 16; ++kc)
-          mma_ts(tmem + SM::kColO + ob * D, tmem + SM::kColP + sb * 32 + kc * 8,
+          mma_ts(tmem + SM::kColO + ob * D, tmem + SM::kColP + pb * 32 + kc * 8,
                  smem_desc(vtile + kc * 2048, 8192, 1024), kIdescPV, (!first || kc > 0) ? 1u : 0u);
-        mma_commit(bPVDone + 8 * sb);
+        mma_commit(bPVDone + 8 * pb);
         mma_commit(bEmpty + 8 * s);
       };
       for (int layer = 0; layer < n_layers && ok; ++layer) {
         for (int item = 0; item < n_items && ok; ++item) {
           const uint32_t q = item_ctr & 1;
-          ok = mbar_wait(bQFull + 8 * q, (item_ctr >> 1) & 1);
+          ok = mbar_spin(bQFull + 8 * q, (item_ctr >> 1) & 1);
           if (!ok) break;
           const ItemInfo it = info[q];
           const int n_tiles = (it.key1 - it.key0 + kAttnTileKeys - 1) / kAttnTileKeys;
@@ -710,7 +826,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           for (int t = 0; t < n_tiles && ok; ++t) {
             const uint32_t gt = tile_ctr;
             const uint32_t s = gt % STAGES, sb = gt & 1;
-            ok = mbar_wait(bFull + 8 * s, (gt / STAGES) & 1) && mbar_wait(bSFree + 8 * sb, ((gt >> 1) & 1) ^ 1);
+            ok = mbar_spin(bFull + 8 * s, (gt / STAGES) & 1) && mbar_spin(bSFree + 8 * sb, ((gt >> 1) & 1) ^ 1);
             if (!ok) break;
             tc_fence_after();
             const uint32_t ktile = sK + s * SM::kTileBytes;
@@ -738,7 +854,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       mbar_wait(bDrain, 0);
     }
     __syncwarp();
-  } else {
+  } else if (warp < kSoftmaxWarps) {
     // ======================= softmax warpgroup =======================
     const int row = warp * 32 + lane;  // tensor-memory lane
     const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
@@ -763,22 +879,33 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       float* lse = set.p[layer].lse;
       for (int item = 0; item < n_items && ok; ++item) {
         const uint32_t q = item_ctr & 1, ob = item_ctr & 1;
-        ok = __all_sync(0xffffffffu, mbar_wait(bQFull + 8 * q, (item_ctr >> 1) & 1));
+        ok = warp_wait(bQFull + 8 * q, (item_ctr >> 1) & 1);
         if (!ok) break;
         const ItemInfo it = info[q];
         __syncwarp();
         if (lane == 0) mbar_arrive(bQEmpty + 8 * q);  // info read; the Q slot is freed by the MMA commit
         const int n_tiles = (it.key1 - it.key0 + kAttnTileKeys - 1) / kAttnTileKeys;
         const bool valid = row < it.rows;
+        // a warp without valid rows only keeps the barrier counts in step
+        const bool warp_live = warp * 32 < it.rows;
         const int t_row = (it.mg * R + row) / g;
         const int lim = it.kv + t_row;  // last visible key of this row
         float m_run = -INFINITY, l_run = 0.f;
         for (int t = 0; t < n_tiles && ok; ++t) {
           const uint32_t gt = tile_ctr;
-          const uint32_t sb = gt & 1;
+          const uint32_t sb = gt & 1, pb = gt % kPBufs;
           const int kt0 = it.key0 + t * kAttnTileKeys;
-          ok = __all_sync(0xffffffffu, mbar_wait(bSFull + 8 * sb, (gt >> 1) & 1));
+          ok = warp_wait(bSFull + 8 * sb, (gt >> 1) & 1);
           if (!ok) break;
+          if (!warp_live) {
+            __syncwarp();
+            if (lane == 0) {
+              mbar_arrive(bSFree + 8 * sb);
+              mbar_arrive(bPFull + 8 * pb);
+            }
+            ++tile_ctr;
+            continue;
+          }
           tc_fence_after();
           uint32_t sr[2][32];
           tmem_ld32(tmem + lane_off + SM::kColS + sb * kAttnTileKeys, sr[0]);
@@ -787,16 +914,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(bSFree + 8 * sb);
-          // scores in the log2 domain, masked
-          float x[kAttnTileKeys];
-          float tmax = -INFINITY;
+          // raw scores; keys past this row's last visible key (and rows past
+          // the group) count as -inf; the scale (> 0) is applied below
+          const bool need_mask = !valid || kt0 + kAttnTileKeys - 1 > lim;
+          float xs[kAttnTileKeys];
+          float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
           for (int c = 0; c < kAttnTileKeys; ++c) {
-            float v = __uint_as_float(sr[c >> 5][c & 31]) * scale_log2;
-            if (!valid || kt0 + c > lim) v = -INFINITY;
-            x[c] = v;
-            tmax = fmaxf(tmax, v);
+            float v = __uint_as_float(sr[c >> 5][c & 31]);
+            if (need_mask && (!valid || kt0 + c > lim)) v = -INFINITY;
+            xs[c] = v;
+            mx[c & 3] = fmaxf(mx[c & 3], v);
           }
+          const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * scale_log2;
           // raise the reference max only when it grows by more than 2^8
           float f = 1.f;
           const bool raise = tmax > m_run + kRescaleLog2;
@@ -804,20 +934,21 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             f = (m_run == -INFINITY) ? 0.f : ex2_approx(m_run - tmax);
             m_run = tmax;
           }
-          const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
-          float lsum = 0.f;
+          const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
+          float ls[4] = {0.f, 0.f, 0.f, 0.f};
           uint32_t pk[32];
 #pragma unroll
           for (int c = 0; c < kAttnTileKeys; c += 2) {
-            const float p0 = ex2_approx(x[c] - m_use), p1 = ex2_approx(x[c + 1] - m_use);
-            lsum += p0 + p1;
+            const float p0 = ex2_approx(fmaf(xs[c], scale_log2, neg_m));
+            const float p1 = ex2_approx(fmaf(xs[c + 1], scale_log2, neg_m));
+            ls[(c >> 1) & 3] += p0 + p1;
             pk[c >> 1] = pack_bf16(p0, p1);
           }
-          l_run = l_run * f + lsum;
+          l_run = l_run * f + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
           // O holds the earlier tiles of this item: rescale its rows once the
           // previous tile's PV has landed (rare: the max rose by > 2^8)
           if (t > 0 && __any_sync(0xffffffffu, raise)) {
-            ok = __all_sync(0xffffffffu, mbar_wait(bPVDone + 8 * ((gt - 1) & 1), ((gt - 1) >> 1) & 1));
+            ok = warp_wait(bPVDone + 8 * ((gt - 1) % kPBufs), ((gt - 1) / kPBufs) & 1);
             if (!ok) break;
             tc_fence_after();
 #pragma unroll 1
@@ -831,56 +962,60 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             }
             tmem_wait_st();
           }
-          // P buffer sb is free once PV(gt - 2) has read it
-          if (gt >= 2) {
-            ok = __all_sync(0xffffffffu, mbar_wait(bPVDone + 8 * sb, ((gt >> 1) & 1) ^ 1));
+          // P buffer pb is free once PV(gt - kPBufs) has read it
+          if (gt >= kPBufs) {
+            ok = warp_wait(bPVDone + 8 * pb, ((gt / kPBufs) & 1) ^ 1);
             if (!ok) break;
             tc_fence_after();
           }
-          tmem_st32(tmem + lane_off + SM::kColP + sb * 32, pk);
+          tmem_st32(tmem + lane_off + SM::kColP + pb * 32, pk);
           tmem_wait_st();
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(bPFull + 8 * sb);
+          if (lane == 0) mbar_arrive(bPFull + 8 * pb);
           ++tile_ctr;
         }
         if (!ok) break;
         // epilogue: O of this item is complete once the last PV has landed
         {
           const uint32_t last = tile_ctr - 1;
-          ok = __all_sync(0xffffffffu, mbar_wait(bPVDone + 8 * (last & 1), (last >> 1) & 1));
+          ok = warp_wait(bPVDone + 8 * (last % kPBufs), (last / kPBufs) & 1);
           if (!ok) break;
           tc_fence_after();
-          const int rr = it.mg * R + row;
-          const int hq = it.kvh * g + rr % g;
-          const float inv = 1.f / l_run;
-          const size_t slot = (size_t)it.slot;
+          if (warp_live) {
+            const int rr = it.mg * R + row;
+            const int hq = it.kvh * g + rr % g;
+            const float inv = 1.f / l_run;
+            const size_t slot = (size_t)it.slot;
 #pragma unroll 1
-          for (int c0 = 0; c0 < D; c0 += 32) {
-            uint32_t o[32];
-            tmem_ld32(tmem + lane_off + SM::kColO + ob * D + c0, o);
-            tmem_wait_ld();
-            if (valid) {
-              if (!it.partial) {
-                uint4* dst = reinterpret_cast<uint4*>(O + (((size_t)it.b * (K + 1) + t_row) * Hq + hq) * D + c0);
+            for (int c0 = 0; c0 < D; c0 += 32) {
+              uint32_t o[32];
+              tmem_ld32(tmem + lane_off + SM::kColO + ob * D + c0, o);
+              tmem_wait_ld();
+              if (valid) {
+                if (!it.partial) {
+                  uint4* dst =
+                      reinterpret_cast<uint4*>(O + (((size_t)it.b * (K + 1) + t_row) * Hq + hq) * D + c0);
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                  dst[i] = make_uint4(pack_bf16(__uint_as_float(o[8 * i]) * inv, __uint_as_float(o[8 * i + 1]) * inv),
-                                      pack_bf16(__uint_as_float(o[8 * i + 2]) * inv, __uint_as_float(o[8 * i + 3]) * inv),
-                                      pack_bf16(__uint_as_float(o[8 * i + 4]) * inv, __uint_as_float(o[8 * i + 5]) * inv),
-                                      pack_bf16(__uint_as_float(o[8 * i + 6]) * inv, __uint_as_float(o[8 * i + 7]) * inv));
-              } else {
-                uint4* dst = reinterpret_cast<uint4*>(part_o + (slot * kAttnRows + row) * D + c0);
+                  for (int i = 0; i < 4; ++i)
+                    dst[i] = make_uint4(
+                        pack_bf16(__uint_as_float(o[8 * i]) * inv, __uint_as_float(o[8 * i + 1]) * inv),
+                        pack_bf16(__uint_as_float(o[8 * i + 2]) * inv, __uint_as_float(o[8 * i + 3]) * inv),
+                        pack_bf16(__uint_as_float(o[8 * i + 4]) * inv, __uint_as_float(o[8 * i + 5]) * inv),
+                        pack_bf16(__uint_as_float(o[8 * i + 6]) * inv, __uint_as_float(o[8 * i + 7]) * inv));
+                } else {
+                  uint4* dst = reinterpret_cast<uint4*>(part_o + (slot * kAttnRows + row) * D + c0);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) dst[i] = make_uint4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+                  for (int i = 0; i < 8; ++i) dst[i] = make_uint4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+                }
               }
             }
-          }
-          if (valid) {
-            if (it.partial) {
-              *reinterpret_cast<float2*>(part_ml + (slot * kAttnRows + row) * 2) = make_float2(m_run, l_run);
-            } else if (lse) {
-              lse[((size_t)it.b * (K + 1) + t_row) * Hq + hq] = (m_run + __log2f(l_run)) * kLn2;
+            if (valid) {
+              if (it.partial) {
+                *reinterpret_cast<float2*>(part_ml + (slot * kAttnRows + row) * 2) = make_float2(m_run, l_run);
+              } else if (lse) {
+                lse[((size_t)it.b * (K + 1) + t_row) * Hq + hq] = (m_run + __log2f(l_run)) * kLn2;
+              }
             }
           }
           tc_fence_before();
@@ -890,46 +1025,78 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         ++item_ctr;
       }
       if (!ok) break;
-      // the previous layer's split groups: its partials (the other parity
-      // buffer) stay untouched until every CTA has passed this layer's
-      // barrier, and the producer already streams the next layer's first
-      // tiles meanwhile
+      // this CTA is done with the layer's items; the previous layer's partials
+      // (the other parity buffer) must be merged before any CTA may start the
+      // next layer and overwrite them: help with what the merge warp has left
+      if (layer > 0 && merge_n > 0) {
+        if (weights_ready(layer))
+          merge_chunks<D, STAGES>(smem, layer - 1, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq,
+                                  Hkv, R, part_buf_o + ((layer - 1) & 1) * part_o_stride, set.p[layer - 1].O,
+                                  set.p[layer - 1].lse);
+        if (warp == 0 && !warp_wait(bMerged, (layer - 1) & 1) && tid == 0) {
+          raise_status(status, LIBRASPEC_ST_TIMEOUT);
+          misc[0] = 1;
+        }
+      }
       softmax_sync();
-      if (layer > 0)
-        merge_layer<D, STAGES>(smem, tasks, n_tasks, K, Hq, Hkv, R, part_buf_o + ((layer - 1) & 1) * part_o_stride,
-                               part_buf_ml + ((layer - 1) & 1) * part_ml_stride, set.p[layer - 1].O,
-                               set.p[layer - 1].lse);
-      // this CTA is done with the layer
-      softmax_sync();
+      if (misc[0]) {
+        ok = false;
+        break;
+      }
       if (tid == 0)
         asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(bar_cnt + layer), "r"(1u) : "memory");
     }
     if (!ok) {
       if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
       misc[0] = 1;
-    } else if (n_layers > 0) {
-      // merge the last layer, then the last CTA out resets the counters
-      if (tid == 0 && !wait_counter(bar_cnt + (n_layers - 1), n_ctas)) {
+    } else if (n_layers > 0 && merge_n > 0) {
+      // help with the last layer's merge
+      if (weights_ready(n_layers))
+        merge_chunks<D, STAGES>(smem, n_layers - 1, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq,
+                                Hkv, R, part_buf_o + ((n_layers - 1) & 1) * part_o_stride, set.p[n_layers - 1].O,
+                                set.p[n_layers - 1].lse);
+    }
+  } else if (warp == kMergeWarp) {
+    // ======================= merge warp =======================
+    // Layer l's split groups, once every CTA has finished layer l (its grid
+    // barrier), while the softmax warps already run layer l+1.
+    bool ok = true;
+    for (int layer = 0; layer < n_layers && ok; ++layer) {
+      if (lane == 0) ok = wait_counter(bar_cnt + layer, n_ctas) && !misc[0];
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      if (merge_n > 0) {
+        merge_weights<D, STAGES>(smem, tasks, n_tasks, part_buf_ml + (layer & 1) * part_ml_stride);
+        if (lane == 0) {
+          __threadfence_block();
+          misc[6] = layer + 1;
+        }
+        __syncwarp();
+        merge_chunks<D, STAGES>(smem, layer, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv,
+                                R, part_buf_o + (layer & 1) * part_o_stride, set.p[layer].O, set.p[layer].lse);
+      }
+    }
+    // every chunk of the last layer is merged (by whichever warp) before the exit count
+    if (ok && merge_n > 0 && n_layers > 0) {
+      if (lane == 0) ok = mbar_wait(bMerged, (n_layers - 1) & 1);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+    }
+    if (!ok) {
+      if (lane == 0 && !misc[0]) {
         raise_status(status, LIBRASPEC_ST_TIMEOUT);
         misc[0] = 1;
       }
-      softmax_sync();
-      if (!misc[0]) {
-        merge_layer<D, STAGES>(smem, tasks, n_tasks, K, Hq, Hkv, R,
-                               part_buf_o + ((n_layers - 1) & 1) * part_o_stride,
-                               part_buf_ml + ((n_layers - 1) & 1) * part_ml_stride, set.p[n_layers - 1].O,
-                               set.p[n_layers - 1].lse);
-        softmax_sync();
-        if (tid == 0) {
-          const uint32_t done = atomicAdd(exit_cnt, 1u);
-          if (done == n_ctas - 1) {
-            for (int l = 0; l < n_layers; ++l) bar_cnt[l] = 0u;
-            *exit_cnt = 0u;
-            __threadfence();
-          }
-        }
+    } else if (lane == 0 && n_layers > 0) {
+      // the last CTA out resets the barrier counters for the next launch
+      __threadfence();
+      const uint32_t done = atomicAdd(exit_cnt, 1u);
+      if (done == n_ctas - 1) {
+        for (int l = 0; l < n_layers; ++l) bar_cnt[l] = 0u;
+        *exit_cnt = 0u;
+        __threadfence();
       }
     }
+    __syncwarp();
   }
   // every role is done with the tensor memory
   tc_fence_before();
