@@ -435,46 +435,48 @@ template <int D, int STAGES>
 __device__ void merge_weights(uint8_t* smem, const MergeTask* tasks, int n_tasks, const float* __restrict__ part_ml) {
   const MergeScratch sc = merge_scratch<D, STAGES>(smem);
   const int lane = threadIdx.x & 31;
-  int off = 0;
-  for (int ti = 0; ti < n_tasks; ++ti) {
+  // (m, l) of every part of every row of both tasks, all loads in flight together
+  for (int ti = 0, off = 0; ti < n_tasks; ++ti) {
     const MergeTask it = tasks[ti];
     const int c0 = it.c0, np = it.np;
     const int k_me = (int)blockIdx.x - c0;
     const int u0 = (int)((long long)it.rows * k_me / np), u1 = (int)((long long)it.rows * (k_me + 1) / np);
     const int nr = u1 - u0;
-    float* w = sc.w + off;
-    float* l = sc.l + off;
-    float* row = sc.row + 2 * kAttnRows * ti;
-    auto slot_of = [&](int p) { return (size_t)(p == 0 ? 2 * c0 + 1 : 2 * (c0 + p)); };
     for (int idx = lane; idx < nr * np; idx += 32) {
       const int r = idx / np, p = idx - r * np;
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(part_ml + (slot_of(p) * kAttnRows + u0 + r) * 2));
-      w[idx] = ml.x;
-      l[idx] = ml.y;
+      const size_t slot = (size_t)(p == 0 ? 2 * c0 + 1 : 2 * (c0 + p));
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(part_ml + (slot * kAttnRows + u0 + r) * 2));
+      sc.w[off + idx] = ml.x;
+      sc.l[off + idx] = ml.y;
     }
-    __syncwarp();
-    for (int r = 0; r < nr; ++r) {
-      float M = -INFINITY;
-      for (int p = lane; p < np; p += 32) M = fmaxf(M, w[r * np + p]);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-      float Ls = 0.f;
-      for (int p = lane; p < np; p += 32) {
-        const float mp = w[r * np + p];
-        const float wp = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
-        w[r * np + p] = wp;
-        Ls += wp * l[r * np + p];
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
-      if (lane == 0) {
-        row[r] = 1.f / Ls;
-        row[kAttnRows + r] = M + __log2f(Ls);
-      }
-    }
-    __syncwarp();
     off += nr * np;
   }
+  __syncwarp();
+  // weights, 1/L and lse: one row per lane, no cross-lane reductions
+  for (int ti = 0, off = 0; ti < n_tasks; ++ti) {
+    const MergeTask it = tasks[ti];
+    const int np = it.np;
+    const int k_me = (int)blockIdx.x - it.c0;
+    const int nr = (int)((long long)it.rows * (k_me + 1) / np) - (int)((long long)it.rows * k_me / np);
+    float* row = sc.row + 2 * kAttnRows * ti;
+    for (int r = lane; r < nr; r += 32) {
+      float* wr = sc.w + off + r * np;
+      const float* lr = sc.l + off + r * np;
+      float M = -INFINITY;
+      for (int p = 0; p < np; ++p) M = fmaxf(M, wr[p]);
+      float Ls = 0.f;
+      for (int p = 0; p < np; ++p) {
+        const float mp = wr[p];
+        const float wp = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
+        wr[p] = wp;
+        Ls += wp * lr[p];
+      }
+      row[r] = 1.f / Ls;
+      row[kAttnRows + r] = M + __log2f(Ls);
+    }
+    off += nr * np;
+  }
+  __syncwarp();
 }
 
 // Claims and merges chunks of layer `layer` until none is left; the warp
