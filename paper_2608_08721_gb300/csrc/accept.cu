@@ -240,16 +240,21 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
     for (int t = 0; t < 4; ++t) {
       const int v = 4 * g + t;
       if (v >= c1) break;
-      float wv = exp2f((yv[t] - mp) * c);
-      if (residual) {
-        const float pv = wv * invZp;
-        const float qv = exp2f((dv[t] - mq) * c) * invZq;
-        wv = pv - qv;
-      }
+      // exponents are <= 0 (below the row maxima), so the fast base-2
+      // exponential is exact to a few ulp
+      const float e = (yv[t] - mp) * c;
+      float wv = ex2_approx(e);
+      if (residual) wv = wv * invZp - ex2_approx((dv[t] - mq) * c) * invZq;
       if (wv > 0.f) {
-        const float E = -logf(word_to_uniform(ws[t]));
-        const float key = E / wv;
-        argmin_combine(best, besti, key, v);
+        // E / w < best  <=>  u > exp(-best * w): a candidate whose uniform is
+        // below that (with a margin far above the rounding of the test)
+        // cannot win, and skips the logarithm
+        const float u = word_to_uniform(ws[t]);
+        if (best == INFINITY || u > ex2_approx(-best * wv * kLog2e) * (1.f - 9.5367431640625e-7f)) {
+          const float E = -logf(u);
+          const float key = residual ? __fdividef(E, wv) : E * ex2_approx(-e);
+          argmin_combine(best, besti, key, v);
+        }
       }
     }
   }
@@ -365,7 +370,7 @@ cudaError_t launch_accept(const float* target, const float* draft, const int32_t
   }
   {
     // race slices: enough CTAs per sequence to stream one or two V-rows fast
-    long target_ctas = 2L * sms;
+    long target_ctas = 4L * sms;
     int nsplit = (int)((target_ctas + B - 1) / B);
     const int cap = (V + 4095) / 4096;
     if (nsplit > cap) nsplit = cap;

@@ -184,7 +184,7 @@ __device__ __forceinline__ void warp_merge_partials(const RowPartial* __restrict
 // several times over, each with at least min_elems elements.
 inline int row_splits(long rows, int V, int num_sms, int max_splits, int min_elems) {
   if (rows <= 0) return 1;
-  const long target = 4L * 8 * num_sms;
+  const long target = 2L * 8 * num_sms;
   long ns = (target + rows - 1) / rows;
   const long cap = (V + min_elems - 1) / min_elems;  // at least min_elems per CTA
   if (ns > cap) ns = cap;
