@@ -394,102 +394,138 @@ struct AttnSmem {
   static constexpr int kTasks = kInfo + 2 * 64;
   static constexpr int kTmem = kTasks + 64;
   // [0] abort, [1] merge tasks, [2] items per layer, [3] merge chunks per
-  // layer, [4] chunks claimed, [5] chunks done, [6] layers whose weights are ready
+  // layer, [4] chunks claimed, [5] chunks done
   static constexpr int kMisc = kTmem + 16;
-  // merge scratch: weights and l for rows x parts of at most two tasks (each
-  // product at most kAttnRows + kMaxParts), then per task 1/L and lse per row
-  static constexpr int kMergeCap = 2 * (kAttnRows + kMaxParts);
-  static constexpr int kMergeW = kMisc + 32;
-  static constexpr int kBytes = kMergeW + (2 * kMergeCap + 4 * kAttnRows) * 4;
+  static constexpr int kBytes = kMisc + 32;
   static constexpr int kAlloc = kBytes + 1024;           // room to align the base to 1024
   // tensor-memory columns
   static constexpr int kColS = 0;                        // S[2]: 64 fp32 columns each
   static constexpr int kColP = 128;                      // P[4]: 64 bf16 = 32 columns each
   static constexpr int kColO = 256;                      // O[2]: D fp32 columns each
   static_assert(kColP + 32 * kPBufs <= kColO && kColO + 2 * D <= kTmemCols, "tensor memory");
+  static_assert(kAlloc <= 227 * 1024, "shared memory per CTA");
 };
 
 // Merging a layer's split groups. This CTA merges its share of rows
 // [rows*k/np, rows*(k+1)/np) of each group it contributed to (k = its index
-// among the group's np CTAs): O = sum_p w_p O_p / sum_p w_p l_p,
-// w_p = 2^(m_p - M), M = max m_p, parts in CTA order. The merge warp computes
-// every weight and 1/L of the layer into shared memory (merge_weights, right
-// after the layer's grid barrier, beside the next layer's items); the
-// weighted sums are cut into chunks of 32 (row, 4-column) items that any warp
-// may claim (merge_chunks): the merge warp first, the softmax warps once
-// their own items of the next layer are done.
-struct MergeScratch {
-  float* w;    // per task t at w_off[t]: [nr][np] weights
-  float* l;    // same layout: l, then unused
-  float* row;  // per task t at 2 * kAttnRows * t: [nr] 1/L, then [nr] lse (log2)
-};
+// among the group's np CTAs): O = sum_p w_p O_p / sum_p w_p l_p with
+// w_p = 2^(m_p - M), M = max m_p, parts in CTA order. The share is cut into
+// chunks of (row, 4-column) items that any warp may claim once the layer's
+// grid barrier has passed: the merge warp right away (beside the next
+// layer's items), the softmax warps once their own items are done. A lane
+// loads (m_p, l_p) and its 4 columns of O_p for a batch of parts at once and
+// folds the batch in with a running maximum, so a chunk costs one memory
+// round trip per batch and no weights are staged in shared memory.
 
-template <int D, int STAGES>
-__device__ __forceinline__ MergeScratch merge_scratch(uint8_t* smem) {
-  using SM = AttnSmem<D, STAGES>;
-  float* base = reinterpret_cast<float*>(smem + SM::kMergeW);
-  return MergeScratch{base, base + SM::kMergeCap, base + 2 * SM::kMergeCap};
+// This CTA's share [u0, u0 + nr) of task t's rows.
+__device__ __forceinline__ int merge_share(const MergeTask& t, int& u0) {
+  const int k_me = (int)blockIdx.x - t.c0;
+  u0 = (int)((long long)t.rows * k_me / t.np);
+  return (int)((long long)t.rows * (k_me + 1) / t.np) - u0;
 }
 
-template <int D, int STAGES>
-__device__ void merge_weights(uint8_t* smem, const MergeTask* tasks, int n_tasks, const float* __restrict__ part_ml) {
-  const MergeScratch sc = merge_scratch<D, STAGES>(smem);
+// Items per lane in a chunk of a group of np parts: J items x 16/J parts are
+// in flight per batch.
+__device__ __forceinline__ int merge_j(int np) { return np > 8 ? 1 : (np > 4 ? 2 : 4); }
+
+template <int D>
+__device__ __forceinline__ int merge_chunk_count(const MergeTask* tasks, int n_tasks) {
+  int n = 0;
+  for (int ti = 0; ti < n_tasks; ++ti) {
+    int u0;
+    const int items = merge_share(tasks[ti], u0) * (D / 4);
+    const int ci = 32 * merge_j(tasks[ti].np);
+    n += (items + ci - 1) / ci;
+  }
+  return n;
+}
+
+// Chunk lc of task t: items (lc*J + j)*32 + lane, j < J.
+template <int J, int D>
+__device__ __forceinline__ void merge_chunk(const MergeTask& t, int u0, int nr, int lc, const float* __restrict__ part_o,
+                                            const float* __restrict__ part_ml, int K, int Hq, int g, int R,
+                                            __nv_bfloat16* __restrict__ O, float* __restrict__ lse) {
+  constexpr int PB = 16 / J, C4 = D / 4;
   const int lane = threadIdx.x & 31;
-  // (m, l) of every part of every row of both tasks, all loads in flight together
-  for (int ti = 0, off = 0; ti < n_tasks; ++ti) {
-    const MergeTask it = tasks[ti];
-    const int c0 = it.c0, np = it.np;
-    const int k_me = (int)blockIdx.x - c0;
-    const int u0 = (int)((long long)it.rows * k_me / np), u1 = (int)((long long)it.rows * (k_me + 1) / np);
-    const int nr = u1 - u0;
-    for (int idx = lane; idx < nr * np; idx += 32) {
-      const int r = idx / np, p = idx - r * np;
-      const size_t slot = (size_t)(p == 0 ? 2 * c0 + 1 : 2 * (c0 + p));
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(part_ml + (slot * kAttnRows + u0 + r) * 2));
-      sc.w[off + idx] = ml.x;
-      sc.l[off + idx] = ml.y;
-    }
-    off += nr * np;
+  const int np = t.np, c0 = t.c0, items = nr * C4;
+  float M[J], Ls[J];
+  float4 acc[J];
+#pragma unroll
+  for (int j = 0; j < J; ++j) {
+    M[j] = -INFINITY;
+    Ls[j] = 0.f;
+    acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  __syncwarp();
-  // weights, 1/L and lse: one row per lane, no cross-lane reductions
-  for (int ti = 0, off = 0; ti < n_tasks; ++ti) {
-    const MergeTask it = tasks[ti];
-    const int np = it.np;
-    const int k_me = (int)blockIdx.x - it.c0;
-    const int nr = (int)((long long)it.rows * (k_me + 1) / np) - (int)((long long)it.rows * k_me / np);
-    float* row = sc.row + 2 * kAttnRows * ti;
-    for (int r = lane; r < nr; r += 32) {
-      float* wr = sc.w + off + r * np;
-      const float* lr = sc.l + off + r * np;
-      float M = -INFINITY;
-      for (int p = 0; p < np; ++p) M = fmaxf(M, wr[p]);
-      float Ls = 0.f;
-      for (int p = 0; p < np; ++p) {
-        const float mp = wr[p];
-        const float wp = (mp == -INFINITY) ? 0.f : ex2_approx(mp - M);
-        wr[p] = wp;
-        Ls += wp * lr[p];
+  for (int p0 = 0; p0 < np; p0 += PB) {
+    float2 ml[J][PB];
+    float4 v[J][PB];
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+      const int i = (lc * J + j) * 32 + lane;
+      const int r = i / C4, c = i - r * C4;
+#pragma unroll
+      for (int k = 0; k < PB; ++k) {
+        const int p = p0 + k;
+        if (i < items && p < np) {
+          const size_t at = (size_t)(p == 0 ? 2 * c0 + 1 : 2 * (c0 + p)) * kAttnRows + u0 + r;
+          ml[j][k] = __ldcg(reinterpret_cast<const float2*>(part_ml + at * 2));
+          v[j][k] = __ldcg(reinterpret_cast<const float4*>(part_o + at * D) + c);
+        } else {
+          ml[j][k] = make_float2(-INFINITY, 0.f);
+          v[j][k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
       }
-      row[r] = 1.f / Ls;
-      row[kAttnRows + r] = M + __log2f(Ls);
     }
-    off += nr * np;
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+      float bm = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < PB; ++k) bm = fmaxf(bm, ml[j][k].x);
+      const float Mn = fmaxf(M[j], bm);
+      if (Mn == -INFINITY) continue;  // no visible key in these parts yet
+      const float f = ex2_approx(M[j] - Mn);  // 0 while M is still -inf
+      acc[j].x *= f;
+      acc[j].y *= f;
+      acc[j].z *= f;
+      acc[j].w *= f;
+      Ls[j] *= f;
+      M[j] = Mn;
+#pragma unroll
+      for (int k = 0; k < PB; ++k) {
+        const float w = ex2_approx(ml[j][k].x - Mn);  // 0 for a part with no visible key
+        acc[j].x += w * v[j][k].x;
+        acc[j].y += w * v[j][k].y;
+        acc[j].z += w * v[j][k].z;
+        acc[j].w += w * v[j][k].w;
+        Ls[j] += w * ml[j][k].y;
+      }
+    }
   }
-  __syncwarp();
+#pragma unroll
+  for (int j = 0; j < J; ++j) {
+    const int i = (lc * J + j) * 32 + lane;
+    if (i >= items) continue;
+    const int r = i / C4, c = i - r * C4;
+    const float inv = 1.f / Ls[j];
+    const int rr = t.mg * R + u0 + r;
+    const int tt = rr / g, hq = t.kvh * g + rr % g;
+    uint2 o;
+    o.x = pack_bf16(acc[j].x * inv, acc[j].y * inv);
+    o.y = pack_bf16(acc[j].z * inv, acc[j].w * inv);
+    *reinterpret_cast<uint2*>(O + (((size_t)t.b * (K + 1) + tt) * Hq + hq) * D + c * 4) = o;
+    if (lse && c == 0) lse[((size_t)t.b * (K + 1) + tt) * Hq + hq] = (M[j] + __log2f(Ls[j])) * kLn2;
+  }
 }
 
 // Claims and merges chunks of layer `layer` until none is left; the warp
 // that completes the layer's last chunk arrives on `merged`. Chunks are
 // numbered [layer * C, (layer + 1) * C) on the CTA's monotonic counters.
-template <int D, int STAGES>
-__device__ void merge_chunks(uint8_t* smem, int layer, const MergeTask* tasks, int n_tasks, int C, int* ctr_claim,
-                             int* ctr_done, uint32_t merged, int K, int Hq, int Hkv, int R,
-                             const float* __restrict__ part_o, __nv_bfloat16* __restrict__ O,
+template <int D>
+__device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int C, int* ctr_claim, int* ctr_done,
+                             uint32_t merged, int K, int Hq, int Hkv, int R, const float* __restrict__ part_o,
+                             const float* __restrict__ part_ml, __nv_bfloat16* __restrict__ O,
                              float* __restrict__ lse) {
-  const MergeScratch sc = merge_scratch<D, STAGES>(smem);
   const int lane = threadIdx.x & 31;
-  constexpr int C4 = D / 4;
   const int g = Hq / Hkv;
   const int hi = (layer + 1) * C;
   for (;;) {
@@ -504,45 +540,22 @@ __device__ void merge_chunks(uint8_t* smem, int layer, const MergeTask* tasks, i
     }
     u = __shfl_sync(0xffffffffu, u, 0);
     if (u >= hi) return;
-    // item of this lane: (task, row, float4 column), tasks' items back to back
-    int i = (u - layer * C) * 32 + lane, ti = 0, off = 0;
-    bool live = false;
-    int nr = 0, u0 = 0;
+    // the chunk's task and its index within the task
+    int lc = u - layer * C, ti = 0, u0 = 0, nr = 0;
     for (; ti < n_tasks; ++ti) {
-      const MergeTask& t = tasks[ti];
-      const int k_me = (int)blockIdx.x - t.c0;
-      u0 = (int)((long long)t.rows * k_me / t.np);
-      nr = (int)((long long)t.rows * (k_me + 1) / t.np) - u0;
-      if (i < nr * C4) {
-        live = true;
-        break;
-      }
-      i -= nr * C4;
-      off += nr * t.np;
+      nr = merge_share(tasks[ti], u0);
+      const int ci = 32 * merge_j(tasks[ti].np);
+      const int nc = (nr * (D / 4) + ci - 1) / ci;
+      if (lc < nc) break;
+      lc -= nc;
     }
-    if (live) {
+    if (ti < n_tasks) {
       const MergeTask& t = tasks[ti];
-      const int r = i / C4, c = i - r * C4, np = t.np, c0 = t.c0;
-      const float* wr = sc.w + off + r * np;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-      for (int p = 0; p < np; ++p) {
-        const size_t slot = (size_t)(p == 0 ? 2 * c0 + 1 : 2 * (c0 + p));
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(part_o + (slot * kAttnRows + u0 + r) * D) + c);
-        const float w = wr[p];
-        acc.x += w * v.x;
-        acc.y += w * v.y;
-        acc.z += w * v.z;
-        acc.w += w * v.w;
+      switch (merge_j(t.np)) {
+        case 1: merge_chunk<1, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse); break;
+        case 2: merge_chunk<2, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse); break;
+        default: merge_chunk<4, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse); break;
       }
-      const float* row = sc.row + 2 * kAttnRows * ti;
-      const float inv = row[r];
-      const int rr = t.mg * R + u0 + r;
-      const int tt = rr / g, hq = t.kvh * g + rr % g;
-      __nv_bfloat16* dst = O + (((size_t)t.b * (K + 1) + tt) * Hq + hq) * D + c * 4;
-      *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-      *reinterpret_cast<__nv_bfloat162*>(dst + 2) = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-      if (lse && c == 0) lse[((size_t)t.b * (K + 1) + tt) * Hq + hq] = row[kAttnRows + r] * kLn2;
     }
     __syncwarp();
     if (lane == 0 && atomicAdd(ctr_done, 1) + 1 == hi) mbar_arrive(merged);
@@ -605,7 +618,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     misc[0] = 0;
     misc[4] = 0;
     misc[5] = 0;
-    misc[6] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == kMmaWarp) {
@@ -655,15 +667,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       }
     }
     if (lane == 0) {
-      int U = 0;  // this CTA's share of rows of its split groups
-      for (int ti = 0; ti < n_tasks; ++ti) {
-        const MergeTask& t = tasks[ti];
-        const int k_me = (int)blockIdx.x - t.c0;
-        U += (int)((long long)t.rows * (k_me + 1) / t.np) - (int)((long long)t.rows * k_me / t.np);
-      }
       misc[1] = n_tasks;
       misc[2] = n_items;
-      misc[3] = (U * (D / 4) + 31) / 32;  // merge chunks of 32 (row, 4-column) items
+      misc[3] = merge_chunk_count<D>(tasks, n_tasks);  // merge chunks per layer
     }
   }
   tc_fence_before();
@@ -672,18 +678,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   const int n_tasks = misc[1], n_items = misc[2], merge_n = misc[3];
   int* merge_claimed = const_cast<int*>(misc) + 4;
   int* merge_done = const_cast<int*>(misc) + 5;
-  // bounded wait until the merge warp has the weights of `layers` layers ready
-  auto weights_ready = [&](int layers) {
-    bool ok = true;
-    if ((threadIdx.x & 31) == 0) {
-      int i = 0;
-      while (misc[6] < layers && i < kMaxWaitIters) {
-        __nanosleep(32);
-        ++i;
-      }
-      ok = misc[6] >= layers;
-      __threadfence_block();  // the weights written before the flag are read after it
-    }
+  // bounded wait until every CTA has finished `layer` (lane 0 polls)
+  auto layer_done = [&](int layer) {
+    bool ok = false;
+    if ((threadIdx.x & 31) == 0) ok = wait_counter(bar_cnt + layer, n_ctas) && !misc[0];
     return __shfl_sync(0xffffffffu, ok, 0) != 0;
   };
   const uint32_t tmem = *tmem_slot;
@@ -1031,10 +1029,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       // (the other parity buffer) must be merged before any CTA may start the
       // next layer and overwrite them: help with what the merge warp has left
       if (layer > 0 && merge_n > 0) {
-        if (weights_ready(layer))
-          merge_chunks<D, STAGES>(smem, layer - 1, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq,
-                                  Hkv, R, part_buf_o + ((layer - 1) & 1) * part_o_stride, set.p[layer - 1].O,
-                                  set.p[layer - 1].lse);
+        merge_chunks<D>(layer - 1, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv, R,
+                        part_buf_o + ((layer - 1) & 1) * part_o_stride,
+                        part_buf_ml + ((layer - 1) & 1) * part_ml_stride, set.p[layer - 1].O, set.p[layer - 1].lse);
         if (warp == 0 && !warp_wait(bMerged, (layer - 1) & 1) && tid == 0) {
           raise_status(status, LIBRASPEC_ST_TIMEOUT);
           misc[0] = 1;
@@ -1052,11 +1049,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
       misc[0] = 1;
     } else if (n_layers > 0 && merge_n > 0) {
-      // help with the last layer's merge
-      if (weights_ready(n_layers))
-        merge_chunks<D, STAGES>(smem, n_layers - 1, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq,
-                                Hkv, R, part_buf_o + ((n_layers - 1) & 1) * part_o_stride, set.p[n_layers - 1].O,
-                                set.p[n_layers - 1].lse);
+      // help with the last layer's merge once its grid barrier has passed
+      const int l = n_layers - 1;
+      if (layer_done(l))
+        merge_chunks<D>(l, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv, R,
+                        part_buf_o + (l & 1) * part_o_stride, part_buf_ml + (l & 1) * part_ml_stride, set.p[l].O,
+                        set.p[l].lse);
     }
   } else if (warp == kMergeWarp) {
     // ======================= merge warp =======================
@@ -1064,19 +1062,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     // barrier), while the softmax warps already run layer l+1.
     bool ok = true;
     for (int layer = 0; layer < n_layers && ok; ++layer) {
-      if (lane == 0) ok = wait_counter(bar_cnt + layer, n_ctas) && !misc[0];
-      ok = __shfl_sync(0xffffffffu, ok, 0);
+      ok = layer_done(layer);
       if (!ok) break;
-      if (merge_n > 0) {
-        merge_weights<D, STAGES>(smem, tasks, n_tasks, part_buf_ml + (layer & 1) * part_ml_stride);
-        if (lane == 0) {
-          __threadfence_block();
-          misc[6] = layer + 1;
-        }
-        __syncwarp();
-        merge_chunks<D, STAGES>(smem, layer, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv,
-                                R, part_buf_o + (layer & 1) * part_o_stride, set.p[layer].O, set.p[layer].lse);
-      }
+      if (merge_n > 0)
+        merge_chunks<D>(layer, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv, R,
+                        part_buf_o + (layer & 1) * part_o_stride, part_buf_ml + (layer & 1) * part_ml_stride,
+                        set.p[layer].O, set.p[layer].lse);
     }
     // every chunk of the last layer is merged (by whichever warp) before the exit count
     if (ok && merge_n > 0 && n_layers > 0) {
