@@ -358,7 +358,6 @@ struct MergeTask {
 };
 
 constexpr int kMaxLayers = kAttnMaxLayers;
-constexpr int kMaxParts = kAttnMaxCtas;  // parts of one split group <= grid size
 
 struct LayerPtrs {
   const __nv_bfloat16* Q;
@@ -424,9 +423,16 @@ __device__ __forceinline__ int merge_share(const MergeTask& t, int& u0) {
   return (int)((long long)t.rows * (k_me + 1) / t.np) - u0;
 }
 
+// Between layers the softmax warps help with a merge of at least this many
+// chunks; a smaller one is left to the merge warp, which keeps cold code off
+// the softmax warps' path from one layer to the next (instruction fetch
+// misses cost about a memory round trip). The last layer's merge, the tail
+// of the launch, is always shared.
+constexpr int kMergeHelpChunks = 8;
+
 // Items per lane in a chunk of a group of np parts: J items x 16/J parts are
 // in flight per batch.
-__device__ __forceinline__ int merge_j(int np) { return np > 8 ? 1 : (np > 4 ? 2 : 4); }
+__device__ __forceinline__ int merge_j(int np) { return np > 4 ? 1 : 4; }
 
 template <int D>
 __device__ __forceinline__ int merge_chunk_count(const MergeTask* tasks, int n_tasks) {
@@ -551,11 +557,8 @@ __device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int
     }
     if (ti < n_tasks) {
       const MergeTask& t = tasks[ti];
-      switch (merge_j(t.np)) {
-        case 1: merge_chunk<1, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse); break;
-        case 2: merge_chunk<2, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse); break;
-        default: merge_chunk<4, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse); break;
-      }
+      if (merge_j(t.np) == 1) merge_chunk<1, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
+      else merge_chunk<4, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
     }
     __syncwarp();
     if (lane == 0 && atomicAdd(ctr_done, 1) + 1 == hi) mbar_arrive(merged);
@@ -860,10 +863,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
     uint32_t item_ctr = 0, tile_ctr = 0;
     bool ok = true;
-    for (int layer = 0; layer < n_layers && ok; ++layer) {
+    // layer n_layers has no items: it only helps with the last layer's merge
+    for (int layer = 0; layer <= n_layers && ok; ++layer) {
+      const bool has_items = layer < n_layers;
       float* part_o = part_buf_o + (layer & 1) * part_o_stride;
       float* part_ml = part_buf_ml + (layer & 1) * part_ml_stride;
-      if (layer > 0) {
+      if (layer > 0 && has_items) {
         // layer's inputs are ready once every CTA is done with the previous layer
         if (tid == 0 && !wait_counter(bar_cnt + (layer - 1), n_ctas)) {
           raise_status(status, LIBRASPEC_ST_TIMEOUT);
@@ -875,9 +880,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           break;
         }
       }
-      __nv_bfloat16* O = set.p[layer].O;
-      float* lse = set.p[layer].lse;
-      for (int item = 0; item < n_items && ok; ++item) {
+      __nv_bfloat16* O = has_items ? set.p[layer].O : nullptr;
+      float* lse = has_items ? set.p[layer].lse : nullptr;
+      for (int item = 0; item < n_items && ok && has_items; ++item) {
         const uint32_t q = item_ctr & 1, ob = item_ctr & 1;
         ok = warp_wait(bQFull + 8 * q, (item_ctr >> 1) & 1);
         if (!ok) break;
@@ -1028,10 +1033,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       // this CTA is done with the layer's items; the previous layer's partials
       // (the other parity buffer) must be merged before any CTA may start the
       // next layer and overwrite them: help with what the merge warp has left
-      if (layer > 0 && merge_n > 0) {
+      // if that is much; after the last layer, help with its merge (the tail
+      // of the launch) once its grid barrier has passed
+      if (layer > 0 && merge_n > 0 && (has_items ? merge_n >= kMergeHelpChunks : layer_done(layer - 1)))
         merge_chunks<D>(layer - 1, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv, R,
-                        part_buf_o + ((layer - 1) & 1) * part_o_stride,
-                        part_buf_ml + ((layer - 1) & 1) * part_ml_stride, set.p[layer - 1].O, set.p[layer - 1].lse);
+                        part_buf_o + ((layer - 1) & 1) * part_o_stride, part_buf_ml + ((layer - 1) & 1) * part_ml_stride,
+                        set.p[layer - 1].O, set.p[layer - 1].lse);
+      if (!has_items) break;
+      if (layer > 0 && merge_n > 0) {
         if (warp == 0 && !warp_wait(bMerged, (layer - 1) & 1) && tid == 0) {
           raise_status(status, LIBRASPEC_ST_TIMEOUT);
           misc[0] = 1;
@@ -1048,13 +1057,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     if (!ok) {
       if (lane == 0) raise_status(status, LIBRASPEC_ST_TIMEOUT);
       misc[0] = 1;
-    } else if (n_layers > 0 && merge_n > 0) {
-      // help with the last layer's merge once its grid barrier has passed
-      const int l = n_layers - 1;
-      if (layer_done(l))
-        merge_chunks<D>(l, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv, R,
-                        part_buf_o + (l & 1) * part_o_stride, part_buf_ml + (l & 1) * part_ml_stride, set.p[l].O,
-                        set.p[l].lse);
     }
   } else if (warp == kMergeWarp) {
     // ======================= merge warp =======================
