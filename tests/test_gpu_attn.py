@@ -68,6 +68,34 @@ def test_attn_long_split_kv_merge(orc, kv):
     check_attn(O, lse, O_ref, lse_ref, L)
 
 
+@pytest.mark.parametrize("kv", [300, 20000])
+@pytest.mark.parametrize("Hq,Hkv,d,L", [(32, 8, 128, 7), (32, 8, 64, 3), (64, 8, 128, 3), (8, 8, 128, 16),
+                                        (32, 8, 128, 12)])
+def test_attn_small_groups_long_cache(orc, kv, Hq, Hkv, d, L):
+    """Row groups of 16 to 52 rows (a few block positions of g heads) over a
+    short and a long cache: one CTA per group, and groups split over many
+    CTAs whose parts are merged."""
+    K = 16
+    Q, Kc, Vc = _inputs(1, K, Hq, Hkv, d, [kv], kv + K + 1, seed=kv + Hq + L, scale_k=2.0)
+    O, lse = _run(Q, Kc, Vc, [kv], [L], K)
+    O_ref, lse_ref = orc.verify_attn(Q, Kc, Vc, np.array([kv]), np.array([L]))
+    check_attn(O, lse, O_ref, lse_ref, [L])
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_attn_small_groups_ragged(orc, d):
+    """Several sequences with small row groups of different sizes, some
+    covered by one CTA, some split."""
+    K, Hq, Hkv = 9, 32, 8
+    kv = [0, 3000, 64, 700, 9000]
+    L = [7, 0, 3, 5, 1]
+    S_cap = max(k + l + 1 for k, l in zip(kv, L)) + 3
+    Q, Kc, Vc = _inputs(len(kv), K, Hq, Hkv, d, kv, S_cap, seed=d + 5, scale_k=2.0)
+    O, lse = _run(Q, Kc, Vc, kv, L, K)
+    O_ref, lse_ref = orc.verify_attn(Q, Kc, Vc, np.array(kv), np.array(L))
+    check_attn(O, lse, O_ref, lse_ref, L)
+
+
 def test_attn_peaky_scores(orc):
     w = workloads.WORKLOADS["sampling"].scaled(B=4, kv=("uniform", 100, 3000))
     kv = workloads.kv_lengths(w)
@@ -159,14 +187,15 @@ def test_attn_many_sequences_stream_k_ranges(orc, B, kv_hi, d, seed):
         check_attn(O, lse, O_ref, lse_ref, L, rows=[tuple(r) for r in rows])
 
 
-@pytest.mark.parametrize("name,n_layers", [("8b", 4), ("sampling", 3), ("tiny", 3)])
-def test_attn_layer_chain_matches_per_layer_oracle(orc, name, n_layers):
+@pytest.mark.parametrize("name,n_layers,L_max", [("8b", 4, None), ("sampling", 3, None), ("tiny", 3, None),
+                                                 ("8b", 3, 4)])
+def test_attn_layer_chain_matches_per_layer_oracle(orc, name, n_layers, L_max):
     """libraspec_verify_attn_layers: all layers in one persistent launch; each
     layer's split groups are merged after the grid barrier that ends it."""
     w = workloads.WORKLOADS[name]
     kv = workloads.kv_lengths(w)
     rng = np.random.default_rng(7)
-    L = rng.integers(0, w.K + 1, size=w.B).astype(np.int32)
+    L = rng.integers(0, (L_max if L_max is not None else w.K) + 1, size=w.B).astype(np.int32)
     layers = [workloads.layer(w, l, kv, device=cuda()) for l in range(n_layers)]
     S = layers[0]["Kc"].shape[2]
     ws = lr.Workspace(w.B, w.K, 1, w.Hq, w.Hkv, w.d, S, device=cuda())
