@@ -58,9 +58,10 @@ def _load():
     lib.oracle_confidence.argtypes = [P, P, P, i32, i32, i32, P, P]
     lib.oracle_select_lengths.argtypes = [P, P, i32, i32, f64, P, P]
     lib.oracle_select_iterate.argtypes = [P, P, i32, f64, i32, P, i32]
+    lib.oracle_select_alpha.argtypes = [P, i32, i32, i32, f64, P, P, P]
     lib.oracle_verify_attn.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, i32, f64, P, P, P, i32]
     lib.oracle_accept.argtypes = [P, P, P, P, P, i32, i32, i32, u64, u64, u32, P, P, P]
-    for name in ("oracle_confidence", "oracle_select_lengths", "oracle_select_iterate",
+    for name in ("oracle_confidence", "oracle_select_lengths", "oracle_select_iterate", "oracle_select_alpha",
                  "oracle_verify_attn", "oracle_accept"):
         getattr(lib, name).restype = i32
     _lib = lib
@@ -147,6 +148,18 @@ def select_iterate(q, cost_table, start: int, e0: float = 1.0):
     n = _check(_load().oracle_select_iterate(_ptr(qq), _ptr(cost), K, float(e0), int(start),
                                              _ptr(path), cap), "oracle_select_iterate")
     return [int(v) for v in path[:n]]
+
+
+def select_alpha(conf, n: int, alpha: float):
+    """Algorithm 1's alpha-mode search: L[B], blocks drafted[B], flag[B] (int32)."""
+    q = _c(conf, np.float64)
+    B, K = q.shape
+    L = np.zeros(B, np.int32)
+    blocks = np.zeros(B, np.int32)
+    flag = np.zeros(B, np.int32)
+    _check(_load().oracle_select_alpha(_ptr(q), B, K, int(n), float(alpha), _ptr(L), _ptr(blocks), _ptr(flag)),
+           "oracle_select_alpha")
+    return L, blocks, flag
 
 
 def verify_attn(Q, Kc, Vc, kv_len, L, scale=None, rows=None, fill=np.nan):

@@ -18,6 +18,10 @@
  *                          cumulative products, proof of Thm. 2).
  *   oracle_select_iterate  iterated single beneficial adjustments (Def. 1,
  *                          Thm. 1 both cases, Thm. 5) from any start length.
+ *   oracle_select_alpha    the alpha-mode length search of Algorithm 1:
+ *                          position-wise bounds eps_i (Thm. 2 / Thm. 3 with
+ *                          the trade-off weight alpha), eps* = min_i eps_i,
+ *                          block-wise drafting budget, one rollback.
  *   oracle_verify_attn     block-causal GQA attention of the d+1 verified
  *                          positions against the target KV cache (Sec. 3.1:
  *                          the target scores all drafted positions in one
@@ -292,6 +296,77 @@ int oracle_select_iterate(const double* q, const double* cost_table, int K, doub
     path[n++] = d;
   }
   return n;
+}
+
+/* ------------------------------------------------------------------ */
+/* Alpha-mode length search (Algorithm 1, Sec. 3.3; Thm. 2 and Thm. 3 */
+/* give the position-wise bounds it evaluates, alpha = 2.0 / 2.2 in    */
+/* Sec. 4).                                                            */
+/*                                                                     */
+/* With q_k the drafter confidence of position k (1-based, q_k =       */
+/* conf[b, k-1]) and the current length d:                              */
+/*   eps_i = floor(alpha * sum_{j=i}^{d} prod_{k=i}^{j} q_k + i),       */
+/*           i = 1 .. d,   eps* = min_i eps_i.                          */
+/* Starting from one drafted block, d = n, budget B = 0, while          */
+/* d < d_max: if eps* <= d, d = eps* and stop (the single rollback);    */
+/* otherwise B -= eps* - d, d = eps*, and when B < 0 ceil(-B/n) more    */
+/* blocks are drafted and B += ceil(-B/n) * n. d tokens are verified.  */
+/* Readings of points the algorithm leaves open:                        */
+/*  * the floor form of Algorithm 1 is used as printed (the theorems'   */
+/*    strict "<" bound would give ceil(x) - 1; the two differ only when */
+/*    alpha*S_i + i is an integer, which is flagged);                  */
+/*  * the sum runs to the current d, as in Algorithm 1;                 */
+/*  * eps* above d_max is clamped to d_max (the loop then ends);        */
+/*  * the first block holds n <= d_max positions (1 <= n <= d_max);     */
+/*  * q_k of every position up to d_max is given: the search only ever  */
+/*    reads q_1 .. q_d of the current d, so this matches drafting the   */
+/*    blocks on demand; blocks_out counts the blocks drafted.          */
+/* The sums are written out as the definition reads (a fresh product   */
+/* for every j). A sequence is flagged when some alpha*S_i + i lies     */
+/* within a relative 1e-6 of an integer (there floor is ambiguous      */
+/* between binary64 evaluations in different orders).                  */
+/* ------------------------------------------------------------------ */
+int oracle_select_alpha(const double* conf, int B, int K, int n, double alpha, int32_t* L_out,
+                        int32_t* blocks_out, int32_t* flag_out) {
+  if (B < 0 || K < 1 || n < 1 || n > K || !conf || !L_out || !(alpha > 0.0) || !isfinite(alpha))
+    return ORACLE_EINVAL;
+  for (int b = 0; b < B; ++b) {
+    const double* q = conf + (size_t)b * K; /* q_k = q[k - 1] */
+    int d = n, blocks = 1, flag = 0;
+    long budget = 0;
+    while (d < K) {
+      long eps_star = 0;
+      for (int i = 1; i <= d; ++i) {
+        double S = 0.0;
+        for (int j = i; j <= d; ++j) {
+          double P = 1.0;
+          for (int k = i; k <= j; ++k) P = P * q[k - 1];
+          S = S + P;
+        }
+        const double x = alpha * S + (double)i;
+        const double fl = floor(x);
+        if (fabs(x - nearbyint(x)) <= FLAG_REL * fmax(1.0, fabs(x))) flag = 1;
+        const long eps_i = (long)fl;
+        if (i == 1 || eps_i < eps_star) eps_star = eps_i;
+      }
+      if (eps_star <= d) {
+        d = (int)eps_star; /* the single rollback */
+        break;
+      }
+      if (eps_star > K) eps_star = K;
+      budget -= eps_star - d;
+      d = (int)eps_star;
+      if (budget < 0) {
+        const long more = (-budget + n - 1) / n;
+        blocks += (int)more;
+        budget += more * n;
+      }
+    }
+    L_out[b] = d;
+    if (blocks_out) blocks_out[b] = blocks;
+    if (flag_out) flag_out[b] = flag;
+  }
+  return ORACLE_OK;
 }
 
 /* ------------------------------------------------------------------ */
