@@ -43,6 +43,11 @@ def parse():
     p.add_argument("--e2e-steps", type=int, default=50)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle sample")
+    p.add_argument("--selector", default="gain", choices=["gain", "alpha"],
+                   help="gain: the Thm. 4 marginal-gain scan; alpha: Algorithm 1's alpha-mode search")
+    p.add_argument("--alpha", type=float, default=2.2, help="alpha of the alpha-mode search (Sec. 4: 2.2)")
+    p.add_argument("--block-size", type=int, default=0,
+                   help="first drafted block of the alpha-mode search (0: 2/3 of K, as 16 of d_max 24)")
     return p.parse_args()
 
 
@@ -271,10 +276,16 @@ def run_ours(args, rank, world, local_rank):
     n_acc = torch.empty((w.B,), dtype=torch.int32, device=dev)
     bonus = torch.empty((w.B,), dtype=torch.int32, device=dev)
 
+    block_size = args.block_size if args.block_size > 0 else max(1, (2 * w.K) // 3)
+    n_blocks = torch.empty((w.B,), dtype=torch.int32, device=dev)
+
     def seg_select():
         lr.libraspec_confidence(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], ws, conf=conf,
                                 dstat=dstat)
-        lr.libraspec_select_lengths(conf, cost, ws, L=L)
+        if args.selector == "alpha":
+            lr.libraspec_select_alpha(conf, block_size, args.alpha, L=L, n_blocks=n_blocks)
+        else:
+            lr.libraspec_select_lengths(conf, cost, ws, L=L)
 
     def seg_attn():
         lr.libraspec_verify_attn_layers(layers, kv_t, L, ws)
@@ -379,6 +390,8 @@ def run_ours(args, rank, world, local_rank):
         "config": {"workload": w.name, "B": w.B, "K": w.K, "V": w.V, "layers": w.n_layers,
                    "resident_kv_layers": n_res, "gqa": "%d/%d" % (w.Hq, w.Hkv), "head_dim": w.d,
                    "kv_len": [int(kv.min()), int(kv.max())], "selected_L": [int(Lh.min()), int(Lh.max())],
+                   "selector": ("alpha (Algorithm 1, alpha %g, first block %d)" % (args.alpha, block_size)
+                                if args.selector == "alpha" else "marginal gain (Thm. 4)"),
                    "parallelism": "dp%d (independent sequences)" % world,
                    "l2": "no flush: %.0f MB of distinct inputs per step > 129 MB L2" % (by["total"] / 1e6),
                    "timing": "3 CUDA graphs per step (conf+select | attention layers | accept), events between"},

@@ -155,6 +155,31 @@ int libraspec_select_lengths(const float* conf, const float* cost_table, int B, 
                              void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * Step 2, alpha mode — the length search of the paper's Algorithm 1 (its
+ * position-wise bounds are Thm. 2 and Thm. 3 with the trade-off weight
+ * alpha; Sec. 4 uses alpha = 2.0 for FastdLLM and 2.2 for DFlash / DDTree,
+ * block size 16 and d_max = 24 for the latter two).
+ *
+ * With q_k = conf[b, k-1] (k = 1 .. K, K = d_max) and the current length d,
+ *     eps_i = floor(alpha * sum_{j=i}^{d} prod_{k=i}^{j} q_k + i),  i = 1..d,
+ *     eps*  = min_i eps_i.
+ * Starting from one drafted block, d = block_size and a budget of 0 drafted
+ * but unused tokens, while d < K: if eps* <= d then d = eps* and the search
+ * stops (the single rollback); otherwise the budget drops by eps* - d,
+ * d = min(eps*, K), and when the budget is negative ceil(-budget /
+ * block_size) more blocks are drafted (each adds block_size to it).
+ * L[b] = d, the number of draft tokens to verify (1 .. K); n_blocks[b] (if
+ * not NULL) = the blocks drafted. The search reads only q_1 .. q_d of the
+ * current d, so giving all K confidences up front matches drafting blocks
+ * on demand. Computed in binary64; eps* above K is clamped to K.
+ * conf [B,K] f32 (finite, in [0,1]), L and n_blocks [B] i32, device
+ * pointers; 1 <= block_size <= K <= LIBRASPEC_MAX_K, alpha > 0 and finite,
+ * else LIBRASPEC_EINVAL. One warp per sequence; no workspace.
+ */
+int libraspec_select_alpha(const float* conf, int B, int K, int block_size, float alpha, int32_t* L,
+                           int32_t* n_blocks, void* stream);
+
+/*
  * Step 3 — block-causal GQA verify attention, one layer (paper Sec. 3.1:
  * the target scores all drafted positions in one forward pass).
  *

@@ -32,6 +32,7 @@ SIGNATURES = {
     "libraspec_confidence": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "libraspec_confidence_noalloc": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P]),
     "libraspec_select_lengths": (_I, [_P, _P, _I, _I, _P, _P, _SZ, _P]),
+    "libraspec_select_alpha": (_I, [_P, _I, _I, _I, _F, _P, _P, _P]),
     "libraspec_verify_attn": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_attn_layers": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
@@ -184,6 +185,21 @@ def libraspec_select_lengths(conf, cost_table, ws: Workspace, L=None, stream=Non
                                          _stream(stream))
     _check(rc, "libraspec_select_lengths")
     return L
+
+
+def libraspec_select_alpha(conf, block_size: int, alpha: float, L=None, n_blocks=None, stream=None):
+    """Algorithm 1's alpha-mode search: L[B] and blocks drafted[B] (int32, device)."""
+    B, K = conf.shape
+    _req(conf, torch.float32, "conf")
+    L = torch.empty((B,), dtype=torch.int32, device=conf.device) if L is None else _req(L, torch.int32, "L", (B,))
+    if n_blocks is None:
+        n_blocks = torch.empty((B,), dtype=torch.int32, device=conf.device)
+    else:
+        _req(n_blocks, torch.int32, "n_blocks", (B,))
+    rc = load().libraspec_select_alpha(_ptr(conf), B, K, int(block_size), float(alpha), _ptr(L), _ptr(n_blocks),
+                                       _stream(stream))
+    _check(rc, "libraspec_select_alpha")
+    return L, n_blocks
 
 
 def libraspec_verify_attn(Q, Kc, Vc, kv_len, L, ws: Workspace, softmax_scale=None, O=None, lse=None,

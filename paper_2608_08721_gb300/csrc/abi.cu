@@ -11,6 +11,7 @@ namespace libraspec {
 cudaError_t launch_confidence(const float*, const int32_t*, const float*, int, int, int, float*, float*, char*,
                               const WsLayout&, cudaStream_t);
 cudaError_t launch_select(const float*, const float*, int, int, int32_t*, char*, const WsLayout&, cudaStream_t);
+cudaError_t launch_select_alpha(const float*, int, int, int, double, int32_t*, int32_t*, cudaStream_t);
 cudaError_t launch_verify_attn(const uint16_t*, const uint16_t*, const uint16_t*, const int32_t*, const int32_t*,
                                int, int, int, int, int, int, float, uint16_t*, float*, char*, const WsLayout&,
                                cudaStream_t);
@@ -128,6 +129,16 @@ int libraspec_select_lengths(const float* conf, const float* cost_table, int B, 
   if (!workspace || !aligned(workspace, 256) || ws_bytes < 256) return LIBRASPEC_EINVAL;
   return from_cuda(
       launch_select(conf, cost_table, B, K, L, static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+}
+
+int libraspec_select_alpha(const float* conf, int B, int K, int block_size, float alpha, int32_t* L,
+                           int32_t* n_blocks, void* stream) {
+  if (B < 0 || K < 1 || K > LIBRASPEC_MAX_K || block_size < 1 || block_size > K) return LIBRASPEC_EINVAL;
+  if (!(alpha > 0.f) || !isfinite(alpha)) return LIBRASPEC_EINVAL;
+  if (B == 0) return LIBRASPEC_OK;
+  if (!conf || !L) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_select_alpha(conf, B, K, block_size, (double)alpha, L, n_blocks,
+                                       static_cast<cudaStream_t>(stream)));
 }
 
 int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc, const int32_t* kv_len,

@@ -141,6 +141,84 @@ __global__ void __launch_bounds__(128) select_kernel(const float* __restrict__ c
 }
 
 // ---------------------------------------------------------------------------
+// Alpha-mode length search (Algorithm 1), one warp per sequence, binary64.
+// eps_i = floor(alpha * S_i + i) with S_i = sum_{j=i}^{d} prod_{k=i}^{j} q_k,
+// eps* = min_i eps_i. S_i = q_i (1 + S_{i+1}), S_{d+1} = 0: lane i-1 holds
+// the affine map x -> q_i + q_i x and a suffix scan of map compositions
+// gives every S_i at once (positions 33..64 in a second chunk whose S_33
+// feeds the first). From d = n: eps* <= d rolls back once and stops, else
+// d = min(eps*, K) and ceil(-budget/n) blocks are drafted when the budget
+// of drafted-but-unused tokens turns negative.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void suffix_compose(double& a, double& b) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const double ao = __shfl_down_sync(0xffffffffu, a, off);
+    const double bo = __shfl_down_sync(0xffffffffu, b, off);
+    if (lane + off < 32) {
+      b = __dadd_rn(__dmul_rn(a, bo), b);  // (this map) o (the maps after it)
+      a = __dmul_rn(a, ao);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(128) select_alpha_kernel(const float* __restrict__ conf, int B, int K, int n,
+                                                           double alpha, int32_t* __restrict__ L,
+                                                           int32_t* __restrict__ n_blocks) {
+  const int seq = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (seq >= B) return;
+  const float* q = conf + (size_t)seq * K;
+  const double q0 = lane < K ? (double)q[lane] : 0.0;            // q_{lane+1}
+  const double q1 = lane + 32 < K ? (double)q[lane + 32] : 0.0;  // q_{lane+33}
+  int d = n, blocks = 1;
+  int budget = 0;
+  while (d < K) {
+    int best = K + 1;
+    double carry = 0.0;  // S_33
+    if (d > 32) {
+      const bool live = lane + 33 <= d;
+      double a = live ? q1 : 1.0, b = live ? q1 : 0.0;
+      suffix_compose(a, b);
+      carry = __shfl_sync(0xffffffffu, b, 0);
+      if (live) {
+        const double x = __dadd_rn(__dmul_rn(alpha, b), (double)(lane + 33));
+        const double f = floor(x);
+        best = min(best, f >= (double)(K + 1) ? K + 1 : (f >= 1.0 ? (int)f : 1));
+      }
+    }
+    const bool live = lane + 1 <= d;
+    double a = live ? q0 : 1.0, b = live ? q0 : 0.0;
+    suffix_compose(a, b);
+    if (live) {
+      const double S = __dadd_rn(__dmul_rn(a, carry), b);
+      const double x = __dadd_rn(__dmul_rn(alpha, S), (double)(lane + 1));
+      const double f = floor(x);
+      best = min(best, f >= (double)(K + 1) ? K + 1 : (f >= 1.0 ? (int)f : 1));
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) best = min(best, __shfl_xor_sync(0xffffffffu, best, off));
+    if (best <= d) {
+      d = best;  // the single rollback
+      break;
+    }
+    if (best > K) best = K;
+    budget -= best - d;
+    d = best;
+    if (budget < 0) {
+      const int more = (-budget + n - 1) / n;
+      blocks += more;
+      budget += more * n;
+    }
+  }
+  if (lane == 0) {
+    L[seq] = d;
+    if (n_blocks) n_blocks[seq] = blocks;
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Host launchers (arguments already validated by the ABI layer).
 // ---------------------------------------------------------------------------
 int num_sms_current();
@@ -164,6 +242,15 @@ cudaError_t launch_confidence(const float* x, const int32_t* tokens, const float
   else
     conf_kernel<false><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
                                                          dstat, part, cnt, st);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select_alpha(const float* conf, int B, int K, int n, double alpha, int32_t* L,
+                                int32_t* n_blocks, cudaStream_t stream) {
+  if (B == 0) return cudaSuccess;
+  const int threads = 128;
+  const int blocks = (B * 32 + threads - 1) / threads;
+  select_alpha_kernel<<<blocks, threads, 0, stream>>>(conf, B, K, n, alpha, L, n_blocks);
   return cudaGetLastError();
 }
 

@@ -1,0 +1,90 @@
+"""GPU parity: Algorithm 1's alpha-mode length search vs. the oracle.
+
+L and the blocks drafted are integers: bit-exact on every sequence the
+oracle does not flag (a bound alpha*S_i + i within 1e-6 of an integer)."""
+import numpy as np
+import pytest
+import torch
+
+from helpers import assert_exact_unless_flagged, cuda
+from paper_2608_08721_gb300 import binding as lr
+from paper_2608_08721_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def _conf(kind, B, K, rng):
+    if kind == "uniform":
+        q = rng.uniform(0.0, 1.0, size=(B, K))
+    elif kind == "confident":  # mostly high with occasional drops, as a good drafter gives
+        q = 1.0 - rng.uniform(0.0, 1.0, size=(B, K)) ** 4
+        drop = rng.uniform(size=(B, K)) < 0.08
+        q[drop] = rng.uniform(0.0, 0.3, size=int(drop.sum()))
+    elif kind == "decaying":  # confidence falling along the block
+        q = np.clip(rng.uniform(0.85, 1.0, size=(B, 1)) * np.exp(-np.arange(K) / rng.uniform(4, 40, size=(B, 1))),
+                    0.0, 1.0)
+    else:
+        raise ValueError(kind)
+    return q.astype(np.float32)
+
+
+def _check(orc, q, n, alpha):
+    conf = torch.from_numpy(q).to(cuda())
+    L, blocks = lr.libraspec_select_alpha(conf, n, alpha)
+    torch.cuda.synchronize()
+    L_ref, b_ref, flag = orc.select_alpha(q.astype(np.float64), n, alpha)
+    nf = assert_exact_unless_flagged(L.cpu().numpy(), L_ref, flag, "L")
+    assert_exact_unless_flagged(blocks.cpu().numpy(), b_ref, flag, "blocks")
+    return nf
+
+
+@pytest.mark.parametrize("K", [1, 8, 16, 24, 32, 33, 40, 64])
+@pytest.mark.parametrize("kind", ["uniform", "confident", "decaying"])
+@pytest.mark.parametrize("alpha", [0.5, 2.0, 2.2, 4.0])
+def test_select_alpha_random(orc, K, kind, alpha):
+    rng = np.random.default_rng(K * 131 + int(alpha * 10))
+    B = 700
+    q = _conf(kind, B, K, rng)
+    for n in sorted({1, max(1, K // 3), min(16, K), K}):
+        nf = _check(orc, q, n, alpha)
+        # flags come from bounds that are exact integers (q = 1.0 in float32
+        # runs, alpha = 2); most sequences must still be compared
+        assert nf <= B // 4, "too many flagged sequences (%d)" % nf
+
+
+@pytest.mark.parametrize("K,n", [(24, 16), (16, 10), (32, 16), (64, 7)])
+def test_select_alpha_degenerate_confidences(orc, K, n):
+    zeros = np.zeros((3, K), np.float32)
+    ones = np.ones((3, K), np.float32)
+    L, blocks = lr.libraspec_select_alpha(torch.from_numpy(zeros).to(cuda()), n, 2.2)
+    assert L.cpu().tolist() == [1, 1, 1] and blocks.cpu().tolist() == [1, 1, 1]
+    L, blocks = lr.libraspec_select_alpha(torch.from_numpy(ones).to(cuda()), n, 2.2)
+    assert L.cpu().tolist() == [K] * 3 and blocks.cpu().tolist() == [-(-K // n)] * 3
+    # one block of ones then zeros: the rollback lands one past the block (see the oracle pins)
+    q = np.array([[1.0] * n + [0.0] * (K - n)], np.float32)
+    L, blocks = lr.libraspec_select_alpha(torch.from_numpy(q).to(cuda()), n, 2.0)
+    L_ref, b_ref, _ = orc.select_alpha(q.astype(np.float64), n, 2.0)
+    assert (int(L.item()), int(blocks.item())) == (int(L_ref[0]), int(b_ref[0]))
+
+
+@pytest.mark.parametrize("name", ["8b", "sampling", "ragged", "70b"])
+def test_select_alpha_on_drafter_confidences(orc, name):
+    """The workload's drafter logits through the confidence kernel, then the
+    alpha search with the paper's DFlash setting scaled to the block length
+    (alpha 2.2, first block 2/3 of d_max, as 16 of 24)."""
+    w = workloads.WORKLOADS[name]
+    inp = workloads.logits(w, device=cuda())
+    ws = lr.Workspace(w.B, w.K, w.V, device=cuda())
+    conf, _ = lr.libraspec_confidence(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], ws)
+    torch.cuda.synchronize()
+    q = conf.cpu().numpy()
+    _check(orc, q, max(1, (2 * w.K) // 3), 2.2)
+
+
+def test_select_alpha_empty_and_invalid():
+    conf = torch.full((4, 8), 0.5, device=cuda())
+    L, _ = lr.libraspec_select_alpha(conf[:0], 4, 2.2)
+    assert L.numel() == 0
+    for n, alpha in [(0, 2.2), (9, 2.2), (4, 0.0), (4, float("nan"))]:
+        with pytest.raises(lr.LibraspecError):
+            lr.libraspec_select_alpha(conf, n, alpha)
