@@ -43,6 +43,8 @@ def parse():
     p.add_argument("--e2e-steps", type=int, default=50)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle sample")
+    p.add_argument("--logits", default="f32", choices=["f32", "bf16"],
+                   help="dtype of the drafter and target logits (bf16: libraspec_*_bf16, half the bytes)")
     p.add_argument("--selector", default="gain", choices=["gain", "alpha"],
                    help="gain: the Thm. 4 marginal-gain scan; alpha: Algorithm 1's alpha-mode search")
     p.add_argument("--alpha", type=float, default=2.2, help="alpha of the alpha-mode search (Sec. 4: 2.2)")
@@ -133,12 +135,12 @@ def physical_gpu(local_rank):
 # ---------------------------------------------------------------------------
 # algorithmic bytes (what the method must move)
 # ---------------------------------------------------------------------------
-def round_bytes(w, kv, L, temperature, n_acc):
-    conf = w.B * w.K * w.V * 4
+def round_bytes(w, kv, L, temperature, n_acc, logit_bytes=4):
+    conf = w.B * w.K * w.V * logit_bytes
     select = w.B * w.K * 4 + (w.K + 1) * 4
-    accept = float(np.sum((L + 1).astype(np.int64) * w.V * 4))
+    accept = float(np.sum((L + 1).astype(np.int64) * w.V * logit_bytes))
     rejected_sampling = np.sum((n_acc < L) & (temperature > 0))
-    accept += float(rejected_sampling) * 2 * w.V * 4
+    accept += float(rejected_sampling) * 2 * w.V * logit_bytes
     from paper_2608_08721_gb300 import workloads
 
     attn_launch = workloads.attn_bytes(w, kv, L)
@@ -258,6 +260,9 @@ def run_ours(args, rank, world, local_rank):
     kv = workloads.kv_lengths(w)
     seq_offset = rank * w.B  # weak scaling: each rank verifies its own B sequences
     inp = workloads.logits(w, device=dev)
+    if args.logits == "bf16":  # as an engine's LM head emits them
+        inp["draft_logits"] = inp["draft_logits"].to(torch.bfloat16)
+        inp["target_logits"] = inp["target_logits"].to(torch.bfloat16)
     n_res = w.resident_layers if w.resident_layers else w.n_layers
     S = workloads.s_cap(w, kv)
     caches = [workloads.layer(w, l, kv, device=dev) for l in range(n_res)]
@@ -353,7 +358,7 @@ def run_ours(args, rank, world, local_rank):
     Lh = L.cpu().numpy()
     nh = n_acc.cpu().numpy()
     temp = inp["temperature"].cpu().numpy()
-    by = round_bytes(w, kv, Lh, temp, nh)
+    by = round_bytes(w, kv, Lh, temp, nh, logit_bytes=2 if args.logits == "bf16" else 4)
     us_per_round = elapsed_ms * 1000.0 / K_steps
     # one persistent attention launch runs up to ATTN_LAYERS_PER_LAUNCH layers
     attn_launches = -(-w.n_layers // ATTN_LAYERS_PER_LAUNCH)
@@ -392,6 +397,7 @@ def run_ours(args, rank, world, local_rank):
                    "kv_len": [int(kv.min()), int(kv.max())], "selected_L": [int(Lh.min()), int(Lh.max())],
                    "selector": ("alpha (Algorithm 1, alpha %g, first block %d)" % (args.alpha, block_size)
                                 if args.selector == "alpha" else "marginal gain (Thm. 4)"),
+                   "logits": args.logits,
                    "parallelism": "dp%d (independent sequences)" % world,
                    "l2": "no flush: %.0f MB of distinct inputs per step > 129 MB L2" % (by["total"] / 1e6),
                    "timing": "3 CUDA graphs per step (conf+select | attention layers | accept), events between"},
@@ -423,7 +429,7 @@ def run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset):
     n_res = len({id(l["Kc"]) for l in layers})
     caches = [{"Kc": l["Kc"], "Vc": l["Vc"]} for l in layers]
     runner = VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, layers[0]["Kc"].shape[2], caches, torch.tensor(kv),
-                         device=dev)
+                         device=dev, logits_dtype=inp["draft_logits"].dtype)
     K1 = w.K + 1
     host = {k: v.cpu().pin_memory() for k, v in inp.items()}
     host["cost_table"] = cost.cpu().pin_memory()

@@ -112,6 +112,17 @@ int libraspec_confidence(const float* draft_logits, const int32_t* draft_tokens,
                          void* stream);
 
 /*
+ * libraspec_confidence on bf16 logits (the 16-bit patterns, as an engine's
+ * LM head emits them): each logit widens to fp32 exactly, then the same
+ * fp32 / binary64 arithmetic runs on the widened values. Half the bytes:
+ * B*K*V*2. draft_logits must be 2-byte aligned; rows whose start is 16-byte
+ * aligned with V % 8 == 0 stream in 128-bit loads.
+ */
+int libraspec_confidence_bf16(const uint16_t* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                              int B, int K, int V, float* conf, float* dstat, void* workspace, size_t ws_bytes,
+                              void* stream);
+
+/*
  * libraspec_confidence without a workspace, for callers that cannot allocate
  * device memory. The paper has no counterpart: this is an integration
  * variant of Step 1 with the same results (the same kernels run).
@@ -261,6 +272,17 @@ int libraspec_accept(const float* target_logits, const float* draft_logits, cons
                      int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * libraspec_accept on bf16 target and drafter logits (16-bit patterns,
+ * widened to fp32 exactly; same arithmetic and generator). conf and dstat
+ * come from libraspec_confidence_bf16 on the same drafter logits.
+ */
+int libraspec_accept_bf16(const uint16_t* target_logits, const uint16_t* draft_logits, const int32_t* draft_tokens,
+                          const float* conf, const float* dstat, const int32_t* L, const float* temperature, int B,
+                          int K, int V, uint64_t seed, uint64_t round_offset, uint32_t seq_offset,
+                          int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                          void* stream);
+
+/*
  * The whole round on one stream: confidence -> selection -> n_layers verify
  * attention layers -> acceptance. Q, Kc, Vc, O point to HOST arrays of
  * n_layers DEVICE pointers (layer l uses Q[l], Kc[l], Vc[l], O[l]); lse is a
@@ -275,6 +297,17 @@ int libraspec_verify_round(const float* draft_logits, const int32_t* draft_token
                            uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
                            int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
                            void* stream);
+
+/* libraspec_verify_round on bf16 drafter and target logits (the _bf16 forms
+ * of steps 1 and 4; selection and attention unchanged). */
+int libraspec_verify_round_bf16(const uint16_t* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                                const float* cost_table, const uint16_t* target_logits, const uint16_t* const* Q,
+                                const uint16_t* const* Kc, const uint16_t* const* Vc, uint16_t* const* O,
+                                float* const* lse, int n_layers, const int32_t* kv_len, int B, int K, int V, int Hq,
+                                int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                                uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
+                                int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                                void* stream);
 
 #ifdef __cplusplus
 }

@@ -20,8 +20,12 @@ from . import binding
 
 class VerifyRound:
     def __init__(self, B: int, K: int, V: int, Hq: int, Hkv: int, head_dim: int, S_cap: int,
-                 caches: List[Dict[str, torch.Tensor]], kv_len: torch.Tensor, device=None):
-        """caches: per layer {"Kc", "Vc"} bf16 [B,Hkv,S_cap,d] on the device."""
+                 caches: List[Dict[str, torch.Tensor]], kv_len: torch.Tensor, device=None,
+                 logits_dtype=torch.float32):
+        """caches: per layer {"Kc", "Vc"} bf16 [B,Hkv,S_cap,d] on the device;
+        logits_dtype: float32 or bfloat16 drafter and target logits."""
+        if logits_dtype not in (torch.float32, torch.bfloat16):
+            raise ValueError("logits_dtype must be torch.float32 or torch.bfloat16")
         self.B, self.K, self.V, self.Hq, self.Hkv, self.d, self.S_cap = B, K, V, Hq, Hkv, head_dim, S_cap
         self.device = torch.device("cuda") if device is None else torch.device(device)
         dev = self.device
@@ -31,8 +35,8 @@ class VerifyRound:
         self.kv_len = kv_len.to(dev, torch.int32).contiguous()
         self.kv_len_host = [int(x) for x in kv_len.cpu()]
         f32, i32, bf = torch.float32, torch.int32, torch.bfloat16
-        self.draft_logits = torch.empty((B, K, V), dtype=f32, device=dev)
-        self.target_logits = torch.empty((B, K + 1, V), dtype=f32, device=dev)
+        self.draft_logits = torch.empty((B, K, V), dtype=logits_dtype, device=dev)
+        self.target_logits = torch.empty((B, K + 1, V), dtype=logits_dtype, device=dev)
         self.draft_tokens = torch.empty((B, K), dtype=i32, device=dev)
         self.temperature = torch.empty((B,), dtype=f32, device=dev)
         self.cost_table = torch.empty((K + 1,), dtype=f32, device=dev)
@@ -54,7 +58,8 @@ class VerifyRound:
 
     def h2d_bytes(self) -> int:
         per_layer = self.B * (self.K + 1) * self.Hq * self.d * 2 + 2 * self.B * self.Hkv * (self.K + 1) * self.d * 2
-        return (self.draft_logits.numel() * 4 + self.target_logits.numel() * 4 + self.draft_tokens.numel() * 4 +
+        lb = self.draft_logits.element_size()
+        return (self.draft_logits.numel() * lb + self.target_logits.numel() * lb + self.draft_tokens.numel() * 4 +
                 self.temperature.numel() * 4 + self.cost_table.numel() * 4 + self.n_layers * per_layer)
 
     def d2h_bytes(self) -> int:

@@ -30,14 +30,18 @@ SIGNATURES = {
     "libraspec_workspace_init": (_I, [_P, _SZ, _P]),
     "libraspec_get_status": (_I, [_P, _P, _P]),
     "libraspec_confidence": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
+    "libraspec_confidence_bf16": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "libraspec_confidence_noalloc": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P]),
     "libraspec_select_lengths": (_I, [_P, _P, _I, _I, _P, _P, _SZ, _P]),
     "libraspec_select_alpha": (_I, [_P, _I, _I, _I, _F, _P, _P, _P]),
     "libraspec_verify_attn": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_attn_layers": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
+    "libraspec_accept_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_round": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _I,
                                     _F, _U64, _U64, _U32, _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "libraspec_verify_round_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I,
+                                         _I, _F, _U64, _U64, _U32, _P, _P, _P, _P, _P, _P, _SZ, _P]),
 }
 
 _lib = None
@@ -137,7 +141,8 @@ def libraspec_get_status(ws: Workspace, stream=None) -> int:
 def libraspec_confidence(draft_logits, draft_tokens, temperature, ws: Workspace, conf=None, dstat=None,
                          stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
     B, K, V = draft_logits.shape
-    _req(draft_logits, torch.float32, "draft_logits")
+    bf16 = draft_logits.dtype == torch.bfloat16  # libraspec_confidence_bf16
+    _req(draft_logits, torch.bfloat16 if bf16 else torch.float32, "draft_logits")
     _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
     _req(temperature, torch.float32, "temperature", (B,))
     dev = draft_logits.device
@@ -145,9 +150,10 @@ def libraspec_confidence(draft_logits, draft_tokens, temperature, ws: Workspace,
                                                                                           "conf", (B, K))
     dstat = torch.empty((B, K, 2), dtype=torch.float32, device=dev) if dstat is None else _req(
         dstat, torch.float32, "dstat", (B, K, 2))
-    rc = load().libraspec_confidence(_ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature), B, K, V,
-                                     _ptr(conf), _ptr(dstat), ws.ptr, ws.nbytes, _stream(stream))
-    _check(rc, "libraspec_confidence")
+    name = "libraspec_confidence_bf16" if bf16 else "libraspec_confidence"
+    rc = getattr(load(), name)(_ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature), B, K, V, _ptr(conf),
+                               _ptr(dstat), ws.ptr, ws.nbytes, _stream(stream))
+    _check(rc, name)
     return conf, dstat
 
 
@@ -258,8 +264,10 @@ def libraspec_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, 
                      stream=None):
     B, K1, V = target_logits.shape
     K = K1 - 1
-    _req(target_logits, torch.float32, "target_logits")
-    _req(draft_logits, torch.float32, "draft_logits", (B, K, V))
+    bf16 = target_logits.dtype == torch.bfloat16  # libraspec_accept_bf16: both logit tensors bf16
+    ldt = torch.bfloat16 if bf16 else torch.float32
+    _req(target_logits, ldt, "target_logits")
+    _req(draft_logits, ldt, "draft_logits", (B, K, V))
     _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
     if conf is not None:
         _req(conf, torch.float32, "conf", (B, K))
@@ -270,11 +278,12 @@ def libraspec_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, 
     dev = target_logits.device
     n_accepted = torch.empty((B,), dtype=torch.int32, device=dev) if n_accepted is None else n_accepted
     bonus_token = torch.empty((B,), dtype=torch.int32, device=dev) if bonus_token is None else bonus_token
-    rc = load().libraspec_accept(_ptr(target_logits), _ptr(draft_logits), _ptr(draft_tokens), _ptr(conf),
-                                 _ptr(dstat), _ptr(L), _ptr(temperature), B, K, V, int(seed) & (2**64 - 1),
-                                 int(round_offset), int(seq_offset), _ptr(n_accepted), _ptr(bonus_token), ws.ptr,
-                                 ws.nbytes, _stream(stream))
-    _check(rc, "libraspec_accept")
+    name = "libraspec_accept_bf16" if bf16 else "libraspec_accept"
+    rc = getattr(load(), name)(_ptr(target_logits), _ptr(draft_logits), _ptr(draft_tokens), _ptr(conf), _ptr(dstat),
+                               _ptr(L), _ptr(temperature), B, K, V, int(seed) & (2**64 - 1), int(round_offset),
+                               int(seq_offset), _ptr(n_accepted), _ptr(bonus_token), ws.ptr, ws.nbytes,
+                               _stream(stream))
+    _check(rc, name)
     return n_accepted, bonus_token
 
 
@@ -298,8 +307,10 @@ def libraspec_verify_round(draft_logits, draft_tokens, temperature, cost_table, 
                            stream=None) -> RoundOutputs:
     """layers: sequence of dicts with Q, Kc, Vc (and optionally O)."""
     B, K, V = draft_logits.shape
-    _req(draft_logits, torch.float32, "draft_logits")
-    _req(target_logits, torch.float32, "target_logits", (B, K + 1, V))
+    bf16 = draft_logits.dtype == torch.bfloat16  # libraspec_verify_round_bf16: both logit tensors bf16
+    ldt = torch.bfloat16 if bf16 else torch.float32
+    _req(draft_logits, ldt, "draft_logits")
+    _req(target_logits, ldt, "target_logits", (B, K + 1, V))
     _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
     _req(temperature, torch.float32, "temperature", (B,))
     _req(cost_table, torch.float32, "cost_table", (K + 1,))
@@ -326,10 +337,11 @@ def libraspec_verify_round(draft_logits, draft_tokens, temperature, cost_table, 
     va = _ptr_array([lay["Vc"] for lay in layers])
     oa = _ptr_array(outputs.O)
     la = _ptr_array(outputs.lse) if outputs.lse is not None else None
-    rc = load().libraspec_verify_round(
+    name = "libraspec_verify_round_bf16" if bf16 else "libraspec_verify_round"
+    rc = getattr(load(), name)(
         _ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature), _ptr(cost_table), _ptr(target_logits), qa, ka, va,
         oa, la, n_layers, _ptr(kv_len), B, K, V, Hq, Hkv, D, S_cap, float(softmax_scale), int(seed) & (2**64 - 1),
         int(round_offset), int(seq_offset), _ptr(outputs.conf), _ptr(outputs.dstat), _ptr(outputs.L),
         _ptr(outputs.n_accepted), _ptr(outputs.bonus_token), ws.ptr, ws.nbytes, _stream(stream))
-    _check(rc, "libraspec_verify_round")
+    _check(rc, name)
     return outputs

@@ -8,7 +8,8 @@
 
 namespace libraspec {
 
-cudaError_t launch_confidence(const float*, const int32_t*, const float*, int, int, int, float*, float*, char*,
+template <typename T>
+cudaError_t launch_confidence(const T*, const int32_t*, const float*, int, int, int, float*, float*, char*,
                               const WsLayout&, cudaStream_t);
 cudaError_t launch_select(const float*, const float*, int, int, int32_t*, char*, const WsLayout&, cudaStream_t);
 cudaError_t launch_select_alpha(const float*, int, int, int, double, int32_t*, int32_t*, cudaStream_t);
@@ -18,7 +19,8 @@ cudaError_t launch_verify_attn(const uint16_t*, const uint16_t*, const uint16_t*
 cudaError_t launch_verify_attn_layers(const uint16_t* const*, const uint16_t* const*, const uint16_t* const*, int,
                                       const int32_t*, const int32_t*, int, int, int, int, int, int, float,
                                       uint16_t* const*, float* const*, char*, const WsLayout&, cudaStream_t);
-cudaError_t launch_accept(const float*, const float*, const int32_t*, const float*, const float*, const int32_t*,
+template <typename T>
+cudaError_t launch_accept(const T*, const T*, const int32_t*, const float*, const float*, const int32_t*,
                           const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, char*,
                           const WsLayout&, cudaStream_t);
 
@@ -108,16 +110,31 @@ static bool ws_ok(const void* ws, size_t ws_bytes, const WsLayout& lay) {
   return ws && aligned(ws, 256) && ws_bytes >= lay.total;
 }
 
-int libraspec_confidence(const float* draft_logits, const int32_t* draft_tokens, const float* temperature, int B,
-                         int K, int V, float* conf, float* dstat, void* workspace, size_t ws_bytes, void* stream) {
+extern "C++" {
+template <typename T>
+static int confidence_t(const T* draft_logits, const int32_t* draft_tokens, const float* temperature, int B, int K,
+                        int V, float* conf, float* dstat, void* workspace, size_t ws_bytes, void* stream) {
   if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
   if (B * K == 0) return LIBRASPEC_OK;
   if (!draft_logits || !draft_tokens || !temperature || !conf) return LIBRASPEC_EINVAL;
-  if (!aligned(draft_logits, 4) || !aligned(conf, 4) || (dstat && !aligned(dstat, 4))) return LIBRASPEC_EINVAL;
+  if (!aligned(draft_logits, sizeof(T)) || !aligned(conf, 4) || (dstat && !aligned(dstat, 4)))
+    return LIBRASPEC_EINVAL;
   const WsLayout lay = ws_layout(B, K, V, 1, 1, 64, 1);
   if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
-  return from_cuda(launch_confidence(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat,
-                                     static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+  return from_cuda(launch_confidence<T>(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat,
+                                        static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+}
+}  // extern "C++"
+
+int libraspec_confidence(const float* draft_logits, const int32_t* draft_tokens, const float* temperature, int B,
+                         int K, int V, float* conf, float* dstat, void* workspace, size_t ws_bytes, void* stream) {
+  return confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream);
+}
+
+int libraspec_confidence_bf16(const uint16_t* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                              int B, int K, int V, float* conf, float* dstat, void* workspace, size_t ws_bytes,
+                              void* stream) {
+  return confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream);
 }
 
 int libraspec_select_lengths(const float* conf, const float* cost_table, int B, int K, int32_t* L, void* workspace,
@@ -179,25 +196,48 @@ int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const
                                              static_cast<cudaStream_t>(stream)));
 }
 
-int libraspec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
-                     const float* conf, const float* dstat, const int32_t* L, const float* temperature, int B, int K,
-                     int V, uint64_t seed, uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted,
-                     int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
+extern "C++" {
+template <typename T>
+static int accept_t(const T* target_logits, const T* draft_logits, const int32_t* draft_tokens, const float* conf,
+                    const float* dstat, const int32_t* L, const float* temperature, int B, int K, int V, uint64_t seed,
+                    uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted, int32_t* bonus_token,
+                    void* workspace, size_t ws_bytes, void* stream) {
   if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
   if (B == 0) return LIBRASPEC_OK;
   if (!target_logits || (!draft_logits && K > 0) || (!draft_tokens && K > 0) || !L || !temperature ||
       !n_accepted || !bonus_token)
     return LIBRASPEC_EINVAL;
-  if (!aligned(target_logits, 4) || (draft_logits && !aligned(draft_logits, 4))) return LIBRASPEC_EINVAL;
+  if (!aligned(target_logits, sizeof(T)) || (draft_logits && !aligned(draft_logits, sizeof(T))))
+    return LIBRASPEC_EINVAL;
   const WsLayout lay = ws_layout(B, K, V, 1, 1, 64, 1);
   if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
-  return from_cuda(launch_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V,
-                                 seed, round_offset, seq_offset, n_accepted, bonus_token,
-                                 static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+  return from_cuda(launch_accept<T>(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V,
+                                    seed, round_offset, seq_offset, n_accepted, bonus_token,
+                                    static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+}
+}  // extern "C++"
+
+int libraspec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
+                     const float* conf, const float* dstat, const int32_t* L, const float* temperature, int B, int K,
+                     int V, uint64_t seed, uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted,
+                     int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
+  return accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed,
+                  round_offset, seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
 }
 
-int libraspec_verify_round(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
-                           const float* cost_table, const float* target_logits, const uint16_t* const* Q,
+int libraspec_accept_bf16(const uint16_t* target_logits, const uint16_t* draft_logits, const int32_t* draft_tokens,
+                          const float* conf, const float* dstat, const int32_t* L, const float* temperature, int B,
+                          int K, int V, uint64_t seed, uint64_t round_offset, uint32_t seq_offset,
+                          int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                          void* stream) {
+  return accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed,
+                  round_offset, seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
+}
+
+extern "C++" {
+template <typename T>
+static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                           const float* cost_table, const T* target_logits, const uint16_t* const* Q,
                            const uint16_t* const* Kc, const uint16_t* const* Vc, uint16_t* const* O,
                            float* const* lse, int n_layers, const int32_t* kv_len, int B, int K, int V, int Hq,
                            int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
@@ -222,8 +262,7 @@ int libraspec_verify_round(const float* draft_logits, const int32_t* draft_token
   char* ws = static_cast<char*>(workspace);
   int rc = LIBRASPEC_OK;
   if (K > 0) {
-    rc = libraspec_confidence(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes,
-                              stream);
+    rc = confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream);
     if (rc != LIBRASPEC_OK) return rc;
   }
   rc = from_cuda(launch_select(conf, cost_table, B, K, L, ws, lay, s));
@@ -231,8 +270,35 @@ int libraspec_verify_round(const float* draft_logits, const int32_t* draft_token
   rc = from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap,
                                            softmax_scale, O, lse, ws, lay, s));
   if (rc != LIBRASPEC_OK) return rc;
-  return libraspec_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed,
-                          round_offset, seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
+  return accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed, round_offset,
+                  seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
+}
+}  // extern "C++"
+
+int libraspec_verify_round(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                           const float* cost_table, const float* target_logits, const uint16_t* const* Q,
+                           const uint16_t* const* Kc, const uint16_t* const* Vc, uint16_t* const* O,
+                           float* const* lse, int n_layers, const int32_t* kv_len, int B, int K, int V, int Hq,
+                           int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                           uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
+                           int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                           void* stream) {
+  return verify_round_t(draft_logits, draft_tokens, temperature, cost_table, target_logits, Q, Kc, Vc, O, lse,
+                        n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed, round_offset,
+                        seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace, ws_bytes, stream);
+}
+
+int libraspec_verify_round_bf16(const uint16_t* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                                const float* cost_table, const uint16_t* target_logits, const uint16_t* const* Q,
+                                const uint16_t* const* Kc, const uint16_t* const* Vc, uint16_t* const* O,
+                                float* const* lse, int n_layers, const int32_t* kv_len, int B, int K, int V, int Hq,
+                                int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                                uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
+                                int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                                void* stream) {
+  return verify_round_t(draft_logits, draft_tokens, temperature, cost_table, target_logits, Q, Kc, Vc, O, lse,
+                        n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed, round_offset,
+                        seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace, ws_bytes, stream);
 }
 
 }  // extern "C"

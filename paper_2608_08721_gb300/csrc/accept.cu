@@ -9,9 +9,9 @@ namespace libraspec {
 // sequences need (m, Z) at their temperature. Partials of a row are merged by
 // the last CTA to finish (atomic ticket) into row_stat[b, j].
 // ---------------------------------------------------------------------------
-template <bool VEC>
+template <bool VEC, typename E>
 __global__ void __launch_bounds__(kRowThreads) accept_rows_kernel(
-    const float* __restrict__ target, const int32_t* __restrict__ Ls, const float* __restrict__ temperature,
+    const E* __restrict__ target, const int32_t* __restrict__ Ls, const float* __restrict__ temperature,
     int K, int V, int nsplit, int chunk, RowPartial* __restrict__ part, uint32_t* __restrict__ cnt,
     RowStat* __restrict__ stat, int* __restrict__ status) {
   __shared__ float smf[64];
@@ -29,7 +29,7 @@ __global__ void __launch_bounds__(kRowThreads) accept_rows_kernel(
   const bool sampling = tb > 0.f;
   const float T = sampling ? tb : 1.f;
   const float c = (float)(1.4426950408889634 / (double)T);
-  const float* xr = target + (size_t)row * V;
+  const E* xr = target + (size_t)row * V;
   const int c0 = split * chunk, c1 = min(V, c0 + chunk);
 
   SumAcc sa;
@@ -40,12 +40,12 @@ __global__ void __launch_bounds__(kRowThreads) accept_rows_kernel(
   int arg = 0;
   float s = 0.f;
   if (sampling) {
-    row_slice_pass<true, false, VEC>(xr, c0, c1, c, sa, aa);
+    row_slice_pass<true, false, VEC, E>(xr, c0, c1, c, sa, aa);
     m = sa.m;
     s = sa.value();
     cta_reduce_sum(m, s, c, smf);
   } else {
-    row_slice_pass<false, true, VEC>(xr, c0, c1, c, sa, aa);
+    row_slice_pass<false, true, VEC, E>(xr, c0, c1, c, sa, aa);
     m = aa.m;
     arg = aa.arg;
     cta_reduce_arg(m, arg, smf, smi);
@@ -101,7 +101,8 @@ struct Decision {
   bool ok;
 };
 
-__device__ Decision decide(int b, int K, int V, const float* __restrict__ target,
+template <typename E>
+__device__ Decision decide(int b, int K, int V, const E* __restrict__ target,
                            const int32_t* __restrict__ tokens, const float* __restrict__ conf,
                            const int32_t* __restrict__ Ls, const float* __restrict__ temperature,
                            const RowStat* __restrict__ stat, uint64_t seed, uint64_t round_offset,
@@ -131,7 +132,7 @@ __device__ Decision decide(int b, int K, int V, const float* __restrict__ target
         reject = true;
       } else {
         const float c = (float)(1.4426950408889634 / (double)tb);
-        const float y = target[((size_t)b * (K + 1) + jj) * V + x];
+        const float y = Logit<E>::at(target, ((size_t)b * (K + 1) + jj) * V + x);
         const double p = (double)exp2f((y - __ldcg(&st[jj].m)) * c) / __ldcg(&st[jj].Z);
         const double q = (double)conf[(size_t)b * K + jj];
         const double ratio = (q <= p) ? 1.0 : p / q;
@@ -151,9 +152,9 @@ __device__ Decision decide(int b, int K, int V, const float* __restrict__ target
   return d;
 }
 
-template <bool VEC>
+template <bool VEC, typename E>
 __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
-    const float* __restrict__ target, const float* __restrict__ draft, const int32_t* __restrict__ tokens,
+    const E* __restrict__ target, const E* __restrict__ draft, const int32_t* __restrict__ tokens,
     const float* __restrict__ conf, const float* __restrict__ dstat, const int32_t* __restrict__ Ls,
     const float* __restrict__ temperature, int K, int V, int nsplit, int chunk, uint64_t seed,
     uint64_t round_offset, uint32_t seq_offset, const RowStat* __restrict__ stat,
@@ -164,8 +165,8 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
   __shared__ int smi[32];
   const int split = blockIdx.x, b = blockIdx.y;
   if (threadIdx.x < 32) {
-    const Decision d = decide(b, K, V, target, tokens, conf, Ls, temperature, stat, seed, round_offset,
-                              seq_offset, status);
+    const Decision d = decide<E>(b, K, V, target, tokens, conf, Ls, temperature, stat, seed, round_offset,
+                                 seq_offset, status);
     if (threadIdx.x == 0) {
       sh_n = d.n;
       sh_bonus = d.bonus;
@@ -203,8 +204,8 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
   const bool residual = n < Lb;
   const float c = (float)(1.4426950408889634 / (double)tb);
   const RowStat st = stat[(size_t)b * (K + 1) + n];
-  const float* yr = target + ((size_t)b * (K + 1) + n) * V;
-  const float* dr = residual ? draft + ((size_t)b * K + n) * V : nullptr;
+  const E* yr = target + ((size_t)b * (K + 1) + n) * V;
+  const E* dr = residual ? draft + ((size_t)b * K + n) * V : nullptr;
   const float mp = st.m;
   const float invZp = (float)(1.0 / st.Z);
   float mq = 0.f, invZq = 0.f;
@@ -222,18 +223,14 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
     const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
     float yv[4], dv[4];
     if (VEC) {
-      const float4 a = ld_stream4(yr + 4 * g);
-      yv[0] = a.x; yv[1] = a.y; yv[2] = a.z; yv[3] = a.w;
-      if (residual) {
-        const float4 e = ld_stream4(dr + 4 * g);
-        dv[0] = e.x; dv[1] = e.y; dv[2] = e.z; dv[3] = e.w;
-      }
+      Logit<E>::stream4(yr + 4 * g, yv);
+      if (residual) Logit<E>::stream4(dr + 4 * g, dv);
     } else {
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
         const int v = 4 * g + t;
-        yv[t] = v < V ? yr[v] : -INFINITY;
-        dv[t] = (residual && v < V) ? dr[v] : 0.f;
+        yv[t] = v < V ? Logit<E>::at(yr, v) : -INFINITY;
+        dv[t] = (residual && v < V) ? Logit<E>::at(dr, v) : 0.f;
       }
     }
 #pragma unroll
@@ -316,7 +313,7 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
   for (int v = threadIdx.x; v < V; v += kRowThreads) {
     const uint4 w4 = philox_block(seed, (uint32_t)(v >> 2), (uint32_t)n, seq, 1u, round_offset);
     const uint32_t wsel = (v & 3) == 0 ? w4.x : (v & 3) == 1 ? w4.y : (v & 3) == 2 ? w4.z : w4.w;
-    const float wv = exp2f((yr[v] - mp) * c);
+    const float wv = exp2f((Logit<E>::at(yr, v) - mp) * c);
     if (wv > 0.f) argmin_combine(best, besti, -logf(word_to_uniform(wsel)) / wv, v);
   }
 #pragma unroll
@@ -341,14 +338,15 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
 // ---------------------------------------------------------------------------
 int num_sms_current();
 
-cudaError_t launch_accept(const float* target, const float* draft, const int32_t* tokens, const float* conf,
+template <typename T>
+cudaError_t launch_accept(const T* target, const T* draft, const int32_t* tokens, const float* conf,
                           const float* dstat, const int32_t* L, const float* temperature, int B, int K, int V,
                           uint64_t seed, uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted,
                           int32_t* bonus, char* ws, const WsLayout& lay, cudaStream_t stream) {
   if (B == 0) return cudaSuccess;
   const int sms = num_sms_current();
-  const bool vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(target) & 15) == 0) &&
-                   (draft == nullptr || (reinterpret_cast<uintptr_t>(draft) & 15) == 0);
+  // the race reads groups of 4 logits: both rows must allow those loads too
+  const bool vec = rows_vectorizable(target, V) && (draft == nullptr || rows_vectorizable(draft, V));
   auto* st = reinterpret_cast<int*>(ws + lay.status);
   auto* rstat = reinterpret_cast<RowStat*>(ws + lay.row_stat);
   {
@@ -360,11 +358,11 @@ cudaError_t launch_accept(const float* target, const float* draft, const int32_t
     auto* part = reinterpret_cast<RowPartial*>(ws + lay.row_part);
     auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.row_cnt);
     if (vec)
-      accept_rows_kernel<true><<<grid, kRowThreads, 0, stream>>>(target, L, temperature, K, V, nsplit, chunk,
-                                                                  part, cnt, rstat, st);
+      accept_rows_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(target, L, temperature, K, V, nsplit, chunk,
+                                                                     part, cnt, rstat, st);
     else
-      accept_rows_kernel<false><<<grid, kRowThreads, 0, stream>>>(target, L, temperature, K, V, nsplit, chunk,
-                                                                   part, cnt, rstat, st);
+      accept_rows_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(target, L, temperature, K, V, nsplit, chunk,
+                                                                      part, cnt, rstat, st);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -382,15 +380,22 @@ cudaError_t launch_accept(const float* target, const float* draft, const int32_t
     auto* part = reinterpret_cast<RacePartial*>(ws + lay.race_part);
     auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.race_cnt);
     if (vec)
-      accept_decide_kernel<true><<<grid, kRowThreads, 0, stream>>>(
+      accept_decide_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(
           target, draft, tokens, conf, dstat, L, temperature, K, V, nsplit, chunk, seed, round_offset, seq_offset,
           rstat, part, cnt, n_accepted, bonus, st);
     else
-      accept_decide_kernel<false><<<grid, kRowThreads, 0, stream>>>(
+      accept_decide_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(
           target, draft, tokens, conf, dstat, L, temperature, K, V, nsplit, chunk, seed, round_offset, seq_offset,
           rstat, part, cnt, n_accepted, bonus, st);
     return cudaGetLastError();
   }
 }
+template cudaError_t launch_accept<float>(const float*, const float*, const int32_t*, const float*, const float*,
+                                          const int32_t*, const float*, int, int, int, uint64_t, uint64_t, uint32_t,
+                                          int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
+template cudaError_t launch_accept<uint16_t>(const uint16_t*, const uint16_t*, const int32_t*, const float*,
+                                             const float*, const int32_t*, const float*, int, int, int, uint64_t,
+                                             uint64_t, uint32_t, int32_t*, int32_t*, char*, const WsLayout&,
+                                             cudaStream_t);
 
 }  // namespace libraspec

@@ -141,6 +141,54 @@ __device__ __forceinline__ float ld_stream(const float* p) {
   return v;
 }
 
+// Logit element types: fp32, or bf16 passed as its 16-bit pattern. A bf16
+// value widens to fp32 exactly (its bits are the top half of the fp32 word).
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+template <typename T>
+struct Logit;
+
+template <>
+struct Logit<float> {
+  static constexpr int kVec = 4;  // elements per 16-byte load
+  __device__ static __forceinline__ float at(const float* p, size_t i) { return p[i]; }
+  __device__ static __forceinline__ float stream1(const float* p) { return ld_stream(p); }
+  // kVec elements from a 16-byte-aligned address
+  __device__ static __forceinline__ void stream_vec(const float* p, float (&v)[4]) {
+    const float4 a = ld_stream4(p);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  }
+  // 4 elements from an address aligned to 4 elements
+  __device__ static __forceinline__ void stream4(const float* p, float (&v)[4]) { stream_vec(p, v); }
+};
+
+template <>
+struct Logit<uint16_t> {
+  static constexpr int kVec = 8;
+  __device__ static __forceinline__ float at(const uint16_t* p, size_t i) {
+    return __uint_as_float((uint32_t)p[i] << 16);
+  }
+  __device__ static __forceinline__ float stream1(const uint16_t* p) {
+    unsigned short h;
+    asm volatile("ld.global.nc.L1::no_allocate.u16 %0, [%1];" : "=h"(h) : "l"(p));
+    return __uint_as_float((uint32_t)h << 16);
+  }
+  __device__ static __forceinline__ void stream_vec(const uint16_t* p, float (&v)[8]) {
+    uint32_t w0, w1, w2, w3;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
+                 : "l"(p));
+    v[0] = bf16_lo(w0); v[1] = bf16_hi(w0); v[2] = bf16_lo(w1); v[3] = bf16_hi(w1);
+    v[4] = bf16_lo(w2); v[5] = bf16_hi(w2); v[6] = bf16_lo(w3); v[7] = bf16_hi(w3);
+  }
+  __device__ static __forceinline__ void stream4(const uint16_t* p, float (&v)[4]) {
+    uint32_t w0, w1;
+    asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];" : "=r"(w0), "=r"(w1) : "l"(p));
+    v[0] = bf16_lo(w0); v[1] = bf16_hi(w0); v[2] = bf16_lo(w1); v[3] = bf16_hi(w1);
+  }
+};
+
 // Combine two (m, s) pairs (binary64 sums); c = log2(e) / T.
 __device__ __forceinline__ void combine_ms(float& m, double& s, float m2, double s2, float c) {
   if (m2 == -INFINITY) return;

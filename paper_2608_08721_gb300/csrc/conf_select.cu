@@ -11,9 +11,9 @@ namespace libraspec {
 // q = exp((x_tok - m)/T) / Z (Assumption 1: q_k, the drafter's probability
 // of its drafted token).
 // ---------------------------------------------------------------------------
-template <bool VEC>
+template <bool VEC, typename E>
 __global__ void __launch_bounds__(kRowThreads) conf_kernel(
-    const float* __restrict__ x, const int32_t* __restrict__ tokens, const float* __restrict__ temperature,
+    const E* __restrict__ x, const int32_t* __restrict__ tokens, const float* __restrict__ temperature,
     int K, int V, int nsplit, int chunk, float* __restrict__ conf, float* __restrict__ dstat,
     RowPartial* __restrict__ part, uint32_t* __restrict__ cnt, int* __restrict__ status) {
   __shared__ float sm[64];
@@ -23,13 +23,13 @@ __global__ void __launch_bounds__(kRowThreads) conf_kernel(
   const float tb = temperature[b];
   const float T = tb > 0.f ? tb : 1.f;
   const float c = (float)(1.4426950408889634 / (double)T);
-  const float* xr = x + (size_t)row * V;
+  const E* xr = x + (size_t)row * V;
   const int c0 = split * chunk, c1 = min(V, c0 + chunk);
 
   SumAcc sa;
   ArgAcc aa;
   sa.init();
-  row_slice_pass<true, false, VEC>(xr, c0, c1, c, sa, aa);
+  row_slice_pass<true, false, VEC, E>(xr, c0, c1, c, sa, aa);
   float m = sa.m, s = sa.value();
   cta_reduce_sum(m, s, c, sm);
 
@@ -65,7 +65,7 @@ __global__ void __launch_bounds__(kRowThreads) conf_kernel(
     raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
   } else {
     // x_tok - M is exact for the near-maximal tokens that matter (Sterbenz)
-    q = (float)((double)exp2f((xr[tok] - M) * c) / Z);
+    q = (float)((double)exp2f((Logit<E>::at(xr, tok) - M) * c) / Z);
   }
   conf[row] = q;
   if (dstat) {
@@ -223,27 +223,31 @@ __global__ void __launch_bounds__(128) select_alpha_kernel(const float* __restri
 // ---------------------------------------------------------------------------
 int num_sms_current();
 
-cudaError_t launch_confidence(const float* x, const int32_t* tokens, const float* temperature, int B, int K,
-                              int V, float* conf, float* dstat, char* ws, const WsLayout& lay,
-                              cudaStream_t stream) {
+template <typename T>
+cudaError_t launch_confidence(const T* x, const int32_t* tokens, const float* temperature, int B, int K, int V,
+                              float* conf, float* dstat, char* ws, const WsLayout& lay, cudaStream_t stream) {
   const long rows = (long)B * K;
   if (rows == 0) return cudaSuccess;
   const int nsplit0 = row_splits(rows, V, num_sms_current(), kConfMaxSplits, 4096);
   const int chunk = row_chunk(V, nsplit0);
   const int nsplit = (V + chunk - 1) / chunk;
-  const bool vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
+  const bool vec = rows_vectorizable(x, V);
   dim3 grid(nsplit, (unsigned)rows);
   auto* part = reinterpret_cast<RowPartial*>(ws + lay.conf_part);
   auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.conf_cnt);
   auto* st = reinterpret_cast<int*>(ws + lay.status);
   if (vec)
-    conf_kernel<true><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
-                                                        dstat, part, cnt, st);
+    conf_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
+                                                           dstat, part, cnt, st);
   else
-    conf_kernel<false><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
-                                                         dstat, part, cnt, st);
+    conf_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
+                                                            dstat, part, cnt, st);
   return cudaGetLastError();
 }
+template cudaError_t launch_confidence<float>(const float*, const int32_t*, const float*, int, int, int, float*,
+                                              float*, char*, const WsLayout&, cudaStream_t);
+template cudaError_t launch_confidence<uint16_t>(const uint16_t*, const int32_t*, const float*, int, int, int,
+                                                 float*, float*, char*, const WsLayout&, cudaStream_t);
 
 cudaError_t launch_select_alpha(const float* conf, int B, int K, int n, double alpha, int32_t* L,
                                 int32_t* n_blocks, cudaStream_t stream) {

@@ -10,7 +10,8 @@
 
 namespace libraspec {
 
-cudaError_t launch_confidence(const float*, const int32_t*, const float*, int, int, int, float*, float*, char*,
+template <typename T>
+cudaError_t launch_confidence(const T*, const int32_t*, const float*, int, int, int, float*, float*, char*,
                               const WsLayout&, cudaStream_t);
 
 namespace {

@@ -61,34 +61,45 @@ struct ArgAcc {
   }
 };
 
-// Stream x[c0, c1) (c0 a multiple of 4). VEC: x is 16-byte aligned and the
-// row length is a multiple of 4, so 128-bit loads cover the slice.
-template <bool SUM, bool ARG, bool VEC>
-__device__ __forceinline__ void row_slice_pass(const float* __restrict__ x, int c0, int c1, float c,
-                                               SumAcc& sa, ArgAcc& aa) {
+// Stream x[c0, c1) of logits of type T (c0 a multiple of kRowAlign). VEC: x
+// is 16-byte aligned and the row length a multiple of the elements one
+// 128-bit load holds, so 128-bit loads cover the slice.
+template <bool SUM, bool ARG, bool VEC, typename T>
+__device__ __forceinline__ void row_slice_pass(const T* __restrict__ x, int c0, int c1, float c, SumAcc& sa,
+                                               ArgAcc& aa) {
+  using LT = Logit<T>;
+  constexpr int W = LT::kVec;  // elements per 128-bit load
   const int tid = threadIdx.x;
   if (VEC) {
-    const int g0 = c0 >> 2, g1 = c1 >> 2;  // groups of 4
+    const int g0 = c0 / W, g1 = c1 / W;  // groups of W
     int g = g0 + tid;
-    constexpr int U = 4;
+    constexpr int U = 16 / W;  // 16 elements in flight per thread
     for (; g + (U - 1) * kRowThreads < g1; g += U * kRowThreads) {
-      float4 v[U];
+      float v[U][W];
 #pragma unroll
-      for (int u = 0; u < U; ++u) v[u] = ld_stream4(x + 4 * (g + u * kRowThreads));
+      for (int u = 0; u < U; ++u) LT::stream_vec(x + W * (g + u * kRowThreads), v[u]);
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        if (SUM) sa.add4(v[u], c);
-        if (ARG) aa.add4(v[u], 4 * (g + u * kRowThreads));
-      }
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int h = 0; h < W; h += 4) {
+          const float4 f = make_float4(v[u][h], v[u][h + 1], v[u][h + 2], v[u][h + 3]);
+          if (SUM) sa.add4(f, c);
+          if (ARG) aa.add4(f, W * (g + u * kRowThreads) + h);
+        }
     }
     for (; g < g1; g += kRowThreads) {
-      const float4 v = ld_stream4(x + 4 * g);
-      if (SUM) sa.add4(v, c);
-      if (ARG) aa.add4(v, 4 * g);
+      float v[W];
+      LT::stream_vec(x + W * g, v);
+#pragma unroll
+      for (int h = 0; h < W; h += 4) {
+        const float4 f = make_float4(v[h], v[h + 1], v[h + 2], v[h + 3]);
+        if (SUM) sa.add4(f, c);
+        if (ARG) aa.add4(f, W * g + h);
+      }
     }
   } else {
     for (int i = c0 + tid; i < c1; i += kRowThreads) {
-      const float v = ld_stream(x + i);
+      const float v = LT::stream1(x + i);
       if (SUM) sa.add1(v, c);
       if (ARG) aa.add1(v, i);
     }
@@ -193,10 +204,17 @@ inline int row_splits(long rows, int V, int num_sms, int max_splits, int min_ele
   return (int)ns;
 }
 
-// Split length: a multiple of 4 elements.
+// Split length: a multiple of 8 elements (whole 128-bit loads of fp32 or bf16).
+constexpr int kRowAlign = 8;
 inline int row_chunk(int V, int nsplit) {
   int ch = (V + nsplit - 1) / nsplit;
-  return (ch + 3) & ~3;
+  return (ch + kRowAlign - 1) & ~(kRowAlign - 1);
+}
+
+// 128-bit loads cover a row of V logits of type T at base x.
+template <typename T>
+inline bool rows_vectorizable(const T* x, int V) {
+  return (V % Logit<T>::kVec == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
 }
 
 }  // namespace libraspec

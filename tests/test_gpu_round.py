@@ -12,21 +12,27 @@ pytestmark = pytest.mark.gpu
 
 
 def _oracle_round(orc, w, inp, kv, layers, cost, rows_per_layer=None):
-    q, _ = orc.confidence(inp["draft_logits"].cpu().numpy(), inp["draft_tokens"].cpu().numpy(),
-                          inp["temperature"].cpu().numpy())
+    dl = inp["draft_logits"].float().cpu().numpy()
+    q, _ = orc.confidence(dl, inp["draft_tokens"].cpu().numpy(), inp["temperature"].cpu().numpy())
     L, sflag = orc.select_lengths(q, cost.astype(np.float64))
-    n, bonus, aflag = orc.accept(inp["target_logits"].cpu().numpy(), inp["draft_logits"].cpu().numpy(),
+    n, bonus, aflag = orc.accept(inp["target_logits"].float().cpu().numpy(), dl,
                                  inp["draft_tokens"].cpu().numpy(), L, inp["temperature"].cpu().numpy(),
                                  w.philox_seed)
     outs = [orc.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L, rows=rows_per_layer) for lay in layers]
     return q, L, sflag, n, bonus, aflag, outs
 
 
+@pytest.mark.parametrize("logits", ["f32", "bf16"])
 @pytest.mark.parametrize("name,n_layers", [("tiny", 1), ("8b", 2), ("sampling", 1)])
-def test_verify_round_matches_oracle(orc, name, n_layers):
+def test_verify_round_matches_oracle(orc, name, n_layers, logits):
+    """libraspec_verify_round, and libraspec_verify_round_bf16 on the same
+    logits rounded to bf16 (the oracle gets the rounded values)."""
     w = workloads.WORKLOADS[name]
     kv = workloads.kv_lengths(w)
     inp = workloads.logits(w, device=cuda())
+    if logits == "bf16":
+        for k in ("draft_logits", "target_logits"):
+            inp[k] = inp[k].to(torch.bfloat16)
     layers = [workloads.layer(w, l, kv, device=cuda()) for l in range(n_layers)]
     cost = workloads.cost_table(w)
     S = layers[0]["Kc"].shape[2]
