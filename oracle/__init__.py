@@ -59,9 +59,11 @@ def _load():
     lib.oracle_select_lengths.argtypes = [P, P, i32, i32, f64, P, P]
     lib.oracle_select_iterate.argtypes = [P, P, i32, f64, i32, P, i32]
     lib.oracle_select_alpha.argtypes = [P, i32, i32, i32, f64, P, P, P]
+    lib.oracle_gather_pages.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, P]
     lib.oracle_verify_attn.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, i32, f64, P, P, P, i32]
     lib.oracle_accept.argtypes = [P, P, P, P, P, i32, i32, i32, u64, u64, u32, P, P, P]
     for name in ("oracle_confidence", "oracle_select_lengths", "oracle_select_iterate", "oracle_select_alpha",
+                 "oracle_gather_pages",
                  "oracle_verify_attn", "oracle_accept"):
         getattr(lib, name).restype = i32
     _lib = lib
@@ -160,6 +162,25 @@ def select_alpha(conf, n: int, alpha: float):
     _check(_load().oracle_select_alpha(_ptr(q), B, K, int(n), float(alpha), _ptr(L), _ptr(blocks), _ptr(flag)),
            "oracle_select_alpha")
     return L, blocks, flag
+
+
+def gather_pages(pool, block_table, S_out: int):
+    """Dense [B,Hkv,S_out,d] bf16 bit patterns from a page pool [n_pages,Hkv,P,d] and a block table [B,max_pages]."""
+    pb = _as_bf16_bits(pool)
+    n_pages, Hkv, P, d = pb.shape
+    bt = _c(block_table, np.int32)
+    B, max_pages = bt.shape
+    dense = np.zeros((B, Hkv, S_out, d), np.uint16)
+    _check(_load().oracle_gather_pages(_ptr(pb), _ptr(bt), B, max_pages, P, n_pages, Hkv, d, int(S_out), _ptr(dense)),
+           "oracle_gather_pages")
+    return dense
+
+
+def verify_attn_paged(Q, Kp, Vp, block_table, kv_len, L, scale=None, rows=None, fill=np.nan):
+    """verify_attn over the dense cache the pages describe."""
+    S = int(np.max(np.asarray(kv_len) + np.asarray(L))) + 1 if len(kv_len) else 1
+    return verify_attn(Q, gather_pages(Kp, block_table, S), gather_pages(Vp, block_table, S), kv_len, L,
+                       scale=scale, rows=rows, fill=fill)
 
 
 def verify_attn(Q, Kc, Vc, kv_len, L, scale=None, rows=None, fill=np.nan):

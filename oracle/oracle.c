@@ -22,6 +22,8 @@
  *                          position-wise bounds eps_i (Thm. 2 / Thm. 3 with
  *                          the trade-off weight alpha), eps* = min_i eps_i,
  *                          block-wise drafting budget, one rollback.
+ *   oracle_gather_pages    the dense KV cache a paged cache (page pool and
+ *                          block table) describes.
  *   oracle_verify_attn     block-causal GQA attention of the d+1 verified
  *                          positions against the target KV cache (Sec. 3.1:
  *                          the target scores all drafted positions in one
@@ -366,6 +368,34 @@ int oracle_select_alpha(const double* conf, int B, int K, int n, double alpha, i
     if (blocks_out) blocks_out[b] = blocks;
     if (flag_out) flag_out[b] = flag;
   }
+  return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------ */
+/* Paged KV cache: the dense cache a block table describes.            */
+/* Reading (the paper does not address memory layout): key s of        */
+/* sequence b is row s % page_size of page block_table[b * max_pages + */
+/* s / page_size] of a pool [n_pages, Hkv, page_size, dh]; the verify  */
+/* attention over a paged cache is the dense one on                    */
+/*   dense[b, h, s, :] = pool[block_table[b][s / P], h, s % P, :],      */
+/* s < S_out <= max_pages * P. An entry outside [0, n_pages) that some  */
+/* s < S_out needs is an error.                                        */
+/* ------------------------------------------------------------------ */
+int oracle_gather_pages(const uint16_t* pool, const int32_t* block_table, int B, int max_pages, int page_size,
+                        int n_pages, int Hkv, int dh, int S_out, uint16_t* dense) {
+  if (B < 0 || max_pages < 1 || page_size < 1 || n_pages < 1 || Hkv < 1 || dh < 1 || S_out < 0 ||
+      (long)S_out > (long)max_pages * page_size || !pool || !block_table || !dense)
+    return ORACLE_EINVAL;
+  for (int b = 0; b < B; ++b)
+    for (int s = 0; s < S_out; ++s) {
+      const int page = block_table[(size_t)b * max_pages + s / page_size];
+      if (page < 0 || page >= n_pages) return ORACLE_EINVAL;
+      for (int h = 0; h < Hkv; ++h) {
+        const uint16_t* src = pool + (((size_t)page * Hkv + h) * page_size + s % page_size) * dh;
+        uint16_t* dst = dense + (((size_t)b * Hkv + h) * S_out + s) * dh;
+        for (int c = 0; c < dh; ++c) dst[c] = src[c];
+      }
+    }
   return ORACLE_OK;
 }
 

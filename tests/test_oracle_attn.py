@@ -4,12 +4,14 @@ Pinned against torch's scaled_dot_product_attention run in float64 on the CPU
 (an independent library routine) with an explicit per-row mask, and against
 closed forms: equal keys give the mean of the visible values, a dominant key
 gives its value row, a single visible key gives its value exactly, and equal
-scores give lse = s + ln(n_keys).
+scores give lse = s + ln(n_keys). The paged-cache gather is pinned against
+caches scattered into permuted pages by numpy indexing.
 """
 import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_2608_08721_gb300 import workloads
 
 
@@ -140,3 +142,46 @@ def test_attn_rejects_cache_overflow(orc):
         orc.verify_attn(Q, Kc, Kc, np.array([8], np.int32), np.array([2], np.int32))
     with pytest.raises(orc.OracleError):
         orc.verify_attn(Q, Kc, Kc, np.array([1], np.int32), np.array([3], np.int32))
+
+
+# ---- paged caches (the dense cache a block table describes) ----
+def _scatter_to_pages(dense, page_size, rng, extra_pages=3):
+    """Pool and block table holding `dense` [B,Hkv,S,d] in randomly permuted pages."""
+    B, Hkv, S, d = dense.shape
+    max_pages = -(-S // page_size)
+    n_pages = B * max_pages + extra_pages
+    perm = rng.permutation(n_pages)[: B * max_pages].reshape(B, max_pages).astype(np.int32)
+    pool = rng.integers(0, 2**16, size=(n_pages, Hkv, page_size, d)).astype(np.uint16)
+    for b in range(B):
+        for j in range(max_pages):
+            s0, s1 = j * page_size, min(S, (j + 1) * page_size)
+            pool[perm[b, j], :, : s1 - s0] = dense[b, :, s0:s1]
+    return pool, perm
+
+
+@pytest.mark.parametrize("page_size", [1, 7, 64, 128])
+def test_gather_pages_recovers_the_dense_cache(page_size):
+    rng = np.random.default_rng(page_size)
+    dense = rng.integers(0, 2**16, size=(3, 2, 300, 16)).astype(np.uint16)
+    pool, table = _scatter_to_pages(dense, page_size, rng)
+    np.testing.assert_array_equal(oracle.gather_pages(pool, table, 300), dense)
+    np.testing.assert_array_equal(oracle.gather_pages(pool, table, 17), dense[:, :, :17])
+
+
+def test_gather_pages_identity_table_is_a_reshape():
+    rng = np.random.default_rng(9)
+    B, Hkv, P, d, n = 2, 3, 64, 8, 4
+    pool = rng.integers(0, 2**16, size=(B * n, Hkv, P, d)).astype(np.uint16)
+    table = np.arange(B * n, dtype=np.int32).reshape(B, n)
+    expect = pool.reshape(B, n, Hkv, P, d).transpose(0, 2, 1, 3, 4).reshape(B, Hkv, n * P, d)
+    np.testing.assert_array_equal(oracle.gather_pages(pool, table, n * P), expect)
+
+
+def test_gather_pages_rejects_bad_entries():
+    pool = np.zeros((4, 1, 64, 8), np.uint16)
+    for bad in (-1, 4):
+        table = np.array([[0, bad]], np.int32)
+        with pytest.raises(oracle.OracleError):
+            oracle.gather_pages(pool, table, 100)
+    # an entry no key reads is not looked at
+    oracle.gather_pages(pool, np.array([[0, 99]], np.int32), 64)
