@@ -62,6 +62,7 @@ extern "C" {
 #define LIBRASPEC_ST_BAD_TOKEN 0x8   /* draft token outside [0, V)               */
 #define LIBRASPEC_ST_TIMEOUT 0x10    /* a bounded wait (async copy, grid barrier) expired */
 #define LIBRASPEC_ST_MISSING_INPUT 0x20 /* sampling sequence but conf/dstat NULL  */
+#define LIBRASPEC_ST_BAD_PAGE 0x40   /* a block-table entry outside [0, n_pages)  */
 
 /* Limits of this build. */
 #define LIBRASPEC_MAX_K 64           /* drafter block length / d_max             */
@@ -241,6 +242,31 @@ int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const
                                  int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
                                  int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,
                                  void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * libraspec_verify_attn_layers over a paged KV cache (block tables, as
+ * serving engines keep it): the same per-layer result as the dense call on
+ * the cache the pages describe.
+ *   Kp[l], Vp[l]  [n_pages, Hkv, page_size, head_dim] bf16 page pools;
+ *   block_table   [B, max_pages] i32: key s of sequence b (cache prefix and
+ *                 the verified block alike) is row s % page_size of page
+ *                 block_table[b * max_pages + s / page_size] (all layers
+ *                 share the table);
+ *   page_size     a multiple of 64 (a 64-key tile lies in one page), else
+ *                 LIBRASPEC_EUNSUPPORTED; the logical capacity is
+ *                 max_pages * page_size (kv_len[b] + L[b] + 1 beyond it:
+ *                 LIBRASPEC_ST_KV_OVERFLOW, sequence skipped).
+ * A block-table entry read outside [0, n_pages) sets LIBRASPEC_ST_BAD_PAGE
+ * and page 0 is read instead (that sequence's rows are then meaningless).
+ * The workspace is sized as for the dense call with S_cap = max_pages *
+ * page_size. Each CTA reads the page ids of its tile range once per launch.
+ */
+int libraspec_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp,
+                                       const uint16_t* const* Vp, int n_layers, const int32_t* block_table,
+                                       int max_pages, int page_size, int n_pages, const int32_t* kv_len,
+                                       const int32_t* L, int B, int K, int Hq, int Hkv, int head_dim,
+                                       float softmax_scale, uint16_t* const* O, float* const* lse, void* workspace,
+                                       size_t ws_bytes, void* stream);
 
 /*
  * Step 4 — acceptance (paper Sec. 3.1; the standard speculative-sampling

@@ -36,6 +36,8 @@ SIGNATURES = {
     "libraspec_select_alpha": (_I, [_P, _I, _I, _I, _F, _P, _P, _P]),
     "libraspec_verify_attn": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_attn_layers": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
+    "libraspec_verify_attn_paged_layers": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _P, _P, _I, _I, _I, _I, _I, _F, _P, _P,
+                                                _P, _SZ, _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_round": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _I,
@@ -256,6 +258,41 @@ def libraspec_verify_attn_layers(layers, kv_len, L, ws: Workspace, softmax_scale
         float(softmax_scale), _ptr_array(outs), _ptr_array(lses) if lses is not None else None, ws.ptr, ws.nbytes,
         _stream(stream))
     _check(rc, "libraspec_verify_attn_layers")
+    return outs, lses
+
+
+def libraspec_verify_attn_paged_layers(layers, block_table, kv_len, L, ws: Workspace, softmax_scale=None,
+                                       want_lse=False, stream=None):
+    """layers: dicts with Q [B,K+1,Hq,d] and page pools Kp, Vp [n_pages,Hkv,page_size,d] (optionally O,
+    lse); block_table [B, max_pages] int32. Returns (O list, lse list or None)."""
+    n = len(layers)
+    if n == 0:
+        return [], None
+    B, K1, Hq, D = layers[0]["Q"].shape
+    n_pages, Hkv, page_size, _ = layers[0]["Kp"].shape
+    for i, lay in enumerate(layers):
+        _req(lay["Q"], torch.bfloat16, "Q[%d]" % i, (B, K1, Hq, D))
+        _req(lay["Kp"], torch.bfloat16, "Kp[%d]" % i, (n_pages, Hkv, page_size, D))
+        _req(lay["Vp"], torch.bfloat16, "Vp[%d]" % i, (n_pages, Hkv, page_size, D))
+    _req(block_table, torch.int32, "block_table")
+    if block_table.dim() != 2 or block_table.shape[0] != B:
+        raise ValueError("block_table must be [B, max_pages]")
+    max_pages = block_table.shape[1]
+    _req(kv_len, torch.int32, "kv_len", (B,))
+    _req(L, torch.int32, "L", (B,))
+    if softmax_scale is None:
+        softmax_scale = D ** -0.5
+    outs = [lay.get("O") if lay.get("O") is not None else torch.empty_like(lay["Q"]) for lay in layers]
+    lses = None
+    if want_lse:
+        lses = [lay.get("lse") if lay.get("lse") is not None else
+                torch.empty((B, K1, Hq), dtype=torch.float32, device=layers[0]["Q"].device) for lay in layers]
+    rc = load().libraspec_verify_attn_paged_layers(
+        _ptr_array([l["Q"] for l in layers]), _ptr_array([l["Kp"] for l in layers]),
+        _ptr_array([l["Vp"] for l in layers]), n, _ptr(block_table), max_pages, page_size, n_pages, _ptr(kv_len),
+        _ptr(L), B, K1 - 1, Hq, Hkv, D, float(softmax_scale), _ptr_array(outs),
+        _ptr_array(lses) if lses is not None else None, ws.ptr, ws.nbytes, _stream(stream))
+    _check(rc, "libraspec_verify_attn_paged_layers")
     return outs, lses
 
 

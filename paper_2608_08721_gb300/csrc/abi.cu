@@ -16,6 +16,10 @@ cudaError_t launch_select_alpha(const float*, int, int, int, double, int32_t*, i
 cudaError_t launch_verify_attn(const uint16_t*, const uint16_t*, const uint16_t*, const int32_t*, const int32_t*,
                                int, int, int, int, int, int, float, uint16_t*, float*, char*, const WsLayout&,
                                cudaStream_t);
+cudaError_t launch_verify_attn_paged_layers(const uint16_t* const*, const uint16_t* const*, const uint16_t* const*,
+                                            int, const int32_t*, int, int, int, const int32_t*, const int32_t*, int,
+                                            int, int, int, int, float, uint16_t* const*, float* const*, char*,
+                                            const WsLayout&, cudaStream_t);
 cudaError_t launch_verify_attn_layers(const uint16_t* const*, const uint16_t* const*, const uint16_t* const*, int,
                                       const int32_t*, const int32_t*, int, int, int, int, int, int, float,
                                       uint16_t* const*, float* const*, char*, const WsLayout&, cudaStream_t);
@@ -194,6 +198,36 @@ int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const
   return from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap,
                                              softmax_scale, O, lse, static_cast<char*>(workspace), lay,
                                              static_cast<cudaStream_t>(stream)));
+}
+
+int libraspec_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp,
+                                       const uint16_t* const* Vp, int n_layers, const int32_t* block_table,
+                                       int max_pages, int page_size, int n_pages, const int32_t* kv_len,
+                                       const int32_t* L, int B, int K, int Hq, int Hkv, int head_dim,
+                                       float softmax_scale, uint16_t* const* O, float* const* lse, void* workspace,
+                                       size_t ws_bytes, void* stream) {
+  if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
+  if (page_size < 64 || page_size % 64 != 0 || page_size > 65536) return LIBRASPEC_EUNSUPPORTED;
+  if (max_pages < 1 || n_pages < 1 || (long)max_pages * page_size > 0x7fffffffL ||
+      (long)n_pages * (Hkv > 0 ? Hkv : 1) > 0x7fffffffL || n_layers < 0)
+    return LIBRASPEC_EINVAL;
+  const int S_cap = max_pages * page_size;
+  if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap)) return LIBRASPEC_EINVAL;
+  if (B == 0 || n_layers == 0) return LIBRASPEC_OK;
+  if (!Q || !Kp || !Vp || !O || !kv_len || !L || !block_table || !aligned(block_table, 4)) return LIBRASPEC_EINVAL;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!Q[l] || !Kp[l] || !Vp[l] || !O[l]) return LIBRASPEC_EINVAL;
+    if (!aligned(Q[l], 16) || !aligned(Kp[l], 16) || !aligned(Vp[l], 16) || !aligned(O[l], 16))
+      return LIBRASPEC_EINVAL;
+    if (lse && lse[l] && !aligned(lse[l], 4)) return LIBRASPEC_EINVAL;
+  }
+  if (!(softmax_scale > 0.f)) return LIBRASPEC_EINVAL;
+  const WsLayout lay = ws_layout(B, K, 1, Hq, Hkv, head_dim, S_cap);
+  if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_verify_attn_paged_layers(Q, Kp, Vp, n_layers, block_table, max_pages, page_size, n_pages,
+                                                   kv_len, L, B, K, Hq, Hkv, head_dim, softmax_scale, O, lse,
+                                                   static_cast<char*>(workspace), lay,
+                                                   static_cast<cudaStream_t>(stream)));
 }
 
 extern "C++" {

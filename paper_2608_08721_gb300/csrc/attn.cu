@@ -403,6 +403,10 @@ struct AttnSmem {
   static constexpr int kColO = 256;                      // O[2]: D fp32 columns each
   static_assert(kColP + 32 * kPBufs <= kColO && kColO + 2 * D <= kTmemCols, "tensor memory");
   static_assert(kAlloc <= 227 * 1024, "shared memory per CTA");
+  // paged caches: the page of each of the CTA's tiles, after everything else
+  static constexpr int kPageCap = 4096;
+  static constexpr int kAllocPaged = kAlloc + kPageCap * 4;
+  static_assert(kAllocPaged <= 227 * 1024, "shared memory per CTA (paged)");
 };
 
 // Merging a layer's split groups. This CTA merges its share of rows
@@ -565,9 +569,14 @@ __device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int
   }
 }
 
-template <int D, int STAGES>
+// PAGED: the caches are page pools [n_pages, Hkv, page_size, d] and key s of
+// sequence b lives at page block_table[b * max_pages + s / page_size], row
+// s % page_size (page_size a multiple of 64, so a key tile lies in one page);
+// S_cap is then max_pages * page_size.
+template <int D, int STAGES, bool PAGED>
 __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     const __grid_constant__ LayerSet set, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
+    const int32_t* __restrict__ block_table, int max_pages, int page_size, int n_pages, int page_cache,
     int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, float* __restrict__ part_buf_o,
     float* __restrict__ part_buf_ml, size_t part_o_stride, size_t part_ml_stride, uint32_t* __restrict__ bar_cnt,
     int* __restrict__ status) {
@@ -703,6 +712,32 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     uint32_t item_ctr = 0, tile_ctr = 0;
     // lane 0 reads the abort flag for the whole warp (the loop body has warp-wide steps)
     auto aborted = [&]() { return __shfl_sync(0xffffffffu, misc[0], 0) != 0; };
+    // paged: the page of every tile of the range, read once for all layers
+    // (they share the block table); a range beyond the cache reads the
+    // table tile by tile
+    int32_t* tile_page = reinterpret_cast<int32_t*>(smem + SM::kBytes);
+    const bool pages_cached = PAGED && hi - lo <= page_cache;
+    auto page_of = [&](int b, int key) {
+      int id = __ldg(block_table + (size_t)b * max_pages + key / page_size);
+      if (id < 0 || id >= n_pages) {
+        raise_status(status, LIBRASPEC_ST_BAD_PAGE);
+        id = 0;  // read a valid page; the sequence's output is then meaningless
+      }
+      return id;
+    };
+    if (pages_cached) {
+      for (long long pos = lo; pos < hi;) {
+        const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, R, Hkv, S_cap);
+        const int nt = loc.p.n_tiles;
+        const long long gstart = loc.seq_start + (pos - loc.seq_start) / nt * nt;
+        const long long iend = gstart + nt < hi ? gstart + nt : hi;
+        const int key0 = (int)(pos - gstart) * kAttnTileKeys;
+        for (int i = lane; i < (int)(iend - pos); i += 32)
+          tile_page[pos - lo + i] = page_of(loc.b, key0 + i * kAttnTileKeys);
+        pos = iend;
+      }
+      __syncwarp();
+    }
     for (int layer = 0; layer < n_layers && !aborted(); ++layer) {
       // layer's dependent data (Q, the block's keys) is readable once every
       // CTA has finished the previous layer
@@ -726,6 +761,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         it.slot = (pos == gstart) ? 2 * c + 1 : 2 * c;
         const int n_tiles = (int)(iend - pos);
         const int zc = loc.b * Hkv + it.kvh;
+        const long long item_pos = pos;  // the item's first tile in the tile sequence
         pos = iend;
         const uint32_t q = item_ctr & 1;
         if (lane == 0) {
@@ -735,11 +771,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             const uint32_t s = tile_ctr % STAGES;
             const uint32_t bar = bFull + 8 * s;
             mbar_expect_tx(bar, 2 * SM::kTileBytes);
-            const int y = it.key0 + i * kAttnTileKeys;
+            int y = it.key0 + i * kAttnTileKeys, z = zc;
+            if (PAGED) {
+              const int page = pages_cached ? tile_page[item_pos - lo + i] : page_of(it.b, y);
+              z = page * Hkv + it.kvh;
+              y %= page_size;
+            }
 #pragma unroll
             for (int bx = 0; bx < SM::kBoxes; ++bx) {
-              tma_load_3d(sK + s * SM::kTileBytes + bx * 8192, &set.K[layer], bar, bx * 64, y, zc);
-              tma_load_3d(sV + s * SM::kTileBytes + bx * 8192, &set.V[layer], bar, bx * 64, y, zc);
+              tma_load_3d(sK + s * SM::kTileBytes + bx * 8192, &set.K[layer], bar, bx * 64, y, z);
+              tma_load_3d(sV + s * SM::kTileBytes + bx * 8192, &set.V[layer], bar, bx * 64, y, z);
             }
             ++tile_ctr;
           };
@@ -1161,16 +1202,34 @@ static int attn_min_tiles() {
   return t;
 }
 
-template <int D, int STAGES>
+// Paged caches (block_table != nullptr): Kc / Vc are page pools of n_pages
+// pages of page_size keys and S_cap = max_pages * page_size.
+// Tiles per CTA whose page ids are cached in shared memory (at most cap);
+// the LIBRASPEC_ATTN_PAGE_CACHE environment variable lowers it (0: read the
+// block table tile by tile). Read once per process.
+static int attn_page_cache(int cap) {
+  static int v = [] {
+    int a = -1;
+    if (const char* e = getenv("LIBRASPEC_ATTN_PAGE_CACHE")) {
+      if (sscanf(e, "%d", &a) != 1 || a < 0) a = -1;
+    }
+    return a;
+  }();
+  return v < 0 || v > cap ? cap : v;
+}
+
+template <int D, int STAGES, bool PAGED>
 static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
-                                   int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq,
-                                   int Hkv, int S_cap, float scale, uint16_t* const* O, float* const* lse, char* ws,
-                                   const WsLayout& lay, cudaStream_t stream) {
+                                   int n_layers, const int32_t* kv_len, const int32_t* L, const int32_t* block_table,
+                                   int max_pages, int page_size, int n_pages, int B, int K, int Hq, int Hkv, int S_cap,
+                                   float scale, uint16_t* const* O, float* const* lse, char* ws, const WsLayout& lay,
+                                   cudaStream_t stream) {
   using SM = AttnSmem<D, STAGES>;
-  auto kern = verify_attn_kernel<D, STAGES>;
+  constexpr int kSmem = PAGED ? SM::kAllocPaged : SM::kAlloc;
+  auto kern = verify_attn_kernel<D, STAGES, PAGED>;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kAlloc);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
@@ -1185,7 +1244,10 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     set.n = n;
     for (int i = 0; i < n; ++i) {
       const int l = l0 + i;
-      if (!make_kv_map(&set.K[i], Kc[l], D, S_cap, B * Hkv) || !make_kv_map(&set.V[i], Vc[l], D, S_cap, B * Hkv) ||
+      // dense: [B*Hkv, S_cap, D]; paged: [n_pages*Hkv, page_size, D]
+      const int rows = PAGED ? page_size : S_cap;
+      const int planes = PAGED ? n_pages * Hkv : B * Hkv;
+      if (!make_kv_map(&set.K[i], Kc[l], D, rows, planes) || !make_kv_map(&set.V[i], Vc[l], D, rows, planes) ||
           !make_q_map(&set.Q[i], Q[l], D, Hq, B * (K + 1), g, R))
         return cudaErrorInvalidValue;
       set.p[i].Q = reinterpret_cast<const __nv_bfloat16*>(Q[l]);
@@ -1196,7 +1258,7 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(kAttnThreads);
-    cfg.dynamicSmemBytes = SM::kAlloc;
+    cfg.dynamicSmemBytes = kSmem;
     cfg.stream = stream;
     // cooperative: every CTA is resident at once, which the layer barriers rely on
     cudaLaunchAttribute attr[1];
@@ -1205,7 +1267,8 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(
-        &cfg, kern, set, kv_len, L, B, K, Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(),
+        &cfg, kern, set, kv_len, L, block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
+        Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(),
         reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_half / sizeof(float),
         ml_half / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
     if (e != cudaSuccess) return e;
@@ -1220,10 +1283,25 @@ cudaError_t launch_verify_attn_layers(const uint16_t* const* Q, const uint16_t* 
                                       cudaStream_t stream) {
   if (B == 0 || n_layers == 0) return cudaSuccess;
   if (D == 128)
-    return launch_layers_t<128, 4>(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, S_cap, scale, O, lse, ws, lay,
-                                   stream);
-  return launch_layers_t<64, 8>(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, S_cap, scale, O, lse, ws, lay,
-                                stream);
+    return launch_layers_t<128, 4, false>(Q, Kc, Vc, n_layers, kv_len, L, nullptr, 0, 0, 0, B, K, Hq, Hkv, S_cap,
+                                          scale, O, lse, ws, lay, stream);
+  return launch_layers_t<64, 8, false>(Q, Kc, Vc, n_layers, kv_len, L, nullptr, 0, 0, 0, B, K, Hq, Hkv, S_cap, scale,
+                                       O, lse, ws, lay, stream);
+}
+
+cudaError_t launch_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp,
+                                            const uint16_t* const* Vp, int n_layers, const int32_t* block_table,
+                                            int max_pages, int page_size, int n_pages, const int32_t* kv_len,
+                                            const int32_t* L, int B, int K, int Hq, int Hkv, int D, float scale,
+                                            uint16_t* const* O, float* const* lse, char* ws, const WsLayout& lay,
+                                            cudaStream_t stream) {
+  if (B == 0 || n_layers == 0) return cudaSuccess;
+  const int S_cap = max_pages * page_size;
+  if (D == 128)
+    return launch_layers_t<128, 4, true>(Q, Kp, Vp, n_layers, kv_len, L, block_table, max_pages, page_size, n_pages, B,
+                                         K, Hq, Hkv, S_cap, scale, O, lse, ws, lay, stream);
+  return launch_layers_t<64, 8, true>(Q, Kp, Vp, n_layers, kv_len, L, block_table, max_pages, page_size, n_pages, B,
+                                      K, Hq, Hkv, S_cap, scale, O, lse, ws, lay, stream);
 }
 
 cudaError_t launch_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc, const int32_t* kv_len,
