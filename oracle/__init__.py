@@ -61,9 +61,11 @@ def _load():
     lib.oracle_select_alpha.argtypes = [P, i32, i32, i32, f64, P, P, P]
     lib.oracle_gather_pages.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, P]
     lib.oracle_verify_attn.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, i32, f64, P, P, P, i32]
+    lib.oracle_verify_attn_tree.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32, i32, f64, P, P, P, i32]
     lib.oracle_accept.argtypes = [P, P, P, P, P, i32, i32, i32, u64, u64, u32, P, P, P]
+    lib.oracle_accept_tree_greedy.argtypes = [P, P, P, P, i32, i32, i32, P, P, P]
     for name in ("oracle_confidence", "oracle_select_lengths", "oracle_select_iterate", "oracle_select_alpha",
-                 "oracle_gather_pages",
+                 "oracle_gather_pages", "oracle_verify_attn_tree", "oracle_accept_tree_greedy",
                  "oracle_verify_attn", "oracle_accept"):
         getattr(lib, name).restype = i32
     _lib = lib
@@ -207,6 +209,49 @@ def verify_attn(Q, Kc, Vc, kv_len, L, scale=None, rows=None, fill=np.nan):
                                       Hkv, d, S_cap, float(scale), _ptr(O), _ptr(lse), _ptr(rws), n_rows),
            "oracle_verify_attn")
     return O, lse
+
+
+def verify_attn_tree(Q, Kc, Vc, kv_len, L, parent, scale=None, rows=None, fill=np.nan):
+    """verify_attn of a draft tree: parent [B,K+1] (int32; parent[b,t] in [0,t) for 1 <= t <= L_b)."""
+    Qb, Kb, Vb = (_as_bf16_bits(t) for t in (Q, Kc, Vc))
+    B, K1, Hq, d = Qb.shape
+    _, Hkv, S_cap, d2 = Kb.shape
+    if d2 != d or Vb.shape != Kb.shape or Kb.shape[0] != B:
+        raise OracleError("shape mismatch")
+    par = _c(parent, np.int32)
+    if par.shape != (B, K1):
+        raise OracleError("parent must be [B,K+1]")
+    if scale is None:
+        scale = 1.0 / np.sqrt(d)
+    kl = _c(kv_len, np.int32)
+    LL = _c(L, np.int32)
+    O = np.full((B, K1, Hq, d), fill, np.float64)
+    lse = np.full((B, K1, Hq), fill, np.float64)
+    rws = None if rows is None else _c(rows, np.int32).reshape(-1, 3)
+    n_rows = 0 if rws is None else rws.shape[0]
+    _check(_load().oracle_verify_attn_tree(_ptr(Qb), _ptr(Kb), _ptr(Vb), _ptr(kl), _ptr(LL), _ptr(par), B, K1 - 1,
+                                           Hq, Hkv, d, S_cap, float(scale), _ptr(O), _ptr(lse), _ptr(rws), n_rows),
+           "oracle_verify_attn_tree")
+    return O, lse
+
+
+def accept_tree_greedy(target_logits, draft_tokens, parent, L):
+    """Greedy walk of a draft tree: n_accepted[B], last_node[B], bonus_token[B] (int32)."""
+    t = _c(target_logits, np.float32)
+    B, K1, V = t.shape
+    tok = _c(draft_tokens, np.int32)
+    if tok.shape != (B, K1 - 1):
+        raise OracleError("draft_tokens must be [B,K]")
+    par = _c(parent, np.int32)
+    if par.shape != (B, K1):
+        raise OracleError("parent must be [B,K+1]")
+    LL = _c(L, np.int32)
+    n = np.zeros(B, np.int32)
+    last = np.zeros(B, np.int32)
+    bonus = np.zeros(B, np.int32)
+    _check(_load().oracle_accept_tree_greedy(_ptr(t), _ptr(tok), _ptr(par), _ptr(LL), B, K1 - 1, V,
+                                             _ptr(n), _ptr(last), _ptr(bonus)), "oracle_accept_tree_greedy")
+    return n, last, bonus
 
 
 def accept(target_logits, draft_logits, draft_tokens, L, temperature, seed, round_offset=0,

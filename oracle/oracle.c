@@ -24,6 +24,10 @@
  *                          block-wise drafting budget, one rollback.
  *   oracle_gather_pages    the dense KV cache a paged cache (page pool and
  *                          block table) describes.
+ *   oracle_verify_attn_tree, oracle_accept_tree_greedy
+ *                          verification of a draft tree (the tree drafters
+ *                          of Sec. 2, e.g. DDTree): ancestor-masked
+ *                          attention and the greedy longest accepted path.
  *   oracle_verify_attn     block-causal GQA attention of the d+1 verified
  *                          positions against the target KV cache (Sec. 3.1:
  *                          the target scores all drafted positions in one
@@ -412,13 +416,48 @@ int oracle_gather_pages(const uint16_t* pool, const int32_t* block_table, int B,
 /* bit patterns); lse [B, K+1, Hq] natural log.                        */
 /* If rows != NULL only the n_rows listed triples (b, h, t) are done.  */
 /* ------------------------------------------------------------------ */
-int oracle_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc,
-                       const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
-                       int dh, int S_cap, double scale, double* O, double* lse,
-                       const int32_t* rows, int n_rows) {
+/* One query row over the visible keys keys[0..n_keys) (ascending), as
+ * verify attention computes it: scores, max, exponentials, weighted sum. */
+static void attn_row(const double* qv, const uint16_t* Kh, const uint16_t* Vh, int dh, double scale,
+                     const int* keys, int n_keys, double* s, double* acc, double* out, double* lse_out) {
+  double m = -INFINITY;
+  for (int jj = 0; jj < n_keys; ++jj) {
+    const int j = keys[jj];
+    double dot = 0.0;
+    for (int i = 0; i < dh; ++i) dot += qv[i] * bf16_to_double(Kh[(size_t)j * dh + i]);
+    s[jj] = dot * scale;
+    if (s[jj] > m) m = s[jj];
+  }
+  double l = 0.0;
+  for (int i = 0; i < dh; ++i) acc[i] = 0.0;
+  for (int jj = 0; jj < n_keys; ++jj) {
+    const int j = keys[jj];
+    double w = exp(s[jj] - m);
+    l += w;
+    for (int i = 0; i < dh; ++i) acc[i] += w * bf16_to_double(Vh[(size_t)j * dh + i]);
+  }
+  for (int i = 0; i < dh; ++i) out[i] = acc[i] / l;
+  if (lse_out) *lse_out = m + log(l);
+}
+
+/* parent == NULL: the chain draft (row t sees keys 0 .. kv_len_b + t).
+ * Otherwise a draft tree: node t in [0, L_b] has parent[b * (K+1) + t] in
+ * [0, t) (node 0, the last accepted token, is the root), its keys sit at
+ * kv_len_b + t, and node t sees the cache prefix and the keys of its
+ * ancestors and itself. A chain tree (parent t-1) is the chain draft. */
+static int verify_attn_impl(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc,
+                            const int32_t* kv_len, const int32_t* L, const int32_t* parent, int B, int K,
+                            int Hq, int Hkv, int dh, int S_cap, double scale, double* O, double* lse,
+                            const int32_t* rows, int n_rows) {
   if (B < 0 || K < 0 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || dh < 1 || S_cap < 1) return ORACLE_EINVAL;
   for (int b = 0; b < B; ++b)
     if (L[b] < 0 || L[b] > K || kv_len[b] < 0 || (long)kv_len[b] + L[b] + 1 > S_cap) return ORACLE_EINVAL;
+  if (parent)
+    for (int b = 0; b < B; ++b)
+      for (int t = 1; t <= L[b]; ++t) {
+        const int p = parent[(size_t)b * (K + 1) + t];
+        if (p < 0 || p >= t) return ORACLE_EINVAL;
+      }
   const int g = Hq / Hkv;
   long total = rows ? n_rows : (long)B * Hq * (K + 1);
 #pragma omp parallel
@@ -426,6 +465,8 @@ int oracle_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc
     double* s = (double*)malloc(sizeof(double) * (size_t)S_cap);
     double* qv = (double*)malloc(sizeof(double) * (size_t)dh);
     double* acc = (double*)malloc(sizeof(double) * (size_t)dh);
+    int* keys = (int*)malloc(sizeof(int) * (size_t)S_cap);
+    char* anc = (char*)malloc((size_t)K + 1);
 #pragma omp for schedule(dynamic, 1)
     for (long it = 0; it < total; ++it) {
       int b, h, t;
@@ -442,25 +483,75 @@ int oracle_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc
       for (int i = 0; i < dh; ++i) qv[i] = bf16_to_double(Q[qoff + i]);
       const uint16_t* Kh = Kc + ((size_t)b * Hkv + kvh) * (size_t)S_cap * dh;
       const uint16_t* Vh = Vc + ((size_t)b * Hkv + kvh) * (size_t)S_cap * dh;
-      int n_keys = kv_len[b] + t + 1;
-      double m = -INFINITY;
-      for (int j = 0; j < n_keys; ++j) {
-        double dot = 0.0;
-        for (int i = 0; i < dh; ++i) dot += qv[i] * bf16_to_double(Kh[(size_t)j * dh + i]);
-        s[j] = dot * scale;
-        if (s[j] > m) m = s[j];
+      int n_keys = 0;
+      for (int j = 0; j < kv_len[b]; ++j) keys[n_keys++] = j;
+      if (!parent) {
+        for (int a = 0; a <= t; ++a) keys[n_keys++] = kv_len[b] + a;
+      } else {
+        for (int a = 0; a <= t; ++a) anc[a] = 0;
+        for (int a = t; a > 0; a = parent[(size_t)b * (K + 1) + a]) anc[a] = 1;
+        anc[0] = 1;
+        for (int a = 0; a <= t; ++a)
+          if (anc[a]) keys[n_keys++] = kv_len[b] + a;
       }
-      double l = 0.0;
-      for (int i = 0; i < dh; ++i) acc[i] = 0.0;
-      for (int j = 0; j < n_keys; ++j) {
-        double w = exp(s[j] - m);
-        l += w;
-        for (int i = 0; i < dh; ++i) acc[i] += w * bf16_to_double(Vh[(size_t)j * dh + i]);
-      }
-      for (int i = 0; i < dh; ++i) O[qoff + i] = acc[i] / l;
-      if (lse) lse[((size_t)b * (K + 1) + t) * Hq + h] = m + log(l);
+      attn_row(qv, Kh, Vh, dh, scale, keys, n_keys, s, acc, O + qoff,
+               lse ? lse + ((size_t)b * (K + 1) + t) * Hq + h : NULL);
     }
-    free(s); free(qv); free(acc);
+    free(s); free(qv); free(acc); free(keys); free(anc);
+  }
+  return ORACLE_OK;
+}
+
+int oracle_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc,
+                       const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                       int dh, int S_cap, double scale, double* O, double* lse,
+                       const int32_t* rows, int n_rows) {
+  return verify_attn_impl(Q, Kc, Vc, kv_len, L, NULL, B, K, Hq, Hkv, dh, S_cap, scale, O, lse, rows, n_rows);
+}
+
+/* Verify attention of a draft tree (tree verification as in the tree
+ * drafters the paper builds on, Sec. 2): parent [B, K+1], see above. */
+int oracle_verify_attn_tree(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc,
+                            const int32_t* kv_len, const int32_t* L, const int32_t* parent, int B, int K,
+                            int Hq, int Hkv, int dh, int S_cap, double scale, double* O, double* lse,
+                            const int32_t* rows, int n_rows) {
+  if (!parent) return ORACLE_EINVAL;
+  return verify_attn_impl(Q, Kc, Vc, kv_len, L, parent, B, K, Hq, Hkv, dh, S_cap, scale, O, lse, rows, n_rows);
+}
+
+/* Greedy acceptance of a draft tree: from the root (node 0), follow the
+ * lowest-numbered child whose token is the target's argmax at the current
+ * node (lowest index on ties) while there is one; n = nodes accepted
+ * below the root, last = the final node, bonus = the argmax there. Node
+ * t >= 1 carries draft token tokens[b * K + t - 1] (the chain layout). A
+ * chain tree gives the chain's greedy acceptance. */
+int oracle_accept_tree_greedy(const float* target, const int32_t* tokens, const int32_t* parent,
+                              const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
+                              int32_t* bonus) {
+  if (B < 0 || K < 0 || V < 1 || !target || !tokens || !parent || !L || !n_accepted || !bonus) return ORACLE_EINVAL;
+  for (int b = 0; b < B; ++b) {
+    if (L[b] < 0 || L[b] > K) return ORACLE_EINVAL;
+    for (int t = 1; t <= L[b]; ++t) {
+      const int p = parent[(size_t)b * (K + 1) + t];
+      if (p < 0 || p >= t) return ORACLE_EINVAL;
+      if (tokens[(size_t)b * K + t - 1] < 0 || tokens[(size_t)b * K + t - 1] >= V) return ORACLE_EINVAL;
+    }
+    int cur = 0, n = 0, arg = 0;
+    for (;;) {
+      arg = row_argmax(target + ((size_t)b * (K + 1) + cur) * V, V);
+      int next = -1;
+      for (int c = cur + 1; c <= L[b]; ++c)
+        if (parent[(size_t)b * (K + 1) + c] == cur && tokens[(size_t)b * K + c - 1] == arg) {
+          next = c;
+          break;
+        }
+      if (next < 0) break;
+      cur = next;
+      ++n;
+    }
+    n_accepted[b] = n;
+    if (last_node) last_node[b] = cur;
+    bonus[b] = arg;
   }
   return ORACLE_OK;
 }

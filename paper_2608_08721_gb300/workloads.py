@@ -218,6 +218,45 @@ def layer(w: Workload, l: int, kv: np.ndarray, device="cpu", peaky: bool = False
     return {"Q": Q, "Kc": Kc, "Vc": Vc}
 
 
+def draft_tree(B: int, K: int, L, seed: int, shape: str = "topk") -> np.ndarray:
+    """Parent array [B, K+1] (int32) of a draft tree per sequence.
+
+    Node 0 is the root (the last accepted token); node t in [1, L_b] has
+    parent[b, t] in [0, t), so node numbers are a topological order; entries
+    t > L_b and the root's are 0. Shapes: ``chain`` (parent t-1, the chain
+    draft), ``star`` (every node a child of the root), ``random`` (uniform
+    recursive tree) and ``topk``: the shape tree drafters grow from
+    per-position candidate lists, a main path with up to three alternatives
+    hanging off each depth (breadth-first: depth by depth, candidates in rank
+    order, each alternative a child of the previous depth's best node)."""
+    rng = np.random.default_rng([seed, 77])
+    L = np.broadcast_to(np.asarray(L, np.int64), (B,))
+    par = np.zeros((B, K + 1), np.int32)
+    for b in range(B):
+        n = int(L[b])
+        if shape == "chain":
+            par[b, 1:n + 1] = np.arange(0, n)
+        elif shape == "star":
+            par[b, 1:n + 1] = 0
+        elif shape == "random":
+            for t in range(1, n + 1):
+                par[b, t] = rng.integers(0, t)
+        elif shape == "topk":
+            t, best = 1, 0
+            while t <= n:
+                width = int(rng.integers(1, 5))
+                first = t
+                for _ in range(width):
+                    if t > n:
+                        break
+                    par[b, t] = best
+                    t += 1
+                best = first
+        else:
+            raise ValueError(shape)
+    return par
+
+
 def reference_inputs_summary(w: Workload) -> List[str]:
     """One line per input recipe, for reports."""
     return [
