@@ -18,6 +18,7 @@ LIB_PATH = os.path.join(_HERE, "libraspec.so")
 
 OK, EINVAL, EUNSUPPORTED, ECUDA, EDEVICE = 0, -1, -2, -3, -4
 ST_BAD_LENGTH, ST_BAD_COST, ST_KV_OVERFLOW, ST_BAD_TOKEN, ST_TIMEOUT, ST_MISSING_INPUT = 1, 2, 4, 8, 16, 32
+ST_BAD_PAGE, ST_BAD_TREE = 0x40, 0x80
 MAX_K = 64
 
 # Every entry point declared in include/libraspec.h, with its ctypes signature.
@@ -38,6 +39,12 @@ SIGNATURES = {
     "libraspec_verify_attn_layers": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_attn_paged_layers": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _P, _P, _I, _I, _I, _I, _I, _F, _P, _P,
                                                 _P, _SZ, _P]),
+    "libraspec_verify_attn_tree_layers": (_I, [_P, _P, _P, _I, _P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P,
+                                               _SZ, _P]),
+    "libraspec_verify_attn_tree_paged_layers": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _P, _P, _I, _I, _I, _I, _I,
+                                                     _F, _P, _P, _P, _SZ, _P]),
+    "libraspec_accept_tree_greedy": (_I, [_P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _SZ, _P]),
+    "libraspec_accept_tree_greedy_bf16": (_I, [_P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _SZ, _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_round": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _I,
@@ -234,6 +241,20 @@ def libraspec_verify_attn(Q, Kc, Vc, kv_len, L, ws: Workspace, softmax_scale=Non
 def libraspec_verify_attn_layers(layers, kv_len, L, ws: Workspace, softmax_scale=None, want_lse=False,
                                  stream=None):
     """layers: sequence of dicts with Q, Kc, Vc (and optionally O, lse). Returns (O list, lse list or None)."""
+    return _attn_layers(layers, None, kv_len, L, ws, softmax_scale, want_lse, stream)
+
+
+def libraspec_verify_attn_tree_layers(layers, parent, kv_len, L, ws: Workspace, softmax_scale=None, want_lse=False,
+                                      stream=None):
+    """Draft-tree verify attention; parent [B, K+1] int32 (parent[b, t] < t). As libraspec_verify_attn_layers."""
+    return _attn_layers(layers, parent, kv_len, L, ws, softmax_scale, want_lse, stream)
+
+
+def _check_parent(parent, B, K1):
+    _req(parent, torch.int32, "parent", (B, K1))
+
+
+def _attn_layers(layers, parent, kv_len, L, ws, softmax_scale, want_lse, stream):
     n = len(layers)
     if n == 0:
         return [], None
@@ -245,6 +266,8 @@ def libraspec_verify_attn_layers(layers, kv_len, L, ws: Workspace, softmax_scale
         _req(lay["Vc"], torch.bfloat16, "Vc[%d]" % i, (B, Hkv, S_cap, D))
     _req(kv_len, torch.int32, "kv_len", (B,))
     _req(L, torch.int32, "L", (B,))
+    if parent is not None:
+        _check_parent(parent, B, K1)
     if softmax_scale is None:
         softmax_scale = D ** -0.5
     outs = [lay.get("O") if lay.get("O") is not None else torch.empty_like(lay["Q"]) for lay in layers]
@@ -252,12 +275,16 @@ def libraspec_verify_attn_layers(layers, kv_len, L, ws: Workspace, softmax_scale
     if want_lse:
         lses = [lay.get("lse") if lay.get("lse") is not None else
                 torch.empty((B, K1, Hq), dtype=torch.float32, device=layers[0]["Q"].device) for lay in layers]
-    rc = load().libraspec_verify_attn_layers(
-        _ptr_array([l["Q"] for l in layers]), _ptr_array([l["Kc"] for l in layers]),
-        _ptr_array([l["Vc"] for l in layers]), n, _ptr(kv_len), _ptr(L), B, K1 - 1, Hq, Hkv, D, S_cap,
-        float(softmax_scale), _ptr_array(outs), _ptr_array(lses) if lses is not None else None, ws.ptr, ws.nbytes,
-        _stream(stream))
-    _check(rc, "libraspec_verify_attn_layers")
+    args = [_ptr_array([l["Q"] for l in layers]), _ptr_array([l["Kc"] for l in layers]),
+            _ptr_array([l["Vc"] for l in layers]), n]
+    name = "libraspec_verify_attn_layers"
+    if parent is not None:
+        args.append(_ptr(parent))
+        name = "libraspec_verify_attn_tree_layers"
+    rc = getattr(load(), name)(
+        *args, _ptr(kv_len), _ptr(L), B, K1 - 1, Hq, Hkv, D, S_cap, float(softmax_scale), _ptr_array(outs),
+        _ptr_array(lses) if lses is not None else None, ws.ptr, ws.nbytes, _stream(stream))
+    _check(rc, name)
     return outs, lses
 
 
@@ -265,6 +292,16 @@ def libraspec_verify_attn_paged_layers(layers, block_table, kv_len, L, ws: Works
                                        want_lse=False, stream=None):
     """layers: dicts with Q [B,K+1,Hq,d] and page pools Kp, Vp [n_pages,Hkv,page_size,d] (optionally O,
     lse); block_table [B, max_pages] int32. Returns (O list, lse list or None)."""
+    return _attn_paged_layers(layers, None, block_table, kv_len, L, ws, softmax_scale, want_lse, stream)
+
+
+def libraspec_verify_attn_tree_paged_layers(layers, parent, block_table, kv_len, L, ws: Workspace,
+                                            softmax_scale=None, want_lse=False, stream=None):
+    """Draft-tree verify attention over a paged cache; parent [B, K+1] int32."""
+    return _attn_paged_layers(layers, parent, block_table, kv_len, L, ws, softmax_scale, want_lse, stream)
+
+
+def _attn_paged_layers(layers, parent, block_table, kv_len, L, ws, softmax_scale, want_lse, stream):
     n = len(layers)
     if n == 0:
         return [], None
@@ -280,6 +317,8 @@ def libraspec_verify_attn_paged_layers(layers, block_table, kv_len, L, ws: Works
     max_pages = block_table.shape[1]
     _req(kv_len, torch.int32, "kv_len", (B,))
     _req(L, torch.int32, "L", (B,))
+    if parent is not None:
+        _check_parent(parent, B, K1)
     if softmax_scale is None:
         softmax_scale = D ** -0.5
     outs = [lay.get("O") if lay.get("O") is not None else torch.empty_like(lay["Q"]) for lay in layers]
@@ -287,12 +326,17 @@ def libraspec_verify_attn_paged_layers(layers, block_table, kv_len, L, ws: Works
     if want_lse:
         lses = [lay.get("lse") if lay.get("lse") is not None else
                 torch.empty((B, K1, Hq), dtype=torch.float32, device=layers[0]["Q"].device) for lay in layers]
-    rc = load().libraspec_verify_attn_paged_layers(
-        _ptr_array([l["Q"] for l in layers]), _ptr_array([l["Kp"] for l in layers]),
-        _ptr_array([l["Vp"] for l in layers]), n, _ptr(block_table), max_pages, page_size, n_pages, _ptr(kv_len),
-        _ptr(L), B, K1 - 1, Hq, Hkv, D, float(softmax_scale), _ptr_array(outs),
-        _ptr_array(lses) if lses is not None else None, ws.ptr, ws.nbytes, _stream(stream))
-    _check(rc, "libraspec_verify_attn_paged_layers")
+    args = [_ptr_array([l["Q"] for l in layers]), _ptr_array([l["Kp"] for l in layers]),
+            _ptr_array([l["Vp"] for l in layers]), n]
+    name = "libraspec_verify_attn_paged_layers"
+    if parent is not None:
+        args.append(_ptr(parent))
+        name = "libraspec_verify_attn_tree_paged_layers"
+    rc = getattr(load(), name)(
+        *args, _ptr(block_table), max_pages, page_size, n_pages, _ptr(kv_len), _ptr(L), B, K1 - 1, Hq, Hkv, D,
+        float(softmax_scale), _ptr_array(outs), _ptr_array(lses) if lses is not None else None, ws.ptr, ws.nbytes,
+        _stream(stream))
+    _check(rc, name)
     return outs, lses
 
 
@@ -322,6 +366,28 @@ def libraspec_accept(target_logits, draft_logits, draft_tokens, conf, dstat, L, 
                                _stream(stream))
     _check(rc, name)
     return n_accepted, bonus_token
+
+
+def libraspec_accept_tree_greedy(target_logits, draft_tokens, parent, L, ws: Workspace, n_accepted=None,
+                                 last_node=None, bonus_token=None, stream=None):
+    """Greedy walk of a draft tree. Returns (n_accepted, last_node, bonus_token), int32 [B] each."""
+    B, K1, V = target_logits.shape
+    K = K1 - 1
+    bf16 = target_logits.dtype == torch.bfloat16
+    _req(target_logits, torch.bfloat16 if bf16 else torch.float32, "target_logits")
+    _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+    _check_parent(parent, B, K1)
+    _req(L, torch.int32, "L", (B,))
+    dev = target_logits.device
+    n_accepted = torch.empty((B,), dtype=torch.int32, device=dev) if n_accepted is None else n_accepted
+    last_node = torch.empty((B,), dtype=torch.int32, device=dev) if last_node is None else last_node
+    bonus_token = torch.empty((B,), dtype=torch.int32, device=dev) if bonus_token is None else bonus_token
+    name = "libraspec_accept_tree_greedy_bf16" if bf16 else "libraspec_accept_tree_greedy"
+    rc = getattr(load(), name)(_ptr(target_logits), _ptr(draft_tokens), _ptr(parent), _ptr(L), B, K, V,
+                               _ptr(n_accepted), _ptr(last_node), _ptr(bonus_token), ws.ptr, ws.nbytes,
+                               _stream(stream))
+    _check(rc, name)
+    return n_accepted, last_node, bonus_token
 
 
 def _ptr_array(tensors: Sequence[Optional[torch.Tensor]]):

@@ -17,12 +17,15 @@ cudaError_t launch_verify_attn(const uint16_t*, const uint16_t*, const uint16_t*
                                int, int, int, int, int, int, float, uint16_t*, float*, char*, const WsLayout&,
                                cudaStream_t);
 cudaError_t launch_verify_attn_paged_layers(const uint16_t* const*, const uint16_t* const*, const uint16_t* const*,
-                                            int, const int32_t*, int, int, int, const int32_t*, const int32_t*, int,
-                                            int, int, int, int, float, uint16_t* const*, float* const*, char*,
-                                            const WsLayout&, cudaStream_t);
+                                            int, const int32_t*, const int32_t*, int, int, int, const int32_t*,
+                                            const int32_t*, int, int, int, int, int, float, uint16_t* const*,
+                                            float* const*, char*, const WsLayout&, cudaStream_t);
 cudaError_t launch_verify_attn_layers(const uint16_t* const*, const uint16_t* const*, const uint16_t* const*, int,
-                                      const int32_t*, const int32_t*, int, int, int, int, int, int, float,
-                                      uint16_t* const*, float* const*, char*, const WsLayout&, cudaStream_t);
+                                      const int32_t*, const int32_t*, const int32_t*, int, int, int, int, int, int,
+                                      float, uint16_t* const*, float* const*, char*, const WsLayout&, cudaStream_t);
+template <typename T>
+cudaError_t launch_accept_tree_greedy(const T*, const int32_t*, const int32_t*, const int32_t*, int, int, int,
+                                      int32_t*, int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
 template <typename T>
 cudaError_t launch_accept(const T*, const T*, const int32_t*, const float*, const float*, const int32_t*,
                           const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, char*,
@@ -178,14 +181,16 @@ int libraspec_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t*
                                       static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
 }
 
-int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
-                                 int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
-                                 int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,
-                                 void* workspace, size_t ws_bytes, void* stream) {
+namespace {
+
+int attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc, int n_layers,
+                const int32_t* parent, bool tree, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq,
+                int Hkv, int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,
+                void* workspace, size_t ws_bytes, void* stream) {
   if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
   if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap) || n_layers < 0) return LIBRASPEC_EINVAL;
   if (B == 0 || n_layers == 0) return LIBRASPEC_OK;
-  if (!Q || !Kc || !Vc || !O || !kv_len || !L) return LIBRASPEC_EINVAL;
+  if (!Q || !Kc || !Vc || !O || !kv_len || !L || (tree && !parent)) return LIBRASPEC_EINVAL;
   for (int l = 0; l < n_layers; ++l) {
     if (!Q[l] || !Kc[l] || !Vc[l] || !O[l]) return LIBRASPEC_EINVAL;
     if (!aligned(Q[l], 16) || !aligned(Kc[l], 16) || !aligned(Vc[l], 16) || !aligned(O[l], 16))
@@ -195,17 +200,16 @@ int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const
   if (!(softmax_scale > 0.f)) return LIBRASPEC_EINVAL;
   const WsLayout lay = ws_layout(B, K, 1, Hq, Hkv, head_dim, S_cap);
   if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
-  return from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap,
-                                             softmax_scale, O, lse, static_cast<char*>(workspace), lay,
+  return from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, parent, kv_len, L, B, K, Hq, Hkv, head_dim,
+                                             S_cap, softmax_scale, O, lse, static_cast<char*>(workspace), lay,
                                              static_cast<cudaStream_t>(stream)));
 }
 
-int libraspec_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp,
-                                       const uint16_t* const* Vp, int n_layers, const int32_t* block_table,
-                                       int max_pages, int page_size, int n_pages, const int32_t* kv_len,
-                                       const int32_t* L, int B, int K, int Hq, int Hkv, int head_dim,
-                                       float softmax_scale, uint16_t* const* O, float* const* lse, void* workspace,
-                                       size_t ws_bytes, void* stream) {
+int attn_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp, const uint16_t* const* Vp, int n_layers,
+                      const int32_t* parent, bool tree, const int32_t* block_table, int max_pages, int page_size,
+                      int n_pages, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                      int head_dim, float softmax_scale, uint16_t* const* O, float* const* lse, void* workspace,
+                      size_t ws_bytes, void* stream) {
   if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
   if (page_size < 64 || page_size % 64 != 0 || page_size > 65536) return LIBRASPEC_EUNSUPPORTED;
   if (max_pages < 1 || n_pages < 1 || (long)max_pages * page_size > 0x7fffffffL ||
@@ -215,6 +219,7 @@ int libraspec_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t*
   if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap)) return LIBRASPEC_EINVAL;
   if (B == 0 || n_layers == 0) return LIBRASPEC_OK;
   if (!Q || !Kp || !Vp || !O || !kv_len || !L || !block_table || !aligned(block_table, 4)) return LIBRASPEC_EINVAL;
+  if (tree && !parent) return LIBRASPEC_EINVAL;
   for (int l = 0; l < n_layers; ++l) {
     if (!Q[l] || !Kp[l] || !Vp[l] || !O[l]) return LIBRASPEC_EINVAL;
     if (!aligned(Q[l], 16) || !aligned(Kp[l], 16) || !aligned(Vp[l], 16) || !aligned(O[l], 16))
@@ -224,10 +229,49 @@ int libraspec_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t*
   if (!(softmax_scale > 0.f)) return LIBRASPEC_EINVAL;
   const WsLayout lay = ws_layout(B, K, 1, Hq, Hkv, head_dim, S_cap);
   if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
-  return from_cuda(launch_verify_attn_paged_layers(Q, Kp, Vp, n_layers, block_table, max_pages, page_size, n_pages,
-                                                   kv_len, L, B, K, Hq, Hkv, head_dim, softmax_scale, O, lse,
+  return from_cuda(launch_verify_attn_paged_layers(Q, Kp, Vp, n_layers, parent, block_table, max_pages, page_size,
+                                                   n_pages, kv_len, L, B, K, Hq, Hkv, head_dim, softmax_scale, O, lse,
                                                    static_cast<char*>(workspace), lay,
                                                    static_cast<cudaStream_t>(stream)));
+}
+
+}  // namespace
+
+int libraspec_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
+                                 int n_layers, const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                                 int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,
+                                 void* workspace, size_t ws_bytes, void* stream) {
+  return attn_layers(Q, Kc, Vc, n_layers, nullptr, false, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap, softmax_scale,
+                     O, lse, workspace, ws_bytes, stream);
+}
+
+int libraspec_verify_attn_tree_layers(const uint16_t* const* Q, const uint16_t* const* Kc,
+                                      const uint16_t* const* Vc, int n_layers, const int32_t* parent,
+                                      const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                                      int head_dim, int S_cap, float softmax_scale, uint16_t* const* O,
+                                      float* const* lse, void* workspace, size_t ws_bytes, void* stream) {
+  return attn_layers(Q, Kc, Vc, n_layers, parent, true, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap, softmax_scale, O,
+                     lse, workspace, ws_bytes, stream);
+}
+
+int libraspec_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp,
+                                       const uint16_t* const* Vp, int n_layers, const int32_t* block_table,
+                                       int max_pages, int page_size, int n_pages, const int32_t* kv_len,
+                                       const int32_t* L, int B, int K, int Hq, int Hkv, int head_dim,
+                                       float softmax_scale, uint16_t* const* O, float* const* lse, void* workspace,
+                                       size_t ws_bytes, void* stream) {
+  return attn_paged_layers(Q, Kp, Vp, n_layers, nullptr, false, block_table, max_pages, page_size, n_pages, kv_len, L,
+                           B, K, Hq, Hkv, head_dim, softmax_scale, O, lse, workspace, ws_bytes, stream);
+}
+
+int libraspec_verify_attn_tree_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp,
+                                            const uint16_t* const* Vp, int n_layers, const int32_t* parent,
+                                            const int32_t* block_table, int max_pages, int page_size, int n_pages,
+                                            const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                                            int head_dim, float softmax_scale, uint16_t* const* O,
+                                            float* const* lse, void* workspace, size_t ws_bytes, void* stream) {
+  return attn_paged_layers(Q, Kp, Vp, n_layers, parent, true, block_table, max_pages, page_size, n_pages, kv_len, L,
+                           B, K, Hq, Hkv, head_dim, softmax_scale, O, lse, workspace, ws_bytes, stream);
 }
 
 extern "C++" {
@@ -270,6 +314,39 @@ int libraspec_accept_bf16(const uint16_t* target_logits, const uint16_t* draft_l
 
 extern "C++" {
 template <typename T>
+static int accept_tree_t(const T* target_logits, const int32_t* draft_tokens, const int32_t* parent,
+                         const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
+                         int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
+  if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
+  if (B == 0) return LIBRASPEC_OK;
+  if (!target_logits || (!draft_tokens && K > 0) || (!parent && K > 0) || !L || !n_accepted || !bonus_token)
+    return LIBRASPEC_EINVAL;
+  if (!aligned(target_logits, sizeof(T))) return LIBRASPEC_EINVAL;
+  const WsLayout lay = ws_layout(B, K, V, 1, 1, 64, 1);
+  if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_accept_tree_greedy<T>(target_logits, draft_tokens, parent, L, B, K, V, n_accepted,
+                                                last_node, bonus_token, static_cast<char*>(workspace), lay,
+                                                static_cast<cudaStream_t>(stream)));
+}
+}  // extern "C++"
+
+int libraspec_accept_tree_greedy(const float* target_logits, const int32_t* draft_tokens, const int32_t* parent,
+                                 const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
+                                 int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
+  return accept_tree_t(target_logits, draft_tokens, parent, L, B, K, V, n_accepted, last_node, bonus_token,
+                       workspace, ws_bytes, stream);
+}
+
+int libraspec_accept_tree_greedy_bf16(const uint16_t* target_logits, const int32_t* draft_tokens,
+                                      const int32_t* parent, const int32_t* L, int B, int K, int V,
+                                      int32_t* n_accepted, int32_t* last_node, int32_t* bonus_token, void* workspace,
+                                      size_t ws_bytes, void* stream) {
+  return accept_tree_t(target_logits, draft_tokens, parent, L, B, K, V, n_accepted, last_node, bonus_token,
+                       workspace, ws_bytes, stream);
+}
+
+extern "C++" {
+template <typename T>
 static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, const float* temperature,
                            const float* cost_table, const T* target_logits, const uint16_t* const* Q,
                            const uint16_t* const* Kc, const uint16_t* const* Vc, uint16_t* const* O,
@@ -301,7 +378,7 @@ static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, co
   }
   rc = from_cuda(launch_select(conf, cost_table, B, K, L, ws, lay, s));
   if (rc != LIBRASPEC_OK) return rc;
-  rc = from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap,
+  rc = from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, nullptr, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap,
                                            softmax_scale, O, lse, ws, lay, s));
   if (rc != LIBRASPEC_OK) return rc;
   return accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed, round_offset,

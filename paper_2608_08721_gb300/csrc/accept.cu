@@ -25,7 +25,7 @@ __global__ void __launch_bounds__(kRowThreads) accept_rows_kernel(
   }
   if (j > Lb) return;
   const int row = b * (K + 1) + j;
-  const float tb = temperature[b];
+  const float tb = temperature ? temperature[b] : 0.f;  // none: every sequence greedy
   const bool sampling = tb > 0.f;
   const float T = sampling ? tb : 1.f;
   const float c = (float)(1.4426950408889634 / (double)T);
@@ -334,9 +334,108 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
 }
 
 // ---------------------------------------------------------------------------
+// Greedy walk of a draft tree, one warp per sequence. Node t in [1, L_b]
+// (parent[b, t] < t, token tokens[b, t-1]) is held by lane (t-1) % 32 in
+// slot (t-1) / 32. From the root, the next node is the lowest-numbered child
+// of the current one whose token is the argmax of the current node's target
+// row (argmaxes from accept_rows_kernel, staged in shared memory first so the
+// walk itself issues no global loads); n = nodes walked, last = the final
+// node, bonus = its argmax. A parent outside [0, t) or a token outside [0, V)
+// never matches and raises its status bit.
+// ---------------------------------------------------------------------------
+constexpr int kWalkWarps = 4;
+
+__global__ void __launch_bounds__(kWalkWarps * 32) tree_walk_kernel(
+    const int32_t* __restrict__ tokens, const int32_t* __restrict__ parent, const int32_t* __restrict__ Ls, int B,
+    int K, int V, const RowStat* __restrict__ stat, int32_t* __restrict__ n_accepted,
+    int32_t* __restrict__ last_node, int32_t* __restrict__ bonus, int* __restrict__ status) {
+  __shared__ int arg_s[kWalkWarps][LIBRASPEC_MAX_K + 1];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * kWalkWarps + w;
+  if (b >= B) return;
+  const int Lb = Ls[b];
+  if (Lb < 0 || Lb > K) {  // accept_rows_kernel raised the status
+    if (lane == 0) {
+      n_accepted[b] = 0;
+      if (last_node) last_node[b] = 0;
+      bonus[b] = 0;
+    }
+    return;
+  }
+  int* arg = arg_s[w];
+  for (int t = lane; t <= Lb; t += 32) arg[t] = __ldcg(&stat[(size_t)b * (K + 1) + t].arg);
+  int par[2], tok[2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int t = lane + 1 + 32 * i;
+    par[i] = -1;
+    tok[i] = -1;
+    if (t <= Lb) {
+      const int p = parent[(size_t)b * (K + 1) + t];
+      const int x = tokens[(size_t)b * K + t - 1];
+      if (p < 0 || p >= t) raise_status(status, LIBRASPEC_ST_BAD_TREE);
+      else if (x < 0 || x >= V) raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
+      else {
+        par[i] = p;
+        tok[i] = x;
+      }
+    }
+  }
+  __syncwarp();
+  int cur = 0, n = 0, a = arg[0];
+  for (int step = 0; step < Lb; ++step) {
+    const unsigned lo = __ballot_sync(0xffffffffu, par[0] == cur && tok[0] == a);
+    const unsigned hi = __ballot_sync(0xffffffffu, par[1] == cur && tok[1] == a);
+    if (!lo && !hi) break;
+    cur = lo ? __ffs(lo) : 32 + __ffs(hi);
+    ++n;
+    a = arg[cur];
+  }
+  if (lane == 0) {
+    n_accepted[b] = n;
+    if (last_node) last_node[b] = cur;
+    bonus[b] = a;
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Host launchers.
 // ---------------------------------------------------------------------------
 int num_sms_current();
+
+template <typename T>
+cudaError_t launch_accept_tree_greedy(const T* target, const int32_t* tokens, const int32_t* parent,
+                                      const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
+                                      int32_t* bonus, char* ws, const WsLayout& lay, cudaStream_t stream) {
+  if (B == 0) return cudaSuccess;
+  const int sms = num_sms_current();
+  auto* st = reinterpret_cast<int*>(ws + lay.status);
+  auto* rstat = reinterpret_cast<RowStat*>(ws + lay.row_stat);
+  const long rows = (long)B * (K + 1);
+  const int nsplit0 = row_splits(rows, V, sms, kRowMaxSplits, 4096);
+  const int chunk = row_chunk(V, nsplit0);
+  const int nsplit = (V + chunk - 1) / chunk;
+  dim3 grid(nsplit, K + 1, B);
+  auto* part = reinterpret_cast<RowPartial*>(ws + lay.row_part);
+  auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.row_cnt);
+  if (rows_vectorizable(target, V))
+    accept_rows_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(target, L, nullptr, K, V, nsplit, chunk, part, cnt,
+                                                                   rstat, st);
+  else
+    accept_rows_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(target, L, nullptr, K, V, nsplit, chunk, part, cnt,
+                                                                    rstat, st);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  tree_walk_kernel<<<(B + kWalkWarps - 1) / kWalkWarps, kWalkWarps * 32, 0, stream>>>(
+      tokens, parent, L, B, K, V, rstat, n_accepted, last_node, bonus, st);
+  return cudaGetLastError();
+}
+template cudaError_t launch_accept_tree_greedy<float>(const float*, const int32_t*, const int32_t*, const int32_t*,
+                                                      int, int, int, int32_t*, int32_t*, int32_t*, char*,
+                                                      const WsLayout&, cudaStream_t);
+template cudaError_t launch_accept_tree_greedy<uint16_t>(const uint16_t*, const int32_t*, const int32_t*,
+                                                         const int32_t*, int, int, int, int32_t*, int32_t*, int32_t*,
+                                                         char*, const WsLayout&, cudaStream_t);
 
 template <typename T>
 cudaError_t launch_accept(const T* target, const T* draft, const int32_t* tokens, const float* conf,

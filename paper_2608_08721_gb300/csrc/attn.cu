@@ -229,6 +229,16 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
+// bits [0, n) set (n clamped to [0, 64])
+__device__ __forceinline__ uint64_t low_bits(int n) {
+  return n <= 0 ? 0ull : (n >= 64 ? ~0ull : ((1ull << n) - 1ull));
+}
+
+// x << s for s >= 0, x >> -s for s < 0; 0 once |s| >= 64
+__device__ __forceinline__ uint64_t shift_bits(uint64_t x, int s) {
+  return (s >= 64 || s <= -64) ? 0ull : (s >= 0 ? x << s : x >> -s);
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -573,9 +583,13 @@ __device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int
 // sequence b lives at page block_table[b * max_pages + s / page_size], row
 // s % page_size (page_size a multiple of 64, so a key tile lies in one page);
 // S_cap is then max_pages * page_size.
+// tree_vis (optional, [B, K+1]): the block is a draft tree and row t sees the
+// block keys of the set bits (bit j <-> block position j + 1) besides the root
+// and the prefix; nullptr: the chain draft (block-causal).
 template <int D, int STAGES, bool PAGED>
 __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     const __grid_constant__ LayerSet set, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
+    const uint64_t* __restrict__ tree_vis,
     const int32_t* __restrict__ block_table, int max_pages, int page_size, int n_pages, int page_cache,
     int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, float* __restrict__ part_buf_o,
     float* __restrict__ part_buf_ml, size_t part_o_stride, size_t part_ml_stride, uint32_t* __restrict__ bar_cnt,
@@ -935,7 +949,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         // a warp without valid rows only keeps the barrier counts in step
         const bool warp_live = warp * 32 < it.rows;
         const int t_row = (it.mg * R + row) / g;
-        const int lim = it.kv + t_row;  // last visible key of this row
+        // Block keys seen by this row: bit j <-> key kv + 1 + j (the root, key
+        // kv, and the cache prefix are seen by every row). Chain: the t_row
+        // earlier positions; tree: the ancestors of node t_row and itself.
+        const uint64_t vis =
+            !valid ? 0ull : (tree_vis ? __ldg(tree_vis + (size_t)it.b * (K + 1) + t_row) : low_bits(t_row));
+        const int mask_from = tree_vis ? it.kv : it.kv + t_row;  // tiles past this key need the mask
         float m_run = -INFINITY, l_run = 0.f;
         for (int t = 0; t < n_tiles && ok; ++t) {
           const uint32_t gt = tile_ctr;
@@ -960,15 +979,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(bSFree + 8 * sb);
-          // raw scores; keys past this row's last visible key (and rows past
-          // the group) count as -inf; the scale (> 0) is applied below
-          const bool need_mask = !valid || kt0 + kAttnTileKeys - 1 > lim;
+          // raw scores; keys this row does not see (and rows past the
+          // group) count as -inf; the scale (> 0) is applied below
+          const bool need_mask = !valid || kt0 + kAttnTileKeys - 1 > mask_from;
+          const uint64_t tmask =
+              !valid ? 0ull : (low_bits(it.kv + 1 - kt0) | shift_bits(vis, it.kv + 1 - kt0));
           float xs[kAttnTileKeys];
           float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
           for (int c = 0; c < kAttnTileKeys; ++c) {
             float v = __uint_as_float(sr[c >> 5][c & 31]);
-            if (need_mask && (!valid || kt0 + c > lim)) v = -INFINITY;
+            if (need_mask && !((tmask >> c) & 1ull)) v = -INFINITY;
             xs[c] = v;
             mx[c & 3] = fmaxf(mx[c & 3], v);
           }
@@ -1202,6 +1223,81 @@ static int attn_min_tiles() {
   return t;
 }
 
+// Ancestor sets of a draft tree, one warp per sequence, by pointer jumping:
+// after round r, m[t] holds node t's ancestors at distance < 2^r and up[t]
+// the one at distance 2^r (the root absorbs: m[0] = 0, up[0] = 0), so 7
+// rounds cover depth 64. vis[b, t] bit j <-> block position j + 1 is node t
+// or an ancestor of it; rows t > L_b get 0. A parent outside [0, t) raises
+// LIBRASPEC_ST_BAD_TREE and is read as the root.
+constexpr int kTreeWarps = 4;
+constexpr int kTreeNodes = LIBRASPEC_MAX_K + 1;
+
+__global__ void __launch_bounds__(kTreeWarps * 32) tree_vis_kernel(const int32_t* __restrict__ parent,
+                                                                     const int32_t* __restrict__ Ls, int B, int K,
+                                                                     uint64_t* __restrict__ vis,
+                                                                     int* __restrict__ status) {
+  __shared__ int up_s[kTreeWarps][kTreeNodes];
+  __shared__ uint64_t m_s[kTreeWarps][kTreeNodes];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * kTreeWarps + w;
+  if (b >= B) return;
+  int* up = up_s[w];
+  uint64_t* m = m_s[w];
+  int Lb = Ls[b];
+  if (Lb < 0 || Lb > K) Lb = 0;  // the attention kernel reports the bad length
+  for (int t = lane; t <= K; t += 32) {
+    int p = 0;
+    uint64_t bit = 0ull;
+    if (t >= 1 && t <= Lb) {
+      p = parent[(size_t)b * (K + 1) + t];
+      if (p < 0 || p >= t) {
+        raise_status(status, LIBRASPEC_ST_BAD_TREE);
+        p = 0;
+      }
+      bit = 1ull << (t - 1);
+    }
+    up[t] = p;
+    m[t] = bit;
+  }
+  __syncwarp();
+  for (int r = 0; r < 7; ++r) {
+    int nu[3];
+    uint64_t nm[3];
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+      const int t = lane + 32 * i;
+      if (t <= K) {
+        const int u = up[t];
+        nm[i] = m[t] | m[u];
+        nu[i] = up[u];
+      }
+    }
+    __syncwarp();
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+      const int t = lane + 32 * i;
+      if (t <= K) {
+        m[t] = nm[i];
+        up[t] = nu[i];
+      }
+    }
+    __syncwarp();
+  }
+  for (int t = lane; t <= K; t += 32) vis[(size_t)b * (K + 1) + t] = m[t];
+}
+
+// parent != nullptr: fill the tree visibility masks of the workspace first.
+static cudaError_t tree_vis(const int32_t* parent, const int32_t* L, int B, int K, char* ws, const WsLayout& lay,
+                            cudaStream_t stream, const uint64_t** out) {
+  *out = nullptr;
+  if (!parent) return cudaSuccess;
+  auto* vis = reinterpret_cast<uint64_t*>(ws + lay.tree_vis);
+  tree_vis_kernel<<<(B + kTreeWarps - 1) / kTreeWarps, kTreeWarps * 32, 0, stream>>>(
+      parent, L, B, K, vis, reinterpret_cast<int*>(ws + lay.status));
+  *out = vis;
+  return cudaGetLastError();
+}
+
 // Paged caches (block_table != nullptr): Kc / Vc are page pools of n_pages
 // pages of page_size keys and S_cap = max_pages * page_size.
 // Tiles per CTA whose page ids are cached in shared memory (at most cap);
@@ -1220,7 +1316,8 @@ static int attn_page_cache(int cap) {
 
 template <int D, int STAGES, bool PAGED>
 static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* const* Kc, const uint16_t* const* Vc,
-                                   int n_layers, const int32_t* kv_len, const int32_t* L, const int32_t* block_table,
+                                   int n_layers, const int32_t* kv_len, const int32_t* L, const uint64_t* tree_vis,
+                                   const int32_t* block_table,
                                    int max_pages, int page_size, int n_pages, int B, int K, int Hq, int Hkv, int S_cap,
                                    float scale, uint16_t* const* O, float* const* lse, char* ws, const WsLayout& lay,
                                    cudaStream_t stream) {
@@ -1267,7 +1364,7 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(
-        &cfg, kern, set, kv_len, L, block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
+        &cfg, kern, set, kv_len, L, tree_vis, block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
         Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(),
         reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_half / sizeof(float),
         ml_half / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
@@ -1276,39 +1373,46 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
   return cudaSuccess;
 }
 
+// parent (optional, [B, K+1]): the block is a draft tree (nullptr: the chain).
 cudaError_t launch_verify_attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc,
-                                      const uint16_t* const* Vc, int n_layers, const int32_t* kv_len,
-                                      const int32_t* L, int B, int K, int Hq, int Hkv, int D, int S_cap, float scale,
-                                      uint16_t* const* O, float* const* lse, char* ws, const WsLayout& lay,
-                                      cudaStream_t stream) {
+                                      const uint16_t* const* Vc, int n_layers, const int32_t* parent,
+                                      const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv, int D,
+                                      int S_cap, float scale, uint16_t* const* O, float* const* lse, char* ws,
+                                      const WsLayout& lay, cudaStream_t stream) {
   if (B == 0 || n_layers == 0) return cudaSuccess;
+  const uint64_t* vis = nullptr;
+  cudaError_t e = tree_vis(parent, L, B, K, ws, lay, stream, &vis);
+  if (e != cudaSuccess) return e;
   if (D == 128)
-    return launch_layers_t<128, 4, false>(Q, Kc, Vc, n_layers, kv_len, L, nullptr, 0, 0, 0, B, K, Hq, Hkv, S_cap,
+    return launch_layers_t<128, 4, false>(Q, Kc, Vc, n_layers, kv_len, L, vis, nullptr, 0, 0, 0, B, K, Hq, Hkv, S_cap,
                                           scale, O, lse, ws, lay, stream);
-  return launch_layers_t<64, 8, false>(Q, Kc, Vc, n_layers, kv_len, L, nullptr, 0, 0, 0, B, K, Hq, Hkv, S_cap, scale,
-                                       O, lse, ws, lay, stream);
+  return launch_layers_t<64, 8, false>(Q, Kc, Vc, n_layers, kv_len, L, vis, nullptr, 0, 0, 0, B, K, Hq, Hkv, S_cap,
+                                       scale, O, lse, ws, lay, stream);
 }
 
 cudaError_t launch_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp,
-                                            const uint16_t* const* Vp, int n_layers, const int32_t* block_table,
-                                            int max_pages, int page_size, int n_pages, const int32_t* kv_len,
-                                            const int32_t* L, int B, int K, int Hq, int Hkv, int D, float scale,
-                                            uint16_t* const* O, float* const* lse, char* ws, const WsLayout& lay,
-                                            cudaStream_t stream) {
+                                            const uint16_t* const* Vp, int n_layers, const int32_t* parent,
+                                            const int32_t* block_table, int max_pages, int page_size, int n_pages,
+                                            const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                                            int D, float scale, uint16_t* const* O, float* const* lse, char* ws,
+                                            const WsLayout& lay, cudaStream_t stream) {
   if (B == 0 || n_layers == 0) return cudaSuccess;
   const int S_cap = max_pages * page_size;
+  const uint64_t* vis = nullptr;
+  cudaError_t e = tree_vis(parent, L, B, K, ws, lay, stream, &vis);
+  if (e != cudaSuccess) return e;
   if (D == 128)
-    return launch_layers_t<128, 4, true>(Q, Kp, Vp, n_layers, kv_len, L, block_table, max_pages, page_size, n_pages, B,
-                                         K, Hq, Hkv, S_cap, scale, O, lse, ws, lay, stream);
-  return launch_layers_t<64, 8, true>(Q, Kp, Vp, n_layers, kv_len, L, block_table, max_pages, page_size, n_pages, B,
-                                      K, Hq, Hkv, S_cap, scale, O, lse, ws, lay, stream);
+    return launch_layers_t<128, 4, true>(Q, Kp, Vp, n_layers, kv_len, L, vis, block_table, max_pages, page_size,
+                                         n_pages, B, K, Hq, Hkv, S_cap, scale, O, lse, ws, lay, stream);
+  return launch_layers_t<64, 8, true>(Q, Kp, Vp, n_layers, kv_len, L, vis, block_table, max_pages, page_size, n_pages,
+                                      B, K, Hq, Hkv, S_cap, scale, O, lse, ws, lay, stream);
 }
 
 cudaError_t launch_verify_attn(const uint16_t* Q, const uint16_t* Kc, const uint16_t* Vc, const int32_t* kv_len,
                                const int32_t* L, int B, int K, int Hq, int Hkv, int D, int S_cap, float scale,
                                uint16_t* O, float* lse, char* ws, const WsLayout& lay, cudaStream_t stream) {
   float* lse_arr[1] = {lse};
-  return launch_verify_attn_layers(&Q, &Kc, &Vc, 1, kv_len, L, B, K, Hq, Hkv, D, S_cap, scale, &O,
+  return launch_verify_attn_layers(&Q, &Kc, &Vc, 1, nullptr, kv_len, L, B, K, Hq, Hkv, D, S_cap, scale, &O,
                                    lse ? lse_arr : nullptr, ws, lay, stream);
 }
 

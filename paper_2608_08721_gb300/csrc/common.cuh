@@ -43,7 +43,7 @@ struct RacePartial {
 
 struct WsLayout {
   size_t status, conf_part, conf_cnt, row_part, row_cnt, row_stat, race_part, race_cnt;
-  size_t attn_o, attn_ml, attn_cnt, total;
+  size_t attn_o, attn_ml, attn_cnt, tree_vis, total;
   int max_items, max_groups;
 };
 
@@ -75,6 +75,8 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.attn_ml = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
   // grid-barrier counters, one per layer of a launch, then the exit counter
   w.attn_cnt = take((kAttnMaxLayers + 1) * sizeof(uint32_t));
+  // ancestor masks of a draft tree, one per block position
+  w.tree_vis = take(rows_t * sizeof(uint64_t));
   w.total = off;
   return w;
 }

@@ -1,0 +1,237 @@
+"""GPU parity: draft-tree verification (ancestor-masked verify attention and
+the greedy walk of the tree) vs. the oracle, bit-for-bit vs. the chain
+kernels on a chain tree, and the paged tree kernel vs. the dense one."""
+import numpy as np
+import pytest
+import torch
+
+from helpers import check_attn, cuda
+from paper_2608_08721_gb300 import binding as lr
+from paper_2608_08721_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def _layers(B, K, Hq, Hkv, d, S, seed, n_layers=1):
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    out = []
+    for _ in range(n_layers):
+        Q = torch.randn((B, K + 1, Hq, d), generator=g, device=cuda()).to(torch.bfloat16)
+        Kc = (torch.randn((B, Hkv, S, d), generator=g, device=cuda()) * 2.0).to(torch.bfloat16)
+        Vc = torch.randn((B, Hkv, S, d), generator=g, device=cuda()).to(torch.bfloat16)
+        out.append({"Q": Q, "Kc": Kc, "Vc": Vc})
+    return out
+
+
+def _i32(x):
+    return torch.as_tensor(np.asarray(x), dtype=torch.int32).to(cuda())
+
+
+def _run_tree(layers, parent, kv, L, K):
+    B, _, Hq, d = layers[0]["Q"].shape
+    _, Hkv, S, _ = layers[0]["Kc"].shape
+    ws = lr.Workspace(B, K, 1, Hq, Hkv, d, S, device=cuda())
+    outs, lses = lr.libraspec_verify_attn_tree_layers(layers, _i32(parent), _i32(kv), _i32(L), ws, want_lse=True)
+    torch.cuda.synchronize()
+    return outs, lses, lr.libraspec_get_status(ws)
+
+
+@pytest.mark.parametrize("shape", ["topk", "random", "star"])
+@pytest.mark.parametrize("d,Hq,Hkv", [(128, 32, 8), (64, 8, 2), (128, 28, 4)])
+def test_tree_attn_matches_oracle(orc, shape, d, Hq, Hkv):
+    K = 20
+    # block keys straddling a tile edge (kv % 64 near 63), at a tile start, a
+    # fresh sequence, a long prefix split over CTAs
+    kv = [0, 62, 64, 700, 2900, 127]
+    L = [20, 20, 5, 1, 17, 11]
+    B = len(kv)
+    S = (max(k + l + 1 for k, l in zip(kv, L)) + 63) // 64 * 64
+    parent = workloads.draft_tree(B, K, L, seed=d + Hq, shape=shape)
+    layers = _layers(B, K, Hq, Hkv, d, S, seed=d + Hq + len(shape))
+    outs, lses, status = _run_tree(layers, parent, kv, L, K)
+    assert status == 0
+    O_ref, lse_ref = orc.verify_attn_tree(layers[0]["Q"], layers[0]["Kc"], layers[0]["Vc"], np.array(kv),
+                                          np.array(L), parent)
+    check_attn(outs[0], lses[0], O_ref, lse_ref, L)
+
+
+def test_tree_attn_full_depth_and_width(orc):
+    """K = 64 (the mask's last bit): a depth-64 chain, a 64-leaf star and a
+    random tree, with the block at every offset within a tile."""
+    K, Hq, Hkv, d = 64, 8, 2, 128
+    kv = [0, 1, 63, 64, 65, 191]
+    L = [64] * 6
+    B = len(kv)
+    S = (max(kv) + K + 1 + 63) // 64 * 64
+    layers = _layers(B, K, Hq, Hkv, d, S, seed=64)
+    for shape in ("chain", "star", "random"):
+        parent = workloads.draft_tree(B, K, L, seed=7, shape=shape)
+        outs, lses, status = _run_tree(layers, parent, kv, L, K)
+        assert status == 0
+        O_ref, lse_ref = orc.verify_attn_tree(layers[0]["Q"], layers[0]["Kc"], layers[0]["Vc"], np.array(kv),
+                                              np.array(L), parent)
+        check_attn(outs[0], lses[0], O_ref, lse_ref, L)
+
+
+@pytest.mark.parametrize("d,Hq,Hkv", [(128, 32, 8), (64, 8, 2)])
+def test_chain_tree_is_bit_identical_to_chain_call(d, Hq, Hkv):
+    K = 16
+    kv = [5, 63, 1000, 4096, 0]
+    L = [16, 3, 16, 9, 0]
+    B = len(kv)
+    S = (max(k + l + 1 for k, l in zip(kv, L)) + 63) // 64 * 64
+    layers = _layers(B, K, Hq, Hkv, d, S, seed=3, n_layers=2)
+    parent = workloads.draft_tree(B, K, L, seed=0, shape="chain")
+    outs, lses, status = _run_tree(layers, parent, kv, L, K)
+    assert status == 0
+    ws = lr.Workspace(B, K, 1, Hq, Hkv, d, S, device=cuda())
+    o2, l2 = lr.libraspec_verify_attn_layers(layers, _i32(kv), _i32(L), ws, want_lse=True)
+    torch.cuda.synchronize()
+    for l in range(2):
+        for b in range(B):
+            assert torch.equal(outs[l][b, :L[b] + 1], o2[l][b, :L[b] + 1])
+            assert torch.equal(lses[l][b, :L[b] + 1], l2[l][b, :L[b] + 1])
+
+
+def test_tree_layers_in_one_launch_long_cache(orc):
+    """Three layers in one launch, 8b-like heads, a 20k prefix split over many
+    CTAs: sampled rows against the oracle."""
+    K, Hq, Hkv, d = 16, 32, 8, 128
+    kv, L = [20000, 300], [16, 12]
+    S = (max(kv) + K + 1 + 63) // 64 * 64
+    layers = _layers(2, K, Hq, Hkv, d, S, seed=8, n_layers=3)
+    parent = workloads.draft_tree(2, K, L, seed=8, shape="topk")
+    outs, lses, status = _run_tree(layers, parent, kv, L, K)
+    assert status == 0
+    rows = np.array([(b, h, t) for b in range(2) for h in (0, 13, Hq - 1) for t in range(L[b] + 1)], np.int32)
+    for l in range(3):
+        O_ref, lse_ref = orc.verify_attn_tree(layers[l]["Q"], layers[l]["Kc"], layers[l]["Vc"], np.array(kv),
+                                              np.array(L), parent, rows=rows)
+        check_attn(outs[l], lses[l], O_ref, lse_ref, L, rows=[tuple(r) for r in rows])
+
+
+def test_tree_paged_is_bit_identical_to_dense():
+    K, Hq, Hkv, d, P = 24, 32, 8, 128, 128
+    kv = [0, 63, 700, 3000]
+    L = [24, 10, 24, 7]
+    B = len(kv)
+    rng = np.random.default_rng(31)
+    S = max(k + l + 1 for k, l in zip(kv, L))
+    max_pages = -(-S // P)
+    n_pages = B * max_pages + 3
+    perm = rng.permutation(n_pages)[: B * max_pages].reshape(B, max_pages).astype(np.int32)
+    dense = _layers(B, K, Hq, Hkv, d, max_pages * P, seed=31, n_layers=2)
+    paged = []
+    for lay in dense:
+        Kp = torch.zeros((n_pages, Hkv, P, d), dtype=torch.bfloat16, device=cuda())
+        Vp = torch.zeros_like(Kp)
+        for b in range(B):
+            for j in range(max_pages):
+                Kp[perm[b, j]] = lay["Kc"][b, :, j * P:(j + 1) * P]
+                Vp[perm[b, j]] = lay["Vc"][b, :, j * P:(j + 1) * P]
+        paged.append({"Q": lay["Q"], "Kp": Kp, "Vp": Vp})
+    parent = workloads.draft_tree(B, K, L, seed=31, shape="random")
+    o_d, l_d, st = _run_tree(dense, parent, kv, L, K)
+    assert st == 0
+    ws = lr.Workspace(B, K, 1, Hq, Hkv, d, max_pages * P, device=cuda())
+    o_p, l_p = lr.libraspec_verify_attn_tree_paged_layers(paged, _i32(parent), _i32(perm), _i32(kv), _i32(L), ws,
+                                                         want_lse=True)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) == 0
+    for l in range(2):
+        for b in range(B):
+            assert torch.equal(o_p[l][b, :L[b] + 1], o_d[l][b, :L[b] + 1])
+            assert torch.equal(l_p[l][b, :L[b] + 1], l_d[l][b, :L[b] + 1])
+
+
+def test_tree_bad_parent_sets_status():
+    K, Hq, Hkv, d = 4, 8, 2, 64
+    kv, L = [100, 10], [3, 4]
+    layers = _layers(2, K, Hq, Hkv, d, 128, seed=2)
+    parent = workloads.draft_tree(2, K, L, seed=2, shape="random")
+    parent[1, 3] = 3  # not below its own number
+    _, _, status = _run_tree(layers, parent, kv, L, K)
+    assert status & lr.ST_BAD_TREE
+
+
+# ---------------------------------------------------------------------------
+# greedy walk
+# ---------------------------------------------------------------------------
+def _walk_inputs(B, K, V, shape, seed, dtype=torch.float32):
+    """Trees with distinct sibling tokens; target rows whose argmax is often
+    one of the node's children's tokens."""
+    rng = np.random.default_rng(seed)
+    L = rng.integers(0, K + 1, size=B).astype(np.int32)
+    L[0], L[-1] = K, 0
+    parent = workloads.draft_tree(B, K, L, seed=seed, shape=shape)
+    tok = np.zeros((B, K), np.int32)
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    x = torch.randn((B, K + 1, V), generator=g, device=cuda()) * 0.5
+    for b in range(B):
+        kids = [[] for _ in range(K + 1)]
+        for t in range(1, int(L[b]) + 1):
+            kids[parent[b, t]].append(t)
+        for p in range(K + 1):
+            vals = rng.choice(V, size=len(kids[p]), replace=False)
+            for t, v in zip(kids[p], vals):
+                tok[b, t - 1] = v
+            if kids[p] and rng.random() < 0.85:
+                x[b, p, int(tok[b, kids[p][rng.integers(len(kids[p]))] - 1])] = 6.0
+    return x.to(dtype), tok, parent, L
+
+
+@pytest.mark.parametrize("shape", ["topk", "random", "star", "chain"])
+@pytest.mark.parametrize("V", [32000, 152064, 1000])
+def test_tree_walk_matches_oracle(orc, shape, V):
+    B, K = 48, 24
+    x, tok, parent, L = _walk_inputs(B, K, V, shape, seed=V % 97 + len(shape))
+    ws = lr.Workspace(B, K, V, 1, 1, 64, 1, device=cuda())
+    n, last, bonus = lr.libraspec_accept_tree_greedy(x, _i32(tok), _i32(parent), _i32(L), ws)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) == 0
+    rn, rlast, rbonus = orc.accept_tree_greedy(x.cpu().numpy(), tok, parent, L)
+    np.testing.assert_array_equal(n.cpu().numpy(), rn)
+    np.testing.assert_array_equal(last.cpu().numpy(), rlast)
+    np.testing.assert_array_equal(bonus.cpu().numpy(), rbonus)
+    if shape != "star":
+        assert rn.max() >= 3
+
+
+def test_tree_walk_bf16_matches_oracle(orc):
+    B, K, V = 32, 64, 128256
+    x, tok, parent, L = _walk_inputs(B, K, V, "topk", seed=5, dtype=torch.bfloat16)
+    ws = lr.Workspace(B, K, V, 1, 1, 64, 1, device=cuda())
+    n, last, bonus = lr.libraspec_accept_tree_greedy(x, _i32(tok), _i32(parent), _i32(L), ws)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) == 0
+    # bf16 widens exactly to f32: the oracle sees the same values
+    rn, rlast, rbonus = orc.accept_tree_greedy(x.float().cpu().numpy(), tok, parent, L)
+    np.testing.assert_array_equal(n.cpu().numpy(), rn)
+    np.testing.assert_array_equal(last.cpu().numpy(), rlast)
+    np.testing.assert_array_equal(bonus.cpu().numpy(), rbonus)
+
+
+def test_chain_tree_walk_equals_greedy_accept():
+    B, K, V = 64, 16, 32000
+    x, tok, _, L = _walk_inputs(B, K, V, "chain", seed=9)
+    parent = workloads.draft_tree(B, K, L, seed=0, shape="chain")
+    ws = lr.Workspace(B, K, V, 1, 1, 64, 1, device=cuda())
+    n, last, bonus = lr.libraspec_accept_tree_greedy(x, _i32(tok), _i32(parent), _i32(L), ws)
+    zeros = torch.zeros((B, K, V), device=cuda())
+    n2, b2 = lr.libraspec_accept(x, zeros, _i32(tok), None, None, _i32(L), torch.zeros(B, device=cuda()), 0, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(n, n2) and torch.equal(bonus, b2) and torch.equal(last, n)
+
+
+def test_tree_walk_bad_inputs_set_status():
+    B, K, V = 2, 4, 100
+    x, tok, parent, L = _walk_inputs(B, K, V, "random", seed=1)
+    L = np.array([4, 4], np.int32)
+    parent = workloads.draft_tree(B, K, L, seed=1, shape="random")
+    parent[0, 2] = 2
+    tok[1, 0] = V + 3
+    ws = lr.Workspace(B, K, V, 1, 1, 64, 1, device=cuda())
+    lr.libraspec_accept_tree_greedy(x, _i32(tok), _i32(parent), _i32(L), ws)
+    torch.cuda.synchronize()
+    st = lr.libraspec_get_status(ws)
+    assert st & lr.ST_BAD_TREE and st & lr.ST_BAD_TOKEN
