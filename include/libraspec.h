@@ -68,6 +68,7 @@ extern "C" {
 /* Limits of this build. */
 #define LIBRASPEC_MAX_K 64           /* drafter block length / d_max             */
 #define LIBRASPEC_MAX_B 4096         /* sequences per call                       */
+#define LIBRASPEC_MAX_TREE_NODES 512 /* nodes below the root of a draft tree      */
 
 /* Version string of the library. */
 const char* libraspec_version(void);
@@ -77,9 +78,10 @@ const char* libraspec_status_string(int status);
 
 /*
  * Bytes of workspace a round with these shapes needs (all calls of the
- * round may share it). B sequences, K drafter block length, V vocabulary,
- * Hq / Hkv query / kv heads, head_dim, S_cap cache capacity per (b, kv head).
- * Pure host function; returns 0 for invalid shapes.
+ * round may share it). B sequences, K drafter block length (the node
+ * budget N for the draft-tree calls, up to LIBRASPEC_MAX_TREE_NODES), V
+ * vocabulary, Hq / Hkv query / kv heads, head_dim, S_cap cache capacity per
+ * (b, kv head). Pure host function; returns 0 for invalid shapes.
  */
 size_t libraspec_workspace_size(int B, int K, int V, int Hq, int Hkv, int head_dim, int S_cap);
 
@@ -271,55 +273,63 @@ int libraspec_verify_attn_paged_layers(const uint16_t* const* Q, const uint16_t*
 
 /*
  * Verification of a draft tree (the tree drafters the paper builds on,
- * Sec. 2, e.g. DDTree): the block holds the nodes of a tree instead of a
- * chain. Node 0 is the root (the last accepted token, block position 0);
- * node t in [1, L[b]] sits at block position t, i.e. its query is Q[b, t]
- * and its key / value at cache row kv_len[b] + t, and
- *   parent [B, K+1] i32  parent[b * (K+1) + t] in [0, t) for 1 <= t <= L[b]
+ * Sec. 2, e.g. DDTree, which the paper runs with node budgets of 64 to 512,
+ * Appendix C): the block holds the nodes of a tree instead of a chain. N is
+ * the node budget (0 <= N <= LIBRASPEC_MAX_TREE_NODES) and takes the place
+ * of K in every shape: Q [B, N+1, Hq, d], O and lse likewise. Node 0 is the
+ * root (the last accepted token, block position 0); node t in [1, L[b]]
+ * (L[b] <= N) sits at block position t, i.e. its query is Q[b, t] and its
+ * key / value at cache row kv_len[b] + t, and
+ *   parent [B, N+1] i32  parent[b * (N+1) + t] in [0, t) for 1 <= t <= L[b]
  *                        (node numbers are a topological order; other
  *                        entries are not read).
  * Node t attends to the cache prefix (keys < kv_len[b]) and to the keys of
  * its ancestors and itself (the root included): the block-causal mask of
  * libraspec_verify_attn_layers with each row's earlier block positions
- * replaced by its root path. A chain (parent[t] = t - 1) gives exactly the
- * chain call's result. A parent outside [0, t) sets LIBRASPEC_ST_BAD_TREE
- * and is read as the root. Everything else (shapes, layers per launch,
- * workspace, the ordering rules between layers) is as for the chain calls;
- * each call first runs a small kernel that turns the parents into one
- * 64-bit ancestor mask per node (in the workspace).
+ * replaced by its root path. A chain (parent[t] = t - 1, N <= 64) gives
+ * exactly the chain call's result. A parent outside [0, t) sets
+ * LIBRASPEC_ST_BAD_TREE and is read as the root. Unlike the chain calls,
+ * (N+1) * Hq / Hkv query rows per kv head are not capped beyond N's bound.
+ * Layers per launch, the ordering rules between layers and the paged-cache
+ * rules are those of the chain calls; the workspace is
+ * libraspec_workspace_size(B, N, ...). Each call first runs a small kernel
+ * that turns the parents into ancestor bit sets (ceil(N / 64) 64-bit words
+ * per node, in the workspace).
  */
 int libraspec_verify_attn_tree_layers(const uint16_t* const* Q, const uint16_t* const* Kc,
                                       const uint16_t* const* Vc, int n_layers, const int32_t* parent,
-                                      const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                                      const int32_t* kv_len, const int32_t* L, int B, int N, int Hq, int Hkv,
                                       int head_dim, int S_cap, float softmax_scale, uint16_t* const* O,
                                       float* const* lse, void* workspace, size_t ws_bytes, void* stream);
 int libraspec_verify_attn_tree_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp,
                                             const uint16_t* const* Vp, int n_layers, const int32_t* parent,
                                             const int32_t* block_table, int max_pages, int page_size, int n_pages,
-                                            const int32_t* kv_len, const int32_t* L, int B, int K, int Hq, int Hkv,
+                                            const int32_t* kv_len, const int32_t* L, int B, int N, int Hq, int Hkv,
                                             int head_dim, float softmax_scale, uint16_t* const* O,
                                             float* const* lse, void* workspace, size_t ws_bytes, void* stream);
 
 /*
  * Greedy acceptance of a draft tree (the longest root path the target
- * agrees with). Row t of target_logits [B, K+1, V] is the target's
+ * agrees with). Row t of target_logits [B, N+1, V] is the target's
  * distribution after node t (tree layout as above; node t >= 1 carries
- * draft_tokens[b * K + t - 1]). From the root, the walk moves to the
- * lowest-numbered child of the current node whose token is the argmax of
- * the current node's row (lowest index wins ties), while there is one.
+ * draft_tokens[b * N + t - 1], draft_tokens [B, N]). From the root, the walk
+ * moves to the lowest-numbered child of the current node whose token is the
+ * argmax of the current node's row (lowest index wins ties), while there is
+ * one.
  *   n_accepted [B] i32 out  nodes walked below the root;
  *   last_node  [B] i32 out  the node the walk ends on (may be NULL);
  *   bonus_token [B] i32 out the argmax of that node's row.
  * A chain gives libraspec_accept's greedy result (last_node = n_accepted).
  * Reads target rows 0..L[b] once. A parent outside [0, t) or a token outside
  * [0, V) never matches (LIBRASPEC_ST_BAD_TREE / LIBRASPEC_ST_BAD_TOKEN).
- * Sampling acceptance of a tree is not provided.
+ * Workspace: libraspec_workspace_size(B, N, V, ...). Sampling acceptance of
+ * a tree is not provided.
  */
 int libraspec_accept_tree_greedy(const float* target_logits, const int32_t* draft_tokens, const int32_t* parent,
-                                 const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
+                                 const int32_t* L, int B, int N, int V, int32_t* n_accepted, int32_t* last_node,
                                  int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream);
 int libraspec_accept_tree_greedy_bf16(const uint16_t* target_logits, const int32_t* draft_tokens,
-                                      const int32_t* parent, const int32_t* L, int B, int K, int V,
+                                      const int32_t* parent, const int32_t* L, int B, int N, int V,
                                       int32_t* n_accepted, int32_t* last_node, int32_t* bonus_token, void* workspace,
                                       size_t ws_bytes, void* stream);
 

@@ -20,6 +20,7 @@ OK, EINVAL, EUNSUPPORTED, ECUDA, EDEVICE = 0, -1, -2, -3, -4
 ST_BAD_LENGTH, ST_BAD_COST, ST_KV_OVERFLOW, ST_BAD_TOKEN, ST_TIMEOUT, ST_MISSING_INPUT = 1, 2, 4, 8, 16, 32
 ST_BAD_PAGE, ST_BAD_TREE = 0x40, 0x80
 MAX_K = 64
+MAX_TREE_NODES = 512
 
 # Every entry point declared in include/libraspec.h, with its ctypes signature.
 _P, _I, _U32, _U64, _F, _SZ = (ctypes.c_void_p, ctypes.c_int, ctypes.c_uint32, ctypes.c_uint64, ctypes.c_float,

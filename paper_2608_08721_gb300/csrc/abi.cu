@@ -56,10 +56,12 @@ bool shapes_ok(int B, int K, int V) {
   return B >= 0 && B <= LIBRASPEC_MAX_B && K >= 0 && K <= LIBRASPEC_MAX_K && V >= 1;
 }
 
-bool attn_shapes_ok(int B, int K, int Hq, int Hkv, int D, int S_cap) {
-  if (B < 0 || B > LIBRASPEC_MAX_B || K < 0 || K > LIBRASPEC_MAX_K) return false;
+// tree: K is the node budget N (<= LIBRASPEC_MAX_TREE_NODES) and the block
+// may hold any number of query rows per kv head.
+bool attn_shapes_ok(int B, int K, int Hq, int Hkv, int D, int S_cap, bool tree = false) {
+  if (B < 0 || B > LIBRASPEC_MAX_B || K < 0 || K > (tree ? LIBRASPEC_MAX_TREE_NODES : LIBRASPEC_MAX_K)) return false;
   if (Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || S_cap < 1) return false;
-  if ((long)(K + 1) * (Hq / Hkv) > 512) return false;
+  if (!tree && (long)(K + 1) * (Hq / Hkv) > 512) return false;
   if (Hq / Hkv > kAttnRows) return false;  // a row group holds at least one block position
   if ((long)B * Hkv > (1L << 30)) return false;
   (void)D;
@@ -86,7 +88,7 @@ const char* libraspec_status_string(int status) {
 }
 
 size_t libraspec_workspace_size(int B, int K, int V, int Hq, int Hkv, int head_dim, int S_cap) {
-  if (!shapes_ok(B, K, V) || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || (head_dim != 64 && head_dim != 128) ||
+  if (B < 0 || B > LIBRASPEC_MAX_B || K < 0 || K > LIBRASPEC_MAX_TREE_NODES || V < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || (head_dim != 64 && head_dim != 128) ||
       S_cap < 1)
     return 0;
   return ws_layout(B, K, V, Hq, Hkv, head_dim, S_cap).total;
@@ -188,7 +190,7 @@ int attn_layers(const uint16_t* const* Q, const uint16_t* const* Kc, const uint1
                 int Hkv, int head_dim, int S_cap, float softmax_scale, uint16_t* const* O, float* const* lse,
                 void* workspace, size_t ws_bytes, void* stream) {
   if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
-  if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap) || n_layers < 0) return LIBRASPEC_EINVAL;
+  if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap, tree) || n_layers < 0) return LIBRASPEC_EINVAL;
   if (B == 0 || n_layers == 0) return LIBRASPEC_OK;
   if (!Q || !Kc || !Vc || !O || !kv_len || !L || (tree && !parent)) return LIBRASPEC_EINVAL;
   for (int l = 0; l < n_layers; ++l) {
@@ -216,7 +218,7 @@ int attn_paged_layers(const uint16_t* const* Q, const uint16_t* const* Kp, const
       (long)n_pages * (Hkv > 0 ? Hkv : 1) > 0x7fffffffL || n_layers < 0)
     return LIBRASPEC_EINVAL;
   const int S_cap = max_pages * page_size;
-  if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap)) return LIBRASPEC_EINVAL;
+  if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap, tree)) return LIBRASPEC_EINVAL;
   if (B == 0 || n_layers == 0) return LIBRASPEC_OK;
   if (!Q || !Kp || !Vp || !O || !kv_len || !L || !block_table || !aligned(block_table, 4)) return LIBRASPEC_EINVAL;
   if (tree && !parent) return LIBRASPEC_EINVAL;
@@ -317,7 +319,7 @@ template <typename T>
 static int accept_tree_t(const T* target_logits, const int32_t* draft_tokens, const int32_t* parent,
                          const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
                          int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
-  if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
+  if (B < 0 || B > LIBRASPEC_MAX_B || K < 0 || K > LIBRASPEC_MAX_TREE_NODES || V < 1) return LIBRASPEC_EINVAL;
   if (B == 0) return LIBRASPEC_OK;
   if (!target_logits || (!draft_tokens && K > 0) || (!parent && K > 0) || !L || !n_accepted || !bonus_token)
     return LIBRASPEC_EINVAL;

@@ -334,22 +334,24 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
 }
 
 // ---------------------------------------------------------------------------
-// Greedy walk of a draft tree, one warp per sequence. Node t in [1, L_b]
-// (parent[b, t] < t, token tokens[b, t-1]) is held by lane (t-1) % 32 in
-// slot (t-1) / 32. From the root, the next node is the lowest-numbered child
-// of the current one whose token is the argmax of the current node's target
-// row (argmaxes from accept_rows_kernel, staged in shared memory first so the
-// walk itself issues no global loads); n = nodes walked, last = the final
-// node, bonus = its argmax. A parent outside [0, t) or a token outside [0, V)
-// never matches and raises its status bit.
+// Greedy walk of a draft tree, one warp per sequence. Node t in [1, L_b] has
+// parent parent[b, t] < t and token tokens[b, t-1]. The warp first finds, for
+// every node p, its matching child next[p]: the lowest-numbered child whose
+// token is the argmax of p's target row (argmaxes from accept_rows_kernel),
+// by shared-memory atomicMin over the nodes; then it follows next[] from the
+// root. n = nodes walked, last = the final node, bonus = its argmax. A parent
+// outside [0, t) or a token outside [0, V) never matches and raises its
+// status bit.
 // ---------------------------------------------------------------------------
 constexpr int kWalkWarps = 4;
+constexpr int kWalkNodes = LIBRASPEC_MAX_TREE_NODES + 1;
 
 __global__ void __launch_bounds__(kWalkWarps * 32) tree_walk_kernel(
     const int32_t* __restrict__ tokens, const int32_t* __restrict__ parent, const int32_t* __restrict__ Ls, int B,
     int K, int V, const RowStat* __restrict__ stat, int32_t* __restrict__ n_accepted,
     int32_t* __restrict__ last_node, int32_t* __restrict__ bonus, int* __restrict__ status) {
-  __shared__ int arg_s[kWalkWarps][LIBRASPEC_MAX_K + 1];
+  __shared__ int arg_s[kWalkWarps][kWalkNodes];
+  __shared__ int next_s[kWalkWarps][kWalkNodes];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * kWalkWarps + w;
   if (b >= B) return;
@@ -363,38 +365,30 @@ __global__ void __launch_bounds__(kWalkWarps * 32) tree_walk_kernel(
     return;
   }
   int* arg = arg_s[w];
-  for (int t = lane; t <= Lb; t += 32) arg[t] = __ldcg(&stat[(size_t)b * (K + 1) + t].arg);
-  int par[2], tok[2];
-#pragma unroll
-  for (int i = 0; i < 2; ++i) {
-    const int t = lane + 1 + 32 * i;
-    par[i] = -1;
-    tok[i] = -1;
-    if (t <= Lb) {
-      const int p = parent[(size_t)b * (K + 1) + t];
-      const int x = tokens[(size_t)b * K + t - 1];
-      if (p < 0 || p >= t) raise_status(status, LIBRASPEC_ST_BAD_TREE);
-      else if (x < 0 || x >= V) raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
-      else {
-        par[i] = p;
-        tok[i] = x;
-      }
-    }
+  int* next = next_s[w];
+  constexpr int kNone = 0x7fffffff;
+  for (int t = lane; t <= Lb; t += 32) {
+    arg[t] = __ldcg(&stat[(size_t)b * (K + 1) + t].arg);
+    next[t] = kNone;
   }
   __syncwarp();
-  int cur = 0, n = 0, a = arg[0];
-  for (int step = 0; step < Lb; ++step) {
-    const unsigned lo = __ballot_sync(0xffffffffu, par[0] == cur && tok[0] == a);
-    const unsigned hi = __ballot_sync(0xffffffffu, par[1] == cur && tok[1] == a);
-    if (!lo && !hi) break;
-    cur = lo ? __ffs(lo) : 32 + __ffs(hi);
-    ++n;
-    a = arg[cur];
+  for (int t = lane + 1; t <= Lb; t += 32) {
+    const int p = parent[(size_t)b * (K + 1) + t];
+    const int x = tokens[(size_t)b * K + t - 1];
+    if (p < 0 || p >= t) raise_status(status, LIBRASPEC_ST_BAD_TREE);
+    else if (x < 0 || x >= V) raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
+    else if (x == arg[p]) atomicMin(&next[p], t);
   }
+  __syncwarp();
   if (lane == 0) {
+    int cur = 0, n = 0;
+    while (n < Lb && next[cur] != kNone) {  // next[] only points to higher nodes
+      cur = next[cur];
+      ++n;
+    }
     n_accepted[b] = n;
     if (last_node) last_node[b] = cur;
-    bonus[b] = a;
+    bonus[b] = arg[cur];
   }
 }
 

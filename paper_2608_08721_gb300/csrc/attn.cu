@@ -234,9 +234,13 @@ __device__ __forceinline__ uint64_t low_bits(int n) {
   return n <= 0 ? 0ull : (n >= 64 ? ~0ull : ((1ull << n) - 1ull));
 }
 
-// x << s for s >= 0, x >> -s for s < 0; 0 once |s| >= 64
-__device__ __forceinline__ uint64_t shift_bits(uint64_t x, int s) {
-  return (s >= 64 || s <= -64) ? 0ull : (s >= 0 ? x << s : x >> -s);
+// Bits [o, o + 64) of the bit set row[0 .. words) (bits outside read as 0;
+// o may be negative).
+__device__ __forceinline__ uint64_t bit_window(const uint64_t* __restrict__ row, int words, int o) {
+  const int q = o >> 6, r = o & 63;  // floor division
+  const uint64_t lo = (q >= 0 && q < words) ? __ldg(row + q) : 0ull;
+  const uint64_t hi = (q + 1 >= 0 && q + 1 < words) ? __ldg(row + q + 1) : 0ull;
+  return r == 0 ? lo : (lo >> r) | (hi << (64 - r));
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -583,13 +587,13 @@ __device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int
 // sequence b lives at page block_table[b * max_pages + s / page_size], row
 // s % page_size (page_size a multiple of 64, so a key tile lies in one page);
 // S_cap is then max_pages * page_size.
-// tree_vis (optional, [B, K+1]): the block is a draft tree and row t sees the
-// block keys of the set bits (bit j <-> block position j + 1) besides the root
-// and the prefix; nullptr: the chain draft (block-causal).
+// tree_vis (optional, [B, K+1, tree_words]): the block is a draft tree and
+// row t sees the block keys of the set bits (bit j <-> block position j + 1)
+// besides the root and the prefix; nullptr: the chain draft (block-causal).
 template <int D, int STAGES, bool PAGED>
 __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     const __grid_constant__ LayerSet set, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
-    const uint64_t* __restrict__ tree_vis,
+    const uint64_t* __restrict__ tree_vis, int tree_words,
     const int32_t* __restrict__ block_table, int max_pages, int page_size, int n_pages, int page_cache,
     int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, float* __restrict__ part_buf_o,
     float* __restrict__ part_buf_ml, size_t part_o_stride, size_t part_ml_stride, uint32_t* __restrict__ bar_cnt,
@@ -949,11 +953,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         // a warp without valid rows only keeps the barrier counts in step
         const bool warp_live = warp * 32 < it.rows;
         const int t_row = (it.mg * R + row) / g;
-        // Block keys seen by this row: bit j <-> key kv + 1 + j (the root, key
-        // kv, and the cache prefix are seen by every row). Chain: the t_row
-        // earlier positions; tree: the ancestors of node t_row and itself.
-        const uint64_t vis =
-            !valid ? 0ull : (tree_vis ? __ldg(tree_vis + (size_t)it.b * (K + 1) + t_row) : low_bits(t_row));
+        // Keys seen by this row: the cache prefix and the root (keys <= kv),
+        // then chain: the block positions up to t_row (keys <= kv + t_row);
+        // tree: the ancestors of node t_row and itself, bit j of its
+        // visibility row <-> key kv + 1 + j.
+        const uint64_t* vrow =
+            (tree_vis && valid) ? tree_vis + ((size_t)it.b * (K + 1) + t_row) * tree_words : nullptr;
         const int mask_from = tree_vis ? it.kv : it.kv + t_row;  // tiles past this key need the mask
         float m_run = -INFINITY, l_run = 0.f;
         for (int t = 0; t < n_tiles && ok; ++t) {
@@ -982,8 +987,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           // raw scores; keys this row does not see (and rows past the
           // group) count as -inf; the scale (> 0) is applied below
           const bool need_mask = !valid || kt0 + kAttnTileKeys - 1 > mask_from;
-          const uint64_t tmask =
-              !valid ? 0ull : (low_bits(it.kv + 1 - kt0) | shift_bits(vis, it.kv + 1 - kt0));
+          uint64_t tmask = ~0ull;  // bit c: key kt0 + c is seen
+          if (need_mask) {
+            if (!valid) tmask = 0ull;
+            else if (!vrow) tmask = low_bits(it.kv + t_row + 1 - kt0);
+            else tmask = low_bits(it.kv + 1 - kt0) | bit_window(vrow, tree_words, kt0 - it.kv - 1);
+          }
           float xs[kAttnTileKeys];
           float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
@@ -1223,68 +1232,74 @@ static int attn_min_tiles() {
   return t;
 }
 
-// Ancestor sets of a draft tree, one warp per sequence, by pointer jumping:
-// after round r, m[t] holds node t's ancestors at distance < 2^r and up[t]
-// the one at distance 2^r (the root absorbs: m[0] = 0, up[0] = 0), so 7
-// rounds cover depth 64. vis[b, t] bit j <-> block position j + 1 is node t
-// or an ancestor of it; rows t > L_b get 0. A parent outside [0, t) raises
-// LIBRASPEC_ST_BAD_TREE and is read as the root.
-constexpr int kTreeWarps = 4;
-constexpr int kTreeNodes = LIBRASPEC_MAX_K + 1;
+// Ancestor sets of a draft tree, one CTA per sequence, by pointer jumping:
+// after round r, m[t] holds the nodes on the path from t up to (not
+// including) up[t], the ancestor at distance 2^r (the root absorbs: m[0] =
+// 0, up[0] = 0); rounds stop once every up[] is the root (depth <= 2^r).
+// vis[b, t] = m[t] as `words` 64-bit words, bit j <-> block position j + 1;
+// rows t > L_b get 0. A parent outside [0, t) raises LIBRASPEC_ST_BAD_TREE
+// and is read as the root. Each round reads all (node, word) pairs into
+// registers before any is written.
+constexpr int kTreeThreads = 256;
+constexpr int kTreeWords = (LIBRASPEC_MAX_TREE_NODES + 63) / 64;
+constexpr int kTreePer = ((LIBRASPEC_MAX_TREE_NODES + 1) * kTreeWords + kTreeThreads - 1) / kTreeThreads;
 
-__global__ void __launch_bounds__(kTreeWarps * 32) tree_vis_kernel(const int32_t* __restrict__ parent,
-                                                                     const int32_t* __restrict__ Ls, int B, int K,
-                                                                     uint64_t* __restrict__ vis,
-                                                                     int* __restrict__ status) {
-  __shared__ int up_s[kTreeWarps][kTreeNodes];
-  __shared__ uint64_t m_s[kTreeWarps][kTreeNodes];
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.x * kTreeWarps + w;
-  if (b >= B) return;
-  int* up = up_s[w];
-  uint64_t* m = m_s[w];
+__global__ void __launch_bounds__(kTreeThreads) tree_vis_kernel(const int32_t* __restrict__ parent,
+                                                                 const int32_t* __restrict__ Ls, int K, int words,
+                                                                 uint64_t* __restrict__ vis,
+                                                                 int* __restrict__ status) {
+  __shared__ int up[LIBRASPEC_MAX_TREE_NODES + 1];
+  __shared__ uint64_t m[(LIBRASPEC_MAX_TREE_NODES + 1) * kTreeWords];
+  const int b = blockIdx.x, tid = threadIdx.x;
   int Lb = Ls[b];
   if (Lb < 0 || Lb > K) Lb = 0;  // the attention kernel reports the bad length
-  for (int t = lane; t <= K; t += 32) {
+  const int pairs = (K + 1) * words;
+  for (int t = tid; t <= K; t += kTreeThreads) {
     int p = 0;
-    uint64_t bit = 0ull;
     if (t >= 1 && t <= Lb) {
       p = parent[(size_t)b * (K + 1) + t];
       if (p < 0 || p >= t) {
         raise_status(status, LIBRASPEC_ST_BAD_TREE);
         p = 0;
       }
-      bit = 1ull << (t - 1);
     }
     up[t] = p;
-    m[t] = bit;
   }
-  __syncwarp();
-  for (int r = 0; r < 7; ++r) {
-    int nu[3];
-    uint64_t nm[3];
+  for (int i = tid; i < pairs; i += kTreeThreads) {
+    const int t = i / words, w = i % words;
+    m[i] = (t >= 1 && t <= Lb && (t - 1) / 64 == w) ? 1ull << ((t - 1) % 64) : 0ull;
+  }
+  __syncthreads();
+  for (int r = 0; r < 16; ++r) {  // depth <= 512 needs at most 10 rounds
+    uint64_t nm[kTreePer];
+    int nu[kTreePer];
+    bool more = false;
 #pragma unroll
-    for (int i = 0; i < 3; ++i) {
-      const int t = lane + 32 * i;
-      if (t <= K) {
+    for (int k = 0; k < kTreePer; ++k) {
+      const int i = tid + k * kTreeThreads;
+      if (i < pairs) {
+        const int t = i / words, w = i % words;
         const int u = up[t];
-        nm[i] = m[t] | m[u];
-        nu[i] = up[u];
+        nm[k] = m[i] | m[u * words + w];
+        nu[k] = up[u];
+        more |= nu[k] != 0;
       }
     }
-    __syncwarp();
+    __syncthreads();
 #pragma unroll
-    for (int i = 0; i < 3; ++i) {
-      const int t = lane + 32 * i;
-      if (t <= K) {
-        m[t] = nm[i];
-        up[t] = nu[i];
+    for (int k = 0; k < kTreePer; ++k) {
+      const int i = tid + k * kTreeThreads;
+      if (i < pairs) {
+        m[i] = nm[k];
+        if (i % words == 0) up[i / words] = nu[k];
       }
     }
-    __syncwarp();
+    if (!__syncthreads_or(more)) break;
   }
-  for (int t = lane; t <= K; t += 32) vis[(size_t)b * (K + 1) + t] = m[t];
+  for (int i = tid; i < pairs; i += kTreeThreads) vis[(size_t)b * pairs + i] = m[i];
 }
+
+inline int tree_words(int K) { return K <= 64 ? 1 : (K + 63) / 64; }
 
 // parent != nullptr: fill the tree visibility masks of the workspace first.
 static cudaError_t tree_vis(const int32_t* parent, const int32_t* L, int B, int K, char* ws, const WsLayout& lay,
@@ -1292,8 +1307,8 @@ static cudaError_t tree_vis(const int32_t* parent, const int32_t* L, int B, int 
   *out = nullptr;
   if (!parent) return cudaSuccess;
   auto* vis = reinterpret_cast<uint64_t*>(ws + lay.tree_vis);
-  tree_vis_kernel<<<(B + kTreeWarps - 1) / kTreeWarps, kTreeWarps * 32, 0, stream>>>(
-      parent, L, B, K, vis, reinterpret_cast<int*>(ws + lay.status));
+  tree_vis_kernel<<<B, kTreeThreads, 0, stream>>>(parent, L, K, tree_words(K), vis,
+                                                  reinterpret_cast<int*>(ws + lay.status));
   *out = vis;
   return cudaGetLastError();
 }
@@ -1364,7 +1379,7 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(
-        &cfg, kern, set, kv_len, L, tree_vis, block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
+        &cfg, kern, set, kv_len, L, tree_vis, tree_words(K), block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
         Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(),
         reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_half / sizeof(float),
         ml_half / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));

@@ -75,8 +75,8 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.attn_ml = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
   // grid-barrier counters, one per layer of a launch, then the exit counter
   w.attn_cnt = take((kAttnMaxLayers + 1) * sizeof(uint32_t));
-  // ancestor masks of a draft tree, one per block position
-  w.tree_vis = take(rows_t * sizeof(uint64_t));
+  // ancestor masks of a draft tree, ceil(K / 64) words per block position
+  w.tree_vis = take(rows_t * size_t(K <= 64 ? 1 : (K + 63) / 64) * sizeof(uint64_t));
   w.total = off;
   return w;
 }

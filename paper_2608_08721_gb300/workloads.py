@@ -218,7 +218,7 @@ def layer(w: Workload, l: int, kv: np.ndarray, device="cpu", peaky: bool = False
     return {"Q": Q, "Kc": Kc, "Vc": Vc}
 
 
-def draft_tree(B: int, K: int, L, seed: int, shape: str = "topk") -> np.ndarray:
+def draft_tree(B: int, K: int, L, seed: int, shape: str = "topk", depth: int = 16) -> np.ndarray:
     """Parent array [B, K+1] (int32) of a draft tree per sequence.
 
     Node 0 is the root (the last accepted token); node t in [1, L_b] has
@@ -228,7 +228,14 @@ def draft_tree(B: int, K: int, L, seed: int, shape: str = "topk") -> np.ndarray:
     recursive tree) and ``topk``: the shape tree drafters grow from
     per-position candidate lists, a main path with up to three alternatives
     hanging off each depth (breadth-first: depth by depth, candidates in rank
-    order, each alternative a child of the previous depth's best node)."""
+    order, each alternative a child of the previous depth's best node);
+    ``ddtree``: the shape a diffusion drafter's tree takes under a node budget
+    (DDTree): per depth d <= ``depth`` (the block length) a ranked candidate
+    list with probabilities q_d (softmax of N(0, s^2) scores, s per sequence
+    in [1, 6]); nodes are added best-first by the product of the
+    candidates' probabilities along the path (a child of node t is candidate
+    k at depth(t) + 1), so a confident drafter grows one long path and an
+    unsure one a bushy top."""
     rng = np.random.default_rng([seed, 77])
     L = np.broadcast_to(np.asarray(L, np.int64), (B,))
     par = np.zeros((B, K + 1), np.int32)
@@ -252,9 +259,40 @@ def draft_tree(B: int, K: int, L, seed: int, shape: str = "topk") -> np.ndarray:
                     par[b, t] = best
                     t += 1
                 best = first
+        elif shape == "ddtree":
+            par[b] = _ddtree_parents(rng, n, K, depth)
         else:
             raise ValueError(shape)
     return par
+
+
+def _ddtree_parents(rng: np.random.Generator, n: int, K: int, depth: int) -> np.ndarray:
+    import heapq
+
+    width = 32
+    s = rng.uniform(1.0, 6.0)
+    z = rng.standard_normal((depth + 1, width)) * s
+    q = np.exp(z - z.max(axis=1, keepdims=True))
+    q = -np.sort(-q / q.sum(axis=1, keepdims=True), axis=1)   # ranked, descending
+    logq = np.log(q)
+    out = np.zeros(K + 1, np.int32)
+    node_depth = [0]
+    # candidates: (-path log-prob, tie, parent node, rank at depth(parent)+1)
+    heap = [(-logq[1, 0], 0, 0, 0)]
+    tie, t = 1, 1
+    while t <= n and heap:
+        neg, _, p, k = heapq.heappop(heap)
+        out[t] = p
+        d = node_depth[p] + 1
+        node_depth.append(d)
+        if k + 1 < width:      # the next sibling candidate
+            heapq.heappush(heap, (neg + logq[d, k] - logq[d, k + 1], tie, p, k + 1))
+            tie += 1
+        if d < depth:          # the first child candidate of the new node
+            heapq.heappush(heap, (neg - logq[d + 1, 0], tie, t, 0))
+            tie += 1
+        t += 1
+    return out
 
 
 def reference_inputs_summary(w: Workload) -> List[str]:

@@ -51,7 +51,9 @@ def test_workspace_size_is_host_only_and_validates(lib):
     assert s > 0 and s % 256 == 0
     assert lib.libraspec_workspace_size(1, 16, 32000, 8, 2, 64, 576) < s
     assert lib.libraspec_workspace_size(1, 16, 32000, 8, 3, 64, 576) == 0      # Hq % Hkv != 0
-    assert lib.libraspec_workspace_size(1, 65, 32000, 8, 2, 64, 576) == 0      # K > max
+    # K up to the draft-tree node budget (512) sizes a workspace; beyond, none
+    assert lib.libraspec_workspace_size(1, 512, 32000, 8, 2, 64, 576) > 0
+    assert lib.libraspec_workspace_size(1, 513, 32000, 8, 2, 64, 576) == 0     # K > max
     assert lib.libraspec_workspace_size(1, 16, 32000, 8, 2, 96, 576) == 0      # head dim
 
 

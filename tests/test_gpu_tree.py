@@ -235,3 +235,88 @@ def test_tree_walk_bad_inputs_set_status():
     torch.cuda.synchronize()
     st = lr.libraspec_get_status(ws)
     assert st & lr.ST_BAD_TREE and st & lr.ST_BAD_TOKEN
+
+
+# ---------------------------------------------------------------------------
+# node budgets beyond 64 (DDTree runs 64 to 512 nodes): multi-word masks
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("N", [65, 128, 256, 512])
+def test_large_tree_attn_matches_oracle(orc, N):
+    Hq, Hkv, d = 32, 8, 128
+    kv = [4096, 63, 1]
+    L = [N, N - 1, N // 2]
+    B = len(kv)
+    S = (max(k + l + 1 for k, l in zip(kv, L)) + 63) // 64 * 64
+    parent = workloads.draft_tree(B, N, L, seed=N, shape="ddtree", depth=16)
+    layers = _layers(B, N, Hq, Hkv, d, S, seed=N + 1)
+    outs, lses, status = _run_tree(layers, parent, kv, L, N)
+    assert status == 0
+    if N <= 128:
+        O_ref, lse_ref = orc.verify_attn_tree(layers[0]["Q"], layers[0]["Kc"], layers[0]["Vc"], np.array(kv),
+                                              np.array(L), parent)
+        check_attn(outs[0], lses[0], O_ref, lse_ref, L)
+    else:
+        rng = np.random.default_rng(N)
+        rows = [(b, h, t) for b in range(B) for h in (0, 17, Hq - 1)
+                for t in sorted(set([0, 1, L[b]] + list(rng.integers(0, L[b] + 1, 12))))]
+        rows = np.array(rows, np.int32)
+        O_ref, lse_ref = orc.verify_attn_tree(layers[0]["Q"], layers[0]["Kc"], layers[0]["Vc"], np.array(kv),
+                                              np.array(L), parent, rows=rows)
+        check_attn(outs[0], lses[0], O_ref, lse_ref, L, rows=[tuple(r) for r in rows])
+
+
+def test_large_tree_random_shape_small_heads(orc):
+    """A uniform random recursive tree (deep, irregular ancestor sets) of 300
+    nodes, 8/2 heads, d 64, two layers."""
+    N, Hq, Hkv, d = 300, 8, 2, 64
+    kv, L = [700, 0], [300, 257]
+    S = (max(k + l + 1 for k, l in zip(kv, L)) + 63) // 64 * 64
+    parent = workloads.draft_tree(2, N, L, seed=300, shape="random")
+    layers = _layers(2, N, Hq, Hkv, d, S, seed=300, n_layers=2)
+    outs, lses, status = _run_tree(layers, parent, kv, L, N)
+    assert status == 0
+    for l in range(2):
+        O_ref, lse_ref = orc.verify_attn_tree(layers[l]["Q"], layers[l]["Kc"], layers[l]["Vc"], np.array(kv),
+                                              np.array(L), parent)
+        check_attn(outs[l], lses[l], O_ref, lse_ref, L)
+
+
+@pytest.mark.parametrize("N", [128, 512])
+def test_large_tree_walk_matches_oracle(orc, N):
+    B, V = 16, 32000
+    rng = np.random.default_rng(N)
+    L = np.full(B, N, np.int32)
+    L[1] = N // 3
+    parent = workloads.draft_tree(B, N, L, seed=N, shape="ddtree", depth=16)
+    tok = np.zeros((B, N), np.int32)
+    g = torch.Generator(device="cuda").manual_seed(N)
+    x = torch.randn((B, N + 1, V), generator=g, device=cuda()) * 0.5
+    for b in range(B):
+        kids = [[] for _ in range(N + 1)]
+        for t in range(1, int(L[b]) + 1):
+            kids[parent[b, t]].append(t)
+        for p in range(N + 1):
+            vals = rng.choice(V, size=len(kids[p]), replace=False)
+            for t, v in zip(kids[p], vals):
+                tok[b, t - 1] = v
+            if kids[p] and rng.random() < 0.9:
+                x[b, p, int(tok[b, kids[p][0] - 1])] = 6.0   # the best-ranked child
+    ws = lr.Workspace(B, N, V, 1, 1, 64, 1, device=cuda())
+    n, last, bonus = lr.libraspec_accept_tree_greedy(x, _i32(tok), _i32(parent), _i32(L), ws)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) == 0
+    rn, rlast, rbonus = orc.accept_tree_greedy(x.cpu().numpy(), tok, parent, L)
+    np.testing.assert_array_equal(n.cpu().numpy(), rn)
+    np.testing.assert_array_equal(last.cpu().numpy(), rlast)
+    np.testing.assert_array_equal(bonus.cpu().numpy(), rbonus)
+    assert rn.max() >= 4
+
+
+def test_tree_rejects_node_budget_over_limit():
+    N = lr.MAX_TREE_NODES + 1
+    Q = torch.zeros((1, N + 1, 8, 64), dtype=torch.bfloat16, device=cuda())
+    Kc = torch.zeros((1, 2, 1024, 64), dtype=torch.bfloat16, device=cuda())
+    ws = lr.Workspace(1, lr.MAX_TREE_NODES, 1, 8, 2, 64, 1024, device=cuda())
+    with pytest.raises(lr.LibraspecError):
+        lr.libraspec_verify_attn_tree_layers([{"Q": Q, "Kc": Kc, "Vc": Kc}], _i32(np.zeros((1, N + 1))),
+                                             _i32([0]), _i32([0]), ws)

@@ -37,14 +37,15 @@ def _inputs(rng, B, K, Hq, Hkv, d, kv_len, S):
     return (_bf16((B, K + 1, Hq, d), rng), _bf16((B, Hkv, S, d), rng, 2.0), _bf16((B, Hkv, S, d), rng))
 
 
-@pytest.mark.parametrize("shape", ["random", "topk", "star"])
+@pytest.mark.parametrize("shape,K", [("random", 9), ("topk", 9), ("star", 9), ("ddtree", 9), ("ddtree", 130),
+                                     ("random", 130)])
 @pytest.mark.parametrize("Hq,Hkv,d", [(4, 2, 16), (3, 1, 8)])
-def test_tree_attn_matches_sdpa_with_closure_mask(shape, Hq, Hkv, d):
+def test_tree_attn_matches_sdpa_with_closure_mask(shape, K, Hq, Hkv, d):
     rng = np.random.default_rng(5 + Hq * 10 + d)
-    B, K = 3, 9
+    B = 3
     kv_len = np.array([0, 5, 21], np.int32)
-    L = np.array([9, 4, 7], np.int32)
-    S = 32
+    L = np.array([K, K // 2, K - 2], np.int32)
+    S = (21 + K + 1 + 63) // 64 * 64
     Q, Kc, Vc = _inputs(rng, B, K, Hq, Hkv, d, kv_len, S)
     par = workloads.draft_tree(B, K, L, seed=3, shape=shape)
     scale = 1.0 / np.sqrt(d)
@@ -68,6 +69,25 @@ def test_tree_attn_matches_sdpa_with_closure_mask(shape, Hq, Hkv, d):
             m = s.max(axis=1)
             np.testing.assert_allclose(lse[b, :n + 1, h], m + np.log(np.exp(s - m[:, None]).sum(1)), rtol=1e-12)
         assert np.all(np.isnan(O[b, n + 1:]))
+
+
+@pytest.mark.parametrize("budget", [64, 512])
+def test_ddtree_generator_shape(budget):
+    """Node numbers are a topological order, depth stays within the block
+    length, and every node but the budget's last is a candidate's best-first
+    expansion (siblings appear in rank order: a node's children are
+    numbered after it)."""
+    L = np.full(8, budget)
+    par = workloads.draft_tree(8, budget, L, seed=1, shape="ddtree", depth=16)
+    assert par.shape == (8, budget + 1)
+    for b in range(8):
+        dep = np.zeros(budget + 1, int)
+        for t in range(1, budget + 1):
+            assert 0 <= par[b, t] < t
+            dep[t] = dep[par[b, t]] + 1
+        assert dep.max() <= 16
+    # the same seed gives the same trees
+    np.testing.assert_array_equal(par, workloads.draft_tree(8, budget, L, seed=1, shape="ddtree", depth=16))
 
 
 def test_chain_tree_is_the_chain_verify():
