@@ -7,6 +7,13 @@ over a 4096-token cache).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
 
+Variants of the round (the default is the chain draft on dense caches):
+  --selector alpha   Algorithm 1's alpha-mode length search instead of Thm. 4's scan;
+  --logits bf16      bf16 drafter and target logits;
+  --page-size P      KV caches in pages of P keys behind block tables;
+  --tree N           a DDTree-shaped draft tree of N nodes: tree-masked attention and the
+                     greedy tree walk replace the chain's attention and acceptance.
+
 N > 1 runs under torchrun, one process per GPU; every rank verifies its own
 batch (weak scaling, no data-path collective) and rank 0 prints one JSON line.
 """
@@ -48,6 +55,10 @@ def parse():
     p.add_argument("--selector", default="gain", choices=["gain", "alpha"],
                    help="gain: the Thm. 4 marginal-gain scan; alpha: Algorithm 1's alpha-mode search")
     p.add_argument("--alpha", type=float, default=2.2, help="alpha of the alpha-mode search (Sec. 4: 2.2)")
+    p.add_argument("--tree", type=int, default=0,
+                   help="verify a DDTree-shaped draft tree of this many nodes (depth <= K) instead of the chain")
+    p.add_argument("--page-size", type=int, default=0,
+                   help="keep the KV cache in pages of this many keys behind block tables (0: dense)")
     p.add_argument("--block-size", type=int, default=0,
                    help="first drafted block of the alpha-mode search (0: 2/3 of K, as 16 of d_max 24)")
     return p.parse_args()
@@ -135,15 +146,19 @@ def physical_gpu(local_rank):
 # ---------------------------------------------------------------------------
 # algorithmic bytes (what the method must move)
 # ---------------------------------------------------------------------------
-def round_bytes(w, kv, L, temperature, n_acc, logit_bytes=4):
+def round_bytes(w, kv, L, temperature, n_acc, logit_bytes=4, L_tree=None):
+    """Algorithmic bytes of one round. L_tree: node counts of draft trees
+    (their attention and acceptance read every node's rows)."""
     conf = w.B * w.K * w.V * logit_bytes
     select = w.B * w.K * 4 + (w.K + 1) * 4
-    accept = float(np.sum((L + 1).astype(np.int64) * w.V * logit_bytes))
-    rejected_sampling = np.sum((n_acc < L) & (temperature > 0))
-    accept += float(rejected_sampling) * 2 * w.V * logit_bytes
+    Lv = L if L_tree is None else L_tree
+    accept = float(np.sum((Lv + 1).astype(np.int64) * w.V * logit_bytes))
+    if L_tree is None:
+        rejected_sampling = np.sum((n_acc < L) & (temperature > 0))
+        accept += float(rejected_sampling) * 2 * w.V * logit_bytes
     from paper_2608_08721_gb300 import workloads
 
-    attn_launch = workloads.attn_bytes(w, kv, L)
+    attn_launch = workloads.attn_bytes(w, kv, Lv)
     return {"conf": conf, "select": select, "attn_per_launch": attn_launch, "attn": attn_launch * w.n_layers,
             "accept": accept, "total": conf + select + accept + attn_launch * w.n_layers}
 
@@ -182,6 +197,51 @@ def oracle_round_time(w, inp_host, layers_host, kv, budget_s):
               "attention layers (fp64 C oracle, %d threads); attention time scaled by %d layers" %
               (len(times_attn), w.n_layers, threads, w.n_layers))
     return per_round * 1e6, threads, sample
+
+
+def oracle_tree_round_time(w, host, tree_host, layer_host, kv, budget_s):
+    """The oracle's tree round on a bounded sample: confidence and selection
+    on the batch, the greedy tree walk, and ONE attention layer scaled to all."""
+    import oracle
+
+    oracle.build()
+    threads = os.cpu_count() or 1
+    oracle.set_threads(threads)
+    cost = np.asarray(host["cost_table"], np.float64)
+    t_logits, t_attn = [], []
+    t_end = time.perf_counter() + budget_s
+    while True:
+        t0 = time.perf_counter()
+        q, _ = oracle.confidence(host["draft_logits"], host["draft_tokens"], host["temperature"])
+        oracle.select_lengths(q, cost)
+        oracle.accept_tree_greedy(tree_host["target_logits"], tree_host["draft_tokens"], tree_host["parent"],
+                                  tree_host["L"])
+        t1 = time.perf_counter()
+        oracle.verify_attn_tree(layer_host["Q"], layer_host["Kc"], layer_host["Vc"], kv, tree_host["L"],
+                                tree_host["parent"])
+        t2 = time.perf_counter()
+        t_logits.append(t1 - t0)
+        t_attn.append(t2 - t1)
+        if time.perf_counter() > t_end or len(t_attn) >= 50:
+            break
+    per_round = statistics.median(t_logits) + statistics.median(t_attn) * w.n_layers
+    sample = ("%d repetition(s) of: confidence, selection and the greedy tree walk on the full batch plus ONE of "
+              "the %d tree-attention layers (fp64 C oracle, %d threads); attention time scaled by %d layers" %
+              (len(t_attn), w.n_layers, threads, w.n_layers))
+    return per_round * 1e6, threads, sample
+
+
+def tree_flops(parent, kv, L, Hq, d):
+    """Attention flops of one tree layer counting visible keys only:
+    Σ_b Σ_t Hq · 4d · (kv_b + depth_t + 1)."""
+    tot = 0.0
+    for b in range(parent.shape[0]):
+        n = int(L[b])
+        dep = np.zeros(n + 1, np.int64)
+        for t in range(1, n + 1):
+            dep[t] = dep[parent[b, t]] + 1
+        tot += float(Hq) * 4.0 * d * float(np.sum(int(kv[b]) + dep + 1))
+    return tot
 
 
 def host_inputs(w, kv, n_layer_samples=1):
@@ -264,17 +324,47 @@ def run_ours(args, rank, world, local_rank):
         inp["draft_logits"] = inp["draft_logits"].to(torch.bfloat16)
         inp["target_logits"] = inp["target_logits"].to(torch.bfloat16)
     n_res = w.resident_layers if w.resident_layers else w.n_layers
-    S = workloads.s_cap(w, kv)
-    caches = [workloads.layer(w, l, kv, device=dev) for l in range(n_res)]
+    N = args.tree  # draft-tree node budget (0: the chain draft)
+    if N and not 1 <= N <= lr.MAX_TREE_NODES:
+        raise SystemExit("--tree must be in [1, %d]" % lr.MAX_TREE_NODES)
+    K1 = N + 1 if N else w.K + 1   # verified positions per sequence
+    S = workloads.s_cap(w, kv) if not N else (int(kv.max()) + N + 1 + 63) // 64 * 64
+    P = args.page_size
+    if P:
+        if P % 64:
+            raise SystemExit("--page-size must be a multiple of 64")
+        S = -(-S // P) * P
+    caches = [workloads.layer(w, l, kv, device=dev, scap=S) for l in range(n_res)]
+    table = None
+    if P:  # the same caches, moved into randomly permuted pages behind block tables
+        max_pages = S // P
+        perm = np.random.default_rng([w.data_seed, 55]).permutation(w.B * max_pages).astype(np.int32)
+        table = torch.from_numpy(perm.reshape(w.B, max_pages)).to(dev)
+        idx = torch.from_numpy(perm).long().to(dev)
+        for c in caches:
+            for key, pk in (("Kc", "Kp"), ("Vc", "Vp")):
+                pages = c.pop(key).view(w.B, w.Hkv, max_pages, P, w.d).permute(0, 2, 1, 3, 4)
+                pool = torch.empty((w.B * max_pages, w.Hkv, P, w.d), dtype=torch.bfloat16, device=dev)
+                pool[idx] = pages.reshape(w.B * max_pages, w.Hkv, P, w.d)
+                c[pk] = pool
     g = torch.Generator(device=dev).manual_seed(w.data_seed * 31 + 5)
-    Qs = [torch.randn((w.B, w.K + 1, w.Hq, w.d), generator=g, device=dev).to(torch.bfloat16)
+    Qs = [torch.randn((w.B, K1, w.Hq, w.d), generator=g, device=dev).to(torch.bfloat16)
           for _ in range(w.n_layers)]
     Os = [torch.empty_like(q) for q in Qs]
-    layers = [{"Q": Qs[l], "Kc": caches[l % n_res]["Kc"], "Vc": caches[l % n_res]["Vc"], "O": Os[l]}
-              for l in range(w.n_layers)]
+    layers = [dict(caches[l % n_res], Q=Qs[l], O=Os[l]) for l in range(w.n_layers)]
     cost = torch.tensor(workloads.cost_table(w, kv), device=dev)
     kv_t = torch.tensor(kv, device=dev)
     ws = lr.Workspace(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, S, device=dev)
+    tree = None
+    if N:
+        parent = workloads.draft_tree(w.B, N, N, seed=w.data_seed, shape="ddtree", depth=w.K)
+        tl = workloads.tree_logits(w, parent, N, device=dev)
+        if args.logits == "bf16":
+            tl["target_logits"] = tl["target_logits"].to(torch.bfloat16)
+        tree = {"parent_np": parent, "parent": torch.from_numpy(parent).to(dev), "tokens": tl["draft_tokens"],
+                "target": tl["target_logits"], "L": torch.full((w.B,), N, dtype=torch.int32, device=dev),
+                "last": torch.empty((w.B,), dtype=torch.int32, device=dev),
+                "ws": lr.Workspace(w.B, N, w.V, w.Hq, w.Hkv, w.d, S, device=dev)}
     conf = torch.empty((w.B, w.K), device=dev)
     dstat = torch.empty((w.B, w.K, 2), device=dev)
     L = torch.empty((w.B,), dtype=torch.int32, device=dev)
@@ -293,18 +383,33 @@ def run_ours(args, rank, world, local_rank):
             lr.libraspec_select_lengths(conf, cost, ws, L=L)
 
     def seg_attn():
-        lr.libraspec_verify_attn_layers(layers, kv_t, L, ws)
+        if N and P:
+            lr.libraspec_verify_attn_tree_paged_layers(layers, tree["parent"], table, kv_t, tree["L"], tree["ws"])
+        elif N:
+            lr.libraspec_verify_attn_tree_layers(layers, tree["parent"], kv_t, tree["L"], tree["ws"])
+        elif P:
+            lr.libraspec_verify_attn_paged_layers(layers, table, kv_t, L, ws)
+        else:
+            lr.libraspec_verify_attn_layers(layers, kv_t, L, ws)
 
     def seg_accept():
+        if N:
+            lr.libraspec_accept_tree_greedy(tree["target"], tree["tokens"], tree["parent"], tree["L"], tree["ws"],
+                                            n_accepted=n_acc, last_node=tree["last"], bonus_token=bonus)
+            return
         lr.libraspec_accept(inp["target_logits"], inp["draft_logits"], inp["draft_tokens"], conf, dstat, L,
                             inp["temperature"], w.philox_seed, ws, seq_offset=seq_offset, n_accepted=n_acc,
                             bonus_token=bonus)
+
+    def device_status():
+        st = lr.libraspec_get_status(ws)
+        return st | (lr.libraspec_get_status(tree["ws"]) if N else 0)
 
     # eager warm-up (also configures kernels), then capture three graphs
     for _ in range(3):
         seg_select(); seg_attn(); seg_accept()
     torch.cuda.synchronize()
-    if lr.libraspec_get_status(ws) != 0:
+    if device_status() != 0:
         raise RuntimeError("device status set during warm-up")
     graphs = []
     side = torch.cuda.Stream(device=dev)
@@ -352,13 +457,14 @@ def run_ours(args, rank, world, local_rank):
     elapsed_ms = start.elapsed_time(end)
     attn_ms = sum(a.elapsed_time(b) for a, b in zip(ev_a, ev_b))
     elapsed_max = pdist.max_over_ranks(elapsed_ms, device=dev)
-    if lr.libraspec_get_status(ws) != 0:
+    if device_status() != 0:
         raise RuntimeError("device status set during the timed steps")
 
     Lh = L.cpu().numpy()
     nh = n_acc.cpu().numpy()
     temp = inp["temperature"].cpu().numpy()
-    by = round_bytes(w, kv, Lh, temp, nh, logit_bytes=2 if args.logits == "bf16" else 4)
+    L_tree = np.full(w.B, N, np.int64) if N else None
+    by = round_bytes(w, kv, Lh, temp, nh, logit_bytes=2 if args.logits == "bf16" else 4, L_tree=L_tree)
     us_per_round = elapsed_ms * 1000.0 / K_steps
     # one persistent attention launch runs up to ATTN_LAYERS_PER_LAUNCH layers
     attn_launches = -(-w.n_layers // ATTN_LAYERS_PER_LAUNCH)
@@ -366,27 +472,54 @@ def run_ours(args, rank, world, local_rank):
     attn_bytes_launch = by["attn_per_launch"] * w.n_layers / attn_launches
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks["hbm_gbs"])
+    tensor_peak = float(peaks.get("bf16_tflops_sustained") or peaks.get("bf16_tflops") or 1700.0)
     achieved = attn_bytes_launch / attn_launch_s / 1e9
-    trec = traffic_record(os.path.join(ROOT, "paper_2608_08721_gb300", "csrc", "attn.cu"))
+    trec = None
+    if not N and not P:
+        trec = traffic_record(os.path.join(ROOT, "paper_2608_08721_gb300", "csrc", "attn.cu"))
+    roof = {"kernel": "verify_attn", "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
+            "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
+            "traffic": None if trec is None else trec.get("traffic_bytes_per_launch"),
+            "algorithmic_bytes_per_launch": attn_bytes_launch,
+            "layers_per_launch": round(w.n_layers / attn_launches, 2),
+            "launch_us": round(attn_launch_s * 1e6, 3),
+            "peak_source": peak_src + " (MEASURED_PEAKS.json hbm_gbs)"}
+    if N:
+        # a tree's query rows share every key: bound by whichever roofline is slower
+        fl = tree_flops(tree["parent_np"], kv, np.full(w.B, N), w.Hq, w.d) * w.n_layers / attn_launches
+        roof["algorithmic_flops_per_launch"] = fl
+        roof["kernel"] = "verify_attn (draft tree)"
+        if fl / (tensor_peak * 1e12) > attn_bytes_launch / (hbm_peak * 1e9):
+            tf = fl / attn_launch_s / 1e12
+            roof.update({"bound": "tensor", "achieved": round(tf, 2), "peak": tensor_peak, "unit": "TFLOP/s",
+                         "frac": round(tf / tensor_peak, 4),
+                         "peak_source": peak_src + " (MEASURED_PEAKS.json bf16_tflops_sustained)"})
 
-    # end to end through the public API with host buffers
+    # end to end through the public API with host buffers (the chain round on dense caches)
     e2e = None
-    if args.e2e_steps > 0:
+    if args.e2e_steps > 0 and not N and not P:
         e2e = run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset)
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        host = {k: v.cpu().numpy() for k, v in inp.items()}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not P:
+        # bf16 logits widen exactly to f32 for the oracle
+        host = {k: (v.float() if v.dtype == torch.bfloat16 else v).cpu().numpy() for k, v in inp.items()}
         host["cost_table"] = workloads.cost_table(w, kv)
         lay_host = [{"Q": layers[0]["Q"].cpu(), "Kc": layers[0]["Kc"].cpu(), "Vc": layers[0]["Vc"].cpu()}]
-        us, cores, sample = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds)
+        if N:
+            th = {"target_logits": tree["target"].float().cpu().numpy(), "draft_tokens": tree["tokens"].cpu().numpy(),
+                  "parent": tree["parent_np"], "L": np.full(w.B, N, np.int32)}
+            us, cores, sample = oracle_tree_round_time(w, host, th, lay_host[0], kv, args.cpu_seconds)
+        else:
+            us, cores, sample = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds)
         cpu = {"value": round(us, 1), "unit": "us", "cores": cores, "kind": "oracle", "sample": sample}
 
     if rank != 0:
         return
     clk = clocks.summary()
     value = elapsed_max * 1000.0 / (K_steps * world)
-    launches = K_steps * (attn_launches + 4)  # attention, conf, select, 2 accept
+    # attention (+ the tree-mask kernel per launch), conf, select, 2 accept
+    launches = K_steps * (attn_launches * (2 if N else 1) + 4)
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "us", "n_gpus": world, "steps": K_steps,
         "warmup": max(3, args.warmup), "ms_per_step": round(elapsed_max / K_steps, 6), "higher_is_better": False,
@@ -398,18 +531,16 @@ def run_ours(args, rank, world, local_rank):
                    "selector": ("alpha (Algorithm 1, alpha %g, first block %d)" % (args.alpha, block_size)
                                 if args.selector == "alpha" else "marginal gain (Thm. 4)"),
                    "logits": args.logits,
+                   "draft": ("DDTree-shaped tree of %d nodes (best-first, depth <= %d), greedy tree walk" % (N, w.K)
+                             if N else "chain"),
+                   "kv_cache": "paged, %d keys per page" % P if P else "dense",
                    "parallelism": "dp%d (independent sequences)" % world,
                    "l2": "no flush: %.0f MB of distinct inputs per step > 129 MB L2" % (by["total"] / 1e6),
                    "timing": "3 CUDA graphs per step (conf+select | attention layers | accept), events between"},
         "hbm_tbs": round(by["total"] / (us_per_round * 1e-6) / 1e12, 3),
         "hbm_frac_of_measured": round(by["total"] / (us_per_round * 1e-6) / 1e9 / hbm_peak, 4),
         "hbm_frac_of_nominal_8tbs": round(by["total"] / (us_per_round * 1e-6) / 1e9 / NOMINAL_HBM_GBS, 4),
-        "roofline": {"kernel": "verify_attn", "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
-                     "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
-                     "traffic": None if trec is None else trec.get("traffic_bytes_per_launch"),
-                     "algorithmic_bytes_per_launch": attn_bytes_launch,
-                     "layers_per_launch": round(w.n_layers / attn_launches, 2),
-                     "launch_us": round(attn_launch_s * 1e6, 3), "peak_source": peak_src + " (MEASURED_PEAKS.json hbm_gbs)"},
+        "roofline": roof,
         "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
                    "samples": clk["samples"]},
         "gpu_launches": launches,

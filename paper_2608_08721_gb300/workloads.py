@@ -295,6 +295,40 @@ def _ddtree_parents(rng: np.random.Generator, n: int, K: int, depth: int) -> np.
     return out
 
 
+def tree_logits(w: Workload, parent: np.ndarray, L, device="cpu", p_follow: float = 0.8) -> dict:
+    """Draft tokens [B, N] (int32) and target logits [B, N+1, V] (f32) of draft trees.
+
+    Siblings carry distinct random tokens. Node p's target row is N(0, 4^2)
+    with +12 at one token: with probability ``p_follow`` (when p has
+    children) the token of its lowest-numbered child (the drafter's
+    best-ranked candidate), else a uniformly random token."""
+    B, N1 = parent.shape
+    N = N1 - 1
+    L = np.broadcast_to(np.asarray(L, np.int64), (B,))
+    rng = np.random.default_rng([w.data_seed, 91])
+    tok = np.zeros((B, N), np.int32)
+    peak = np.zeros((B, N1), np.int64)
+    for b in range(B):
+        kids = [[] for _ in range(N1)]
+        for t in range(1, int(L[b]) + 1):
+            kids[int(parent[b, t])].append(t)
+        for p in range(N1):
+            if kids[p]:
+                vals = rng.choice(w.V, size=len(kids[p]), replace=False)
+                for t, v in zip(kids[p], vals):
+                    tok[b, t - 1] = v
+            if kids[p] and rng.random() < p_follow:
+                peak[b, p] = tok[b, kids[p][0] - 1]
+            else:
+                peak[b, p] = rng.integers(0, w.V)
+    g = torch.Generator(device=device)
+    g.manual_seed(w.data_seed * 7919 + 77)
+    target = _randn((B, N1, w.V), g, device) * 4.0
+    idx = torch.from_numpy(peak).to(device)
+    target.scatter_add_(2, idx[:, :, None], torch.full((B, N1, 1), 12.0, device=device))
+    return {"draft_tokens": torch.from_numpy(tok).to(device), "target_logits": target.contiguous()}
+
+
 def reference_inputs_summary(w: Workload) -> List[str]:
     """One line per input recipe, for reports."""
     return [
