@@ -449,8 +449,16 @@ __device__ __forceinline__ int merge_share(const MergeTask& t, int& u0) {
 constexpr int kMergeHelpChunks = 8;
 
 // Items per lane in a chunk of a group of np parts: J items x 16/J parts are
-// in flight per batch.
-__device__ __forceinline__ int merge_j(int np) { return np > 4 ? 1 : 4; }
+// in flight per batch, and a share of `items` items costs ceil(items / 32J)
+// chunks x ceil(np / (16/J)) batches, one memory round trip each. J = 4 wins
+// for many rows over few parts (tree and long blocks), J = 1 for one row
+// over many parts (short blocks at B = 1); ties go to J = 1 (more chunks to
+// share among helping warps).
+__device__ __forceinline__ int merge_j(int np, int items) {
+  const int trips1 = ((items + 31) / 32) * ((np + 15) / 16);
+  const int trips4 = ((items + 127) / 128) * ((np + 3) / 4);
+  return trips4 < trips1 ? 4 : 1;
+}
 
 template <int D>
 __device__ __forceinline__ int merge_chunk_count(const MergeTask* tasks, int n_tasks) {
@@ -458,7 +466,7 @@ __device__ __forceinline__ int merge_chunk_count(const MergeTask* tasks, int n_t
   for (int ti = 0; ti < n_tasks; ++ti) {
     int u0;
     const int items = merge_share(tasks[ti], u0) * (D / 4);
-    const int ci = 32 * merge_j(tasks[ti].np);
+    const int ci = 32 * merge_j(tasks[ti].np, items);
     n += (items + ci - 1) / ci;
   }
   return n;
@@ -568,14 +576,14 @@ __device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int
     int lc = u - layer * C, ti = 0, u0 = 0, nr = 0;
     for (; ti < n_tasks; ++ti) {
       nr = merge_share(tasks[ti], u0);
-      const int ci = 32 * merge_j(tasks[ti].np);
+      const int ci = 32 * merge_j(tasks[ti].np, nr * (D / 4));
       const int nc = (nr * (D / 4) + ci - 1) / ci;
       if (lc < nc) break;
       lc -= nc;
     }
     if (ti < n_tasks) {
       const MergeTask& t = tasks[ti];
-      if (merge_j(t.np) == 1) merge_chunk<1, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
+      if (merge_j(t.np, nr * (D / 4)) == 1) merge_chunk<1, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
       else merge_chunk<4, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
     }
     __syncwarp();
