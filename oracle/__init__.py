@@ -64,8 +64,9 @@ def _load():
     lib.oracle_verify_attn_tree.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32, i32, f64, P, P, P, i32]
     lib.oracle_accept.argtypes = [P, P, P, P, P, i32, i32, i32, u64, u64, u32, P, P, P]
     lib.oracle_accept_tree_greedy.argtypes = [P, P, P, P, i32, i32, i32, P, P, P]
+    lib.oracle_accept_tree.argtypes = [P, P, P, P, P, i32, i32, i32, u64, u64, u32, P, P, P, P]
     for name in ("oracle_confidence", "oracle_select_lengths", "oracle_select_iterate", "oracle_select_alpha",
-                 "oracle_gather_pages", "oracle_verify_attn_tree", "oracle_accept_tree_greedy",
+                 "oracle_gather_pages", "oracle_verify_attn_tree", "oracle_accept_tree_greedy", "oracle_accept_tree",
                  "oracle_verify_attn", "oracle_accept"):
         getattr(lib, name).restype = i32
     _lib = lib
@@ -252,6 +253,29 @@ def accept_tree_greedy(target_logits, draft_tokens, parent, L):
     _check(_load().oracle_accept_tree_greedy(_ptr(t), _ptr(tok), _ptr(par), _ptr(LL), B, K1 - 1, V,
                                              _ptr(n), _ptr(last), _ptr(bonus)), "oracle_accept_tree_greedy")
     return n, last, bonus
+
+
+def accept_tree(target_logits, draft_tokens, parent, L, temperature, seed, round_offset=0, seq_offset=0):
+    """Walk of a draft tree drawing the target's token at each node (greedy where temperature is 0):
+    n_accepted[B], last_node[B], bonus_token[B], flag[B] (int32)."""
+    t = _c(target_logits, np.float32)
+    B, K1, V = t.shape
+    tok = _c(draft_tokens, np.int32)
+    if tok.shape != (B, K1 - 1):
+        raise OracleError("draft_tokens must be [B,K]")
+    par = _c(parent, np.int32)
+    if par.shape != (B, K1):
+        raise OracleError("parent must be [B,K+1]")
+    LL = _c(L, np.int32)
+    T = _c(temperature, np.float32)
+    n = np.zeros(B, np.int32)
+    last = np.zeros(B, np.int32)
+    bonus = np.zeros(B, np.int32)
+    flag = np.zeros(B, np.int32)
+    _check(_load().oracle_accept_tree(_ptr(t), _ptr(tok), _ptr(par), _ptr(LL), _ptr(T), B, K1 - 1, V,
+                                      int(seed) & (2**64 - 1), int(round_offset), int(seq_offset), _ptr(n),
+                                      _ptr(last), _ptr(bonus), _ptr(flag)), "oracle_accept_tree")
+    return n, last, bonus, flag
 
 
 def accept(target_logits, draft_logits, draft_tokens, L, temperature, seed, round_offset=0,

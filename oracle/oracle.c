@@ -24,10 +24,11 @@
  *                          block-wise drafting budget, one rollback.
  *   oracle_gather_pages    the dense KV cache a paged cache (page pool and
  *                          block table) describes.
- *   oracle_verify_attn_tree, oracle_accept_tree_greedy
+ *   oracle_verify_attn_tree, oracle_accept_tree_greedy, oracle_accept_tree
  *                          verification of a draft tree (the tree drafters
  *                          of Sec. 2, e.g. DDTree): ancestor-masked
- *                          attention and the greedy longest accepted path.
+ *                          attention, the greedy longest accepted path and
+ *                          its sampling counterpart.
  *   oracle_verify_attn     block-causal GQA attention of the d+1 verified
  *                          positions against the target KV cache (Sec. 3.1:
  *                          the target scores all drafted positions in one
@@ -552,6 +553,83 @@ int oracle_accept_tree_greedy(const float* target, const int32_t* tokens, const 
     n_accepted[b] = n;
     if (last_node) last_node[b] = cur;
     bonus[b] = arg;
+  }
+  return ORACLE_OK;
+}
+
+/* Acceptance of a draft tree at temperature[b] (the greedy walk above when
+ * it is 0). At the current node the walk draws the target's token x from
+ * softmax(row / T) and moves to the lowest-numbered child carrying x while
+ * there is one; the round emits the walked nodes' tokens and then the last
+ * draw (bonus). Every emitted token is a draw from the target given the
+ * prefix it extends, so the output follows the target's distribution; a
+ * child is accepted with the target's probability of its token. Draw at
+ * node t: the race x = argmin_v key_v, key_v = log2(E_v) - y_v log2(e) / T,
+ * E_v = -ln u_v, u_v the Philox uniform of (v >> 2, position t, sequence
+ * seq_offset + b, purpose 2), word v & 3 (the exponential race in log2
+ * units; lowest index on equal keys). flag[b] = 1 when at a visited node
+ * the two smallest keys lie within 4e-5 + 1e-6 |y_v log2(e) / T| of each
+ * other (the fp32 keys of a GPU could order them differently). */
+static const uint32_t TREE_PURPOSE = 2u;
+
+static int tree_draw(const float* row, int V, double T, uint64_t seed, uint32_t t, uint32_t seq,
+                     uint64_t round_offset, int* flag) {
+  const double c = 1.4426950408889634 / T;
+  double best = INFINITY, second = INFINITY, yc_best = 0.0, yc_second = 0.0;
+  int arg = 0;
+  for (int v = 0; v < V; ++v) {
+    const double yc = (double)row[v] * c;
+    if (!(yc > -INFINITY)) continue;
+    const double u = oracle_uniform(seed, (uint32_t)(v >> 2), t, seq, TREE_PURPOSE, round_offset, v & 3);
+    const double key = log2(-log(u)) - yc;
+    if (key < best) {
+      second = best; yc_second = yc_best;
+      best = key; yc_best = yc; arg = v;
+    } else if (key < second) {
+      second = key; yc_second = yc;
+    }
+  }
+  if (second < INFINITY && second - best <= 4e-5 + 1e-6 * fmax(fabs(yc_best), fabs(yc_second))) *flag = 1;
+  return arg;
+}
+
+int oracle_accept_tree(const float* target, const int32_t* tokens, const int32_t* parent, const int32_t* L,
+                       const float* temperature, int B, int K, int V, uint64_t seed, uint64_t round_offset,
+                       uint32_t seq_offset, int32_t* n_accepted, int32_t* last_node, int32_t* bonus,
+                       int32_t* flag_out) {
+  if (B < 0 || K < 0 || V < 1 || !target || !tokens || !parent || !L || !temperature || !n_accepted || !bonus)
+    return ORACLE_EINVAL;
+  for (int b = 0; b < B; ++b) {
+    if (L[b] < 0 || L[b] > K) return ORACLE_EINVAL;
+    if (!(temperature[b] >= 0.0f) || !isfinite(temperature[b])) return ORACLE_EINVAL;
+    for (int t = 1; t <= L[b]; ++t) {
+      const int p = parent[(size_t)b * (K + 1) + t];
+      if (p < 0 || p >= t) return ORACLE_EINVAL;
+      if (tokens[(size_t)b * K + t - 1] < 0 || tokens[(size_t)b * K + t - 1] >= V) return ORACLE_EINVAL;
+    }
+  }
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int b = 0; b < B; ++b) {
+    const double T = (double)temperature[b];
+    const uint32_t seq = seq_offset + (uint32_t)b;
+    int cur = 0, n = 0, x = 0, flag = 0;
+    for (;;) {
+      const float* row = target + ((size_t)b * (K + 1) + cur) * V;
+      x = T == 0.0 ? row_argmax(row, V) : tree_draw(row, V, T, seed, (uint32_t)cur, seq, round_offset, &flag);
+      int next = -1;
+      for (int c = cur + 1; c <= L[b]; ++c)
+        if (parent[(size_t)b * (K + 1) + c] == cur && tokens[(size_t)b * K + c - 1] == x) {
+          next = c;
+          break;
+        }
+      if (next < 0) break;
+      cur = next;
+      ++n;
+    }
+    n_accepted[b] = n;
+    if (last_node) last_node[b] = cur;
+    bonus[b] = x;
+    if (flag_out) flag_out[b] = flag;
   }
   return ORACLE_OK;
 }

@@ -321,3 +321,134 @@ def test_tree_walk_rejects_bad_input(case):
         L = np.array([3], np.int32)
     with pytest.raises(oracle.OracleError):
         oracle.accept_tree_greedy(x, tok, par, L)
+
+
+# ---------------------------------------------------------------------------
+# sampling walk (temperature > 0)
+# ---------------------------------------------------------------------------
+def _softmax(y, T):
+    z = np.asarray(y, np.float64) / T
+    e = np.exp(z - z.max())
+    return e / e.sum()
+
+
+def _chi2_ok(counts, probs, n):
+    """Pearson chi-square against expected counts, cells with >= 5 expected;
+    accept unless the statistic is beyond the 1e-4 upper tail."""
+    from scipy.stats import chi2
+
+    exp = probs * n
+    keep = exp >= 5
+    stat = float(((counts[keep] - exp[keep]) ** 2 / exp[keep]).sum()) + 0.0
+    rest_o, rest_e = counts[~keep].sum(), exp[~keep].sum()
+    dof = int(keep.sum()) - 1
+    if rest_e >= 5:
+        stat += (rest_o - rest_e) ** 2 / rest_e
+        dof += 1
+    return stat < chi2.ppf(1 - 1e-4, max(dof, 1)), stat
+
+
+def test_tree_sampling_at_zero_temperature_is_the_greedy_walk():
+    rng = np.random.default_rng(40)
+    B, K, V = 40, 12, 30
+    L = rng.integers(0, K + 1, size=B).astype(np.int32)
+    par = workloads.draft_tree(B, K, L, seed=3, shape="random")
+    x = rng.standard_normal((B, K + 1, V)).astype(np.float32)
+    tok = rng.integers(0, V, size=(B, K)).astype(np.int32)
+    for b in range(B):   # make some matches
+        for t in range(1, int(L[b]) + 1):
+            if rng.random() < 0.7:
+                tok[b, t - 1] = int(np.argmax(x[b, par[b, t]]))
+    n, last, bonus, flag = oracle.accept_tree(x, tok, par, L, np.zeros(B, np.float32), seed=7)
+    n2, last2, bonus2 = oracle.accept_tree_greedy(x, tok, par, L)
+    np.testing.assert_array_equal(n, n2)
+    np.testing.assert_array_equal(last, last2)
+    np.testing.assert_array_equal(bonus, bonus2)
+    assert not flag.any()
+
+
+def test_tree_sampling_root_draw_follows_the_target():
+    """With no children the round emits one draw from softmax(row / T)."""
+    V, T, B = 7, 0.8, 40000
+    y = np.array([1.0, -0.5, 2.0, 0.3, 0.3, -2.0, 1.5], np.float32)
+    x = np.broadcast_to(y, (B, 1, V)).copy()
+    n, last, bonus, flag = oracle.accept_tree(x, np.zeros((B, 0), np.int32), np.zeros((B, 1), np.int32),
+                                              np.zeros(B, np.int32), np.full(B, T, np.float32), seed=123)
+    assert not n.any() and not last.any()
+    ok, stat = _chi2_ok(np.bincount(bonus, minlength=V).astype(float), _softmax(y, T), B)
+    assert ok, stat
+
+
+def test_tree_sampling_is_lossless_on_a_small_tree():
+    """The emitted token sequence follows the target's own sampling along the
+    tree, P(x1, x2, ...) = p_0(x1) p_{node(x1)}(x2) ..., enumerated exactly.
+
+    Tree (V = 4): node 1 (token 0) and node 2 (token 2) under the root, node 3
+    (token 1) under node 1, node 4 (token 3) under node 2."""
+    V, T, B = 4, 0.7, 60000
+    par = np.array([0, 0, 0, 1, 2], np.int32)
+    tok = np.array([0, 2, 1, 3], np.int32)
+    rows = np.array([[0.5, -1.0, 0.2, 0.0],     # root
+                     [-0.3, 0.9, 0.1, -1.2],    # node 1
+                     [0.0, 0.4, -0.6, 0.7],     # node 2
+                     [1.1, -0.2, 0.3, 0.0],     # node 3 (leaf)
+                     [-0.5, 0.5, 0.2, 0.8]],    # node 4 (leaf)
+                    np.float32)
+    p = [_softmax(r, T) for r in rows]
+    child = {(0, 0): 1, (0, 2): 2, (1, 1): 3, (2, 3): 4}
+    probs = {}
+
+    def walk(node, prefix, pr):
+        for v in range(V):
+            q = pr * p[node][v]
+            if (node, v) in child:
+                walk(child[(node, v)], prefix + (v,), q)
+            else:
+                probs[prefix + (v,)] = q
+    walk(0, (), 1.0)
+    assert abs(sum(probs.values()) - 1.0) < 1e-12
+    x = np.broadcast_to(rows, (B, 5, V)).copy()
+    n, last, bonus, flag = oracle.accept_tree(x, np.broadcast_to(tok, (B, 4)).copy(),
+                                              np.broadcast_to(par, (B, 5)).copy(), np.full(B, 4, np.int32),
+                                              np.full(B, T, np.float32), seed=2024, round_offset=3)
+    keys = sorted(probs)
+    index = {k: i for i, k in enumerate(keys)}
+    counts = np.zeros(len(keys))
+    node_token = {1: 0, 2: 2, 3: 1, 4: 3}
+    for b in range(B):
+        path, t = [], int(last[b])
+        while t != 0:
+            path.append(node_token[t])
+            t = int(par[t])
+        assert len(path) == n[b]
+        counts[index[tuple(path[::-1]) + (int(bonus[b]),)]] += 1
+    ok, stat = _chi2_ok(counts, np.array([probs[k] for k in keys]), B)
+    assert ok, stat
+    # the root's children are accepted with the target's probability of their tokens
+    acc = float((n >= 1).mean())
+    assert abs(acc - (p[0][0] + p[0][2])) < 4 * np.sqrt(acc * (1 - acc) / B)
+
+
+def test_tree_sampling_sequence_offset_and_rounds():
+    """Draws depend on the global sequence index and the round: a batch split
+    with seq_offset reproduces the unsplit batch; another round differs."""
+    rng = np.random.default_rng(41)
+    B, K, V = 24, 10, 50
+    L = np.full(B, K, np.int32)
+    par = workloads.draft_tree(B, K, L, seed=8, shape="topk")
+    x = (rng.standard_normal((B, K + 1, V)) * 2).astype(np.float32)
+    tok = rng.integers(0, V, size=(B, K)).astype(np.int32)
+    T = np.full(B, 1.0, np.float32)
+    full = oracle.accept_tree(x, tok, par, L, T, seed=5, round_offset=2)
+    part = oracle.accept_tree(x[10:], tok[10:], par[10:], L[10:], T[10:], seed=5, round_offset=2, seq_offset=10)
+    for a, b in zip(full, part):
+        np.testing.assert_array_equal(a[10:], b)
+    other = oracle.accept_tree(x, tok, par, L, T, seed=5, round_offset=3)
+    assert (other[2] != full[2]).any()
+
+
+def test_tree_sampling_rejects_bad_temperature():
+    x = np.zeros((1, 2, 4), np.float32)
+    with pytest.raises(oracle.OracleError):
+        oracle.accept_tree(x, np.array([[1]], np.int32), np.array([[0, 0]], np.int32), np.array([1], np.int32),
+                           np.array([-1.0], np.float32), seed=0)
