@@ -322,8 +322,8 @@ int libraspec_verify_attn_tree_paged_layers(const uint16_t* const* Q, const uint
  * A chain gives libraspec_accept's greedy result (last_node = n_accepted).
  * Reads target rows 0..L[b] once. A parent outside [0, t) or a token outside
  * [0, V) never matches (LIBRASPEC_ST_BAD_TREE / LIBRASPEC_ST_BAD_TOKEN).
- * Workspace: libraspec_workspace_size(B, N, V, ...). Sampling acceptance of
- * a tree is not provided.
+ * Workspace: libraspec_workspace_size(B, N, V, ...). libraspec_accept_tree
+ * is the same walk with per-sequence temperatures.
  */
 int libraspec_accept_tree_greedy(const float* target_logits, const int32_t* draft_tokens, const int32_t* parent,
                                  const int32_t* L, int B, int N, int V, int32_t* n_accepted, int32_t* last_node,
@@ -332,6 +332,32 @@ int libraspec_accept_tree_greedy_bf16(const uint16_t* target_logits, const int32
                                       const int32_t* parent, const int32_t* L, int B, int N, int V,
                                       int32_t* n_accepted, int32_t* last_node, int32_t* bonus_token, void* workspace,
                                       size_t ws_bytes, void* stream);
+
+/*
+ * Acceptance of a draft tree at temperature[b] (temperature [B] f32, >= 0;
+ * 0 gives the greedy walk above). At the current node the walk draws the
+ * target's token x from softmax(row / T) and moves to the lowest-numbered
+ * child carrying x while there is one; bonus_token is the last draw. Every
+ * emitted token is a draw from the target given the prefix it extends, so
+ * the output follows the target's distribution (lossless), and a child is
+ * accepted with the target's probability of its token; the drafter's own
+ * probabilities are not used (a tree drafter's candidates are chosen, not
+ * sampled). Draw at node t: x = argmin_v log2(-ln u_v) - y_v log2(e) / T,
+ * u_v the Philox4x32-10 uniform of counter (v >> 2, t, seq_offset + b,
+ * 2 + 4 * round_offset), word v & 3, key (seed lo, seed hi) (the generator
+ * and uniform mapping of libraspec_accept, purpose 2). The GPU ranks keys
+ * in binary32. Every node row 0..L[b] is read once and drawn from (the
+ * walk's path is known only after the draws). Shapes, outputs and
+ * workspace as for libraspec_accept_tree_greedy.
+ */
+int libraspec_accept_tree(const float* target_logits, const int32_t* draft_tokens, const int32_t* parent,
+                          const int32_t* L, const float* temperature, int B, int N, int V, uint64_t seed,
+                          uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted, int32_t* last_node,
+                          int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream);
+int libraspec_accept_tree_bf16(const uint16_t* target_logits, const int32_t* draft_tokens, const int32_t* parent,
+                               const int32_t* L, const float* temperature, int B, int N, int V, uint64_t seed,
+                               uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted, int32_t* last_node,
+                               int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream);
 
 /*
  * Step 4 — acceptance (paper Sec. 3.1; the standard speculative-sampling

@@ -46,6 +46,9 @@ SIGNATURES = {
                                                      _F, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_tree_greedy": (_I, [_P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_tree_greedy_bf16": (_I, [_P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _SZ, _P]),
+    "libraspec_accept_tree": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _P, _SZ, _P]),
+    "libraspec_accept_tree_bf16": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _P, _SZ,
+                                        _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_round": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _I,
@@ -387,6 +390,31 @@ def libraspec_accept_tree_greedy(target_logits, draft_tokens, parent, L, ws: Wor
     rc = getattr(load(), name)(_ptr(target_logits), _ptr(draft_tokens), _ptr(parent), _ptr(L), B, K, V,
                                _ptr(n_accepted), _ptr(last_node), _ptr(bonus_token), ws.ptr, ws.nbytes,
                                _stream(stream))
+    _check(rc, name)
+    return n_accepted, last_node, bonus_token
+
+
+def libraspec_accept_tree(target_logits, draft_tokens, parent, L, temperature, seed: int, ws: Workspace,
+                          round_offset: int = 0, seq_offset: int = 0, n_accepted=None, last_node=None,
+                          bonus_token=None, stream=None):
+    """Walk of a draft tree drawing the target's token at each node (greedy where temperature is 0).
+    Returns (n_accepted, last_node, bonus_token), int32 [B] each."""
+    B, K1, V = target_logits.shape
+    K = K1 - 1
+    bf16 = target_logits.dtype == torch.bfloat16
+    _req(target_logits, torch.bfloat16 if bf16 else torch.float32, "target_logits")
+    _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+    _check_parent(parent, B, K1)
+    _req(L, torch.int32, "L", (B,))
+    _req(temperature, torch.float32, "temperature", (B,))
+    dev = target_logits.device
+    n_accepted = torch.empty((B,), dtype=torch.int32, device=dev) if n_accepted is None else n_accepted
+    last_node = torch.empty((B,), dtype=torch.int32, device=dev) if last_node is None else last_node
+    bonus_token = torch.empty((B,), dtype=torch.int32, device=dev) if bonus_token is None else bonus_token
+    name = "libraspec_accept_tree_bf16" if bf16 else "libraspec_accept_tree"
+    rc = getattr(load(), name)(_ptr(target_logits), _ptr(draft_tokens), _ptr(parent), _ptr(L), _ptr(temperature), B,
+                               K, V, int(seed) & (2**64 - 1), int(round_offset), int(seq_offset), _ptr(n_accepted),
+                               _ptr(last_node), _ptr(bonus_token), ws.ptr, ws.nbytes, _stream(stream))
     _check(rc, name)
     return n_accepted, last_node, bonus_token
 

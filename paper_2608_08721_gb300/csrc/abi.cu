@@ -24,8 +24,9 @@ cudaError_t launch_verify_attn_layers(const uint16_t* const*, const uint16_t* co
                                       const int32_t*, const int32_t*, const int32_t*, int, int, int, int, int, int,
                                       float, uint16_t* const*, float* const*, char*, const WsLayout&, cudaStream_t);
 template <typename T>
-cudaError_t launch_accept_tree_greedy(const T*, const int32_t*, const int32_t*, const int32_t*, int, int, int,
-                                      int32_t*, int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
+cudaError_t launch_accept_tree(const T*, const int32_t*, const int32_t*, const int32_t*, const float*, int, int, int,
+                               uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, int32_t*, char*, const WsLayout&,
+                               cudaStream_t);
 template <typename T>
 cudaError_t launch_accept(const T*, const T*, const int32_t*, const float*, const float*, const int32_t*,
                           const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, char*,
@@ -317,7 +318,8 @@ int libraspec_accept_bf16(const uint16_t* target_logits, const uint16_t* draft_l
 extern "C++" {
 template <typename T>
 static int accept_tree_t(const T* target_logits, const int32_t* draft_tokens, const int32_t* parent,
-                         const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
+                         const int32_t* L, const float* temperature, int B, int K, int V, uint64_t seed,
+                         uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted, int32_t* last_node,
                          int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
   if (B < 0 || B > LIBRASPEC_MAX_B || K < 0 || K > LIBRASPEC_MAX_TREE_NODES || V < 1) return LIBRASPEC_EINVAL;
   if (B == 0) return LIBRASPEC_OK;
@@ -326,25 +328,43 @@ static int accept_tree_t(const T* target_logits, const int32_t* draft_tokens, co
   if (!aligned(target_logits, sizeof(T))) return LIBRASPEC_EINVAL;
   const WsLayout lay = ws_layout(B, K, V, 1, 1, 64, 1);
   if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
-  return from_cuda(launch_accept_tree_greedy<T>(target_logits, draft_tokens, parent, L, B, K, V, n_accepted,
-                                                last_node, bonus_token, static_cast<char*>(workspace), lay,
-                                                static_cast<cudaStream_t>(stream)));
+  return from_cuda(launch_accept_tree<T>(target_logits, draft_tokens, parent, L, temperature, B, K, V, seed,
+                                         round_offset, seq_offset, n_accepted, last_node, bonus_token,
+                                         static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
 }
 }  // extern "C++"
 
 int libraspec_accept_tree_greedy(const float* target_logits, const int32_t* draft_tokens, const int32_t* parent,
                                  const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
                                  int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
-  return accept_tree_t(target_logits, draft_tokens, parent, L, B, K, V, n_accepted, last_node, bonus_token,
-                       workspace, ws_bytes, stream);
+  return accept_tree_t(target_logits, draft_tokens, parent, L, nullptr, B, K, V, 0, 0, 0, n_accepted, last_node,
+                       bonus_token, workspace, ws_bytes, stream);
 }
 
 int libraspec_accept_tree_greedy_bf16(const uint16_t* target_logits, const int32_t* draft_tokens,
                                       const int32_t* parent, const int32_t* L, int B, int K, int V,
                                       int32_t* n_accepted, int32_t* last_node, int32_t* bonus_token, void* workspace,
                                       size_t ws_bytes, void* stream) {
-  return accept_tree_t(target_logits, draft_tokens, parent, L, B, K, V, n_accepted, last_node, bonus_token,
-                       workspace, ws_bytes, stream);
+  return accept_tree_t(target_logits, draft_tokens, parent, L, nullptr, B, K, V, 0, 0, 0, n_accepted, last_node,
+                       bonus_token, workspace, ws_bytes, stream);
+}
+
+int libraspec_accept_tree(const float* target_logits, const int32_t* draft_tokens, const int32_t* parent,
+                          const int32_t* L, const float* temperature, int B, int N, int V, uint64_t seed,
+                          uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted, int32_t* last_node,
+                          int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
+  if (!temperature && B > 0) return LIBRASPEC_EINVAL;
+  return accept_tree_t(target_logits, draft_tokens, parent, L, temperature, B, N, V, seed, round_offset, seq_offset,
+                       n_accepted, last_node, bonus_token, workspace, ws_bytes, stream);
+}
+
+int libraspec_accept_tree_bf16(const uint16_t* target_logits, const int32_t* draft_tokens, const int32_t* parent,
+                               const int32_t* L, const float* temperature, int B, int N, int V, uint64_t seed,
+                               uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted, int32_t* last_node,
+                               int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
+  if (!temperature && B > 0) return LIBRASPEC_EINVAL;
+  return accept_tree_t(target_logits, draft_tokens, parent, L, temperature, B, N, V, seed, round_offset, seq_offset,
+                       n_accepted, last_node, bonus_token, workspace, ws_bytes, stream);
 }
 
 extern "C++" {

@@ -334,6 +334,120 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
 }
 
 // ---------------------------------------------------------------------------
+// Per-node draws of a draft tree. Grid (nsplit, N+1, B); nodes t > L_b exit
+// at once. A greedy sequence (temperature 0) takes the argmax of the node's
+// target row; a sampling one draws from softmax(row / T) by the exponential
+// race x = argmin_v key_v, key_v = log2(E_v) - y_v log2(e) / T, E_v = -ln u_v,
+// u_v from Philox at (v >> 2, node t, sequence, purpose 2), word v & 3. The
+// race is carried as an argmax of -key so the partials merge like argmaxes
+// (lowest index on ties). A candidate can only win if key_v < best, i.e.
+// u_v > exp(-2^(best + y_v c)); that test (two fast exponentials, with a
+// margin above their error) skips the logarithms of almost every token.
+// The draw of node t lands in stat[b, t].arg for the walk.
+// ---------------------------------------------------------------------------
+template <bool VEC, typename E>
+__global__ void __launch_bounds__(kRowThreads) tree_rows_kernel(
+    const E* __restrict__ target, const int32_t* __restrict__ Ls, const float* __restrict__ temperature, int K,
+    int V, int nsplit, int chunk, uint64_t seed, uint64_t round_offset, uint32_t seq_offset,
+    RowPartial* __restrict__ part, uint32_t* __restrict__ cnt, RowStat* __restrict__ stat, int* __restrict__ status) {
+  __shared__ float smf[64];
+  __shared__ int smi[32];
+  __shared__ int last;
+  const int split = blockIdx.x, j = blockIdx.y, b = blockIdx.z;
+  const int Lb = Ls[b];
+  if (Lb < 0 || Lb > K) {
+    if (split == 0 && j == 0 && threadIdx.x == 0) raise_status(status, LIBRASPEC_ST_BAD_LENGTH);
+    return;
+  }
+  if (j > Lb) return;
+  const int row = b * (K + 1) + j;
+  const float tb = temperature[b];
+  const E* xr = target + (size_t)row * V;
+  const int c0 = split * chunk, c1 = min(V, c0 + chunk);
+  float m;
+  int arg;
+  if (!(tb > 0.f)) {
+    SumAcc sa;
+    ArgAcc aa;
+    sa.init();
+    aa.init();
+    row_slice_pass<false, true, VEC, E>(xr, c0, c1, 1.f, sa, aa);
+    m = aa.m;
+    arg = aa.arg;
+  } else {
+    const float c = (float)(1.4426950408889634 / (double)tb);
+    const uint32_t seq = seq_offset + (uint32_t)b;
+    float best = INFINITY;
+    int besti = 0x7fffffff;
+    for (int g = (c0 >> 2) + threadIdx.x; 4 * g < c1; g += kRowThreads) {
+      const uint4 w4 = philox_block(seed, (uint32_t)g, (uint32_t)j, seq, 2u, round_offset);
+      const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
+      float yv[4];
+      if (VEC) {
+        Logit<E>::stream4(xr + 4 * g, yv);
+      } else {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) yv[t] = 4 * g + t < V ? Logit<E>::at(xr, 4 * g + t) : -INFINITY;
+      }
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int v = 4 * g + t;
+        if (v >= c1) break;
+        const float yc = yv[t] * c;
+        if (!(yc > -INFINITY)) continue;
+        const float u = word_to_uniform(ws[t]);
+        // key < best  <=>  u > exp(-2^(best + yc)) =: h. The fast exponentials
+        // give h to a relative 2e-4 while h is a normal float (exponent above
+        // -150; below, h flushes to 0 and every candidate passes): a margin of
+        // 2^-12 keeps every possible winner, whose key is then compared exactly.
+        if (best == INFINITY || u > ex2_approx(-ex2_approx(best + yc) * kLog2e) * 0.999755859375f) {
+          const float key = log2f(-logf(u)) - yc;
+          argmin_combine(best, besti, key, v);
+        }
+      }
+    }
+    m = -best;
+    arg = besti;
+  }
+  cta_reduce_arg(m, arg, smf, smi);
+  if (nsplit == 1) {
+    if (threadIdx.x == 0) {
+      RowStat st;
+      st.m = m;
+      st.arg = arg;
+      st.Z = 0.0;
+      stat[row] = st;
+    }
+    return;
+  }
+  if (threadIdx.x == 0) {
+    RowPartial p;
+    p.m = m;
+    p.arg = arg;
+    p.s = 0.0;
+    part[(size_t)row * kRowMaxSplits + split] = p;
+    __threadfence();
+    const uint32_t ticket = atomicAdd(&cnt[row], 1u);
+    last = (ticket == (uint32_t)(nsplit - 1));
+  }
+  __syncthreads();
+  if (!last || threadIdx.x >= 32) return;
+  __threadfence();
+  float M;
+  int A;
+  double Z;
+  warp_merge_partials(part + (size_t)row * kRowMaxSplits, nsplit, 0.f, true, M, A, Z);
+  if (threadIdx.x == 0) {
+    RowStat st;
+    st.m = M;
+    st.arg = A;
+    st.Z = 0.0;
+    stat[row] = st;
+    cnt[row] = 0u;
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Greedy walk of a draft tree, one warp per sequence. Node t in [1, L_b] has
 // parent parent[b, t] < t and token tokens[b, t-1]. The warp first finds, for
 // every node p, its matching child next[p]: the lowest-numbered child whose
@@ -368,7 +482,8 @@ __global__ void __launch_bounds__(kWalkWarps * 32) tree_walk_kernel(
   int* next = next_s[w];
   constexpr int kNone = 0x7fffffff;
   for (int t = lane; t <= Lb; t += 32) {
-    arg[t] = __ldcg(&stat[(size_t)b * (K + 1) + t].arg);
+    const int a = __ldcg(&stat[(size_t)b * (K + 1) + t].arg);
+    arg[t] = a == 0x7fffffff ? 0 : a;  // a row without a finite logit
     next[t] = kNone;
   }
   __syncwarp();
@@ -397,10 +512,13 @@ __global__ void __launch_bounds__(kWalkWarps * 32) tree_walk_kernel(
 // ---------------------------------------------------------------------------
 int num_sms_current();
 
+// temperature == nullptr: every sequence greedy (argmax rows); else per
+// sequence, greedy at 0 and drawing at T > 0 (tree_rows_kernel).
 template <typename T>
-cudaError_t launch_accept_tree_greedy(const T* target, const int32_t* tokens, const int32_t* parent,
-                                      const int32_t* L, int B, int K, int V, int32_t* n_accepted, int32_t* last_node,
-                                      int32_t* bonus, char* ws, const WsLayout& lay, cudaStream_t stream) {
+cudaError_t launch_accept_tree(const T* target, const int32_t* tokens, const int32_t* parent, const int32_t* L,
+                               const float* temperature, int B, int K, int V, uint64_t seed, uint64_t round_offset,
+                               uint32_t seq_offset, int32_t* n_accepted, int32_t* last_node, int32_t* bonus,
+                               char* ws, const WsLayout& lay, cudaStream_t stream) {
   if (B == 0) return cudaSuccess;
   const int sms = num_sms_current();
   auto* st = reinterpret_cast<int*>(ws + lay.status);
@@ -412,24 +530,33 @@ cudaError_t launch_accept_tree_greedy(const T* target, const int32_t* tokens, co
   dim3 grid(nsplit, K + 1, B);
   auto* part = reinterpret_cast<RowPartial*>(ws + lay.row_part);
   auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.row_cnt);
-  if (rows_vectorizable(target, V))
-    accept_rows_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(target, L, nullptr, K, V, nsplit, chunk, part, cnt,
-                                                                   rstat, st);
-  else
-    accept_rows_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(target, L, nullptr, K, V, nsplit, chunk, part, cnt,
-                                                                    rstat, st);
+  const bool vec = rows_vectorizable(target, V);
+  if (temperature == nullptr) {
+    if (vec)
+      accept_rows_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(target, L, nullptr, K, V, nsplit, chunk, part,
+                                                                     cnt, rstat, st);
+    else
+      accept_rows_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(target, L, nullptr, K, V, nsplit, chunk, part,
+                                                                      cnt, rstat, st);
+  } else if (vec) {
+    tree_rows_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(target, L, temperature, K, V, nsplit, chunk, seed,
+                                                                 round_offset, seq_offset, part, cnt, rstat, st);
+  } else {
+    tree_rows_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(target, L, temperature, K, V, nsplit, chunk, seed,
+                                                                  round_offset, seq_offset, part, cnt, rstat, st);
+  }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   tree_walk_kernel<<<(B + kWalkWarps - 1) / kWalkWarps, kWalkWarps * 32, 0, stream>>>(
       tokens, parent, L, B, K, V, rstat, n_accepted, last_node, bonus, st);
   return cudaGetLastError();
 }
-template cudaError_t launch_accept_tree_greedy<float>(const float*, const int32_t*, const int32_t*, const int32_t*,
-                                                      int, int, int, int32_t*, int32_t*, int32_t*, char*,
-                                                      const WsLayout&, cudaStream_t);
-template cudaError_t launch_accept_tree_greedy<uint16_t>(const uint16_t*, const int32_t*, const int32_t*,
-                                                         const int32_t*, int, int, int, int32_t*, int32_t*, int32_t*,
-                                                         char*, const WsLayout&, cudaStream_t);
+template cudaError_t launch_accept_tree<float>(const float*, const int32_t*, const int32_t*, const int32_t*,
+                                               const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*,
+                                               int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
+template cudaError_t launch_accept_tree<uint16_t>(const uint16_t*, const int32_t*, const int32_t*, const int32_t*,
+                                                  const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*,
+                                                  int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
 
 template <typename T>
 cudaError_t launch_accept(const T* target, const T* draft, const int32_t* tokens, const float* conf,

@@ -157,7 +157,7 @@ def test_tree_bad_parent_sets_status():
 # ---------------------------------------------------------------------------
 # greedy walk
 # ---------------------------------------------------------------------------
-def _walk_inputs(B, K, V, shape, seed, dtype=torch.float32):
+def _walk_inputs(B, K, V, shape, seed, dtype=torch.float32, peak=6.0):
     """Trees with distinct sibling tokens; target rows whose argmax is often
     one of the node's children's tokens."""
     rng = np.random.default_rng(seed)
@@ -176,7 +176,7 @@ def _walk_inputs(B, K, V, shape, seed, dtype=torch.float32):
             for t, v in zip(kids[p], vals):
                 tok[b, t - 1] = v
             if kids[p] and rng.random() < 0.85:
-                x[b, p, int(tok[b, kids[p][rng.integers(len(kids[p]))] - 1])] = 6.0
+                x[b, p, int(tok[b, kids[p][rng.integers(len(kids[p]))] - 1])] = peak
     return x.to(dtype), tok, parent, L
 
 
@@ -320,3 +320,66 @@ def test_tree_rejects_node_budget_over_limit():
     with pytest.raises(lr.LibraspecError):
         lr.libraspec_verify_attn_tree_layers([{"Q": Q, "Kc": Kc, "Vc": Kc}], _i32(np.zeros((1, N + 1))),
                                              _i32([0]), _i32([0]), ws)
+
+
+# ---------------------------------------------------------------------------
+# sampling walk (per-sequence temperature)
+# ---------------------------------------------------------------------------
+def _assert_exact_unless_flagged(gpu, ref, flag, what):
+    gpu, ref, flag = (np.asarray(x) for x in (gpu, ref, flag))
+    bad = (gpu != ref) & (flag == 0)
+    assert not bad.any(), "%s differs on unflagged sequences %s" % (what, np.nonzero(bad)[0].tolist())
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("N,V", [(24, 32000), (24, 152064), (512, 32000), (130, 1003)])
+def test_tree_sampling_walk_matches_oracle(orc, dtype, N, V):
+    B = 24 if N <= 130 else 6
+    x, tok, parent, L = _walk_inputs(B, N, V, "ddtree" if N > 24 else "topk", seed=N + V % 89, dtype=dtype,
+                                     peak=14.0)
+    # mixed batch: greedy, cool, neutral and hot sequences
+    temps = np.array([[0.0, 0.6, 1.0, 1.6][b % 4] for b in range(B)], np.float32)
+    ws = lr.Workspace(B, N, V, 1, 1, 64, 1, device=cuda())
+    n, last, bonus = lr.libraspec_accept_tree(x, _i32(tok), _i32(parent), _i32(L),
+                                              torch.from_numpy(temps).to(cuda()), 99, ws, round_offset=5,
+                                              seq_offset=1000)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) == 0
+    rn, rlast, rbonus, flag = orc.accept_tree(x.float().cpu().numpy(), tok, parent, L, temps, seed=99,
+                                              round_offset=5, seq_offset=1000)
+    assert flag.sum() <= max(1, B // 10)
+    _assert_exact_unless_flagged(n.cpu().numpy(), rn, flag, "n_accepted")
+    _assert_exact_unless_flagged(last.cpu().numpy(), rlast, flag, "last_node")
+    _assert_exact_unless_flagged(bonus.cpu().numpy(), rbonus, flag, "bonus")
+    assert (rn[temps > 0] > 0).any()
+
+
+def test_tree_sampling_at_zero_temperature_equals_greedy_entry():
+    B, N, V = 16, 64, 32000
+    x, tok, parent, L = _walk_inputs(B, N, V, "ddtree", seed=12)
+    ws = lr.Workspace(B, N, V, 1, 1, 64, 1, device=cuda())
+    a = lr.libraspec_accept_tree(x, _i32(tok), _i32(parent), _i32(L), torch.zeros(B, device=cuda()), 3, ws)
+    b = lr.libraspec_accept_tree_greedy(x, _i32(tok), _i32(parent), _i32(L), ws)
+    torch.cuda.synchronize()
+    for u, v in zip(a, b):
+        assert torch.equal(u, v)
+
+
+def test_tree_sampling_root_draw_distribution_on_gpu():
+    """Sequences that share one row and have no children: the bonus draws
+    follow softmax(row / T) (chi-square, independent of the oracle)."""
+    from scipy.stats import chi2
+
+    B, V, T = 4096, 6, 0.9
+    y = torch.tensor([0.3, 1.2, -0.4, 0.8, 0.0, 2.0])
+    x = y.expand(B, 1, V).contiguous().to(cuda())
+    ws = lr.Workspace(B, 0, V, 1, 1, 64, 1, device=cuda())
+    _, _, bonus = lr.libraspec_accept_tree(x, torch.zeros((B, 0), dtype=torch.int32, device=cuda()),
+                                           torch.zeros((B, 1), dtype=torch.int32, device=cuda()),
+                                           torch.zeros(B, dtype=torch.int32, device=cuda()),
+                                           torch.full((B,), T, device=cuda()), 11, ws)
+    torch.cuda.synchronize()
+    counts = np.bincount(bonus.cpu().numpy(), minlength=V)
+    p = torch.softmax(y.double() / T, 0).numpy()
+    stat = float(((counts - p * B) ** 2 / (p * B)).sum())
+    assert stat < chi2.ppf(1 - 1e-4, V - 1), stat
