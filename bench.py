@@ -12,7 +12,8 @@ Variants of the round (the default is the chain draft on dense caches):
   --logits bf16      bf16 drafter and target logits;
   --page-size P      KV caches in pages of P keys behind block tables;
   --tree N           a DDTree-shaped draft tree of N nodes: tree-masked attention and the
-                     greedy tree walk replace the chain's attention and acceptance.
+                     tree walk (greedy or drawing, per the workload's temperatures) replace
+                     the chain's attention and acceptance.
 
 N > 1 runs under torchrun, one process per GPU; every rank verifies its own
 batch (weak scaling, no data-path collective) and rank 0 prints one JSON line.
@@ -214,8 +215,8 @@ def oracle_tree_round_time(w, host, tree_host, layer_host, kv, budget_s):
         t0 = time.perf_counter()
         q, _ = oracle.confidence(host["draft_logits"], host["draft_tokens"], host["temperature"])
         oracle.select_lengths(q, cost)
-        oracle.accept_tree_greedy(tree_host["target_logits"], tree_host["draft_tokens"], tree_host["parent"],
-                                  tree_host["L"])
+        oracle.accept_tree(tree_host["target_logits"], tree_host["draft_tokens"], tree_host["parent"],
+                           tree_host["L"], host["temperature"], w.philox_seed)
         t1 = time.perf_counter()
         oracle.verify_attn_tree(layer_host["Q"], layer_host["Kc"], layer_host["Vc"], kv, tree_host["L"],
                                 tree_host["parent"])
@@ -225,7 +226,7 @@ def oracle_tree_round_time(w, host, tree_host, layer_host, kv, budget_s):
         if time.perf_counter() > t_end or len(t_attn) >= 50:
             break
     per_round = statistics.median(t_logits) + statistics.median(t_attn) * w.n_layers
-    sample = ("%d repetition(s) of: confidence, selection and the greedy tree walk on the full batch plus ONE of "
+    sample = ("%d repetition(s) of: confidence, selection and the tree walk on the full batch plus ONE of "
               "the %d tree-attention layers (fp64 C oracle, %d threads); attention time scaled by %d layers" %
               (len(t_attn), w.n_layers, threads, w.n_layers))
     return per_round * 1e6, threads, sample
@@ -394,8 +395,9 @@ def run_ours(args, rank, world, local_rank):
 
     def seg_accept():
         if N:
-            lr.libraspec_accept_tree_greedy(tree["target"], tree["tokens"], tree["parent"], tree["L"], tree["ws"],
-                                            n_accepted=n_acc, last_node=tree["last"], bonus_token=bonus)
+            lr.libraspec_accept_tree(tree["target"], tree["tokens"], tree["parent"], tree["L"], inp["temperature"],
+                                     w.philox_seed, tree["ws"], seq_offset=seq_offset, n_accepted=n_acc,
+                                     last_node=tree["last"], bonus_token=bonus)
             return
         lr.libraspec_accept(inp["target_logits"], inp["draft_logits"], inp["draft_tokens"], conf, dstat, L,
                             inp["temperature"], w.philox_seed, ws, seq_offset=seq_offset, n_accepted=n_acc,
@@ -531,7 +533,7 @@ def run_ours(args, rank, world, local_rank):
                    "selector": ("alpha (Algorithm 1, alpha %g, first block %d)" % (args.alpha, block_size)
                                 if args.selector == "alpha" else "marginal gain (Thm. 4)"),
                    "logits": args.logits,
-                   "draft": ("DDTree-shaped tree of %d nodes (best-first, depth <= %d), greedy tree walk" % (N, w.K)
+                   "draft": ("DDTree-shaped tree of %d nodes (best-first, depth <= %d), tree walk" % (N, w.K)
                              if N else "chain"),
                    "kv_cache": "paged, %d keys per page" % P if P else "dense",
                    "parallelism": "dp%d (independent sequences)" % world,
