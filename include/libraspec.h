@@ -360,6 +360,31 @@ int libraspec_accept_tree_bf16(const uint16_t* target_logits, const int32_t* dra
                                int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * Appending the verified block's keys and values to the caches (the target
+ * computes them for the block positions, Sec. 3.1; the verify attention
+ * reads them at rows kv_len[b] .. kv_len[b] + T - 1):
+ *   kv_new [n_layers, 2, B, Hkv, T, head_dim] bf16 (device, 16-byte aligned):
+ *          layer l's keys ([l, 0]) and values ([l, 1]) of block positions
+ *          0 .. T-1 (T = K+1 for a chain block, N+1 for a tree);
+ *   Kc[l], Vc[l]: HOST arrays of device pointers to the layer caches,
+ *          [B, Hkv, S_cap, head_dim] (dense) or page pools [n_pages, Hkv,
+ *          page_size, head_dim] with block_table [B, max_pages] (paged: row s
+ *          of sequence b at page block_table[b * max_pages + s / page_size],
+ *          row s % page_size).
+ * Row kv_len[b] + r lands in the cache for r < T; a row past the capacity
+ * sets LIBRASPEC_ST_KV_OVERFLOW and a block-table entry outside [0, n_pages)
+ * LIBRASPEC_ST_BAD_PAGE (the row is skipped). The workspace holds the status
+ * word only (>= 256 bytes). One launch per 64 layers, 16 bytes per thread.
+ */
+int libraspec_kv_append(const uint16_t* kv_new, uint16_t* const* Kc, uint16_t* const* Vc, int n_layers,
+                        const int32_t* kv_len, int B, int T, int Hkv, int head_dim, int S_cap, void* workspace,
+                        size_t ws_bytes, void* stream);
+int libraspec_kv_append_paged(const uint16_t* kv_new, uint16_t* const* Kp, uint16_t* const* Vp, int n_layers,
+                              const int32_t* block_table, int max_pages, int page_size, int n_pages,
+                              const int32_t* kv_len, int B, int T, int Hkv, int head_dim, void* workspace,
+                              size_t ws_bytes, void* stream);
+
+/*
  * Step 4 — acceptance (paper Sec. 3.1; the standard speculative-sampling
  * rule of Leviathan et al. that the paper cites, lossless with respect to
  * the target distribution).

@@ -1,21 +1,33 @@
 """Public API: a verify round over device-resident state, fed from host buffers.
 
-``VerifyRound`` owns the device buffers of one round's shapes (per-round
-inputs, outputs, workspace) and runs the whole round through
-``libraspec_verify_round``. The KV caches are model state and stay on the
-device; the per-round inputs (logits, drafts, temperatures, cost table, the
-verified block's queries and its new K/V rows) can be passed as pinned host
-tensors, in which case they are copied in on the round's stream and the
-accepted counts and bonus tokens are copied back.
+``VerifyRound`` owns the device buffers of one round's shapes and runs the
+whole round through ``libraspec_verify_round``. The KV caches are model state
+and stay on the device. Every per-round input (drafter and target logits,
+draft tokens, temperatures, the cost table, each layer's queries and the
+verified block's new keys and values) lives in ONE pinned host buffer and its
+device mirror: a round is one host-to-device copy, ``libraspec_kv_append``
+(the block's keys and values into the caches), the round's kernels, and an
+8-byte-per-sequence copy of the accepted counts and bonus tokens back.
 """
 from __future__ import annotations
 
-from typing import Dict, List, Optional
+from typing import Dict, List
 
-import numpy as np
 import torch
 
 from . import binding
+
+
+def _layout(regions):
+    """Byte offsets of the regions, each 256-byte aligned; returns (offsets, total)."""
+    offs, off = {}, 0
+    for name, shape, dtype in regions:
+        offs[name] = off
+        n = 1
+        for s in shape:
+            n *= s
+        off += (n * torch.empty((), dtype=dtype).element_size() + 255) // 256 * 256
+    return offs, off
 
 
 class VerifyRound:
@@ -30,64 +42,80 @@ class VerifyRound:
         self.device = torch.device("cuda") if device is None else torch.device(device)
         dev = self.device
         self.caches = caches
-        self.n_layers = len(caches)
+        self.n_layers = n = len(caches)
         self.ws = binding.Workspace(B, K, V, Hq, Hkv, head_dim, S_cap, device=dev)
         self.kv_len = kv_len.to(dev, torch.int32).contiguous()
-        self.kv_len_host = [int(x) for x in kv_len.cpu()]
         f32, i32, bf = torch.float32, torch.int32, torch.bfloat16
-        self.draft_logits = torch.empty((B, K, V), dtype=logits_dtype, device=dev)
-        self.target_logits = torch.empty((B, K + 1, V), dtype=logits_dtype, device=dev)
-        self.draft_tokens = torch.empty((B, K), dtype=i32, device=dev)
-        self.temperature = torch.empty((B,), dtype=f32, device=dev)
-        self.cost_table = torch.empty((K + 1,), dtype=f32, device=dev)
-        self.layers = [{"Q": torch.empty((B, K + 1, Hq, head_dim), dtype=bf, device=dev),
-                        "Kc": c["Kc"], "Vc": c["Vc"]} for c in caches]
+        K1 = K + 1
+        regions = [("draft_logits", (B, K, V), logits_dtype), ("target_logits", (B, K1, V), logits_dtype),
+                   ("draft_tokens", (B, K), i32), ("temperature", (B,), f32), ("cost_table", (K1,), f32),
+                   ("Q", (n, B, K1, Hq, head_dim), bf), ("kv_new", (n, 2, B, Hkv, K1, head_dim), bf)]
+        offs, total = _layout(regions)
+        self._host_stage = torch.empty(total, dtype=torch.uint8, pin_memory=True)
+        self._dev_stage = torch.empty(total, dtype=torch.uint8, device=dev)
+
+        def views(buf):
+            out = {}
+            for name, shape, dtype in regions:
+                nbytes = torch.empty((), dtype=dtype).element_size()
+                for s in shape:
+                    nbytes *= s
+                out[name] = buf[offs[name]:offs[name] + nbytes].view(dtype).view(shape)
+            return out
+
+        self._host = views(self._host_stage)
+        self._dev = views(self._dev_stage)
+        d = self._dev
+        self.draft_logits, self.target_logits = d["draft_logits"], d["target_logits"]
+        self.draft_tokens, self.temperature, self.cost_table = d["draft_tokens"], d["temperature"], d["cost_table"]
+        self.layers = [{"Q": d["Q"][l], "Kc": c["Kc"], "Vc": c["Vc"]} for l, c in enumerate(caches)]
         self.out = binding.RoundOutputs(
             torch.empty((B, K), dtype=f32, device=dev), torch.empty((B, K, 2), dtype=f32, device=dev),
             torch.empty((B,), dtype=i32, device=dev), torch.empty((B,), dtype=i32, device=dev),
             torch.empty((B,), dtype=i32, device=dev),
-            [torch.empty((B, K + 1, Hq, head_dim), dtype=bf, device=dev) for _ in caches], None)
+            [torch.empty((B, K1, Hq, head_dim), dtype=bf, device=dev) for _ in caches], None)
         self.result_host = torch.empty((2, B), dtype=i32, pin_memory=True)
 
+    def host_inputs(self) -> Dict[str, torch.Tensor]:
+        """Pinned host views to fill before ``run_staged``: draft_logits [B,K,V], target_logits [B,K+1,V],
+        draft_tokens [B,K], temperature [B], cost_table [K+1], Q [n_layers,B,K+1,Hq,d] and kv_new
+        [n_layers,2,B,Hkv,K+1,d] (layer l's new keys [l,0] and values [l,1] of the verified block)."""
+        return self._host
+
     def run_device(self, seed: int, round_offset: int = 0, seq_offset: int = 0, stream=None):
-        """The round on inputs already resident in this object's device buffers."""
+        """The round on inputs already resident in this object's device buffers
+        (the new keys and values already in the caches)."""
         return binding.libraspec_verify_round(
             self.draft_logits, self.draft_tokens, self.temperature, self.cost_table, self.target_logits,
             self.layers, self.kv_len, seed, self.ws, round_offset=round_offset, seq_offset=seq_offset,
             outputs=self.out, stream=stream)
 
     def h2d_bytes(self) -> int:
-        per_layer = self.B * (self.K + 1) * self.Hq * self.d * 2 + 2 * self.B * self.Hkv * (self.K + 1) * self.d * 2
-        lb = self.draft_logits.element_size()
-        return (self.draft_logits.numel() * lb + self.target_logits.numel() * lb + self.draft_tokens.numel() * 4 +
-                self.temperature.numel() * 4 + self.cost_table.numel() * 4 + self.n_layers * per_layer)
+        return self._host_stage.numel()
 
     def d2h_bytes(self) -> int:
         return self.result_host.numel() * 4
 
-    def run_host(self, host: Dict, seed: int, round_offset: int = 0, seq_offset: int = 0):
-        """Copy one round's host inputs in, run the round, copy the results out.
-
-        host: draft_logits, target_logits, draft_tokens, temperature, cost_table
-        (pinned CPU tensors) and "layers": per layer {"Q", "K_new", "V_new"}
-        with K_new / V_new [B,Hkv,K+1,d], the verified block's keys and values,
-        written into the caches at kv_len_b .. kv_len_b + K.
-        Returns (n_accepted, bonus_token) as numpy arrays."""
-        nb = True
-        self.draft_logits.copy_(host["draft_logits"], non_blocking=nb)
-        self.target_logits.copy_(host["target_logits"], non_blocking=nb)
-        self.draft_tokens.copy_(host["draft_tokens"], non_blocking=nb)
-        self.temperature.copy_(host["temperature"], non_blocking=nb)
-        self.cost_table.copy_(host["cost_table"], non_blocking=nb)
-        K1 = self.K + 1
-        for l, hl in enumerate(host["layers"]):
-            self.layers[l]["Q"].copy_(hl["Q"], non_blocking=nb)
-            for b in range(self.B):
-                kv = self.kv_len_host[b]
-                self.layers[l]["Kc"][b, :, kv:kv + K1].copy_(hl["K_new"][b], non_blocking=nb)
-                self.layers[l]["Vc"][b, :, kv:kv + K1].copy_(hl["V_new"][b], non_blocking=nb)
+    def run_staged(self, seed: int, round_offset: int = 0, seq_offset: int = 0):
+        """One round from the pinned host inputs (``host_inputs``): copy them in, append the block's keys
+        and values, run the round, read the results back. Returns (n_accepted, bonus_token) numpy arrays."""
+        self._dev_stage.copy_(self._host_stage, non_blocking=True)
+        binding.libraspec_kv_append(self._dev["kv_new"], self.caches, self.kv_len, self.ws)
         self.run_device(seed, round_offset, seq_offset)
-        self.result_host[0].copy_(self.out.n_accepted, non_blocking=nb)
-        self.result_host[1].copy_(self.out.bonus_token, non_blocking=nb)
+        self.result_host[0].copy_(self.out.n_accepted, non_blocking=True)
+        self.result_host[1].copy_(self.out.bonus_token, non_blocking=True)
         torch.cuda.current_stream().synchronize()
         return self.result_host[0].numpy().copy(), self.result_host[1].numpy().copy()
+
+    def run_host(self, host: Dict, seed: int, round_offset: int = 0, seq_offset: int = 0):
+        """``run_staged`` from separate host tensors: draft_logits, target_logits, draft_tokens,
+        temperature, cost_table and "layers": per layer {"Q", "K_new", "V_new"} (K_new / V_new
+        [B,Hkv,K+1,d]), first gathered into the pinned buffer on the host."""
+        h = self._host
+        for name in ("draft_logits", "target_logits", "draft_tokens", "temperature", "cost_table"):
+            h[name].copy_(host[name])
+        for l, hl in enumerate(host["layers"]):
+            h["Q"][l].copy_(hl["Q"])
+            h["kv_new"][l, 0].copy_(hl["K_new"])
+            h["kv_new"][l, 1].copy_(hl["V_new"])
+        return self.run_staged(seed, round_offset, seq_offset)

@@ -49,6 +49,8 @@ SIGNATURES = {
     "libraspec_accept_tree": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_tree_bf16": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _P, _SZ,
                                         _P]),
+    "libraspec_kv_append": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _P, _SZ, _P]),
+    "libraspec_kv_append_paged": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _P, _I, _I, _I, _I, _P, _SZ, _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
     "libraspec_verify_round": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _I,
@@ -417,6 +419,36 @@ def libraspec_accept_tree(target_logits, draft_tokens, parent, L, temperature, s
                                _ptr(last_node), _ptr(bonus_token), ws.ptr, ws.nbytes, _stream(stream))
     _check(rc, name)
     return n_accepted, last_node, bonus_token
+
+
+def libraspec_kv_append(kv_new, caches, kv_len, ws: Workspace, block_table=None, stream=None) -> None:
+    """kv_new [n_layers, 2, B, Hkv, T, d] bf16; caches: per layer {"Kc", "Vc"} (dense [B,Hkv,S_cap,d]) or
+    {"Kp", "Vp"} (page pools [n_pages,Hkv,page_size,d], with block_table [B, max_pages])."""
+    n_layers, two, B, Hkv, T, d = kv_new.shape
+    if two != 2 or len(caches) != n_layers:
+        raise ValueError("kv_new must be [n_layers, 2, B, Hkv, T, d] with one cache per layer")
+    _req(kv_new, torch.bfloat16, "kv_new")
+    _req(kv_len, torch.int32, "kv_len", (B,))
+    if block_table is None:
+        S_cap = caches[0]["Kc"].shape[2] if n_layers else 1
+        for i, c in enumerate(caches):
+            _req(c["Kc"], torch.bfloat16, "Kc[%d]" % i, (B, Hkv, S_cap, d))
+            _req(c["Vc"], torch.bfloat16, "Vc[%d]" % i, (B, Hkv, S_cap, d))
+        rc = load().libraspec_kv_append(_ptr(kv_new), _ptr_array([c["Kc"] for c in caches]),
+                                        _ptr_array([c["Vc"] for c in caches]), n_layers, _ptr(kv_len), B, T, Hkv,
+                                        d, S_cap, ws.ptr, ws.nbytes, _stream(stream))
+        _check(rc, "libraspec_kv_append")
+        return
+    _req(block_table, torch.int32, "block_table")
+    n_pages, _, page_size, _ = caches[0]["Kp"].shape
+    for i, c in enumerate(caches):
+        _req(c["Kp"], torch.bfloat16, "Kp[%d]" % i, (n_pages, Hkv, page_size, d))
+        _req(c["Vp"], torch.bfloat16, "Vp[%d]" % i, (n_pages, Hkv, page_size, d))
+    rc = load().libraspec_kv_append_paged(_ptr(kv_new), _ptr_array([c["Kp"] for c in caches]),
+                                          _ptr_array([c["Vp"] for c in caches]), n_layers, _ptr(block_table),
+                                          block_table.shape[1], page_size, n_pages, _ptr(kv_len), B, T, Hkv, d,
+                                          ws.ptr, ws.nbytes, _stream(stream))
+    _check(rc, "libraspec_kv_append_paged")
 
 
 def _ptr_array(tensors: Sequence[Optional[torch.Tensor]]):

@@ -23,6 +23,8 @@ cudaError_t launch_verify_attn_paged_layers(const uint16_t* const*, const uint16
 cudaError_t launch_verify_attn_layers(const uint16_t* const*, const uint16_t* const*, const uint16_t* const*, int,
                                       const int32_t*, const int32_t*, const int32_t*, int, int, int, int, int, int,
                                       float, uint16_t* const*, float* const*, char*, const WsLayout&, cudaStream_t);
+cudaError_t launch_kv_append(const uint16_t*, uint16_t* const*, uint16_t* const*, int, const int32_t*,
+                             const int32_t*, int, int, int, int, int, int, int, int, int*, cudaStream_t);
 template <typename T>
 cudaError_t launch_accept_tree(const T*, const int32_t*, const int32_t*, const int32_t*, const float*, int, int, int,
                                uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, int32_t*, char*, const WsLayout&,
@@ -313,6 +315,45 @@ int libraspec_accept_bf16(const uint16_t* target_logits, const uint16_t* draft_l
                           void* stream) {
   return accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed,
                   round_offset, seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
+}
+
+namespace {
+
+int kv_append_checked(const uint16_t* kv_new, uint16_t* const* Kc, uint16_t* const* Vc, int n_layers,
+                      const int32_t* kv_len, const int32_t* block_table, int max_pages, int page_size, int n_pages,
+                      int B, int T, int Hkv, int head_dim, int S_cap, void* workspace, size_t ws_bytes,
+                      void* stream) {
+  if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
+  if (B < 0 || B > LIBRASPEC_MAX_B || T < 0 || T > LIBRASPEC_MAX_TREE_NODES + 1 || Hkv < 1 || n_layers < 0 ||
+      S_cap < 1)
+    return LIBRASPEC_EINVAL;
+  if (B == 0 || T == 0 || n_layers == 0) return LIBRASPEC_OK;
+  if (!kv_new || !aligned(kv_new, 16) || !Kc || !Vc || !kv_len) return LIBRASPEC_EINVAL;
+  for (int l = 0; l < n_layers; ++l)
+    if (!Kc[l] || !Vc[l] || !aligned(Kc[l], 16) || !aligned(Vc[l], 16)) return LIBRASPEC_EINVAL;
+  if (!workspace || !aligned(workspace, 256) || ws_bytes < 256) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_kv_append(kv_new, Kc, Vc, n_layers, kv_len, block_table, max_pages, page_size, n_pages, B,
+                                    T, Hkv, head_dim, S_cap, static_cast<int*>(workspace),
+                                    static_cast<cudaStream_t>(stream)));
+}
+
+}  // namespace
+
+int libraspec_kv_append(const uint16_t* kv_new, uint16_t* const* Kc, uint16_t* const* Vc, int n_layers,
+                        const int32_t* kv_len, int B, int T, int Hkv, int head_dim, int S_cap, void* workspace,
+                        size_t ws_bytes, void* stream) {
+  return kv_append_checked(kv_new, Kc, Vc, n_layers, kv_len, nullptr, 0, 0, 0, B, T, Hkv, head_dim, S_cap, workspace,
+                           ws_bytes, stream);
+}
+
+int libraspec_kv_append_paged(const uint16_t* kv_new, uint16_t* const* Kp, uint16_t* const* Vp, int n_layers,
+                              const int32_t* block_table, int max_pages, int page_size, int n_pages,
+                              const int32_t* kv_len, int B, int T, int Hkv, int head_dim, void* workspace,
+                              size_t ws_bytes, void* stream) {
+  if (page_size < 1 || max_pages < 1 || n_pages < 1 || (long)max_pages * page_size > 0x7fffffffL) return LIBRASPEC_EINVAL;
+  if (B > 0 && (!block_table || !aligned(block_table, 4))) return LIBRASPEC_EINVAL;
+  return kv_append_checked(kv_new, Kp, Vp, n_layers, kv_len, block_table, max_pages, page_size, n_pages, B, T, Hkv,
+                           head_dim, max_pages * page_size, workspace, ws_bytes, stream);
 }
 
 extern "C++" {
