@@ -451,6 +451,44 @@ int libraspec_verify_round_bf16(const uint16_t* draft_logits, const int32_t* dra
                                 int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
                                 void* stream);
 
+/*
+ * The round fed from pinned host memory with the copies overlapped: three
+ * host parts (host_parts[i], part_bytes[i] bytes, pinned) are copied to
+ * dev_parts[i] on copy_stream, in order: part 0 must hold the drafter block
+ * (draft_logits, draft_tokens, temperature, cost_table), part 1 the layers'
+ * Q and kv_new, part 2 target_logits (the typed pointers below point into
+ * the device parts). On `stream`, confidence and selection wait for part 0;
+ * libraspec_kv_append of kv_new ([n_layers, 2, B, Hkv, K+1, head_dim]) and
+ * the attention layers wait for part 1; acceptance waits for part 2; then
+ * n_accepted and bonus_token are copied to n_accepted_host / bonus_host
+ * (pinned, B entries each). copy_stream first waits for the work already on
+ * `stream`, so a round never overwrites buffers an earlier one still reads.
+ * The call returns after enqueuing; synchronise `stream` before reading the
+ * host results. Other arguments as libraspec_verify_round (lse is not
+ * produced).
+ */
+int libraspec_verify_round_staged(const void* const* host_parts, void* const* dev_parts, const size_t* part_bytes,
+                                  void* copy_stream, const uint16_t* kv_new, int32_t* n_accepted_host,
+                                  int32_t* bonus_host, const float* draft_logits, const int32_t* draft_tokens,
+                                  const float* temperature, const float* cost_table, const float* target_logits,
+                                  const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
+                                  uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V,
+                                  int Hq, int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                                  uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
+                                  int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                                  void* stream);
+int libraspec_verify_round_staged_bf16(const void* const* host_parts, void* const* dev_parts,
+                                       const size_t* part_bytes, void* copy_stream, const uint16_t* kv_new,
+                                       int32_t* n_accepted_host, int32_t* bonus_host, const uint16_t* draft_logits,
+                                       const int32_t* draft_tokens, const float* temperature,
+                                       const float* cost_table, const uint16_t* target_logits,
+                                       const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
+                                       uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V,
+                                       int Hq, int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                                       uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat,
+                                       int32_t* L, int32_t* n_accepted, int32_t* bonus_token, void* workspace,
+                                       size_t ws_bytes, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -5,9 +5,12 @@ whole round through ``libraspec_verify_round``. The KV caches are model state
 and stay on the device. Every per-round input (drafter and target logits,
 draft tokens, temperatures, the cost table, each layer's queries and the
 verified block's new keys and values) lives in ONE pinned host buffer and its
-device mirror: a round is one host-to-device copy, ``libraspec_kv_append``
-(the block's keys and values into the caches), the round's kernels, and an
-8-byte-per-sequence copy of the accepted counts and bonus tokens back.
+device mirror, laid out in the order the round needs them: the drafter block
+(confidence and selection), the layers' queries and new keys/values
+(``libraspec_kv_append``, then attention), the target rows (acceptance). A
+round copies the three parts in on a side stream while the round's kernels
+start as soon as their part has landed, then reads the accepted counts and
+bonus tokens back (8 bytes per sequence).
 """
 from __future__ import annotations
 
@@ -47,10 +50,13 @@ class VerifyRound:
         self.kv_len = kv_len.to(dev, torch.int32).contiguous()
         f32, i32, bf = torch.float32, torch.int32, torch.bfloat16
         K1 = K + 1
-        regions = [("draft_logits", (B, K, V), logits_dtype), ("target_logits", (B, K1, V), logits_dtype),
-                   ("draft_tokens", (B, K), i32), ("temperature", (B,), f32), ("cost_table", (K1,), f32),
-                   ("Q", (n, B, K1, Hq, head_dim), bf), ("kv_new", (n, 2, B, Hkv, K1, head_dim), bf)]
+        regions = [("draft_logits", (B, K, V), logits_dtype), ("draft_tokens", (B, K), i32),
+                   ("temperature", (B,), f32), ("cost_table", (K1,), f32),
+                   ("Q", (n, B, K1, Hq, head_dim), bf), ("kv_new", (n, 2, B, Hkv, K1, head_dim), bf),
+                   ("target_logits", (B, K1, V), logits_dtype)]
         offs, total = _layout(regions)
+        # the three parts a round copies in, in the order its steps need them
+        self._parts = [(0, offs["Q"]), (offs["Q"], offs["target_logits"]), (offs["target_logits"], total)]
         self._host_stage = torch.empty(total, dtype=torch.uint8, pin_memory=True)
         self._dev_stage = torch.empty(total, dtype=torch.uint8, device=dev)
 
@@ -75,6 +81,10 @@ class VerifyRound:
             torch.empty((B,), dtype=i32, device=dev),
             [torch.empty((B, K1, Hq, head_dim), dtype=bf, device=dev) for _ in caches], None)
         self.result_host = torch.empty((2, B), dtype=i32, pin_memory=True)
+        self._staged = binding.StagedRound(
+            [self._host_stage[a:b] for a, b in self._parts], [self._dev_stage[a:b] for a, b in self._parts],
+            d["kv_new"], self.result_host[0], self.result_host[1], self.draft_logits, self.draft_tokens,
+            self.temperature, self.cost_table, self.target_logits, self.layers, self.kv_len, self.out, self.ws)
 
     def host_inputs(self) -> Dict[str, torch.Tensor]:
         """Pinned host views to fill before ``run_staged``: draft_logits [B,K,V], target_logits [B,K+1,V],
@@ -97,14 +107,13 @@ class VerifyRound:
         return self.result_host.numel() * 4
 
     def run_staged(self, seed: int, round_offset: int = 0, seq_offset: int = 0):
-        """One round from the pinned host inputs (``host_inputs``): copy them in, append the block's keys
-        and values, run the round, read the results back. Returns (n_accepted, bonus_token) numpy arrays."""
-        self._dev_stage.copy_(self._host_stage, non_blocking=True)
-        binding.libraspec_kv_append(self._dev["kv_new"], self.caches, self.kv_len, self.ws)
-        self.run_device(seed, round_offset, seq_offset)
-        self.result_host[0].copy_(self.out.n_accepted, non_blocking=True)
-        self.result_host[1].copy_(self.out.bonus_token, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
+        """One round from the pinned host inputs (``host_inputs``), by libraspec_verify_round_staged: the
+        three parts are copied in on a side stream; confidence and selection start once the drafter
+        part has landed, the key/value append and the attention layers once the layer part has,
+        acceptance once the target rows have; the results come back into pinned memory. Returns
+        (n_accepted, bonus_token) numpy arrays."""
+        self._staged(seed, round_offset, seq_offset)
+        torch.cuda.current_stream(self.device).synchronize()
         return self.result_host[0].numpy().copy(), self.result_host[1].numpy().copy()
 
     def run_host(self, host: Dict, seed: int, round_offset: int = 0, seq_offset: int = 0):

@@ -49,6 +49,12 @@ SIGNATURES = {
     "libraspec_accept_tree": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_tree_bf16": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _P, _SZ,
                                         _P]),
+    "libraspec_verify_round_staged": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P,
+                                           _I, _I, _I, _I, _I, _I, _I, _F, _U64, _U64, _U32, _P, _P, _P, _P, _P, _P,
+                                           _SZ, _P]),
+    "libraspec_verify_round_staged_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I,
+                                                _P, _I, _I, _I, _I, _I, _I, _I, _F, _U64, _U64, _U32, _P, _P, _P, _P,
+                                                _P, _P, _SZ, _P]),
     "libraspec_kv_append": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _P, _SZ, _P]),
     "libraspec_kv_append_paged": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _P, _I, _I, _I, _I, _P, _SZ, _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
@@ -509,3 +515,74 @@ def libraspec_verify_round(draft_logits, draft_tokens, temperature, cost_table, 
         _ptr(outputs.n_accepted), _ptr(outputs.bonus_token), ws.ptr, ws.nbytes, _stream(stream))
     _check(rc, name)
     return outputs
+
+
+class StagedRound:
+    """Marshalled arguments of libraspec_verify_round_staged for fixed buffers: built (and checked)
+    once, then each call enqueues one round.
+
+    host_parts / dev_parts: three (pinned host, device) uint8 tensors, the drafter part, the layers
+    part and the target part; the typed inputs (draft_logits ... target_logits, each layer's Q,
+    kv_new) are device tensors inside dev_parts; layers: per layer {"Q", "Kc", "Vc"};
+    outputs: RoundOutputs; n_host / bonus_host: pinned int32 [B] tensors."""
+
+    def __init__(self, host_parts, dev_parts, kv_new, n_host, bonus_host, draft_logits, draft_tokens, temperature,
+                 cost_table, target_logits, layers, kv_len, outputs: "RoundOutputs", ws: Workspace,
+                 softmax_scale=None, copy_stream=None):
+        B, K, V = draft_logits.shape
+        bf16 = draft_logits.dtype == torch.bfloat16
+        ldt = torch.bfloat16 if bf16 else torch.float32
+        _req(draft_logits, ldt, "draft_logits")
+        _req(target_logits, ldt, "target_logits", (B, K + 1, V))
+        _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+        _req(temperature, torch.float32, "temperature", (B,))
+        _req(cost_table, torch.float32, "cost_table", (K + 1,))
+        _req(kv_len, torch.int32, "kv_len", (B,))
+        n_layers = len(layers)
+        Hq, D = layers[0]["Q"].shape[2], layers[0]["Q"].shape[3]
+        Hkv, S_cap = layers[0]["Kc"].shape[1], layers[0]["Kc"].shape[2]
+        for i, lay in enumerate(layers):
+            _req(lay["Q"], torch.bfloat16, "Q[%d]" % i, (B, K + 1, Hq, D))
+            _req(lay["Kc"], torch.bfloat16, "Kc[%d]" % i, (B, Hkv, S_cap, D))
+            _req(lay["Vc"], torch.bfloat16, "Vc[%d]" % i, (B, Hkv, S_cap, D))
+        _req(kv_new, torch.bfloat16, "kv_new", (n_layers, 2, B, Hkv, K + 1, D))
+        if len(host_parts) != 3 or len(dev_parts) != 3:
+            raise ValueError("three host and three device parts")
+        for h, d in zip(host_parts, dev_parts):
+            if not h.is_pinned() or h.numel() != d.numel() or not d.is_cuda:
+                raise ValueError("each part: a pinned host tensor and a device tensor of the same size")
+        if softmax_scale is None:
+            softmax_scale = D ** -0.5
+        self._keep = (host_parts, dev_parts, layers, outputs, n_host, bonus_host)
+        self._hp = (ctypes.c_void_p * 3)(*[h.data_ptr() for h in host_parts])
+        self._dp = (ctypes.c_void_p * 3)(*[d.data_ptr() for d in dev_parts])
+        self._nb = (ctypes.c_size_t * 3)(*[h.numel() * h.element_size() for h in host_parts])
+        self._copy = copy_stream if copy_stream is not None else torch.cuda.Stream(device=draft_logits.device)
+        self._qa = _ptr_array([l["Q"] for l in layers])
+        self._ka = _ptr_array([l["Kc"] for l in layers])
+        self._va = _ptr_array([l["Vc"] for l in layers])
+        self._oa = _ptr_array(outputs.O)
+        self._name = "libraspec_verify_round_staged_bf16" if bf16 else "libraspec_verify_round_staged"
+        self._fn = getattr(load(), self._name)
+        self._pre = (self._hp, self._dp, self._nb, ctypes.c_void_p(self._copy.cuda_stream), _ptr(kv_new),
+                     _ptr(n_host), _ptr(bonus_host), _ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature),
+                     _ptr(cost_table), _ptr(target_logits), self._qa, self._ka, self._va, self._oa, n_layers,
+                     _ptr(kv_len), B, K, V, Hq, Hkv, D, S_cap, float(softmax_scale))
+        self._post = (_ptr(outputs.conf), _ptr(outputs.dstat), _ptr(outputs.L), _ptr(outputs.n_accepted),
+                      _ptr(outputs.bonus_token), ws.ptr, ws.nbytes)
+
+    def __call__(self, seed: int, round_offset: int = 0, seq_offset: int = 0, stream=None) -> None:
+        rc = self._fn(*self._pre, int(seed) & (2**64 - 1), int(round_offset), int(seq_offset), *self._post,
+                      _stream(stream))
+        _check(rc, self._name)
+
+
+def libraspec_verify_round_staged(host_parts, dev_parts, kv_new, n_host, bonus_host, draft_logits, draft_tokens,
+                                  temperature, cost_table, target_logits, layers, kv_len, outputs, ws, seed: int,
+                                  round_offset: int = 0, seq_offset: int = 0, softmax_scale=None, copy_stream=None,
+                                  stream=None) -> None:
+    """One staged round (see StagedRound); returns after enqueuing."""
+    StagedRound(host_parts, dev_parts, kv_new, n_host, bonus_host, draft_logits, draft_tokens, temperature,
+                cost_table, target_logits, layers, kv_len, outputs, ws, softmax_scale, copy_stream)(
+        seed, round_offset, seq_offset, stream)
+

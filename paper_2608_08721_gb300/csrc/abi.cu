@@ -408,6 +408,51 @@ int libraspec_accept_tree_bf16(const uint16_t* target_logits, const int32_t* dra
                        n_accepted, last_node, bonus_token, workspace, ws_bytes, stream);
 }
 
+namespace {
+
+// Inputs of a staged round: three host parts copied in on copy_stream (the
+// drafter part, then the layers' queries and new keys/values, then the
+// target rows), each step of the round waiting only for its part; the block's
+// keys and values appended from kv_new; results read back into host memory.
+struct Staged {
+  const void* const* host_parts;
+  void* const* dev_parts;
+  const size_t* part_bytes;
+  cudaStream_t copy_stream;
+  const uint16_t* kv_new;
+  int32_t* n_host;
+  int32_t* bonus_host;
+  cudaEvent_t ev[4];
+};
+
+// Creates the events, orders copy_stream after the work already on `s` and
+// enqueues the three copies, recording one event after each.
+int staged_begin(Staged* st, cudaStream_t s) {
+  for (int i = 0; i < 4; ++i) st->ev[i] = nullptr;
+  for (int i = 0; i < 4; ++i)
+    if (cudaEventCreateWithFlags(&st->ev[i], cudaEventDisableTiming) != cudaSuccess) return LIBRASPEC_ECUDA;
+  cudaError_t e = cudaEventRecord(st->ev[3], s);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(st->copy_stream, st->ev[3], 0);
+  for (int i = 0; i < 3 && e == cudaSuccess; ++i) {
+    if (st->part_bytes[i] > 0)
+      e = cudaMemcpyAsync(st->dev_parts[i], st->host_parts[i], st->part_bytes[i], cudaMemcpyHostToDevice,
+                          st->copy_stream);
+    if (e == cudaSuccess) e = cudaEventRecord(st->ev[i], st->copy_stream);
+  }
+  return from_cuda(e);
+}
+
+void staged_end(Staged* st) {
+  for (int i = 0; i < 4; ++i)
+    if (st->ev[i]) cudaEventDestroy(st->ev[i]);  // released once the recorded work completes
+}
+
+int staged_wait(const Staged* st, int part, cudaStream_t s) {
+  return st ? from_cuda(cudaStreamWaitEvent(s, st->ev[part], 0)) : LIBRASPEC_OK;
+}
+
+}  // namespace
+
 extern "C++" {
 template <typename T>
 static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, const float* temperature,
@@ -417,7 +462,7 @@ static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, co
                            int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
                            uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
                            int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
-                           void* stream) {
+                           void* stream, Staged* st = nullptr) {
   if (!shapes_ok(B, K, V) || n_layers < 0) return LIBRASPEC_EINVAL;
   if (head_dim != 64 && head_dim != 128) return LIBRASPEC_EUNSUPPORTED;
   if (!attn_shapes_ok(B, K, Hq, Hkv, head_dim, S_cap)) return LIBRASPEC_EINVAL;
@@ -435,19 +480,91 @@ static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, co
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* ws = static_cast<char*>(workspace);
   int rc = LIBRASPEC_OK;
+  if (st && (rc = staged_begin(st, s)) != LIBRASPEC_OK) return rc;
+  if ((rc = staged_wait(st, 0, s)) != LIBRASPEC_OK) return rc;
   if (K > 0) {
     rc = confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream);
     if (rc != LIBRASPEC_OK) return rc;
   }
   rc = from_cuda(launch_select(conf, cost_table, B, K, L, ws, lay, s));
   if (rc != LIBRASPEC_OK) return rc;
+  if ((rc = staged_wait(st, 1, s)) != LIBRASPEC_OK) return rc;
+  if (st && (rc = from_cuda(launch_kv_append(st->kv_new, const_cast<uint16_t* const*>(Kc),
+                                             const_cast<uint16_t* const*>(Vc), n_layers, kv_len, nullptr, 0, 0, 0, B,
+                                             K + 1, Hkv, head_dim, S_cap, reinterpret_cast<int*>(ws + lay.status),
+                                             s))) != LIBRASPEC_OK)
+    return rc;
   rc = from_cuda(launch_verify_attn_layers(Q, Kc, Vc, n_layers, nullptr, kv_len, L, B, K, Hq, Hkv, head_dim, S_cap,
                                            softmax_scale, O, lse, ws, lay, s));
   if (rc != LIBRASPEC_OK) return rc;
-  return accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed, round_offset,
-                  seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
+  if ((rc = staged_wait(st, 2, s)) != LIBRASPEC_OK) return rc;
+  rc = accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed, round_offset,
+                seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
+  if (rc != LIBRASPEC_OK || !st) return rc;
+  cudaError_t e = cudaMemcpyAsync(st->n_host, n_accepted, sizeof(int32_t) * B, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(st->bonus_host, bonus_token, sizeof(int32_t) * B, cudaMemcpyDeviceToHost, s);
+  return from_cuda(e);
+}
+
+template <typename T>
+static int verify_round_staged_t(const void* const* host_parts, void* const* dev_parts, const size_t* part_bytes,
+                                 void* copy_stream, const uint16_t* kv_new, int32_t* n_accepted_host,
+                                 int32_t* bonus_host, const T* draft_logits, const int32_t* draft_tokens,
+                                 const float* temperature, const float* cost_table, const T* target_logits,
+                                 const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
+                                 uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V, int Hq,
+                                 int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                                 uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
+                                 int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                                 void* stream) {
+  if (!host_parts || !dev_parts || !part_bytes || !n_accepted_host || !bonus_host || !n_accepted || !bonus_token)
+    return LIBRASPEC_EINVAL;
+  for (int i = 0; i < 3; ++i)
+    if (part_bytes[i] > 0 && (!host_parts[i] || !dev_parts[i])) return LIBRASPEC_EINVAL;
+  if (n_layers > 0 && (!kv_new || !aligned(kv_new, 16))) return LIBRASPEC_EINVAL;
+  Staged st{host_parts, dev_parts, part_bytes, static_cast<cudaStream_t>(copy_stream), kv_new, n_accepted_host,
+            bonus_host, {}};
+  const int rc = verify_round_t(draft_logits, draft_tokens, temperature, cost_table, target_logits, Q, Kc, Vc, O,
+                                nullptr, n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed,
+                                round_offset, seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace,
+                                ws_bytes, stream, &st);
+  staged_end(&st);
+  return rc;
 }
 }  // extern "C++"
+
+int libraspec_verify_round_staged(const void* const* host_parts, void* const* dev_parts, const size_t* part_bytes,
+                                  void* copy_stream, const uint16_t* kv_new, int32_t* n_accepted_host,
+                                  int32_t* bonus_host, const float* draft_logits, const int32_t* draft_tokens,
+                                  const float* temperature, const float* cost_table, const float* target_logits,
+                                  const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
+                                  uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V,
+                                  int Hq, int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                                  uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
+                                  int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
+                                  void* stream) {
+  return verify_round_staged_t(host_parts, dev_parts, part_bytes, copy_stream, kv_new, n_accepted_host, bonus_host,
+                               draft_logits, draft_tokens, temperature, cost_table, target_logits, Q, Kc, Vc, O,
+                               n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed, round_offset,
+                               seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace, ws_bytes, stream);
+}
+
+int libraspec_verify_round_staged_bf16(const void* const* host_parts, void* const* dev_parts,
+                                       const size_t* part_bytes, void* copy_stream, const uint16_t* kv_new,
+                                       int32_t* n_accepted_host, int32_t* bonus_host, const uint16_t* draft_logits,
+                                       const int32_t* draft_tokens, const float* temperature,
+                                       const float* cost_table, const uint16_t* target_logits,
+                                       const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
+                                       uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V,
+                                       int Hq, int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
+                                       uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat,
+                                       int32_t* L, int32_t* n_accepted, int32_t* bonus_token, void* workspace,
+                                       size_t ws_bytes, void* stream) {
+  return verify_round_staged_t(host_parts, dev_parts, part_bytes, copy_stream, kv_new, n_accepted_host, bonus_host,
+                               draft_logits, draft_tokens, temperature, cost_table, target_logits, Q, Kc, Vc, O,
+                               n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed, round_offset,
+                               seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace, ws_bytes, stream);
+}
 
 int libraspec_verify_round(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
                            const float* cost_table, const float* target_logits, const uint16_t* const* Q,
