@@ -65,8 +65,9 @@ def _load():
     lib.oracle_accept.argtypes = [P, P, P, P, P, i32, i32, i32, u64, u64, u32, P, P, P]
     lib.oracle_accept_tree_greedy.argtypes = [P, P, P, P, i32, i32, i32, P, P, P]
     lib.oracle_accept_tree.argtypes = [P, P, P, P, P, i32, i32, i32, u64, u64, u32, P, P, P, P]
+    lib.oracle_lm_head_stats.argtypes = [P, P, P, i32, P, i32, i32, i32, P, P, P, P, P]
     for name in ("oracle_confidence", "oracle_select_lengths", "oracle_select_iterate", "oracle_select_alpha",
-                 "oracle_gather_pages", "oracle_verify_attn_tree", "oracle_accept_tree_greedy", "oracle_accept_tree",
+                 "oracle_gather_pages", "oracle_verify_attn_tree", "oracle_accept_tree_greedy", "oracle_accept_tree", "oracle_lm_head_stats",
                  "oracle_verify_attn", "oracle_accept"):
         getattr(lib, name).restype = i32
     _lib = lib
@@ -276,6 +277,23 @@ def accept_tree(target_logits, draft_tokens, parent, L, temperature, seed, round
                                       int(seed) & (2**64 - 1), int(round_offset), int(seq_offset), _ptr(n),
                                       _ptr(last), _ptr(bonus), _ptr(flag)), "oracle_accept_tree")
     return n, last, bonus, flag
+
+
+def lm_head_stats(H, W, temperature=None, rows_per_seq=1, tokens=None):
+    """Row statistics of logits H @ W^T (bf16 inputs, binary64 sums): row_max, row_Z (at the row's
+    temperature, 1 where 0), row_argmax, token_prob (0 where token < 0 or tokens is None), flag."""
+    Hb, Wb = _as_bf16_bits(H), _as_bf16_bits(W)
+    M, Dm = Hb.shape
+    V, Dm2 = Wb.shape
+    if Dm2 != Dm:
+        raise OracleError("H and W disagree on the model dimension")
+    T = None if temperature is None else _c(temperature, np.float32)
+    tok = None if tokens is None else _c(tokens, np.int32)
+    mx, Z, tp = (np.zeros(M, np.float64) for _ in range(3))
+    arg, flag = np.zeros(M, np.int32), np.zeros(M, np.int32)
+    _check(_load().oracle_lm_head_stats(_ptr(Hb), _ptr(Wb), _ptr(T), int(rows_per_seq), _ptr(tok), M, V, Dm,
+                                        _ptr(mx), _ptr(Z), _ptr(arg), _ptr(tp), _ptr(flag)), "oracle_lm_head_stats")
+    return mx, Z, arg, tp, flag
 
 
 def accept(target_logits, draft_logits, draft_tokens, L, temperature, seed, round_offset=0,

@@ -29,6 +29,9 @@
  *                          of Sec. 2, e.g. DDTree): ancestor-masked
  *                          attention, the greedy longest accepted path and
  *                          its sampling counterpart.
+ *   oracle_lm_head_stats   confidence / acceptance row statistics from an LM
+ *                          head's hidden states and weights (logits
+ *                          never stored).
  *   oracle_verify_attn     block-causal GQA attention of the d+1 verified
  *                          positions against the target KV cache (Sec. 3.1:
  *                          the target scores all drafted positions in one
@@ -674,6 +677,64 @@ static race_result exp_race(const double* w, const double* rel, int V, uint64_t 
     }
   }
   return res;
+}
+
+/* ------------------------------------------------------------------ */
+/* Row statistics straight from an LM head (the confidence of Assumption */
+/* 1 and the acceptance row statistics of Sec. 3.1, with the logits     */
+/* x[r, v] = sum_k H[r, k] W[v, k] never stored): H [M, Dm] and W [V, Dm]  */
+/* bf16 bit patterns; T_r = temperature[r / rows_per_seq] (1 when 0 or   */
+/* when temperature is NULL). Per row: max m, lowest-index argmax, Z =   */
+/* sum_v exp((x_v - m) / T_r), and for token[r] >= 0 the probability     */
+/* exp((x_tok - m) / T_r) / Z. Logits are sums of exact bf16 products in */
+/* binary64. flag[r] = 1 when the two largest logits lie within          */
+/* 2^-16 (a_1 + a_2), a_v = sum_k |H[r,k] W[v,k]|: a binary32            */
+/* accumulation may order them differently.                              */
+/* ------------------------------------------------------------------ */
+int oracle_lm_head_stats(const uint16_t* H, const uint16_t* W, const float* temperature, int rows_per_seq,
+                         const int32_t* token, int M, int V, int Dm, double* row_max, double* row_Z,
+                         int32_t* row_arg, double* token_prob, int32_t* flag) {
+  if (M < 0 || V < 1 || Dm < 1 || !H || !W || rows_per_seq < 1) return ORACLE_EINVAL;
+  for (int r = 0; r < M; ++r)
+    if (token && token[r] >= V) return ORACLE_EINVAL;
+#pragma omp parallel
+  {
+    double* x = (double*)malloc(sizeof(double) * (size_t)V);
+    double* a = (double*)malloc(sizeof(double) * (size_t)V);
+    double* h = (double*)malloc(sizeof(double) * (size_t)Dm);
+#pragma omp for schedule(dynamic, 1)
+    for (int r = 0; r < M; ++r) {
+      for (int k = 0; k < Dm; ++k) h[k] = bf16_to_double(H[(size_t)r * Dm + k]);
+      for (int v = 0; v < V; ++v) {
+        double s = 0.0, sa = 0.0;
+        const uint16_t* w = W + (size_t)v * Dm;
+        for (int k = 0; k < Dm; ++k) {
+          const double p = h[k] * bf16_to_double(w[k]);
+          s += p;
+          sa += fabs(p);
+        }
+        x[v] = s;
+        a[v] = sa;
+      }
+      double T = temperature ? (double)temperature[r / rows_per_seq] : 1.0;
+      if (!(T > 0.0)) T = 1.0;
+      int arg = 0, second = -1;
+      for (int v = 1; v < V; ++v) {
+        if (x[v] > x[arg]) { second = arg; arg = v; }
+        else if (second < 0 || x[v] > x[second]) second = v;
+      }
+      const double m = x[arg];
+      double Z = 0.0;
+      for (int v = 0; v < V; ++v) Z += exp((x[v] - m) / T);
+      if (row_max) row_max[r] = m;
+      if (row_Z) row_Z[r] = Z;
+      if (row_arg) row_arg[r] = arg;
+      if (token_prob) token_prob[r] = (token && token[r] >= 0) ? exp((x[token[r]] - m) / T) / Z : 0.0;
+      if (flag) flag[r] = (second >= 0 && x[arg] - x[second] <= ldexp(a[arg] + a[second], -16)) ? 1 : 0;
+    }
+    free(x); free(a); free(h);
+  }
+  return ORACLE_OK;
 }
 
 /* ------------------------------------------------------------------ */
