@@ -360,6 +360,33 @@ int libraspec_accept_tree_bf16(const uint16_t* target_logits, const int32_t* dra
                                int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * Row statistics straight from the LM head (steps 1 and 4 without stored
+ * logits; the confidence of Assumption 1, the acceptance row statistics of
+ * Sec. 3.1): the logits x[r, v] = sum_k H[r, k] W[v, k] are accumulated on
+ * the tensor cores and reduced in the GEMM's epilogue.
+ *   H [M, Dm] bf16 hidden states (row r = sequence r / rows_per_seq), W [V, Dm]
+ *   bf16 head weights, Dm a multiple of 64 (else LIBRASPEC_EUNSUPPORTED),
+ *   both 16-byte aligned; temperature [M / rows_per_seq] f32 or NULL (T = 1;
+ *   a row at T = 0 takes T = 1, like libraspec_confidence); tokens [M] i32 or
+ *   NULL (-1: no token).
+ *   row_stat [M, 2] f32 out (m = max_v x, Z = sum_v exp((x_v - m) / T)) or
+ *   NULL; row_argmax [M] i32 out (lowest index on ties) or NULL;
+ *   token_prob [M] f32 out = exp((x_tok - m) / T) / Z (0 for token -1) or
+ *   NULL (needs tokens).
+ * With H the drafter rows (rows_per_seq = K) and tokens the drafted tokens,
+ * token_prob and row_stat are libraspec_confidence's conf and dstat. Logits
+ * are binary32 accumulations of exact bf16 products; partials merge in
+ * binary64. A token outside [-1, V) sets LIBRASPEC_ST_BAD_TOKEN (its
+ * probability NaN). Reads W once per 128-row tile of H.
+ * Workspace: libraspec_lm_head_workspace_size(M, V) bytes (status word and
+ * the per-tile partials).
+ */
+size_t libraspec_lm_head_workspace_size(int M, int V);
+int libraspec_lm_head_stats(const uint16_t* H, const uint16_t* W, const float* temperature, int rows_per_seq,
+                            const int32_t* tokens, int M, int V, int Dm, float* row_stat, int32_t* row_argmax,
+                            float* token_prob, void* workspace, size_t ws_bytes, void* stream);
+
+/*
  * Appending the verified block's keys and values to the caches (the target
  * computes them for the block positions, Sec. 3.1; the verify attention
  * reads them at rows kv_len[b] .. kv_len[b] + T - 1):

@@ -55,6 +55,8 @@ SIGNATURES = {
     "libraspec_verify_round_staged_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I,
                                                 _P, _I, _I, _I, _I, _I, _I, _I, _F, _U64, _U64, _U32, _P, _P, _P, _P,
                                                 _P, _P, _SZ, _P]),
+    "libraspec_lm_head_workspace_size": (_SZ, [_I, _I]),
+    "libraspec_lm_head_stats": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _P, _SZ, _P]),
     "libraspec_kv_append": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _P, _SZ, _P]),
     "libraspec_kv_append_paged": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _P, _I, _I, _I, _I, _P, _SZ, _P]),
     "libraspec_accept": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _SZ, _P]),
@@ -455,6 +457,46 @@ def libraspec_kv_append(kv_new, caches, kv_len, ws: Workspace, block_table=None,
                                           block_table.shape[1], page_size, n_pages, _ptr(kv_len), B, T, Hkv, d,
                                           ws.ptr, ws.nbytes, _stream(stream))
     _check(rc, "libraspec_kv_append_paged")
+
+
+class LmHeadWorkspace:
+    """Device scratch of libraspec_lm_head_stats for M rows and a vocabulary of V."""
+
+    def __init__(self, M, V, device=None):
+        self.nbytes = int(load().libraspec_lm_head_workspace_size(M, V))
+        if self.nbytes == 0:
+            raise ValueError("invalid LM-head workspace shapes")
+        dev = torch.device("cuda") if device is None else torch.device(device)
+        self.buf = torch.zeros(self.nbytes, dtype=torch.uint8, device=dev)
+
+    @property
+    def ptr(self) -> int:
+        return self.buf.data_ptr()
+
+
+def libraspec_lm_head_stats(H, W, ws: "LmHeadWorkspace", temperature=None, rows_per_seq: int = 1, tokens=None,
+                            row_stat=None, row_argmax=None, token_prob=None, stream=None):
+    """Row statistics of H @ W^T without storing it: (row_stat [M,2], row_argmax [M], token_prob [M] or None)."""
+    M, Dm = H.shape
+    V = W.shape[0]
+    _req(H, torch.bfloat16, "H")
+    _req(W, torch.bfloat16, "W", (V, Dm))
+    if temperature is not None:
+        _req(temperature, torch.float32, "temperature")
+        if temperature.numel() * rows_per_seq < M:
+            raise ValueError("temperature needs one entry per sequence of rows_per_seq rows")
+    if tokens is not None:
+        _req(tokens, torch.int32, "tokens", (M,))
+    dev = H.device
+    row_stat = torch.empty((M, 2), dtype=torch.float32, device=dev) if row_stat is None else row_stat
+    row_argmax = torch.empty((M,), dtype=torch.int32, device=dev) if row_argmax is None else row_argmax
+    if tokens is not None and token_prob is None:
+        token_prob = torch.empty((M,), dtype=torch.float32, device=dev)
+    rc = load().libraspec_lm_head_stats(_ptr(H), _ptr(W), _ptr(temperature), int(rows_per_seq), _ptr(tokens), M, V,
+                                        Dm, _ptr(row_stat), _ptr(row_argmax), _ptr(token_prob), ws.ptr, ws.nbytes,
+                                        _stream(stream))
+    _check(rc, "libraspec_lm_head_stats")
+    return row_stat, row_argmax, token_prob
 
 
 def _ptr_array(tensors: Sequence[Optional[torch.Tensor]]):

@@ -16,8 +16,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libraspec.so")
-SOURCES = ["conf_select.cu", "accept.cu", "attn.cu", "abi.cu", "noalloc.cu", "kv.cu"]
-HEADERS = ["common.cuh", "rowpass.cuh"]
+SOURCES = ["conf_select.cu", "accept.cu", "attn.cu", "abi.cu", "noalloc.cu", "kv.cu", "lmhead.cu"]
+HEADERS = ["common.cuh", "rowpass.cuh", "tc.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

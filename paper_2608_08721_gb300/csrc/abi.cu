@@ -23,6 +23,9 @@ cudaError_t launch_verify_attn_paged_layers(const uint16_t* const*, const uint16
 cudaError_t launch_verify_attn_layers(const uint16_t* const*, const uint16_t* const*, const uint16_t* const*, int,
                                       const int32_t*, const int32_t*, const int32_t*, int, int, int, int, int, int,
                                       float, uint16_t* const*, float* const*, char*, const WsLayout&, cudaStream_t);
+size_t lm_head_workspace_bytes(int M, int V);
+cudaError_t launch_lm_head_stats(const uint16_t*, const uint16_t*, const float*, int, const int32_t*, int, int, int,
+                                 float*, int32_t*, float*, char*, cudaStream_t);
 cudaError_t launch_kv_append(const uint16_t*, uint16_t* const*, uint16_t* const*, int, const int32_t*,
                              const int32_t*, int, int, int, int, int, int, int, int, int*, cudaStream_t);
 template <typename T>
@@ -338,6 +341,25 @@ int kv_append_checked(const uint16_t* kv_new, uint16_t* const* Kc, uint16_t* con
 }
 
 }  // namespace
+
+size_t libraspec_lm_head_workspace_size(int M, int V) {
+  if (M < 0 || M > (1 << 20) || V < 1) return 0;
+  return lm_head_workspace_bytes(M, V);
+}
+
+int libraspec_lm_head_stats(const uint16_t* H, const uint16_t* W, const float* temperature, int rows_per_seq,
+                            const int32_t* tokens, int M, int V, int Dm, float* row_stat, int32_t* row_argmax,
+                            float* token_prob, void* workspace, size_t ws_bytes, void* stream) {
+  if (M < 0 || M > (1 << 20) || V < 1 || rows_per_seq < 1) return LIBRASPEC_EINVAL;
+  if (Dm < 64 || Dm % 64 != 0 || Dm > 65536) return LIBRASPEC_EUNSUPPORTED;
+  if (M == 0) return LIBRASPEC_OK;
+  if (!H || !W || !aligned(H, 16) || !aligned(W, 16)) return LIBRASPEC_EINVAL;
+  if (token_prob && !tokens) return LIBRASPEC_EINVAL;
+  if (!workspace || !aligned(workspace, 256) || ws_bytes < lm_head_workspace_bytes(M, V)) return LIBRASPEC_EINVAL;
+  return from_cuda(launch_lm_head_stats(H, W, temperature, rows_per_seq, tokens, M, V, Dm, row_stat, row_argmax,
+                                        token_prob, static_cast<char*>(workspace),
+                                        static_cast<cudaStream_t>(stream)));
+}
 
 int libraspec_kv_append(const uint16_t* kv_new, uint16_t* const* Kc, uint16_t* const* Vc, int n_layers,
                         const int32_t* kv_len, int B, int T, int Hkv, int head_dim, int S_cap, void* workspace,
