@@ -11,6 +11,8 @@ Variants of the round (the default is the chain draft on dense caches):
   --selector alpha   Algorithm 1's alpha-mode length search instead of Thm. 4's scan;
   --logits bf16      bf16 drafter and target logits;
   --page-size P      KV caches in pages of P keys behind block tables;
+  --lm-head          the confidence from the drafter's hidden states and the LM head
+                     (the statistics in the GEMM's epilogue, no drafter logits);
   --tree N           a DDTree-shaped draft tree of N nodes: tree-masked attention and the
                      tree walk (greedy or drawing, per the workload's temperatures) replace
                      the chain's attention and acceptance.
@@ -60,6 +62,9 @@ def parse():
                    help="verify a DDTree-shaped draft tree of this many nodes (depth <= K) instead of the chain")
     p.add_argument("--page-size", type=int, default=0,
                    help="keep the KV cache in pages of this many keys behind block tables (0: dense)")
+    p.add_argument("--lm-head", action="store_true",
+                   help="compute the confidence from the drafter's hidden states and the LM head (fused GEMM "
+                        "epilogue, logits never stored) instead of from drafter logits")
     p.add_argument("--block-size", type=int, default=0,
                    help="first drafted block of the alpha-mode search (0: 2/3 of K, as 16 of d_max 24)")
     return p.parse_args()
@@ -375,9 +380,21 @@ def run_ours(args, rank, world, local_rank):
     block_size = args.block_size if args.block_size > 0 else max(1, (2 * w.K) // 3)
     n_blocks = torch.empty((w.B,), dtype=torch.int32, device=dev)
 
+    head = None
+    if args.lm_head:
+        head = workloads.lm_head(w, w.B * w.K, device=dev)
+        head["ws"] = lr.LmHeadWorkspace(w.B * w.K, w.V, device=dev)
+        head["tokens"] = inp["draft_tokens"].reshape(-1).contiguous()
+        head["argmax"] = torch.empty((w.B * w.K,), dtype=torch.int32, device=dev)
+
     def seg_select():
-        lr.libraspec_confidence(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], ws, conf=conf,
-                                dstat=dstat)
+        if head is not None:
+            lr.libraspec_lm_head_stats(head["H"], head["W"], head["ws"], temperature=inp["temperature"],
+                                       rows_per_seq=w.K, tokens=head["tokens"], row_stat=dstat.view(-1, 2),
+                                       row_argmax=head["argmax"], token_prob=conf.view(-1))
+        else:
+            lr.libraspec_confidence(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], ws, conf=conf,
+                                    dstat=dstat)
         if args.selector == "alpha":
             lr.libraspec_select_alpha(conf, block_size, args.alpha, L=L, n_blocks=n_blocks)
         else:
@@ -404,7 +421,7 @@ def run_ours(args, rank, world, local_rank):
                             bonus_token=bonus)
 
     def device_status():
-        st = lr.libraspec_get_status(ws)
+        st = lr.libraspec_get_status(ws) | (lr.libraspec_get_status(head["ws"]) if head is not None else 0)
         return st | (lr.libraspec_get_status(tree["ws"]) if N else 0)
 
     # eager warm-up (also configures kernels), then capture three graphs
@@ -422,7 +439,9 @@ def run_ours(args, rank, world, local_rank):
         graphs.append(gr)
     stream = torch.cuda.current_stream()
 
-    def step(ev_a=None, ev_b=None):
+    def step(ev_a=None, ev_b=None, ev_0=None):
+        if ev_0 is not None:
+            ev_0.record(stream)
         graphs[0].replay()
         if ev_a is not None:
             ev_a.record(stream)
@@ -444,6 +463,7 @@ def run_ours(args, rank, world, local_rank):
         torch.cuda.synchronize()
         per = (time.perf_counter() - t0) / 20
         K_steps = int(min(20000, max(50, 2.0 / max(per, 1e-6))))
+    ev_0 = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
     ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
     ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -452,12 +472,13 @@ def run_ours(args, rank, world, local_rank):
     with ClockSampler(physical_gpu(local_rank)) as clocks:
         start.record(stream)
         for i in range(K_steps):
-            step(ev_a[i], ev_b[i])
+            step(ev_a[i], ev_b[i], ev_0[i])
         end.record(stream)
         torch.cuda.synchronize()
     pdist.barrier()
     elapsed_ms = start.elapsed_time(end)
     attn_ms = sum(a.elapsed_time(b) for a, b in zip(ev_a, ev_b))
+    select_ms = sum(a.elapsed_time(b) for a, b in zip(ev_0, ev_a))
     elapsed_max = pdist.max_over_ranks(elapsed_ms, device=dev)
     if device_status() != 0:
         raise RuntimeError("device status set during the timed steps")
@@ -503,7 +524,7 @@ def run_ours(args, rank, world, local_rank):
         e2e = run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset)
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and not P:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not P and not args.lm_head:
         # bf16 logits widen exactly to f32 for the oracle
         host = {k: (v.float() if v.dtype == torch.bfloat16 else v).cpu().numpy() for k, v in inp.items()}
         host["cost_table"] = workloads.cost_table(w, kv)
@@ -516,12 +537,21 @@ def run_ours(args, rank, world, local_rank):
             us, cores, sample = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds)
         cpu = {"value": round(us, 1), "unit": "us", "cores": cores, "kind": "oracle", "sample": sample}
 
+    lm = None
+    if head is not None:
+        # the conf+select graph is the head's GEMM plus a selection of a few microseconds
+        head_bytes = (w.V + w.B * w.K) * w.hidden * 2
+        lm_s = select_ms / 1000.0 / K_steps
+        lm = {"kernel": "lm_head_stats (tcgen05 GEMM, statistics in the epilogue)", "us": round(lm_s * 1e6, 3),
+              "bytes": head_bytes, "GBps": round(head_bytes / lm_s / 1e9, 1),
+              "frac_of_measured_hbm": round(head_bytes / lm_s / 1e9 / hbm_peak, 4),
+              "note": "time of the confidence+selection graph; the head's weights dominate its bytes"}
     if rank != 0:
         return
     clk = clocks.summary()
     value = elapsed_max * 1000.0 / (K_steps * world)
     # attention (+ the tree-mask kernel per launch), conf, select, 2 accept
-    launches = K_steps * (attn_launches * (2 if N else 1) + 4)
+    launches = K_steps * (attn_launches * (2 if N else 1) + 4 + (1 if args.lm_head else 0))
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "us", "n_gpus": world, "steps": K_steps,
         "warmup": max(3, args.warmup), "ms_per_step": round(elapsed_max / K_steps, 6), "higher_is_better": False,
@@ -536,6 +566,8 @@ def run_ours(args, rank, world, local_rank):
                    "draft": ("DDTree-shaped tree of %d nodes (best-first, depth <= %d), tree walk" % (N, w.K)
                              if N else "chain"),
                    "kv_cache": "paged, %d keys per page" % P if P else "dense",
+                   "confidence": ("from hidden states [%d, %d] and a %d x %d LM head (fused epilogue)" %
+                                  (w.B * w.K, w.hidden, w.V, w.hidden) if args.lm_head else "from drafter logits"),
                    "parallelism": "dp%d (independent sequences)" % world,
                    "l2": "no flush: %.0f MB of distinct inputs per step > 129 MB L2" % (by["total"] / 1e6),
                    "timing": "3 CUDA graphs per step (conf+select | attention layers | accept), events between"},
@@ -543,6 +575,9 @@ def run_ours(args, rank, world, local_rank):
         "hbm_frac_of_measured": round(by["total"] / (us_per_round * 1e-6) / 1e9 / hbm_peak, 4),
         "hbm_frac_of_nominal_8tbs": round(by["total"] / (us_per_round * 1e-6) / 1e9 / NOMINAL_HBM_GBS, 4),
         "roofline": roof,
+        "lm_head": lm,
+        "segments_us": {"conf_select": round(select_ms * 1000.0 / K_steps, 3),
+                        "attention": round(attn_ms * 1000.0 / K_steps, 3)},
         "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
                    "samples": clk["samples"]},
         "gpu_launches": launches,

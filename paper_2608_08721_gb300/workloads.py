@@ -39,6 +39,7 @@ class Workload:
     philox_seed: int
     data_seed: int
     resident_layers: int = 0   # >0: distinct KV buffers kept on the device (rest reuse them)
+    hidden: int = 4096         # model dimension of the LM head (Llama-3-8B / 70B: 4096 / 8192, Qwen2.5-7B 3584)
 
     def scaled(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
@@ -56,11 +57,11 @@ WORKLOADS = {
     "8b": Workload("8b", B=1, K=16, V=128256, Hq=32, Hkv=8, d=128, n_layers=32,
                    kv=("const", 4096), temperature=("const", 0.0), target=("normal_peak", 6.0, 12.0),
                    draft_noise=("const", 1.5), cost=("poly", 1.0, 0.01, 0.0),
-                   philox_seed=1, data_seed=1),
+                   philox_seed=1, data_seed=1, hidden=4096),
     "sampling": Workload("sampling", B=16, K=16, V=152064, Hq=28, Hkv=4, d=128, n_layers=1,
                          kv=("uniform", 1024, 8192), temperature=("const", 1.0), target=("normal", 4.0),
                          draft_noise=("uniform", 0.5, 3.0), cost=("poly", 1.0, 0.015, 0.0005),
-                         philox_seed=1234, data_seed=2),
+                         philox_seed=1234, data_seed=2, hidden=3584),
     "ragged": Workload("ragged", B=64, K=32, V=128256, Hq=32, Hkv=8, d=128, n_layers=1,
                        kv=("loguniform", 512, 32768), temperature=("alternate", 0.0, 0.8),
                        target=("normal_sigma_u", 1.0, 8.0), draft_noise=("const", 1.0),
@@ -68,7 +69,7 @@ WORKLOADS = {
     "70b": Workload("70b", B=8, K=16, V=128256, Hq=64, Hkv=8, d=128, n_layers=80,
                     kv=("const", 131072), temperature=("const", 0.7), target=("normal", 4.0),
                     draft_noise=("const", 1.0), cost=("poly", 1.0, 0.008, 0.0),
-                    philox_seed=4, data_seed=4, resident_layers=16),
+                    philox_seed=4, data_seed=4, resident_layers=16, hidden=8192),
 }
 
 
@@ -327,6 +328,16 @@ def tree_logits(w: Workload, parent: np.ndarray, L, device="cpu", p_follow: floa
     idx = torch.from_numpy(peak).to(device)
     target.scatter_add_(2, idx[:, :, None], torch.full((B, N1, 1), 12.0, device=device))
     return {"draft_tokens": torch.from_numpy(tok).to(device), "target_logits": target.contiguous()}
+
+
+def lm_head(w: Workload, rows: int, device="cpu", sigma: float = 4.0) -> dict:
+    """Hidden states H [rows, hidden] ~ N(0, 1) and LM-head weights W [V, hidden] ~ N(0, sigma^2 / hidden),
+    bf16, so that logits are ~ N(0, sigma^2)."""
+    g = torch.Generator(device=device)
+    g.manual_seed(w.data_seed * 7919 + 555)
+    H = _randn((rows, w.hidden), g, device).to(torch.bfloat16)
+    W = (_randn((w.V, w.hidden), g, device) * (sigma / w.hidden ** 0.5)).to(torch.bfloat16)
+    return {"H": H, "W": W}
 
 
 def reference_inputs_summary(w: Workload) -> List[str]:
