@@ -392,6 +392,10 @@ def run_ours(args, rank, world, local_rank):
             lr.libraspec_lm_head_stats(head["H"], head["W"], head["ws"], temperature=inp["temperature"],
                                        rows_per_seq=w.K, tokens=head["tokens"], row_stat=dstat.view(-1, 2),
                                        row_argmax=head["argmax"], token_prob=conf.view(-1))
+        elif args.selector == "gain":  # confidence and Thm. 4's selection in one launch
+            lr.libraspec_confidence_select(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], cost, ws,
+                                           conf=conf, dstat=dstat, L=L)
+            return
         else:
             lr.libraspec_confidence(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], ws, conf=conf,
                                     dstat=dstat)
@@ -430,8 +434,15 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     if device_status() != 0:
         raise RuntimeError("device status set during warm-up")
-    graphs = []
+    # the timed step: the whole round in one CUDA graph; the same round split
+    # into three graphs (events between) times the segments in a second pass
     side = torch.cuda.Stream(device=dev)
+    round_graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(round_graph, stream=side):
+        seg_select()
+        seg_attn()
+        seg_accept()
+    graphs = []
     for seg in (seg_select, seg_attn, seg_accept):
         gr = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gr, stream=side):
@@ -439,19 +450,21 @@ def run_ours(args, rank, world, local_rank):
         graphs.append(gr)
     stream = torch.cuda.current_stream()
 
-    def step(ev_a=None, ev_b=None, ev_0=None):
-        if ev_0 is not None:
-            ev_0.record(stream)
+    def step():
+        round_graph.replay()
+
+    def step_split(ev_a, ev_b, ev_0):
+        ev_0.record(stream)
         graphs[0].replay()
-        if ev_a is not None:
-            ev_a.record(stream)
+        ev_a.record(stream)
         graphs[1].replay()
-        if ev_b is not None:
-            ev_b.record(stream)
+        ev_b.record(stream)
         graphs[2].replay()
 
     for _ in range(max(3, args.warmup)):
         step()
+        for gr in graphs:
+            gr.replay()
     torch.cuda.synchronize()
     # steps: enough for ~2 s of timed work unless given
     if args.steps > 0:
@@ -472,8 +485,13 @@ def run_ours(args, rank, world, local_rank):
     with ClockSampler(physical_gpu(local_rank)) as clocks:
         start.record(stream)
         for i in range(K_steps):
-            step(ev_a[i], ev_b[i], ev_0[i])
+            step()
         end.record(stream)
+        torch.cuda.synchronize()
+        pdist.barrier()
+        # second pass: the same K rounds as three graphs, for the kernels' launch durations
+        for i in range(K_steps):
+            step_split(ev_a[i], ev_b[i], ev_0[i])
         torch.cuda.synchronize()
     pdist.barrier()
     elapsed_ms = start.elapsed_time(end)
@@ -550,8 +568,10 @@ def run_ours(args, rank, world, local_rank):
         return
     clk = clocks.summary()
     value = elapsed_max * 1000.0 / (K_steps * world)
-    # attention (+ the tree-mask kernel per launch), conf, select, 2 accept
-    launches = K_steps * (attn_launches * (2 if N else 1) + 4 + (1 if args.lm_head else 0))
+    # attention (+ the tree-mask kernel per launch); confidence and selection (one fused launch for the
+    # Thm. 4 selector, the LM head's GEMM + merge + selection, or confidence + selection); 2 for acceptance
+    conf_launches = 3 if args.lm_head else (1 if args.selector == "gain" else 2)
+    launches = K_steps * (attn_launches * (2 if N else 1) + conf_launches + 2)
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "us", "n_gpus": world, "steps": K_steps,
         "warmup": max(3, args.warmup), "ms_per_step": round(elapsed_max / K_steps, 6), "higher_is_better": False,
@@ -570,7 +590,9 @@ def run_ours(args, rank, world, local_rank):
                                   (w.B * w.K, w.hidden, w.V, w.hidden) if args.lm_head else "from drafter logits"),
                    "parallelism": "dp%d (independent sequences)" % world,
                    "l2": "no flush: %.0f MB of distinct inputs per step > 129 MB L2" % (by["total"] / 1e6),
-                   "timing": "3 CUDA graphs per step (conf+select | attention layers | accept), events between"},
+                   "timing": ("value: K rounds, each one CUDA graph replay, events around the loop; segments and "
+                              "roofline: a second pass of the same K rounds as three graphs (conf+select | "
+                              "attention layers | accept) with events between")},
         "hbm_tbs": round(by["total"] / (us_per_round * 1e-6) / 1e12, 3),
         "hbm_frac_of_measured": round(by["total"] / (us_per_round * 1e-6) / 1e9 / hbm_peak, 4),
         "hbm_frac_of_nominal_8tbs": round(by["total"] / (us_per_round * 1e-6) / 1e9 / NOMINAL_HBM_GBS, 4),

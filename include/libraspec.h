@@ -151,6 +151,20 @@ int libraspec_confidence_noalloc(const float* draft_logits, const int32_t* draft
                                  int B, int K, int V, float* conf, float* dstat, int32_t* status, void* stream);
 
 /*
+ * Steps 1 and 2 in one launch: libraspec_confidence, and as soon as the
+ * last of a sequence's K rows is done, that CTA selects the sequence's
+ * length exactly as libraspec_select_lengths does (same L, same status
+ * bits). Arguments as the two calls; K = 0 only selects.
+ */
+int libraspec_confidence_select(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                                const float* cost_table, int B, int K, int V, float* conf, float* dstat, int32_t* L,
+                                void* workspace, size_t ws_bytes, void* stream);
+int libraspec_confidence_select_bf16(const uint16_t* draft_logits, const int32_t* draft_tokens,
+                                     const float* temperature, const float* cost_table, int B, int K, int V,
+                                     float* conf, float* dstat, int32_t* L, void* workspace, size_t ws_bytes,
+                                     void* stream);
+
+/*
  * Step 2 — LibraSpec length selection (paper Thm. 4, from Thm. 1's
  * ratio comparison; Eq. 2 with negligible drafting cost).
  *

@@ -34,6 +34,8 @@ SIGNATURES = {
     "libraspec_confidence": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "libraspec_confidence_bf16": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "libraspec_confidence_noalloc": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P]),
+    "libraspec_confidence_select": (_I, [_P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _SZ, _P]),
+    "libraspec_confidence_select_bf16": (_I, [_P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _SZ, _P]),
     "libraspec_select_lengths": (_I, [_P, _P, _I, _I, _P, _P, _SZ, _P]),
     "libraspec_select_alpha": (_I, [_P, _I, _I, _I, _F, _P, _P, _P]),
     "libraspec_verify_attn": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _SZ, _P]),
@@ -203,6 +205,26 @@ def libraspec_confidence_noalloc(draft_logits, draft_tokens, temperature, conf, 
     rc = load().libraspec_confidence_noalloc(_ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature), B, K, V,
                                              _ptr(conf), _ptr(dstat), _ptr(status), _stream(stream))
     _check(rc, "libraspec_confidence_noalloc")
+
+
+def libraspec_confidence_select(draft_logits, draft_tokens, temperature, cost_table, ws: Workspace, conf=None,
+                                dstat=None, L=None, stream=None):
+    """Confidence and the Thm. 4 selection in one launch: (conf [B,K], dstat [B,K,2], L [B])."""
+    B, K, V = draft_logits.shape
+    bf16 = draft_logits.dtype == torch.bfloat16
+    _req(draft_logits, torch.bfloat16 if bf16 else torch.float32, "draft_logits")
+    _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+    _req(temperature, torch.float32, "temperature", (B,))
+    _req(cost_table, torch.float32, "cost_table", (K + 1,))
+    dev = draft_logits.device
+    conf = torch.empty((B, K), dtype=torch.float32, device=dev) if conf is None else conf
+    dstat = torch.empty((B, K, 2), dtype=torch.float32, device=dev) if dstat is None else dstat
+    L = torch.empty((B,), dtype=torch.int32, device=dev) if L is None else L
+    name = "libraspec_confidence_select_bf16" if bf16 else "libraspec_confidence_select"
+    rc = getattr(load(), name)(_ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature), _ptr(cost_table), B, K, V,
+                               _ptr(conf), _ptr(dstat), _ptr(L), ws.ptr, ws.nbytes, _stream(stream))
+    _check(rc, name)
+    return conf, dstat, L
 
 
 def libraspec_select_lengths(conf, cost_table, ws: Workspace, L=None, stream=None) -> torch.Tensor:

@@ -10,7 +10,7 @@ namespace libraspec {
 
 template <typename T>
 cudaError_t launch_confidence(const T*, const int32_t*, const float*, int, int, int, float*, float*, char*,
-                              const WsLayout&, cudaStream_t);
+                              const WsLayout&, cudaStream_t, const float*, int32_t*);
 cudaError_t launch_select(const float*, const float*, int, int, int32_t*, char*, const WsLayout&, cudaStream_t);
 cudaError_t launch_select_alpha(const float*, int, int, int, double, int32_t*, int32_t*, cudaStream_t);
 cudaError_t launch_verify_attn(const uint16_t*, const uint16_t*, const uint16_t*, const int32_t*, const int32_t*,
@@ -128,7 +128,8 @@ static bool ws_ok(const void* ws, size_t ws_bytes, const WsLayout& lay) {
 extern "C++" {
 template <typename T>
 static int confidence_t(const T* draft_logits, const int32_t* draft_tokens, const float* temperature, int B, int K,
-                        int V, float* conf, float* dstat, void* workspace, size_t ws_bytes, void* stream) {
+                        int V, float* conf, float* dstat, void* workspace, size_t ws_bytes, void* stream,
+                        const float* cost = nullptr, int32_t* L = nullptr) {
   if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
   if (B * K == 0) return LIBRASPEC_OK;
   if (!draft_logits || !draft_tokens || !temperature || !conf) return LIBRASPEC_EINVAL;
@@ -137,7 +138,8 @@ static int confidence_t(const T* draft_logits, const int32_t* draft_tokens, cons
   const WsLayout lay = ws_layout(B, K, V, 1, 1, 64, 1);
   if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
   return from_cuda(launch_confidence<T>(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat,
-                                        static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+                                        static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream), cost,
+                                        L));
 }
 }  // extern "C++"
 
@@ -150,6 +152,25 @@ int libraspec_confidence_bf16(const uint16_t* draft_logits, const int32_t* draft
                               int B, int K, int V, float* conf, float* dstat, void* workspace, size_t ws_bytes,
                               void* stream) {
   return confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream);
+}
+
+int libraspec_confidence_select(const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                                const float* cost_table, int B, int K, int V, float* conf, float* dstat, int32_t* L,
+                                void* workspace, size_t ws_bytes, void* stream) {
+  if (!cost_table || !L) return LIBRASPEC_EINVAL;
+  if (K == 0) return libraspec_select_lengths(conf, cost_table, B, K, L, workspace, ws_bytes, stream);
+  return confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream,
+                      cost_table, L);
+}
+
+int libraspec_confidence_select_bf16(const uint16_t* draft_logits, const int32_t* draft_tokens,
+                                     const float* temperature, const float* cost_table, int B, int K, int V,
+                                     float* conf, float* dstat, int32_t* L, void* workspace, size_t ws_bytes,
+                                     void* stream) {
+  if (!cost_table || !L) return LIBRASPEC_EINVAL;
+  if (K == 0) return libraspec_select_lengths(conf, cost_table, B, K, L, workspace, ws_bytes, stream);
+  return confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream,
+                      cost_table, L);
 }
 
 int libraspec_select_lengths(const float* conf, const float* cost_table, int B, int K, int32_t* L, void* workspace,
@@ -504,11 +525,13 @@ static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, co
   int rc = LIBRASPEC_OK;
   if (st && (rc = staged_begin(st, s)) != LIBRASPEC_OK) return rc;
   if ((rc = staged_wait(st, 0, s)) != LIBRASPEC_OK) return rc;
-  if (K > 0) {
-    rc = confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream);
-    if (rc != LIBRASPEC_OK) return rc;
+  if (!cost_table) return LIBRASPEC_EINVAL;
+  if (K > 0) {  // confidence, and the selection in the same launch
+    rc = confidence_t(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, workspace, ws_bytes, stream,
+                      cost_table, L);
+  } else {
+    rc = from_cuda(launch_select(conf, cost_table, B, K, L, ws, lay, s));
   }
-  rc = from_cuda(launch_select(conf, cost_table, B, K, L, ws, lay, s));
   if (rc != LIBRASPEC_OK) return rc;
   if ((rc = staged_wait(st, 1, s)) != LIBRASPEC_OK) return rc;
   if (st && (rc = from_cuda(launch_kv_append(st->kv_new, const_cast<uint16_t* const*>(Kc),

@@ -42,7 +42,7 @@ struct RacePartial {
 };
 
 struct WsLayout {
-  size_t status, conf_part, conf_cnt, row_part, row_cnt, row_stat, race_part, race_cnt;
+  size_t status, conf_part, conf_cnt, seq_cnt, row_part, row_cnt, row_stat, race_part, race_cnt;
   size_t attn_o, attn_ml, attn_cnt, tree_vis, total;
   int max_items, max_groups;
 };
@@ -64,6 +64,7 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.status = take(256);
   w.conf_part = take(rows_d * kConfMaxSplits * sizeof(RowPartial));
   w.conf_cnt = take(rows_d * sizeof(uint32_t));
+  w.seq_cnt = take(size_t(B) * sizeof(uint32_t));  // rows of a sequence done (fused selection)
   w.row_part = take(rows_t * kRowMaxSplits * sizeof(RowPartial));
   w.row_cnt = take(rows_t * sizeof(uint32_t));
   w.row_stat = take(rows_t * sizeof(RowStat));

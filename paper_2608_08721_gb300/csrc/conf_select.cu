@@ -11,83 +11,19 @@ namespace libraspec {
 // q = exp((x_tok - m)/T) / Z (Assumption 1: q_k, the drafter's probability
 // of its drafted token).
 // ---------------------------------------------------------------------------
-template <bool VEC, typename E>
-__global__ void __launch_bounds__(kRowThreads) conf_kernel(
-    const E* __restrict__ x, const int32_t* __restrict__ tokens, const float* __restrict__ temperature,
-    int K, int V, int nsplit, int chunk, float* __restrict__ conf, float* __restrict__ dstat,
-    RowPartial* __restrict__ part, uint32_t* __restrict__ cnt, int* __restrict__ status) {
-  __shared__ float sm[64];
-  __shared__ int last;
-  const int row = blockIdx.y, split = blockIdx.x;
-  const int b = row / K;
-  const float tb = temperature[b];
-  const float T = tb > 0.f ? tb : 1.f;
-  const float c = (float)(1.4426950408889634 / (double)T);
-  const E* xr = x + (size_t)row * V;
-  const int c0 = split * chunk, c1 = min(V, c0 + chunk);
-
-  SumAcc sa;
-  ArgAcc aa;
-  sa.init();
-  row_slice_pass<true, false, VEC, E>(xr, c0, c1, c, sa, aa);
-  float m = sa.m, s = sa.value();
-  cta_reduce_sum(m, s, c, sm);
-
-  double Z;
-  float M;
-  if (nsplit == 1) {
-    if (threadIdx.x != 0) return;
-    M = m;
-    Z = (double)s;
-  } else {
-    if (threadIdx.x == 0) {
-      RowPartial p;
-      p.m = m;
-      p.arg = 0;
-      p.s = (double)s;
-      part[(size_t)row * kConfMaxSplits + split] = p;
-      __threadfence();
-      const uint32_t ticket = atomicAdd(&cnt[row], 1u);
-      last = (ticket == (uint32_t)(nsplit - 1));
-    }
-    __syncthreads();
-    if (!last) return;
-    if (threadIdx.x >= 32) return;
-    __threadfence();
-    int dummy;
-    warp_merge_partials(part + (size_t)row * kConfMaxSplits, nsplit, c, false, M, dummy, Z);
-    if (threadIdx.x != 0) return;
-    cnt[row] = 0u;  // ready for the next call
-  }
-  const int tok = tokens[row];
-  float q = 0.f;
-  if (tok < 0 || tok >= V) {
-    raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
-  } else {
-    // x_tok - M is exact for the near-maximal tokens that matter (Sterbenz)
-    q = (float)((double)exp2f((Logit<E>::at(xr, tok) - M) * c) / Z);
-  }
-  conf[row] = q;
-  if (dstat) {
-    dstat[2 * (size_t)row] = M;
-    dstat[2 * (size_t)row + 1] = (float)Z;
-  }
-}
-
 // ---------------------------------------------------------------------------
 // Selection (Thm. 4): one warp per sequence, binary64. Lane k of a 32-wide
 // chunk evaluates the step L = k -> k+1:
 //   P_{k+1} = prod_{i<=k} q_i          (multiplicative inclusive scan)
 //   E_k     = 1 + sum_{j<=k} P_j       (additive exclusive scan of P)
 //   extend  iff P_{k+1} * T(k) > (T(k+1) - T(k)) * E_k
-// L is the first lane (in chunk order) whose test fails, or K.
+// L is the first lane (in chunk order) whose test fails, or K. Executed by
+// one full warp; conf is read through L2 (it may have been written by other
+// CTAs of the same launch).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(128) select_kernel(const float* __restrict__ conf,
-                                                     const float* __restrict__ cost, int B, int K,
-                                                     int32_t* __restrict__ L, int* __restrict__ status) {
-  const int seq = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+__device__ void select_seq(const float* __restrict__ conf, const float* __restrict__ cost, int K, int seq,
+                           int32_t* __restrict__ L, int* __restrict__ status) {
   const int lane = threadIdx.x & 31;
-  if (seq >= B) return;
   bool bad = false;
   for (int l = lane; l <= K; l += 32) {
     const float t = cost[l];
@@ -105,7 +41,7 @@ __global__ void __launch_bounds__(128) select_kernel(const float* __restrict__ c
   for (int base = 0; base < K; base += 32) {
     const int k = base + lane;
     const bool live = k < K;
-    const double q = live ? (double)conf[(size_t)seq * K + k] : 1.0;
+    const double q = live ? (double)__ldcg(&conf[(size_t)seq * K + k]) : 1.0;
     double P = q;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
@@ -138,6 +74,91 @@ __global__ void __launch_bounds__(128) select_kernel(const float* __restrict__ c
     carryE = __dadd_rn(carryE, __shfl_sync(0xffffffffu, S, 31));
   }
   if (lane == 0) L[seq] = result;
+}
+
+__global__ void __launch_bounds__(128) select_kernel(const float* __restrict__ conf,
+                                                     const float* __restrict__ cost, int B, int K,
+                                                     int32_t* __restrict__ L, int* __restrict__ status) {
+  const int seq = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (seq >= B) return;
+  select_seq(conf, cost, K, seq, L, status);
+}
+
+template <bool VEC, typename E>
+__global__ void __launch_bounds__(kRowThreads) conf_kernel(
+    const E* __restrict__ x, const int32_t* __restrict__ tokens, const float* __restrict__ temperature,
+    int K, int V, int nsplit, int chunk, float* __restrict__ conf, float* __restrict__ dstat,
+    RowPartial* __restrict__ part, uint32_t* __restrict__ cnt, const float* __restrict__ cost,
+    int32_t* __restrict__ L, uint32_t* __restrict__ seq_cnt, int* __restrict__ status) {
+  __shared__ float sm[64];
+  __shared__ int last;
+  const int row = blockIdx.y, split = blockIdx.x;
+  const int b = row / K;
+  const float tb = temperature[b];
+  const float T = tb > 0.f ? tb : 1.f;
+  const float c = (float)(1.4426950408889634 / (double)T);
+  const E* xr = x + (size_t)row * V;
+  const int c0 = split * chunk, c1 = min(V, c0 + chunk);
+
+  SumAcc sa;
+  ArgAcc aa;
+  sa.init();
+  row_slice_pass<true, false, VEC, E>(xr, c0, c1, c, sa, aa);
+  float m = sa.m, s = sa.value();
+  cta_reduce_sum(m, s, c, sm);
+
+  double Z;
+  float M;
+  if (nsplit == 1) {
+    if (threadIdx.x >= 32) return;
+    M = m;
+    Z = (double)s;
+  } else {
+    if (threadIdx.x == 0) {
+      RowPartial p;
+      p.m = m;
+      p.arg = 0;
+      p.s = (double)s;
+      part[(size_t)row * kConfMaxSplits + split] = p;
+      __threadfence();
+      const uint32_t ticket = atomicAdd(&cnt[row], 1u);
+      last = (ticket == (uint32_t)(nsplit - 1));
+    }
+    __syncthreads();
+    if (!last) return;
+    if (threadIdx.x >= 32) return;
+    __threadfence();
+    int dummy;
+    warp_merge_partials(part + (size_t)row * kConfMaxSplits, nsplit, c, false, M, dummy, Z);
+    if (threadIdx.x == 0) cnt[row] = 0u;  // ready for the next call
+  }
+  // warp 0 of the CTA that completed the row
+  bool seq_done = false;
+  if (threadIdx.x == 0) {
+    const int tok = tokens[row];
+    float q = 0.f;
+    if (tok < 0 || tok >= V) {
+      raise_status(status, LIBRASPEC_ST_BAD_TOKEN);
+    } else {
+      // x_tok - M is exact for the near-maximal tokens that matter (Sterbenz)
+      q = (float)((double)exp2f((Logit<E>::at(xr, tok) - M) * c) / Z);
+    }
+    conf[row] = q;
+    if (dstat) {
+      dstat[2 * (size_t)row] = M;
+      dstat[2 * (size_t)row + 1] = (float)Z;
+    }
+    if (cost) {
+      __threadfence();
+      seq_done = atomicAdd(&seq_cnt[b], 1u) == (uint32_t)(K - 1);
+    }
+  }
+  // With a cost table, the CTA that completes a sequence's last row selects
+  // its length (Thm. 4) right away instead of in a separate launch.
+  if (cost == nullptr || !__shfl_sync(0xffffffffu, seq_done, 0)) return;
+  __threadfence();
+  if (threadIdx.x == 0) seq_cnt[b] = 0u;  // ready for the next call
+  select_seq(conf, cost, K, b, L, status);
 }
 
 // ---------------------------------------------------------------------------
@@ -223,9 +244,12 @@ __global__ void __launch_bounds__(128) select_alpha_kernel(const float* __restri
 // ---------------------------------------------------------------------------
 int num_sms_current();
 
+// cost != nullptr: also select every sequence's length (Thm. 4) into L, in
+// the same launch (K >= 1).
 template <typename T>
 cudaError_t launch_confidence(const T* x, const int32_t* tokens, const float* temperature, int B, int K, int V,
-                              float* conf, float* dstat, char* ws, const WsLayout& lay, cudaStream_t stream) {
+                              float* conf, float* dstat, char* ws, const WsLayout& lay, cudaStream_t stream,
+                              const float* cost, int32_t* L) {
   const long rows = (long)B * K;
   if (rows == 0) return cudaSuccess;
   const int nsplit0 = row_splits(rows, V, num_sms_current(), kConfMaxSplits, 4096);
@@ -236,18 +260,20 @@ cudaError_t launch_confidence(const T* x, const int32_t* tokens, const float* te
   auto* part = reinterpret_cast<RowPartial*>(ws + lay.conf_part);
   auto* cnt = reinterpret_cast<uint32_t*>(ws + lay.conf_cnt);
   auto* st = reinterpret_cast<int*>(ws + lay.status);
+  auto* seq_cnt = reinterpret_cast<uint32_t*>(ws + lay.seq_cnt);
   if (vec)
     conf_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
-                                                           dstat, part, cnt, st);
+                                                           dstat, part, cnt, cost, L, seq_cnt, st);
   else
     conf_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(x, tokens, temperature, K, V, nsplit, chunk, conf,
-                                                            dstat, part, cnt, st);
+                                                            dstat, part, cnt, cost, L, seq_cnt, st);
   return cudaGetLastError();
 }
 template cudaError_t launch_confidence<float>(const float*, const int32_t*, const float*, int, int, int, float*,
-                                              float*, char*, const WsLayout&, cudaStream_t);
+                                              float*, char*, const WsLayout&, cudaStream_t, const float*, int32_t*);
 template cudaError_t launch_confidence<uint16_t>(const uint16_t*, const int32_t*, const float*, int, int, int,
-                                                 float*, float*, char*, const WsLayout&, cudaStream_t);
+                                                 float*, float*, char*, const WsLayout&, cudaStream_t, const float*,
+                                                 int32_t*);
 
 cudaError_t launch_select_alpha(const float* conf, int B, int K, int n, double alpha, int32_t* L,
                                 int32_t* n_blocks, cudaStream_t stream) {

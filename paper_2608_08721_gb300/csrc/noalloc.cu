@@ -12,7 +12,7 @@ namespace libraspec {
 
 template <typename T>
 cudaError_t launch_confidence(const T*, const int32_t*, const float*, int, int, int, float*, float*, char*,
-                              const WsLayout&, cudaStream_t);
+                              const WsLayout&, cudaStream_t, const float*, int32_t*);
 
 namespace {
 
@@ -77,7 +77,8 @@ extern "C" int libraspec_confidence_noalloc(const float* draft_logits, const int
   lay.status = 0;
   lay.conf_cnt = kCntOff;
   lay.conf_part = kPartOff;
-  e = launch_confidence(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, scratch, lay, s);
+  e = launch_confidence(draft_logits, draft_tokens, temperature, B, K, V, conf, dstat, scratch, lay, s,
+                        static_cast<const float*>(nullptr), nullptr);
   if (e != cudaSuccess) return LIBRASPEC_ECUDA;
   if (status) {
     e = cudaMemcpyAsync(status, scratch, sizeof(int32_t), cudaMemcpyDeviceToDevice, s);

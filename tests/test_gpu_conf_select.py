@@ -143,3 +143,34 @@ def test_select_random_adversarial(orc):
     L = lr.libraspec_select_lengths(torch.tensor(q, device=cuda()), torch.tensor(cost, device=cuda()), ws)
     L_ref, flag = orc.select_lengths(q.astype(np.float64), cost.astype(np.float64))
     assert_exact_unless_flagged(L.cpu().numpy(), L_ref, flag, "L")
+
+
+@pytest.mark.parametrize("name", ["tiny", "8b", "sampling", "ragged"])
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_fused_confidence_select_equals_the_two_calls(name, dtype):
+    """libraspec_confidence_select: the same conf, dstat and L as
+    libraspec_confidence followed by libraspec_select_lengths, bit for bit."""
+    w = workloads.WORKLOADS[name]
+    inp = workloads.logits(w, device=cuda())
+    x = inp["draft_logits"].to(dtype)
+    cost = torch.tensor(workloads.cost_table(w), device=cuda())
+    ws = lr.Workspace(w.B, w.K, w.V, device=cuda())
+    c1, d1 = lr.libraspec_confidence(x, inp["draft_tokens"], inp["temperature"], ws)
+    L1 = lr.libraspec_select_lengths(c1, cost, ws)
+    for _ in range(2):   # the tickets reset themselves between calls
+        c2, d2, L2 = lr.libraspec_confidence_select(x, inp["draft_tokens"], inp["temperature"], cost, ws)
+        torch.cuda.synchronize()
+        assert torch.equal(c1, c2) and torch.equal(d1, d2) and torch.equal(L1, L2)
+    assert lr.libraspec_get_status(ws) == 0
+
+
+def test_fused_confidence_select_bad_cost_sets_status():
+    w = workloads.WORKLOADS["tiny"]
+    inp = workloads.logits(w, device=cuda())
+    cost = torch.tensor(workloads.cost_table(w), device=cuda())
+    cost[3] = -1.0
+    ws = lr.Workspace(w.B, w.K, w.V, device=cuda())
+    _, _, L = lr.libraspec_confidence_select(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], cost, ws)
+    torch.cuda.synchronize()
+    assert lr.libraspec_get_status(ws) & lr.ST_BAD_COST
+    assert (L == 0).all()

@@ -109,3 +109,32 @@ def test_staged_round_appends_and_matches_device_round():
     np.testing.assert_array_equal(runner.out.n_accepted.cpu().numpy(), n2)
     np.testing.assert_array_equal(runner.out.bonus_token.cpu().numpy(), b2)
     assert runner.h2d_bytes() >= h["draft_logits"].numel() * 4 + h["target_logits"].numel() * 4
+
+
+def test_staged_round_bf16_logits_matches_device_round():
+    w = workloads.WORKLOADS["tiny"]
+    kv = workloads.kv_lengths(w)
+    lay = workloads.layer(w, 0, kv, device=cuda())
+    inp = workloads.logits(w)
+    caches = [{"Kc": lay["Kc"].clone(), "Vc": lay["Vc"].clone()}]
+    runner = api.VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, lay["Kc"].shape[2], caches, torch.tensor(kv),
+                             logits_dtype=torch.bfloat16)
+    h = runner.host_inputs()
+    h["draft_logits"].copy_(inp["draft_logits"].to(torch.bfloat16))
+    h["target_logits"].copy_(inp["target_logits"].to(torch.bfloat16))
+    for name in ("draft_tokens", "temperature"):
+        h[name].copy_(inp[name])
+    h["cost_table"].copy_(torch.tensor(workloads.cost_table(w)))
+    h["Q"][0].copy_(lay["Q"].cpu())
+    K1 = w.K + 1
+    kvb = int(kv[0])
+    h["kv_new"][0, 0].copy_(lay["Kc"][:, :, kvb:kvb + K1].cpu())
+    h["kv_new"][0, 1].copy_(lay["Vc"][:, :, kvb:kvb + K1].cpu())
+    n, bonus = runner.run_staged(seed=w.philox_seed, round_offset=2)
+    O = runner.out.O[0].clone()
+    runner.run_device(seed=w.philox_seed, round_offset=2)
+    torch.cuda.synchronize()
+    assert torch.equal(runner.out.O[0], O)
+    np.testing.assert_array_equal(runner.out.n_accepted.cpu().numpy(), n)
+    np.testing.assert_array_equal(runner.out.bonus_token.cpu().numpy(), bonus)
+    assert lr.libraspec_get_status(runner.ws) == 0
