@@ -504,13 +504,19 @@ int libraspec_verify_round_bf16(const uint16_t* draft_logits, const int32_t* dra
  * n_accepted and bonus_token are copied to n_accepted_host / bonus_host
  * (pinned, B entries each). copy_stream first waits for the work already on
  * `stream`, so a round never overwrites buffers an earlier one still reads.
- * The call returns after enqueuing; synchronise `stream` before reading the
- * host results. Other arguments as libraspec_verify_round (lse is not
- * produced).
+ * The generator arguments travel with part 2: the call writes seed,
+ * round_offset and seq_offset to rng_host[0..2] (pinned, inside host part
+ * 2, 8-byte aligned) and acceptance reads them at rng_dev (the same bytes in
+ * device part 2). The first call with a given set of buffers and shapes
+ * runs eagerly; the second captures the round on `stream` as one CUDA graph
+ * (per thread) and later calls with the same set replay it, whatever the
+ * seed and offsets. The call returns after enqueuing; synchronise `stream`
+ * before reading the host results or rewriting the host parts. Other
+ * arguments as libraspec_verify_round (lse is not produced).
  */
 int libraspec_verify_round_staged(const void* const* host_parts, void* const* dev_parts, const size_t* part_bytes,
-                                  void* copy_stream, const uint16_t* kv_new, int32_t* n_accepted_host,
-                                  int32_t* bonus_host, const float* draft_logits, const int32_t* draft_tokens,
+                                  void* copy_stream, const uint16_t* kv_new, uint64_t* rng_host,
+                                  const uint64_t* rng_dev, int32_t* n_accepted_host, int32_t* bonus_host, const float* draft_logits, const int32_t* draft_tokens,
                                   const float* temperature, const float* cost_table, const float* target_logits,
                                   const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
                                   uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V,
@@ -520,7 +526,8 @@ int libraspec_verify_round_staged(const void* const* host_parts, void* const* de
                                   void* stream);
 int libraspec_verify_round_staged_bf16(const void* const* host_parts, void* const* dev_parts,
                                        const size_t* part_bytes, void* copy_stream, const uint16_t* kv_new,
-                                       int32_t* n_accepted_host, int32_t* bonus_host, const uint16_t* draft_logits,
+                                       uint64_t* rng_host, const uint64_t* rng_dev, int32_t* n_accepted_host,
+                                       int32_t* bonus_host, const uint16_t* draft_logits,
                                        const int32_t* draft_tokens, const float* temperature,
                                        const float* cost_table, const uint16_t* target_logits,
                                        const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,

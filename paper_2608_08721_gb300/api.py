@@ -53,7 +53,7 @@ class VerifyRound:
         regions = [("draft_logits", (B, K, V), logits_dtype), ("draft_tokens", (B, K), i32),
                    ("temperature", (B,), f32), ("cost_table", (K1,), f32),
                    ("Q", (n, B, K1, Hq, head_dim), bf), ("kv_new", (n, 2, B, Hkv, K1, head_dim), bf),
-                   ("target_logits", (B, K1, V), logits_dtype)]
+                   ("target_logits", (B, K1, V), logits_dtype), ("rng", (3,), torch.int64)]
         offs, total = _layout(regions)
         # the three parts a round copies in, in the order its steps need them
         self._parts = [(0, offs["Q"]), (offs["Q"], offs["target_logits"]), (offs["target_logits"], total)]
@@ -81,16 +81,19 @@ class VerifyRound:
             torch.empty((B,), dtype=i32, device=dev),
             [torch.empty((B, K1, Hq, head_dim), dtype=bf, device=dev) for _ in caches], None)
         self.result_host = torch.empty((2, B), dtype=i32, pin_memory=True)
+        # the staged round runs on its own stream (a graph cannot be captured on the legacy default one)
+        self._stream = torch.cuda.Stream(device=dev)
         self._staged = binding.StagedRound(
             [self._host_stage[a:b] for a, b in self._parts], [self._dev_stage[a:b] for a, b in self._parts],
             d["kv_new"], self.result_host[0], self.result_host[1], self.draft_logits, self.draft_tokens,
-            self.temperature, self.cost_table, self.target_logits, self.layers, self.kv_len, self.out, self.ws)
+            self.temperature, self.cost_table, self.target_logits, self.layers, self.kv_len, self.out, self.ws,
+            self._host["rng"], d["rng"])
 
     def host_inputs(self) -> Dict[str, torch.Tensor]:
         """Pinned host views to fill before ``run_staged``: draft_logits [B,K,V], target_logits [B,K+1,V],
         draft_tokens [B,K], temperature [B], cost_table [K+1], Q [n_layers,B,K+1,Hq,d] and kv_new
         [n_layers,2,B,Hkv,K+1,d] (layer l's new keys [l,0] and values [l,1] of the verified block)."""
-        return self._host
+        return {k: v for k, v in self._host.items() if k != "rng"}
 
     def run_device(self, seed: int, round_offset: int = 0, seq_offset: int = 0, stream=None):
         """The round on inputs already resident in this object's device buffers
@@ -112,8 +115,9 @@ class VerifyRound:
         part has landed, the key/value append and the attention layers once the layer part has,
         acceptance once the target rows have; the results come back into pinned memory. Returns
         (n_accepted, bonus_token) numpy arrays."""
-        self._staged(seed, round_offset, seq_offset)
-        torch.cuda.current_stream(self.device).synchronize()
+        self._stream.wait_stream(torch.cuda.current_stream(self.device))
+        self._staged(seed, round_offset, seq_offset, stream=self._stream)
+        self._stream.synchronize()
         return self.result_host[0].numpy().copy(), self.result_host[1].numpy().copy()
 
     def run_host(self, host: Dict, seed: int, round_offset: int = 0, seq_offset: int = 0):

@@ -51,12 +51,10 @@ SIGNATURES = {
     "libraspec_accept_tree": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _P, _SZ, _P]),
     "libraspec_accept_tree_bf16": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _U64, _U64, _U32, _P, _P, _P, _P, _SZ,
                                         _P]),
-    "libraspec_verify_round_staged": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P,
-                                           _I, _I, _I, _I, _I, _I, _I, _F, _U64, _U64, _U32, _P, _P, _P, _P, _P, _P,
-                                           _SZ, _P]),
-    "libraspec_verify_round_staged_bf16": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I,
-                                                _P, _I, _I, _I, _I, _I, _I, _I, _F, _U64, _U64, _U32, _P, _P, _P, _P,
-                                                _P, _P, _SZ, _P]),
+    "libraspec_verify_round_staged": (_I, [_P] * 18 + [_I, _P] + [_I] * 7 + [_F, _U64, _U64, _U32] + [_P] * 6 +
+                                      [_SZ, _P]),
+    "libraspec_verify_round_staged_bf16": (_I, [_P] * 18 + [_I, _P] + [_I] * 7 + [_F, _U64, _U64, _U32] + [_P] * 6 +
+                                           [_SZ, _P]),
     "libraspec_lm_head_workspace_size": (_SZ, [_I, _I]),
     "libraspec_lm_head_stats": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _P, _P, _P, _P, _SZ, _P]),
     "libraspec_kv_append": (_I, [_P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _P, _SZ, _P]),
@@ -592,7 +590,7 @@ class StagedRound:
 
     def __init__(self, host_parts, dev_parts, kv_new, n_host, bonus_host, draft_logits, draft_tokens, temperature,
                  cost_table, target_logits, layers, kv_len, outputs: "RoundOutputs", ws: Workspace,
-                 softmax_scale=None, copy_stream=None):
+                 rng_host, rng_dev, softmax_scale=None, copy_stream=None):
         B, K, V = draft_logits.shape
         bf16 = draft_logits.dtype == torch.bfloat16
         ldt = torch.bfloat16 if bf16 else torch.float32
@@ -615,9 +613,13 @@ class StagedRound:
         for h, d in zip(host_parts, dev_parts):
             if not h.is_pinned() or h.numel() != d.numel() or not d.is_cuda:
                 raise ValueError("each part: a pinned host tensor and a device tensor of the same size")
+        _req(rng_dev, torch.int64, "rng_dev", (3,))
+        if (not isinstance(rng_host, torch.Tensor) or rng_host.dtype != torch.int64 or rng_host.numel() != 3
+                or not rng_host.is_pinned()):
+            raise ValueError("rng_host must be 3 int64 of pinned host memory inside host part 2")
         if softmax_scale is None:
             softmax_scale = D ** -0.5
-        self._keep = (host_parts, dev_parts, layers, outputs, n_host, bonus_host)
+        self._keep = (host_parts, dev_parts, layers, outputs, n_host, bonus_host, rng_host, rng_dev)
         self._hp = (ctypes.c_void_p * 3)(*[h.data_ptr() for h in host_parts])
         self._dp = (ctypes.c_void_p * 3)(*[d.data_ptr() for d in dev_parts])
         self._nb = (ctypes.c_size_t * 3)(*[h.numel() * h.element_size() for h in host_parts])
@@ -629,7 +631,7 @@ class StagedRound:
         self._name = "libraspec_verify_round_staged_bf16" if bf16 else "libraspec_verify_round_staged"
         self._fn = getattr(load(), self._name)
         self._pre = (self._hp, self._dp, self._nb, ctypes.c_void_p(self._copy.cuda_stream), _ptr(kv_new),
-                     _ptr(n_host), _ptr(bonus_host), _ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature),
+                     _ptr(rng_host), _ptr(rng_dev), _ptr(n_host), _ptr(bonus_host), _ptr(draft_logits), _ptr(draft_tokens), _ptr(temperature),
                      _ptr(cost_table), _ptr(target_logits), self._qa, self._ka, self._va, self._oa, n_layers,
                      _ptr(kv_len), B, K, V, Hq, Hkv, D, S_cap, float(softmax_scale))
         self._post = (_ptr(outputs.conf), _ptr(outputs.dstat), _ptr(outputs.L), _ptr(outputs.n_accepted),
@@ -642,11 +644,12 @@ class StagedRound:
 
 
 def libraspec_verify_round_staged(host_parts, dev_parts, kv_new, n_host, bonus_host, draft_logits, draft_tokens,
-                                  temperature, cost_table, target_logits, layers, kv_len, outputs, ws, seed: int,
-                                  round_offset: int = 0, seq_offset: int = 0, softmax_scale=None, copy_stream=None,
-                                  stream=None) -> None:
+                                  temperature, cost_table, target_logits, layers, kv_len, outputs, ws, rng_host,
+                                  rng_dev, seed: int, round_offset: int = 0, seq_offset: int = 0, softmax_scale=None,
+                                  copy_stream=None, stream=None) -> None:
     """One staged round (see StagedRound); returns after enqueuing."""
     StagedRound(host_parts, dev_parts, kv_new, n_host, bonus_host, draft_logits, draft_tokens, temperature,
-                cost_table, target_logits, layers, kv_len, outputs, ws, softmax_scale, copy_stream)(
+                cost_table, target_logits, layers, kv_len, outputs, ws, rng_host, rng_dev, softmax_scale,
+                copy_stream)(
         seed, round_offset, seq_offset, stream)
 

@@ -3,6 +3,7 @@
 // accept.cu.
 #include <cstdio>
 #include <cstring>
+#include <vector>
 
 #include "common.cuh"
 
@@ -35,7 +36,7 @@ cudaError_t launch_accept_tree(const T*, const int32_t*, const int32_t*, const i
 template <typename T>
 cudaError_t launch_accept(const T*, const T*, const int32_t*, const float*, const float*, const int32_t*,
                           const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, char*,
-                          const WsLayout&, cudaStream_t);
+                          const WsLayout&, cudaStream_t, const uint64_t*);
 
 int num_sms_current() {
   static int cached_dev = -1, cached_sms = 0;
@@ -308,7 +309,7 @@ template <typename T>
 static int accept_t(const T* target_logits, const T* draft_logits, const int32_t* draft_tokens, const float* conf,
                     const float* dstat, const int32_t* L, const float* temperature, int B, int K, int V, uint64_t seed,
                     uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted, int32_t* bonus_token,
-                    void* workspace, size_t ws_bytes, void* stream) {
+                    void* workspace, size_t ws_bytes, void* stream, const uint64_t* rng = nullptr) {
   if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
   if (B == 0) return LIBRASPEC_OK;
   if (!target_logits || (!draft_logits && K > 0) || (!draft_tokens && K > 0) || !L || !temperature ||
@@ -320,7 +321,7 @@ static int accept_t(const T* target_logits, const T* draft_logits, const int32_t
   if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
   return from_cuda(launch_accept<T>(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V,
                                     seed, round_offset, seq_offset, n_accepted, bonus_token,
-                                    static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream)));
+                                    static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream), rng));
 }
 }  // extern "C++"
 
@@ -465,6 +466,7 @@ struct Staged {
   const uint16_t* kv_new;
   int32_t* n_host;
   int32_t* bonus_host;
+  const uint64_t* rng_dev;  // {seed, round_offset, seq_offset} inside part 2 on the device
   cudaEvent_t ev[4];
 };
 
@@ -544,32 +546,117 @@ static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, co
   if (rc != LIBRASPEC_OK) return rc;
   if ((rc = staged_wait(st, 2, s)) != LIBRASPEC_OK) return rc;
   rc = accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed, round_offset,
-                seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream);
+                seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream, st ? st->rng_dev : nullptr);
   if (rc != LIBRASPEC_OK || !st) return rc;
   cudaError_t e = cudaMemcpyAsync(st->n_host, n_accepted, sizeof(int32_t) * B, cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(st->bonus_host, bonus_token, sizeof(int32_t) * B, cudaMemcpyDeviceToHost, s);
   return from_cuda(e);
 }
 
+// A staged round replays as one CUDA graph: the first call with a set of
+// buffers and shapes runs eagerly, the second captures the round (copies,
+// events, kernels, read-back) on the caller's stream and keeps the
+// instantiated graph; later calls with the same set launch it. The generator
+// arguments travel in part 2 (rng_host -> rng_dev), so a graph serves every
+// seed and round. One cached graph per thread.
+inline uintptr_t float_bits(float f) {
+  uint32_t u;
+  memcpy(&u, &f, sizeof(u));
+  return u;
+}
+
+struct StagedGraph {
+  std::vector<uintptr_t> key;
+  int seen = 0;
+  cudaGraphExec_t exec = nullptr;
+};
+
 template <typename T>
 static int verify_round_staged_t(const void* const* host_parts, void* const* dev_parts, const size_t* part_bytes,
-                                 void* copy_stream, const uint16_t* kv_new, int32_t* n_accepted_host,
-                                 int32_t* bonus_host, const T* draft_logits, const int32_t* draft_tokens,
-                                 const float* temperature, const float* cost_table, const T* target_logits,
-                                 const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
-                                 uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V, int Hq,
-                                 int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
-                                 uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
-                                 int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
-                                 void* stream) {
-  if (!host_parts || !dev_parts || !part_bytes || !n_accepted_host || !bonus_host || !n_accepted || !bonus_token)
+                                 void* copy_stream, const uint16_t* kv_new, uint64_t* rng_host,
+                                 const uint64_t* rng_dev, int32_t* n_accepted_host, int32_t* bonus_host,
+                                 const T* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                                 const float* cost_table, const T* target_logits, const uint16_t* const* Q,
+                                 uint16_t* const* Kc, uint16_t* const* Vc, uint16_t* const* O, int n_layers,
+                                 const int32_t* kv_len, int B, int K, int V, int Hq, int Hkv, int head_dim,
+                                 int S_cap, float softmax_scale, uint64_t seed, uint64_t round_offset,
+                                 uint32_t seq_offset, float* conf, float* dstat, int32_t* L, int32_t* n_accepted,
+                                 int32_t* bonus_token, void* workspace, size_t ws_bytes, void* stream) {
+  if (!host_parts || !dev_parts || !part_bytes || !n_accepted_host || !bonus_host || !n_accepted || !bonus_token ||
+      !rng_host || !rng_dev || !aligned(rng_dev, 8))
     return LIBRASPEC_EINVAL;
   for (int i = 0; i < 3; ++i)
     if (part_bytes[i] > 0 && (!host_parts[i] || !dev_parts[i])) return LIBRASPEC_EINVAL;
-  if (n_layers > 0 && (!kv_new || !aligned(kv_new, 16))) return LIBRASPEC_EINVAL;
+  if (n_layers > 0 && (!kv_new || !aligned(kv_new, 16) || !Q || !Kc || !Vc || !O)) return LIBRASPEC_EINVAL;
+  if (n_layers < 0 || n_layers > 4096) return LIBRASPEC_EINVAL;
+  const uintptr_t fixed[] = {
+      (uintptr_t)host_parts[0], (uintptr_t)host_parts[1], (uintptr_t)host_parts[2], (uintptr_t)dev_parts[0],
+      (uintptr_t)dev_parts[1], (uintptr_t)dev_parts[2], part_bytes[0], part_bytes[1], part_bytes[2],
+      (uintptr_t)copy_stream, (uintptr_t)kv_new, (uintptr_t)rng_dev, (uintptr_t)n_accepted_host,
+      (uintptr_t)bonus_host, (uintptr_t)draft_logits, (uintptr_t)draft_tokens, (uintptr_t)temperature,
+      (uintptr_t)cost_table, (uintptr_t)target_logits, (uintptr_t)n_layers, (uintptr_t)kv_len, (uintptr_t)B,
+      (uintptr_t)K, (uintptr_t)V, (uintptr_t)Hq, (uintptr_t)Hkv, (uintptr_t)head_dim, (uintptr_t)S_cap,
+      float_bits(softmax_scale), (uintptr_t)conf, (uintptr_t)dstat, (uintptr_t)L,
+      (uintptr_t)n_accepted, (uintptr_t)bonus_token, (uintptr_t)workspace, ws_bytes, (uintptr_t)stream,
+      (uintptr_t)sizeof(T)};
+  std::vector<uintptr_t> key(fixed, fixed + sizeof(fixed) / sizeof(fixed[0]));
+  for (int l = 0; l < n_layers; ++l) {
+    key.push_back((uintptr_t)Q[l]);
+    key.push_back((uintptr_t)Kc[l]);
+    key.push_back((uintptr_t)Vc[l]);
+    key.push_back((uintptr_t)O[l]);
+  }
+  // the generator arguments of this round, copied in with part 2
+  rng_host[0] = seed;
+  rng_host[1] = round_offset;
+  rng_host[2] = seq_offset;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  static thread_local StagedGraph cache;
+  if (cache.exec && cache.key == key) return from_cuda(cudaGraphLaunch(cache.exec, s));
+  const bool capture = cache.key == key && cache.seen >= 1;
+  if (cache.key != key) {
+    if (cache.exec) cudaGraphExecDestroy(cache.exec);
+    cache.exec = nullptr;
+    cache.key = key;
+    cache.seen = 0;
+  }
+  ++cache.seen;
   Staged st{host_parts, dev_parts, part_bytes, static_cast<cudaStream_t>(copy_stream), kv_new, n_accepted_host,
-            bonus_host, {}};
-  const int rc = verify_round_t(draft_logits, draft_tokens, temperature, cost_table, target_logits, Q, Kc, Vc, O,
+            bonus_host, rng_dev, {}};
+  bool capturing = false;
+  if (capture) {
+    // not possible on the legacy default stream, for one: then this set of
+    // buffers always runs eagerly
+    capturing = cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+    if (!capturing) {
+      cudaGetLastError();
+      cache.seen = -(1 << 30);
+    }
+  }
+  if (capturing) {
+    int rc = verify_round_t(draft_logits, draft_tokens, temperature, cost_table, target_logits, Q,
+                            const_cast<const uint16_t* const*>(Kc), const_cast<const uint16_t* const*>(Vc), O,
+                            nullptr, n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed,
+                            round_offset, seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace, ws_bytes,
+                            stream, &st);
+    cudaGraph_t graph = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(s, &graph);
+    staged_end(&st);
+    cudaGraphExec_t exec = nullptr;
+    if (rc == LIBRASPEC_OK && e == cudaSuccess && graph &&
+        cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess) {
+      cudaGraphDestroy(graph);
+      cache.exec = exec;
+      return from_cuda(cudaGraphLaunch(exec, s));
+    }
+    if (graph) cudaGraphDestroy(graph);
+    cudaGetLastError();  // the failed capture's error; run the round eagerly below, and from now on
+    cache.seen = -(1 << 30);
+    st = Staged{host_parts, dev_parts, part_bytes, static_cast<cudaStream_t>(copy_stream), kv_new, n_accepted_host,
+                bonus_host, rng_dev, {}};
+  }
+  const int rc = verify_round_t(draft_logits, draft_tokens, temperature, cost_table, target_logits, Q,
+                                const_cast<const uint16_t* const*>(Kc), const_cast<const uint16_t* const*>(Vc), O,
                                 nullptr, n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed,
                                 round_offset, seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace,
                                 ws_bytes, stream, &st);
@@ -579,8 +666,8 @@ static int verify_round_staged_t(const void* const* host_parts, void* const* dev
 }  // extern "C++"
 
 int libraspec_verify_round_staged(const void* const* host_parts, void* const* dev_parts, const size_t* part_bytes,
-                                  void* copy_stream, const uint16_t* kv_new, int32_t* n_accepted_host,
-                                  int32_t* bonus_host, const float* draft_logits, const int32_t* draft_tokens,
+                                  void* copy_stream, const uint16_t* kv_new, uint64_t* rng_host,
+                                  const uint64_t* rng_dev, int32_t* n_accepted_host, int32_t* bonus_host, const float* draft_logits, const int32_t* draft_tokens,
                                   const float* temperature, const float* cost_table, const float* target_logits,
                                   const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
                                   uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V,
@@ -588,7 +675,8 @@ int libraspec_verify_round_staged(const void* const* host_parts, void* const* de
                                   uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat, int32_t* L,
                                   int32_t* n_accepted, int32_t* bonus_token, void* workspace, size_t ws_bytes,
                                   void* stream) {
-  return verify_round_staged_t(host_parts, dev_parts, part_bytes, copy_stream, kv_new, n_accepted_host, bonus_host,
+  return verify_round_staged_t(host_parts, dev_parts, part_bytes, copy_stream, kv_new, rng_host, rng_dev,
+                               n_accepted_host, bonus_host,
                                draft_logits, draft_tokens, temperature, cost_table, target_logits, Q, Kc, Vc, O,
                                n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed, round_offset,
                                seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace, ws_bytes, stream);
@@ -596,7 +684,8 @@ int libraspec_verify_round_staged(const void* const* host_parts, void* const* de
 
 int libraspec_verify_round_staged_bf16(const void* const* host_parts, void* const* dev_parts,
                                        const size_t* part_bytes, void* copy_stream, const uint16_t* kv_new,
-                                       int32_t* n_accepted_host, int32_t* bonus_host, const uint16_t* draft_logits,
+                                       uint64_t* rng_host, const uint64_t* rng_dev, int32_t* n_accepted_host,
+                                       int32_t* bonus_host, const uint16_t* draft_logits,
                                        const int32_t* draft_tokens, const float* temperature,
                                        const float* cost_table, const uint16_t* target_logits,
                                        const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
@@ -605,7 +694,8 @@ int libraspec_verify_round_staged_bf16(const void* const* host_parts, void* cons
                                        uint64_t round_offset, uint32_t seq_offset, float* conf, float* dstat,
                                        int32_t* L, int32_t* n_accepted, int32_t* bonus_token, void* workspace,
                                        size_t ws_bytes, void* stream) {
-  return verify_round_staged_t(host_parts, dev_parts, part_bytes, copy_stream, kv_new, n_accepted_host, bonus_host,
+  return verify_round_staged_t(host_parts, dev_parts, part_bytes, copy_stream, kv_new, rng_host, rng_dev,
+                               n_accepted_host, bonus_host,
                                draft_logits, draft_tokens, temperature, cost_table, target_logits, Q, Kc, Vc, O,
                                n_layers, kv_len, B, K, V, Hq, Hkv, head_dim, S_cap, softmax_scale, seed, round_offset,
                                seq_offset, conf, dstat, L, n_accepted, bonus_token, workspace, ws_bytes, stream);

@@ -157,13 +157,18 @@ __global__ void __launch_bounds__(kRowThreads) accept_decide_kernel(
     const E* __restrict__ target, const E* __restrict__ draft, const int32_t* __restrict__ tokens,
     const float* __restrict__ conf, const float* __restrict__ dstat, const int32_t* __restrict__ Ls,
     const float* __restrict__ temperature, int K, int V, int nsplit, int chunk, uint64_t seed,
-    uint64_t round_offset, uint32_t seq_offset, const RowStat* __restrict__ stat,
+    uint64_t round_offset, uint32_t seq_offset, const uint64_t* __restrict__ rng, const RowStat* __restrict__ stat,
     RacePartial* __restrict__ part, uint32_t* __restrict__ cnt, int32_t* __restrict__ n_accepted,
     int32_t* __restrict__ bonus_token, int* __restrict__ status) {
   __shared__ int sh_n, sh_bonus, sh_ok, last;
   __shared__ float smk[32];
   __shared__ int smi[32];
   const int split = blockIdx.x, b = blockIdx.y;
+  if (rng) {  // the generator's arguments from device memory (a replayed graph of a staged round)
+    seed = rng[0];
+    round_offset = rng[1];
+    seq_offset = (uint32_t)rng[2];
+  }
   if (threadIdx.x < 32) {
     const Decision d = decide<E>(b, K, V, target, tokens, conf, Ls, temperature, stat, seed, round_offset,
                                  seq_offset, status);
@@ -558,11 +563,14 @@ template cudaError_t launch_accept_tree<uint16_t>(const uint16_t*, const int32_t
                                                   const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*,
                                                   int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
 
+// rng (optional, device): {seed, round_offset, seq_offset} read by the
+// kernels in place of the three arguments.
 template <typename T>
 cudaError_t launch_accept(const T* target, const T* draft, const int32_t* tokens, const float* conf,
                           const float* dstat, const int32_t* L, const float* temperature, int B, int K, int V,
                           uint64_t seed, uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted,
-                          int32_t* bonus, char* ws, const WsLayout& lay, cudaStream_t stream) {
+                          int32_t* bonus, char* ws, const WsLayout& lay, cudaStream_t stream,
+                          const uint64_t* rng) {
   if (B == 0) return cudaSuccess;
   const int sms = num_sms_current();
   // the race reads groups of 4 logits: both rows must allow those loads too
@@ -602,20 +610,21 @@ cudaError_t launch_accept(const T* target, const T* draft, const int32_t* tokens
     if (vec)
       accept_decide_kernel<true, T><<<grid, kRowThreads, 0, stream>>>(
           target, draft, tokens, conf, dstat, L, temperature, K, V, nsplit, chunk, seed, round_offset, seq_offset,
-          rstat, part, cnt, n_accepted, bonus, st);
+          rng, rstat, part, cnt, n_accepted, bonus, st);
     else
       accept_decide_kernel<false, T><<<grid, kRowThreads, 0, stream>>>(
           target, draft, tokens, conf, dstat, L, temperature, K, V, nsplit, chunk, seed, round_offset, seq_offset,
-          rstat, part, cnt, n_accepted, bonus, st);
+          rng, rstat, part, cnt, n_accepted, bonus, st);
     return cudaGetLastError();
   }
 }
 template cudaError_t launch_accept<float>(const float*, const float*, const int32_t*, const float*, const float*,
                                           const int32_t*, const float*, int, int, int, uint64_t, uint64_t, uint32_t,
-                                          int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
+                                          int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t,
+                                          const uint64_t*);
 template cudaError_t launch_accept<uint16_t>(const uint16_t*, const uint16_t*, const int32_t*, const float*,
                                              const float*, const int32_t*, const float*, int, int, int, uint64_t,
                                              uint64_t, uint32_t, int32_t*, int32_t*, char*, const WsLayout&,
-                                             cudaStream_t);
+                                             cudaStream_t, const uint64_t*);
 
 }  // namespace libraspec

@@ -138,3 +138,36 @@ def test_staged_round_bf16_logits_matches_device_round():
     np.testing.assert_array_equal(runner.out.n_accepted.cpu().numpy(), n)
     np.testing.assert_array_equal(runner.out.bonus_token.cpu().numpy(), bonus)
     assert lr.libraspec_get_status(runner.ws) == 0
+
+
+def test_staged_round_graph_replays_follow_seed_and_round():
+    """From the second call on, a staged round replays a captured graph; the
+    generator's arguments come from the host buffer, so every round's draws
+    still follow its own seed and round offset (compared with the eager
+    device round)."""
+    w = workloads.WORKLOADS["tiny"].scaled(B=8, temperature=("const", 1.0))
+    kv = workloads.kv_lengths(w)
+    lay = workloads.layer(w, 0, kv, device=cuda())
+    inp = workloads.logits(w)
+    caches = [{"Kc": lay["Kc"].clone(), "Vc": lay["Vc"].clone()}]
+    runner = api.VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, lay["Kc"].shape[2], caches, torch.tensor(kv))
+    h = runner.host_inputs()
+    for name in ("draft_logits", "target_logits", "draft_tokens", "temperature"):
+        h[name].copy_(inp[name])
+    h["cost_table"].copy_(torch.tensor(workloads.cost_table(w)))
+    h["Q"][0].copy_(lay["Q"].cpu())
+    K1 = w.K + 1
+    for b in range(w.B):
+        kvb = int(kv[b])
+        h["kv_new"][0, 0, b].copy_(lay["Kc"][b, :, kvb:kvb + K1].cpu())
+        h["kv_new"][0, 1, b].copy_(lay["Vc"][b, :, kvb:kvb + K1].cpu())
+    seen = set()
+    for r, (seed, ro) in enumerate([(5, 0), (5, 1), (5, 2), (9, 2), (5, 0)]):
+        n, bonus = runner.run_staged(seed=seed, round_offset=ro, seq_offset=3)
+        runner.run_device(seed=seed, round_offset=ro, seq_offset=3)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(runner.out.n_accepted.cpu().numpy(), n)
+        np.testing.assert_array_equal(runner.out.bonus_token.cpu().numpy(), bonus)
+        seen.add(tuple(bonus.tolist()))
+    assert len(seen) >= 3   # different rounds draw differently
+    assert lr.libraspec_get_status(runner.ws) == 0
