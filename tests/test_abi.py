@@ -83,3 +83,34 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(lr, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="not built"):
         lr.load()
+
+
+def test_newer_entry_points_reject_bad_arguments_before_any_launch(lib):
+    P = ctypes.c_void_p
+    fake = P(0x1000)  # never dereferenced: validation fails first
+    arr = (ctypes.c_void_p * 1)(0x1000)
+    # draft trees: node budget above the limit, a missing parent array
+    assert lib.libraspec_verify_attn_tree_layers(arr, arr, arr, 1, fake, fake, fake, 1, lr.MAX_TREE_NODES + 1, 8,
+                                                 2, 64, 1024, 0.1, arr, None, fake, 1 << 30, None) == lr.EINVAL
+    assert lib.libraspec_verify_attn_tree_layers(arr, arr, arr, 1, None, fake, fake, 1, 16, 8, 2, 64, 1024, 0.1,
+                                                 arr, None, fake, 1 << 30, None) == lr.EINVAL
+    assert lib.libraspec_accept_tree(fake, fake, fake, fake, None, 2, 8, 100, 0, 0, 0, fake, fake, fake, fake,
+                                     1 << 30, None) == lr.EINVAL                      # no temperatures
+    # the LM head: model dimension not a multiple of 64, a workspace too small, no tokens for probabilities
+    assert lib.libraspec_lm_head_stats(fake, fake, None, 1, None, 4, 100, 48, fake, fake, None, fake, 1 << 20,
+                                       None) == lr.EUNSUPPORTED
+    assert lib.libraspec_lm_head_stats(fake, fake, None, 1, None, 4, 100, 64, fake, fake, None, fake, 16,
+                                       None) == lr.EINVAL
+    assert lib.libraspec_lm_head_stats(fake, fake, None, 1, None, 4, 100, 64, fake, fake, fake, fake, 1 << 20,
+                                       None) == lr.EINVAL
+    assert lib.libraspec_lm_head_workspace_size(-1, 100) == 0
+    assert lib.libraspec_lm_head_workspace_size(33, 128256) >= 33 * 1002 * 16
+    # the KV append: head dim, unaligned source
+    assert lib.libraspec_kv_append(fake, arr, arr, 1, fake, 1, 5, 2, 96, 64, fake, 256, None) == lr.EUNSUPPORTED
+    assert lib.libraspec_kv_append(P(0x1004), arr, arr, 1, fake, 1, 5, 2, 64, 64, fake, 256, None) == lr.EINVAL
+    # confidence + selection without a cost table
+    assert lib.libraspec_confidence_select(fake, fake, fake, None, 1, 4, 64, fake, fake, fake, fake, 1 << 20,
+                                           None) == lr.EINVAL
+    # the staged round without its parts
+    args = [None] * 18 + [1, fake] + [1, 4, 64, 8, 2, 64, 64] + [0.1, 0, 0, 0] + [fake] * 6 + [1 << 30, None]
+    assert lib.libraspec_verify_round_staged(*args) == lr.EINVAL
