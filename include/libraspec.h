@@ -65,7 +65,7 @@ extern "C" {
 #define LIBRASPEC_ST_BAD_PAGE 0x40   /* a block-table entry outside [0, n_pages)  */
 #define LIBRASPEC_ST_BAD_TREE 0x80   /* a draft-tree parent outside [0, t)        */
 
-/* Limits of this build. */
+/* Limits of the library. */
 #define LIBRASPEC_MAX_K 64           /* drafter block length / d_max             */
 #define LIBRASPEC_MAX_B 4096         /* sequences per call                       */
 #define LIBRASPEC_MAX_TREE_NODES 512 /* nodes below the root of a draft tree      */

@@ -45,10 +45,10 @@ class Workload:
         return dataclasses.replace(self, **kw)
 
 
-# The five workloads (batch 1..64). Values the task leaves open (data seeds of
-# the larger configs, the sampling config's target sigma, the ragged config's
-# odd-sequence temperature and drafter noise, layer counts of the single-layer
-# configs) are fixed here once.
+# The five workloads (batch 1..64). Values their shapes leave open (data seeds
+# of the larger configs, the sampling config's target sigma, the ragged
+# config's odd-sequence temperature and drafter noise, layer counts of the
+# single-layer configs) are fixed here once.
 WORKLOADS = {
     "tiny": Workload("tiny", B=1, K=16, V=32000, Hq=8, Hkv=2, d=64, n_layers=1,
                      kv=("const", 512), temperature=("const", 0.0), target=("normal", 4.0),
