@@ -35,6 +35,7 @@ constexpr uint32_t kLmBTile = kLmBN * kLmBK * 2;  // 16 KB
 constexpr int kLmBarBytes = (2 * kLmMaxStages + 5) * 8 + 16;  // barriers and the tensor-memory slot
 constexpr int kLmSmemMax = 227 * 1024;
 constexpr int kLmTmemCols = 2 * kLmBN;
+constexpr int kLmSub = 2;  // k-slabs per stage (fewer when Dm / 64 is not a multiple)
 constexpr uint32_t kLmIdesc = mma_idesc(kLmBM, kLmBN, 0);
 
 // Shared memory of a ring of `stages` stages of stage_bytes: barriers first,
@@ -54,17 +55,20 @@ struct LmPartial {
 __global__ void __launch_bounds__(kLmThreads, 1) lm_head_stats_kernel(
     const __grid_constant__ CUtensorMap mapH, const __grid_constant__ CUtensorMap mapW,
     const float* __restrict__ temperature, int rows_per_seq, const int32_t* __restrict__ tokens, int M, int V,
-    int Dm, int m_tiles, int n_tiles, int a_rows, int stages, LmPartial* __restrict__ part,
+    int Dm, int m_tiles, int n_tiles, int a_rows, int stages, int sub, LmPartial* __restrict__ part,
     int* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t a_bytes = (uint32_t)a_rows * kLmBK * 2, stage_bytes = a_bytes + kLmBTile;
+  // a stage holds `sub` consecutive k-slabs (H slab, then W slab, each 1024-byte aligned), so every
+  // row of W is read `sub` * 128 contiguous bytes at a time
+  const uint32_t a_bytes = (uint32_t)a_rows * kLmBK * 2, slab_bytes = a_bytes + kLmBTile;
+  const uint32_t stage_bytes = sub * slab_bytes;
   const uint32_t sbase = smem_u32(smem) + lm_ring_offset();
   const uint32_t bFull = smem_u32(smem), bEmpty = bFull + 8 * kLmMaxStages;
   const uint32_t bAccFull = bEmpty + 8 * kLmMaxStages, bAccEmpty = bAccFull + 16, bDrain = bAccEmpty + 16;
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + (2 * kLmMaxStages + 5) * 8);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int items = m_tiles * n_tiles, nk = Dm / kLmBK;
+  const int items = m_tiles * n_tiles, nk = Dm / kLmBK / sub;  // stages per item
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -103,8 +107,11 @@ __global__ void __launch_bounds__(kLmThreads, 1) lm_head_stats_kernel(
           if (!(ok = mbar_wait(bEmpty + 8 * s, ph ^ 1))) break;
           const uint32_t a = sbase + s * stage_bytes;
           mbar_expect_tx(bFull + 8 * s, stage_bytes);
-          tma_load_2d(a, &mapH, bFull + 8 * s, k * kLmBK, m * kLmBM);
-          tma_load_2d(a + a_bytes, &mapW, bFull + 8 * s, k * kLmBK, n * kLmBN);
+          for (int j = 0; j < sub; ++j) {
+            const int kc = (k * sub + j) * kLmBK;
+            tma_load_2d(a + j * slab_bytes, &mapH, bFull + 8 * s, kc, m * kLmBM);
+            tma_load_2d(a + j * slab_bytes + a_bytes, &mapW, bFull + 8 * s, kc, n * kLmBN);
+          }
         }
       }
       if (!ok) raise_status(status, LIBRASPEC_ST_TIMEOUT);
@@ -122,11 +129,13 @@ __global__ void __launch_bounds__(kLmThreads, 1) lm_head_stats_kernel(
           const uint32_t s = it % stages, ph = (it / stages) & 1;
           if (!(ok = mbar_wait(bFull + 8 * s, ph))) break;
           tc_fence_after();
-          const uint32_t a = sbase + s * stage_bytes;
+          for (int j = 0; j < sub; ++j) {
+            const uint32_t a = sbase + s * stage_bytes + j * slab_bytes;
 #pragma unroll
-          for (int kk = 0; kk < kLmBK / 16; ++kk)
-            mma_ss(d, smem_desc(a + kk * 32, 16, 1024), smem_desc(a + a_bytes + kk * 32, 16, 1024), kLmIdesc,
-                   (k | kk) != 0 ? 1u : 0u);
+            for (int kk = 0; kk < kLmBK / 16; ++kk)
+              mma_ss(d, smem_desc(a + kk * 32, 16, 1024), smem_desc(a + a_bytes + kk * 32, 16, 1024), kLmIdesc,
+                     (k | j | kk) != 0 ? 1u : 0u);
+          }
           mma_commit(bEmpty + 8 * s);  // the stage is free once these MMAs have read it
         }
         if (ok) mma_commit(bAccFull + 8 * ab);
@@ -290,8 +299,15 @@ cudaError_t launch_lm_head_stats(const uint16_t* H, const uint16_t* W, const flo
   const int m_tiles = (M + kLmBM - 1) / kLmBM, n_tiles = (V + kLmBN - 1) / kLmBN;
   // one row tile: load only its rows (rounded up to 8), and spend the room on stages
   const int a_rows = m_tiles == 1 ? (M + 7) / 8 * 8 : kLmBM;
-  const int stage_bytes = a_rows * kLmBK * 2 + (int)kLmBTile;
-  int stages = (kLmSmemMax - lm_smem_bytes(0, stage_bytes)) / stage_bytes;
+  const int slab_bytes = a_rows * kLmBK * 2 + (int)kLmBTile;
+  const int nk = Dm / kLmBK;
+  // k-slabs per stage: kLmSub, fewer while they do not divide Dm / 64 or leave under 3 stages
+  int sub = kLmSub, stages = 0;
+  for (;; sub >>= 1) {
+    stages = (kLmSmemMax - lm_smem_bytes(0, sub * slab_bytes)) / (sub * slab_bytes);
+    if (sub == 1 || (nk % sub == 0 && stages >= 3)) break;
+  }
+  const int stage_bytes = sub * slab_bytes;
   if (stages > kLmMaxStages) stages = kLmMaxStages;
   const int smem = lm_smem_bytes(stages, stage_bytes);
   CUtensorMap mapH, mapW;
@@ -308,7 +324,7 @@ cudaError_t launch_lm_head_stats(const uint16_t* H, const uint16_t* W, const flo
   auto* part = reinterpret_cast<LmPartial*>(ws + 256);
   auto* status = reinterpret_cast<int*>(ws);
   lm_head_stats_kernel<<<grid, kLmThreads, smem, stream>>>(mapH, mapW, temperature, rows_per_seq, tokens, M, V, Dm,
-                                                          m_tiles, n_tiles, a_rows, stages, part, status);
+                                                          m_tiles, n_tiles, a_rows, stages, sub, part, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   lm_head_merge_kernel<<<(M + 3) / 4, 128, 0, stream>>>(part, M, V, n_tiles, temperature, rows_per_seq, tokens,
