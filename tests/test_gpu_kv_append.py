@@ -171,3 +171,14 @@ def test_staged_round_graph_replays_follow_seed_and_round():
         seen.add(tuple(bonus.tolist()))
     assert len(seen) >= 3   # different rounds draw differently
     assert lr.libraspec_get_status(runner.ws) == 0
+
+
+def test_kv_append_empty_block_is_a_no_op():
+    g = torch.Generator(device="cuda").manual_seed(4)
+    caches = [{"Kc": _bf((2, 2, 64, 64), g), "Vc": _bf((2, 2, 64, 64), g)}]
+    before = caches[0]["Kc"].clone()
+    ws = lr.Workspace(2, 4, 1, 2, 2, 64, 64, device=cuda())
+    lr.libraspec_kv_append(torch.empty((1, 2, 2, 2, 0, 64), dtype=torch.bfloat16, device=cuda()), caches,
+                           torch.tensor([3, 9], dtype=torch.int32, device=cuda()), ws)
+    torch.cuda.synchronize()
+    assert torch.equal(caches[0]["Kc"], before) and lr.libraspec_get_status(ws) == 0

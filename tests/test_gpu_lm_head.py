@@ -94,3 +94,14 @@ def test_lm_head_rejects_unsupported_model_dim():
     ws = lr.LmHeadWorkspace(4, 100)
     with pytest.raises(lr.LibraspecError):
         lr.libraspec_lm_head_stats(H[:, :48].contiguous(), W[:, :48].contiguous(), ws)
+
+
+def test_lm_head_single_row_and_single_tile_vocabulary(orc):
+    for M, V in ((1, 77), (1, 128), (129, 64)):
+        H, W = _inputs(M, V, 64, seed=M * 1000 + V)
+        ws = lr.LmHeadWorkspace(M, V)
+        tok = torch.arange(M, dtype=torch.int32, device=cuda()) % V
+        out = lr.libraspec_lm_head_stats(H, W, ws, tokens=tok)
+        torch.cuda.synchronize()
+        assert lr.libraspec_get_status(ws) == 0
+        _check(orc, H, W, None, 1, tok.cpu().numpy(), out)

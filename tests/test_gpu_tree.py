@@ -383,3 +383,30 @@ def test_tree_sampling_root_draw_distribution_on_gpu():
     p = torch.softmax(y.double() / T, 0).numpy()
     stat = float(((counts - p * B) ** 2 / (p * B)).sum())
     assert stat < chi2.ppf(1 - 1e-4, V - 1), stat
+
+
+def test_tree_edge_cases_empty_trees_and_fresh_caches(orc):
+    """Trees of zero nodes (only the root), fresh caches (kv_len 0) and one
+    sequence at the node budget, in one batch."""
+    N, Hq, Hkv, d = 40, 8, 2, 128
+    kv = [0, 0, 5, 64, 0]
+    L = [0, N, 0, N, 1]
+    B = len(kv)
+    S = (max(k + l + 1 for k, l in zip(kv, L)) + 63) // 64 * 64
+    parent = workloads.draft_tree(B, N, L, seed=17, shape="ddtree", depth=16)
+    layers = _layers(B, N, Hq, Hkv, d, S, seed=17)
+    outs, lses, status = _run_tree(layers, parent, kv, L, N)
+    assert status == 0
+    O_ref, lse_ref = orc.verify_attn_tree(layers[0]["Q"], layers[0]["Kc"], layers[0]["Vc"], np.array(kv),
+                                          np.array(L), parent)
+    check_attn(outs[0], lses[0], O_ref, lse_ref, L)
+    # the walk of a root-only tree emits the root's argmax
+    V = 500
+    x, tok, _, _ = _walk_inputs(B, N, V, "random", seed=3)
+    ws = lr.Workspace(B, N, V, 1, 1, 64, 1, device=cuda())
+    n, last, bonus = lr.libraspec_accept_tree_greedy(x, _i32(tok), _i32(parent), _i32(L), ws)
+    torch.cuda.synchronize()
+    rn, rlast, rbonus = orc.accept_tree_greedy(x.cpu().numpy(), tok, parent, np.array(L, np.int32))
+    np.testing.assert_array_equal(n.cpu().numpy(), rn)
+    np.testing.assert_array_equal(bonus.cpu().numpy(), rbonus)
+    assert n[0].item() == 0 and bonus[0].item() == int(x[0, 0].argmax())
