@@ -172,10 +172,12 @@ def round_bytes(w, kv, L, temperature, n_acc, logit_bytes=4, L_tree=None):
 # ---------------------------------------------------------------------------
 # the oracle on the host cores (CPU baseline / reference arm)
 # ---------------------------------------------------------------------------
-def oracle_round_time(w, inp_host, layers_host, kv, budget_s):
+def oracle_round_time(w, inp_host, layers_host, kv, budget_s, conf_fn=None, attn_fn=None, variant=""):
     """Time the oracle's round on a bounded sample: the full logits steps and
     one attention layer (scaled to all layers). Repeats the sample until the
-    budget is spent; returns (us per round, threads, sample text)."""
+    budget is spent; returns (us per round, threads, sample text).
+    conf_fn() -> q replaces the confidence from drafter logits (the LM-head
+    variant); attn_fn(layer, L) replaces the dense attention (paged caches)."""
     import oracle
 
     oracle.build()
@@ -186,13 +188,19 @@ def oracle_round_time(w, inp_host, layers_host, kv, budget_s):
     t_end = time.perf_counter() + budget_s
     while True:
         t0 = time.perf_counter()
-        q, _ = oracle.confidence(inp_host["draft_logits"], inp_host["draft_tokens"], inp_host["temperature"])
+        if conf_fn is not None:
+            q = conf_fn()
+        else:
+            q, _ = oracle.confidence(inp_host["draft_logits"], inp_host["draft_tokens"], inp_host["temperature"])
         L, _ = oracle.select_lengths(q, cost)
         oracle.accept(inp_host["target_logits"], inp_host["draft_logits"], inp_host["draft_tokens"], L,
                       inp_host["temperature"], w.philox_seed)
         t1 = time.perf_counter()
         lay = layers_host[len(times_attn) % len(layers_host)]
-        oracle.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L)
+        if attn_fn is not None:
+            attn_fn(lay, L)
+        else:
+            oracle.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L)
         t2 = time.perf_counter()
         times_logits.append(t1 - t0)
         times_attn.append(t2 - t1)
@@ -200,8 +208,8 @@ def oracle_round_time(w, inp_host, layers_host, kv, budget_s):
             break
     per_round = statistics.median(times_logits) + statistics.median(times_attn) * w.n_layers
     sample = ("%d repetition(s) of: confidence, selection and acceptance on the full batch plus ONE of the %d "
-              "attention layers (fp64 C oracle, %d threads); attention time scaled by %d layers" %
-              (len(times_attn), w.n_layers, threads, w.n_layers))
+              "attention layers (fp64 C oracle, %d threads); attention time scaled by %d layers%s" %
+              (len(times_attn), w.n_layers, threads, w.n_layers, variant))
     return per_round * 1e6, threads, sample
 
 
@@ -542,17 +550,42 @@ def run_ours(args, rank, world, local_rank):
         e2e = run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset)
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and not P and not args.lm_head:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+
         # bf16 logits widen exactly to f32 for the oracle
         host = {k: (v.float() if v.dtype == torch.bfloat16 else v).cpu().numpy() for k, v in inp.items()}
         host["cost_table"] = workloads.cost_table(w, kv)
-        lay_host = [{"Q": layers[0]["Q"].cpu(), "Kc": layers[0]["Kc"].cpu(), "Vc": layers[0]["Vc"].cpu()}]
+        conf_fn = attn_fn = None
+        if P:
+            table_np = table.cpu().numpy()
+            lay_host = [{"Q": layers[0]["Q"].cpu(), "Kp": layers[0]["Kp"].cpu(), "Vp": layers[0]["Vp"].cpu()}]
+
+            def attn_fn(lay, L):  # the oracle on the cache the pages describe (gather included)
+                oracle.verify_attn_paged(lay["Q"], lay["Kp"], lay["Vp"], table_np, kv, L)
+        else:
+            lay_host = [{"Q": layers[0]["Q"].cpu(), "Kc": layers[0]["Kc"].cpu(), "Vc": layers[0]["Vc"].cpu()}]
+        if head is not None:
+            H_host, W_host = head["H"].cpu(), head["W"].cpu()
+            tok_host = head["tokens"].cpu().numpy()
+
+            def conf_fn():  # the head's statistics over the full vocabulary, in binary64
+                return oracle.lm_head_stats(H_host, W_host, host["temperature"], w.K, tok_host)[3].reshape(w.B, w.K)
         if N:
             th = {"target_logits": tree["target"].float().cpu().numpy(), "draft_tokens": tree["tokens"].cpu().numpy(),
                   "parent": tree["parent_np"], "L": np.full(w.B, N, np.int32)}
-            us, cores, sample = oracle_tree_round_time(w, host, th, lay_host[0], kv, args.cpu_seconds)
+            lay0 = lay_host[0]
+            if P:
+                S_all = int(table_np.shape[1] * P)
+                lay0 = {"Q": lay0["Q"], "Kc": oracle.gather_pages(lay0["Kp"], table_np, S_all),
+                        "Vc": oracle.gather_pages(lay0["Vp"], table_np, S_all)}
+            us, cores, sample = oracle_tree_round_time(w, host, th, lay0, kv, args.cpu_seconds)
         else:
-            us, cores, sample = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds)
+            variant = "".join([
+                "; the confidence from the hidden states and the LM head" if head is not None else "",
+                "; attention on the cache gathered from its pages" if P else ""])
+            us, cores, sample = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds, conf_fn=conf_fn,
+                                                  attn_fn=attn_fn, variant=variant)
         cpu = {"value": round(us, 1), "unit": "us", "cores": cores, "kind": "oracle", "sample": sample}
 
     lm = None
