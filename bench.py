@@ -461,13 +461,14 @@ def run_ours(args, rank, world, local_rank):
     def step():
         round_graph.replay()
 
-    def step_split(ev_a, ev_b, ev_0):
+    def step_split(ev_a, ev_b, ev_0, ev_c):
         ev_0.record(stream)
         graphs[0].replay()
         ev_a.record(stream)
         graphs[1].replay()
         ev_b.record(stream)
         graphs[2].replay()
+        ev_c.record(stream)
 
     for _ in range(max(3, args.warmup)):
         step()
@@ -487,6 +488,7 @@ def run_ours(args, rank, world, local_rank):
     ev_0 = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
     ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
     ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
+    ev_c = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     pdist.barrier()
     torch.cuda.synchronize()
@@ -499,12 +501,13 @@ def run_ours(args, rank, world, local_rank):
         pdist.barrier()
         # second pass: the same K rounds as three graphs, for the kernels' launch durations
         for i in range(K_steps):
-            step_split(ev_a[i], ev_b[i], ev_0[i])
+            step_split(ev_a[i], ev_b[i], ev_0[i], ev_c[i])
         torch.cuda.synchronize()
     pdist.barrier()
     elapsed_ms = start.elapsed_time(end)
     attn_ms = sum(a.elapsed_time(b) for a, b in zip(ev_a, ev_b))
     select_ms = sum(a.elapsed_time(b) for a, b in zip(ev_0, ev_a))
+    accept_ms = sum(a.elapsed_time(b) for a, b in zip(ev_b, ev_c))
     elapsed_max = pdist.max_over_ranks(elapsed_ms, device=dev)
     if device_status() != 0:
         raise RuntimeError("device status set during the timed steps")
@@ -597,6 +600,16 @@ def run_ours(args, rank, world, local_rank):
               "bytes": head_bytes, "GBps": round(head_bytes / lm_s / 1e9, 1),
               "frac_of_measured_hbm": round(head_bytes / lm_s / 1e9 / hbm_peak, 4),
               "note": "time of the confidence+selection graph; the head's weights dominate its bytes"}
+    # the logits-bound segments: confidence (+ selection) over B*K drafter rows, acceptance over the
+    # verified target rows (+ residual rows); their graph times include the small launches beside them
+    logits = None
+    if head is None:
+        logits = {}
+        for name, nbytes, ms in (("conf_select", by["conf"] + by["select"], select_ms),
+                                 ("accept", by["accept"], accept_ms)):
+            sec = ms / 1000.0 / K_steps
+            logits[name] = {"us": round(sec * 1e6, 3), "bytes": int(nbytes), "GBps": round(nbytes / sec / 1e9, 1),
+                            "frac_of_measured_hbm": round(nbytes / sec / 1e9 / hbm_peak, 4)}
     if rank != 0:
         return
     clk = clocks.summary()
@@ -631,8 +644,10 @@ def run_ours(args, rank, world, local_rank):
         "hbm_frac_of_nominal_8tbs": round(by["total"] / (us_per_round * 1e-6) / 1e9 / NOMINAL_HBM_GBS, 4),
         "roofline": roof,
         "lm_head": lm,
+        "logits_segments": logits,
         "segments_us": {"conf_select": round(select_ms * 1000.0 / K_steps, 3),
-                        "attention": round(attn_ms * 1000.0 / K_steps, 3)},
+                        "attention": round(attn_ms * 1000.0 / K_steps, 3),
+                        "accept": round(accept_ms * 1000.0 / K_steps, 3)},
         "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
                    "samples": clk["samples"]},
         "gpu_launches": launches,
