@@ -151,7 +151,8 @@ int libraspec_confidence_noalloc(const float* draft_logits, const int32_t* draft
                                  int B, int K, int V, float* conf, float* dstat, int32_t* status, void* stream);
 
 /*
- * Steps 1 and 2 in one launch: libraspec_confidence, and as soon as the
+ * Steps 1 and 2 in one launch (Assumption 1's q_k feeding Thm. 4's
+ * criterion, Sec. 3.3-3.4): libraspec_confidence, and as soon as the
  * last of a sequence's K rows is done, that CTA selects the sequence's
  * length exactly as libraspec_select_lengths does (same L, same status
  * bits). Arguments as the two calls; K = 0 only selects.
@@ -324,7 +325,8 @@ int libraspec_verify_attn_tree_paged_layers(const uint16_t* const* Q, const uint
 
 /*
  * Greedy acceptance of a draft tree (the longest root path the target
- * agrees with). Row t of target_logits [B, N+1, V] is the target's
+ * agrees with; the tree drafters of Sec. 2 and Appendix C, verified by the
+ * prefix-match rule of Sec. 3.1 along each root path). Row t of target_logits [B, N+1, V] is the target's
  * distribution after node t (tree layout as above; node t >= 1 carries
  * draft_tokens[b * N + t - 1], draft_tokens [B, N]). From the root, the walk
  * moves to the lowest-numbered child of the current node whose token is the
@@ -349,7 +351,8 @@ int libraspec_accept_tree_greedy_bf16(const uint16_t* target_logits, const int32
 
 /*
  * Acceptance of a draft tree at temperature[b] (temperature [B] f32, >= 0;
- * 0 gives the greedy walk above). At the current node the walk draws the
+ * 0 gives the greedy walk above; Sec. 3.1's lossless verification, applied
+ * to the candidate children of each node). At the current node the walk draws the
  * target's token x from softmax(row / T) and moves to the lowest-numbered
  * child carrying x while there is one; bonus_token is the last draw. Every
  * emitted token is a draw from the target given the prefix it extends, so
@@ -466,7 +469,8 @@ int libraspec_accept_bf16(const uint16_t* target_logits, const uint16_t* draft_l
                           void* stream);
 
 /*
- * The whole round on one stream: confidence -> selection -> n_layers verify
+ * The whole round on one stream (one verification step of Sec. 3.1 with the
+ * length chosen per Thm. 4): confidence -> selection -> n_layers verify
  * attention layers -> acceptance. Q, Kc, Vc, O point to HOST arrays of
  * n_layers DEVICE pointers (layer l uses Q[l], Kc[l], Vc[l], O[l]); lse is a
  * host array of n_layers device pointers or NULL. conf, dstat, L are device
@@ -516,8 +520,9 @@ int libraspec_verify_round_bf16(const uint16_t* draft_logits, const int32_t* dra
  */
 int libraspec_verify_round_staged(const void* const* host_parts, void* const* dev_parts, const size_t* part_bytes,
                                   void* copy_stream, const uint16_t* kv_new, uint64_t* rng_host,
-                                  const uint64_t* rng_dev, int32_t* n_accepted_host, int32_t* bonus_host, const float* draft_logits, const int32_t* draft_tokens,
-                                  const float* temperature, const float* cost_table, const float* target_logits,
+                                  const uint64_t* rng_dev, int32_t* n_accepted_host, int32_t* bonus_host,
+                                  const float* draft_logits, const int32_t* draft_tokens, const float* temperature,
+                                  const float* cost_table, const float* target_logits,
                                   const uint16_t* const* Q, uint16_t* const* Kc, uint16_t* const* Vc,
                                   uint16_t* const* O, int n_layers, const int32_t* kv_len, int B, int K, int V,
                                   int Hq, int Hkv, int head_dim, int S_cap, float softmax_scale, uint64_t seed,
