@@ -449,8 +449,11 @@ int libraspec_kv_append_paged(const uint16_t* kv_new, uint16_t* const* Kp, uint1
  * [B,K] i32, conf [B,K] f32 and dstat [B,K,2] f32 from libraspec_confidence
  * (may be NULL when every temperature is 0), L [B] i32, temperature [B] f32;
  * n_accepted [B] i32 out, bonus_token [B] i32 out.
- * Reads target rows 0..L[b] once, plus one or two V-rows per sampling
- * sequence for its draw.
+ * Reads target rows 0..L[b] of a greedy sequence once; a sampling sequence
+ * reads rows 0..L[b]-1 once, then target row L[b] for its bonus draw or
+ * target and drafter rows r for its residual draw. Three launches on the
+ * stream: the plan of the row slices (one CTA), the row statistics with the
+ * decisions, and the draws.
  */
 int libraspec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
                      const float* conf, const float* dstat, const int32_t* L, const float* temperature, int B,

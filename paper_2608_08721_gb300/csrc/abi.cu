@@ -36,7 +36,10 @@ cudaError_t launch_accept_tree(const T*, const int32_t*, const int32_t*, const i
 template <typename T>
 cudaError_t launch_accept(const T*, const T*, const int32_t*, const float*, const float*, const int32_t*,
                           const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, char*,
-                          const WsLayout&, cudaStream_t, const uint64_t*);
+                          const WsLayout&, cudaStream_t, const uint64_t*, bool);
+template <typename T>
+cudaError_t launch_accept_plan(const T*, const T*, const float*, const float*, const int32_t*, const float*, int,
+                               int, int, int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
 
 int num_sms_current() {
   static int cached_dev = -1, cached_sms = 0;
@@ -309,7 +312,8 @@ template <typename T>
 static int accept_t(const T* target_logits, const T* draft_logits, const int32_t* draft_tokens, const float* conf,
                     const float* dstat, const int32_t* L, const float* temperature, int B, int K, int V, uint64_t seed,
                     uint64_t round_offset, uint32_t seq_offset, int32_t* n_accepted, int32_t* bonus_token,
-                    void* workspace, size_t ws_bytes, void* stream, const uint64_t* rng = nullptr) {
+                    void* workspace, size_t ws_bytes, void* stream, const uint64_t* rng = nullptr,
+                    bool plan_ready = false) {
   if (!shapes_ok(B, K, V)) return LIBRASPEC_EINVAL;
   if (B == 0) return LIBRASPEC_OK;
   if (!target_logits || (!draft_logits && K > 0) || (!draft_tokens && K > 0) || !L || !temperature ||
@@ -321,7 +325,8 @@ static int accept_t(const T* target_logits, const T* draft_logits, const int32_t
   if (!ws_ok(workspace, ws_bytes, lay)) return LIBRASPEC_EINVAL;
   return from_cuda(launch_accept<T>(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V,
                                     seed, round_offset, seq_offset, n_accepted, bonus_token,
-                                    static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream), rng));
+                                    static_cast<char*>(workspace), lay, static_cast<cudaStream_t>(stream), rng,
+                                    plan_ready));
 }
 }  // extern "C++"
 
@@ -535,6 +540,12 @@ static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, co
     rc = from_cuda(launch_select(conf, cost_table, B, K, L, ws, lay, s));
   }
   if (rc != LIBRASPEC_OK) return rc;
+  // the acceptance plan needs only L and the temperatures: it runs here, off
+  // the acceptance's critical path
+  const bool plan = target_logits != nullptr && (draft_logits != nullptr || K == 0) && aligned(target_logits, sizeof(T));
+  if (plan && (rc = from_cuda(launch_accept_plan<T>(target_logits, draft_logits, conf, dstat, L, temperature, B, K,
+                                                    V, n_accepted, bonus_token, ws, lay, s))) != LIBRASPEC_OK)
+    return rc;
   if ((rc = staged_wait(st, 1, s)) != LIBRASPEC_OK) return rc;
   if (st && (rc = from_cuda(launch_kv_append(st->kv_new, const_cast<uint16_t* const*>(Kc),
                                              const_cast<uint16_t* const*>(Vc), n_layers, kv_len, nullptr, 0, 0, 0, B,
@@ -546,7 +557,7 @@ static int verify_round_t(const T* draft_logits, const int32_t* draft_tokens, co
   if (rc != LIBRASPEC_OK) return rc;
   if ((rc = staged_wait(st, 2, s)) != LIBRASPEC_OK) return rc;
   rc = accept_t(target_logits, draft_logits, draft_tokens, conf, dstat, L, temperature, B, K, V, seed, round_offset,
-                seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream, st ? st->rng_dev : nullptr);
+                seq_offset, n_accepted, bonus_token, workspace, ws_bytes, stream, st ? st->rng_dev : nullptr, plan);
   if (rc != LIBRASPEC_OK || !st) return rc;
   cudaError_t e = cudaMemcpyAsync(st->n_host, n_accepted, sizeof(int32_t) * B, cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(st->bonus_host, bonus_token, sizeof(int32_t) * B, cudaMemcpyDeviceToHost, s);

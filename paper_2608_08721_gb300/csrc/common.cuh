@@ -5,6 +5,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <algorithm>
+
 #include "libraspec.h"
 
 namespace libraspec {
@@ -23,6 +25,7 @@ constexpr int kAttnMaxCtas = 192;     // persistent attention grid cap (one CTA 
 constexpr int kAttnRows = 128;        // query rows per attention row group (at most)
 constexpr int kAttnTileKeys = 64;     // keys per KV tile
 constexpr int kAttnMaxLayers = LIBRASPEC_ATTN_LAYERS_PER_LAUNCH;  // layers per attention launch
+constexpr int kAccMaxGrid = 6144;     // acceptance rows grid cap (4 waves of 8 CTAs on <= 192 SMs)
 
 struct RowPartial {      // one CTA's share of a logit row
   float m;               // max
@@ -41,8 +44,30 @@ struct RacePartial {
   int idx;
 };
 
+// A race candidate carried without the row's normaliser: the key of token v
+// is E_v * 2^(-y_v c) (E_v = -ln u_v, c = log2(e) / T), compared between two
+// candidates as E_a < E_b * 2^((y_a - y_b) c).
+struct RaceCand {
+  float E;
+  float y;
+  int idx;
+  int pad;
+};
+
+// The draw that ends a sampling sequence's acceptance: mode 1, the bonus
+// draw from target row n = L_b (all drafts accepted); mode 2, the residual
+// draw max(0, p_n - q_n) after a rejection at n (with row n's max and
+// normaliser); mode 0, none (a greedy sequence, or one without units).
+struct ResEntry {
+  int n;
+  int mode;
+  float mp;     // max of target row n (mode 2)
+  float invZp;  // 1 / sum of exp((y - mp) / T) of target row n (mode 2)
+};
+
 struct WsLayout {
   size_t status, conf_part, conf_cnt, seq_cnt, row_part, row_cnt, row_stat, race_part, race_cnt;
+  size_t acc_seq, acc_yx, acc_res, acc_ready, acc_plan;
   size_t attn_o, attn_ml, attn_cnt, tree_vis, total;
   int max_items, max_groups;
 };
@@ -68,8 +93,16 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.row_part = take(rows_t * kRowMaxSplits * sizeof(RowPartial));
   w.row_cnt = take(rows_t * sizeof(uint32_t));
   w.row_stat = take(rows_t * sizeof(RowStat));
-  w.race_part = take(size_t(B) * kRaceMaxSplits * sizeof(RacePartial));
+  w.race_part = take(size_t(B) * kRaceMaxSplits * sizeof(RaceCand));
   w.race_cnt = take(size_t(B) * sizeof(uint32_t));
+  // acceptance: slices done per sequence, the target logit at each drafted
+  // token, and each sequence's residual draw (or none)
+  w.acc_seq = take(size_t(B) * sizeof(uint32_t));
+  w.acc_yx = take(rows_t * sizeof(float));
+  w.acc_res = take(size_t(B) * sizeof(ResEntry));
+  w.acc_ready = take(size_t(B) * sizeof(uint32_t));  // res[b] published
+  // the acceptance plan: a header, then one 8-byte descriptor per unit
+  w.acc_plan = take(16 + 8 * std::max(size_t(kAccMaxGrid), rows_t));
   // two partial slots per attention CTA (its first and its last item), in two
   // buffers that alternate with the layer parity
   w.attn_o = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * d * sizeof(float));
@@ -127,6 +160,20 @@ __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// c = log2(e) / T in binary32 arithmetic alone (GB300 runs binary64 at a
+// small fraction of the binary32 rate, so one binary64 division per thread
+// costs more than the thread's share of a logit row). log2(e) = hi + lo; the
+// rounded quotient q = hi / T is corrected once by the exact remainder
+// hi - q T (an FMA) plus lo: the result is log2(e) / T rounded to binary32,
+// up to a residual far below half an ulp.
+__device__ __forceinline__ float log2e_over(float T) {
+  const float hi = 1.44269502162933349609375f;  // binary32 log2(e)
+  const float lo = 1.925963033500011e-08f;      // log2(e) - hi
+  const float q = __fdiv_rn(hi, T);
+  const float r = __fadd_rn(__fmaf_rn(-q, T, hi), lo);
+  return __fmaf_rn(r, __frcp_rn(T), q);
 }
 
 // Streaming 128-bit load that does not allocate in L1.

@@ -96,7 +96,7 @@ __global__ void __launch_bounds__(kRowThreads) conf_kernel(
   const int b = row / K;
   const float tb = temperature[b];
   const float T = tb > 0.f ? tb : 1.f;
-  const float c = (float)(1.4426950408889634 / (double)T);
+  const float c = log2e_over(T);
   const E* xr = x + (size_t)row * V;
   const int c0 = split * chunk, c1 = min(V, c0 + chunk);
 

@@ -160,7 +160,7 @@ __global__ void __launch_bounds__(kLmThreads, 1) lm_head_stats_kernel(
       const bool valid = grow < M;
       float T = (valid && temperature) ? temperature[grow / rows_per_seq] : 1.f;
       if (!(T > 0.f)) T = 1.f;
-      const float c = (float)(1.4426950408889634 / (double)T);
+      const float c = log2e_over(T);
       const int tok = (valid && tokens) ? tokens[grow] : -1;
       const int v0 = n * kLmBN;
       float mrun = -INFINITY, z = 0.f, xt = __int_as_float(0x7fc00000);
@@ -235,7 +235,7 @@ __global__ void __launch_bounds__(128) lm_head_merge_kernel(const LmPartial* __r
   const LmPartial* p = part + (size_t)r * n_tiles;
   float T = temperature ? temperature[r / rows_per_seq] : 1.f;
   if (!(T > 0.f)) T = 1.f;
-  const double c = (double)(float)(1.4426950408889634 / (double)T);
+  const double c = (double)log2e_over(T);
   float mx = -INFINITY;
   int arg = 0x7fffffff;
   for (int n = lane; n < n_tiles; n += 32) argmax_combine(mx, arg, __ldg(&p[n].m), __ldg(&p[n].arg));

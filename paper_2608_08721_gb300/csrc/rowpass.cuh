@@ -61,15 +61,24 @@ struct ArgAcc {
   }
 };
 
+// Logit `watch` of a group of four starting at index i0, if it lies there.
+__device__ __forceinline__ void watch4(float4 f, int i0, int watch, float& watched) {
+  const unsigned d = (unsigned)(watch - i0);
+  if (d < 4u) watched = d == 0 ? f.x : d == 1 ? f.y : d == 2 ? f.z : f.w;
+}
+
 // Stream x[c0, c1) of logits of type T (c0 a multiple of kRowAlign). VEC: x
 // is 16-byte aligned and the row length a multiple of the elements one
-// 128-bit load holds, so 128-bit loads cover the slice.
-template <bool SUM, bool ARG, bool VEC, typename T>
+// 128-bit load holds, so 128-bit loads cover the slice. WATCH: the thread
+// that streams logit `watch` also keeps it in `watched` (a drafted token's
+// logit, read with the stream instead of by a dependent load).
+template <bool SUM, bool ARG, bool VEC, typename T, bool WATCH = false>
 __device__ __forceinline__ void row_slice_pass(const T* __restrict__ x, int c0, int c1, float c, SumAcc& sa,
-                                               ArgAcc& aa) {
+                                               ArgAcc& aa, int watch = -1, float* watched = nullptr) {
   using LT = Logit<T>;
   constexpr int W = LT::kVec;  // elements per 128-bit load
   const int tid = threadIdx.x;
+  float wv = 0.f;
   if (VEC) {
     const int g0 = c0 / W, g1 = c1 / W;  // groups of W
     int g = g0 + tid;
@@ -85,6 +94,7 @@ __device__ __forceinline__ void row_slice_pass(const T* __restrict__ x, int c0, 
           const float4 f = make_float4(v[u][h], v[u][h + 1], v[u][h + 2], v[u][h + 3]);
           if (SUM) sa.add4(f, c);
           if (ARG) aa.add4(f, W * (g + u * kRowThreads) + h);
+          if (WATCH) watch4(f, W * (g + u * kRowThreads) + h, watch, wv);
         }
     }
     for (; g < g1; g += kRowThreads) {
@@ -95,6 +105,7 @@ __device__ __forceinline__ void row_slice_pass(const T* __restrict__ x, int c0, 
         const float4 f = make_float4(v[h], v[h + 1], v[h + 2], v[h + 3]);
         if (SUM) sa.add4(f, c);
         if (ARG) aa.add4(f, W * g + h);
+        if (WATCH) watch4(f, W * g + h, watch, wv);
       }
     }
   } else {
@@ -102,8 +113,12 @@ __device__ __forceinline__ void row_slice_pass(const T* __restrict__ x, int c0, 
       const float v = LT::stream1(x + i);
       if (SUM) sa.add1(v, c);
       if (ARG) aa.add1(v, i);
+      if (WATCH && i == watch) wv = v;
     }
   }
+  if (WATCH && watch >= c0 && watch < c1 && (VEC ? ((watch / W) - c0 / W) % kRowThreads == tid
+                                                 : (watch - c0) % kRowThreads == tid))
+    *watched = wv;
 }
 
 // Combine the (m, s) pairs of all threads of the CTA; result valid in thread 0.
