@@ -2,10 +2,12 @@
 
 One step = one verify round over one batch: drafter confidence + length
 selection, every verify-attention layer, acceptance. Default workload: the
-8B-class greedy round (B=1, K=16, V=128256, 32 layers of GQA 32/8 attention
-over a 4096-token cache).
+ragged heavy batch (B=64 sequences, K=32, V=128256, GQA 32/8 attention over
+KV lengths log-uniform in [512, 32768], greedy and T=0.8 sequences
+alternating); the sampling batch (B=16) and the 8B-class greedy round (B=1,
+32 layers) are measured in the same run under "also".
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--also A,B] [--impl ours|reference]
 
 Variants of the round (the default is the chain draft on dense caches):
   --selector alpha   Algorithm 1's alpha-mode length search instead of Thm. 4's scan;
@@ -48,7 +50,10 @@ def parse():
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=0, help="timed steps (0: enough for ~2 s)")
     p.add_argument("--warmup", type=int, default=20)
-    p.add_argument("--config", default="8b")
+    p.add_argument("--config", default="ragged")
+    p.add_argument("--also", default="sampling,8b",
+                   help="workloads also measured in the same run, each under its own key (empty: none)")
+    p.add_argument("--also-steps", type=int, default=20, help="timed rounds of each 'also' workload")
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--e2e-steps", type=int, default=50)
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -172,17 +177,31 @@ def round_bytes(w, kv, L, temperature, n_acc, logit_bytes=4, L_tree=None):
 # ---------------------------------------------------------------------------
 # the oracle on the host cores (CPU baseline / reference arm)
 # ---------------------------------------------------------------------------
-def oracle_round_time(w, inp_host, layers_host, kv, budget_s, conf_fn=None, attn_fn=None, variant=""):
+def _subset(w, inp_host, layers_host, kv, seqs):
+    """The first ``seqs`` sequences of the batch (host inputs and one layer each)."""
+    sub = {k: (v[:seqs] if k != "cost_table" else v) for k, v in inp_host.items()}
+    lays = [{k: v[:seqs] for k, v in lay.items()} for lay in layers_host]
+    return w.scaled(B=seqs), sub, lays, kv[:seqs]
+
+
+def oracle_round_time(w, inp_host, layers_host, kv, budget_s, conf_fn=None, attn_fn=None, variant="",
+                      threads=None, seqs=None):
     """Time the oracle's round on a bounded sample: the full logits steps and
     one attention layer (scaled to all layers). Repeats the sample until the
     budget is spent; returns (us per round, threads, sample text).
     conf_fn() -> q replaces the confidence from drafter logits (the LM-head
-    variant); attn_fn(layer, L) replaces the dense attention (paged caches)."""
+    variant); attn_fn(layer, L) replaces the dense attention (paged caches).
+    threads: OpenMP threads (default: all cores). seqs: time the first seqs
+    sequences only and scale the time by B / seqs."""
     import oracle
 
     oracle.build()
-    threads = os.cpu_count() or 1
+    threads = threads or (os.cpu_count() or 1)
     oracle.set_threads(threads)
+    B = w.B
+    if seqs and seqs < B:
+        w, inp_host, layers_host, kv = _subset(w, inp_host, layers_host, kv, seqs)
+    scale = B / w.B
     cost = np.asarray(inp_host["cost_table"], np.float64)
     times_logits, times_attn = [], []
     t_end = time.perf_counter() + budget_s
@@ -206,11 +225,31 @@ def oracle_round_time(w, inp_host, layers_host, kv, budget_s, conf_fn=None, attn
         times_attn.append(t2 - t1)
         if time.perf_counter() > t_end or len(times_attn) >= 50:
             break
-    per_round = statistics.median(times_logits) + statistics.median(times_attn) * w.n_layers
-    sample = ("%d repetition(s) of: confidence, selection and acceptance on the full batch plus ONE of the %d "
-              "attention layers (fp64 C oracle, %d threads); attention time scaled by %d layers%s" %
-              (len(times_attn), w.n_layers, threads, w.n_layers, variant))
+    per_round = (statistics.median(times_logits) + statistics.median(times_attn) * w.n_layers) * scale
+    sample = ("%d repetition(s) of: confidence, selection and acceptance on %s plus ONE of the %d "
+              "attention layers (fp64 C oracle, %d thread%s); attention time scaled by %d layers%s%s" %
+              (len(times_attn), "the full batch" if scale == 1 else "%d of the %d sequences" % (w.B, B),
+               w.n_layers, threads, "" if threads == 1 else "s", w.n_layers,
+               "" if scale == 1 else ", the round's time scaled by %d/%d sequences" % (B, w.B), variant))
     return per_round * 1e6, threads, sample
+
+
+def oracle_flags(w, host, L_gpu, n_gpu, bonus_gpu):
+    """Oracle flags of the chain round (near-threshold selections and draws)
+    and the GPU's disagreements with the oracle outside them. The acceptance
+    is compared given the GPU's lengths."""
+    import oracle
+
+    oracle.build()
+    oracle.set_threads(os.cpu_count() or 1)
+    q, _ = oracle.confidence(host["draft_logits"], host["draft_tokens"], host["temperature"])
+    L, sflag = oracle.select_lengths(q, np.asarray(host["cost_table"], np.float64))
+    n, bonus, aflag = oracle.accept(host["target_logits"], host["draft_logits"], host["draft_tokens"],
+                                    L_gpu.astype(np.int32), host["temperature"], w.philox_seed)
+    sel_bad = (L != L_gpu) & (sflag == 0)
+    acc_bad = ((n != n_gpu) | (bonus != bonus_gpu)) & (aflag == 0)
+    return {"sequences": int(w.B), "select_flagged": int(sflag.sum()), "accept_flagged": int(aflag.sum()),
+            "select_mismatch_unflagged": int(sel_bad.sum()), "accept_mismatch_unflagged": int(acc_bad.sum())}
 
 
 def oracle_tree_round_time(w, host, tree_host, layer_host, kv, budget_s):
@@ -302,9 +341,10 @@ def run_reference(args, rank, world):
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
-def traffic_record(kernel_file):
-    """DRAM bytes per launch of the dominant kernel from the committed ncu
-    summary, if it was taken on the current kernel source."""
+def attn_profile_record(kernel_file, workload):
+    """ncu figures of the attention kernel on ``workload`` from the committed
+    record (DRAM traffic per launch, tensor-pipe share), if they were taken on
+    the current kernel source."""
     path = os.path.join(ROOT, "profiles", "verify_attn_traffic.json")
     try:
         rec = json.load(open(path))
@@ -313,24 +353,58 @@ def traffic_record(kernel_file):
     sha = hashlib.sha256(open(kernel_file, "rb").read()).hexdigest()
     if rec.get("kernel_source_sha256") != sha:
         return None
-    return rec
+    return rec.get("workloads", {}).get(workload)
 
 
-def run_ours(args, rank, world, local_rank):
+def host_link(nbytes, dev):
+    """Pinned host -> device copy rate: one copy of nbytes, and the same bytes
+    as three copies on three streams (the staged round's parts). Median of 5."""
+    import torch
+
+    nbytes = int(nbytes) // 16 * 16
+    src = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    dst = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    streams = [torch.cuda.Stream(device=dev) for _ in range(3)]
+    third = nbytes // 3 // 16 * 16
+    cuts = [0, third, 2 * third, nbytes]
+
+    def one():
+        dst.copy_(src, non_blocking=True)
+
+    def three():
+        cur = torch.cuda.current_stream()
+        for i, st in enumerate(streams):
+            st.wait_stream(cur)
+            with torch.cuda.stream(st):
+                dst[cuts[i]:cuts[i + 1]].copy_(src[cuts[i]:cuts[i + 1]], non_blocking=True)
+        for st in streams:
+            cur.wait_stream(st)
+
+    out = {"bytes": nbytes}
+    for name, fn in (("single_copy", one), ("three_streams", three)):
+        fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(5):
+            t0 = time.perf_counter()
+            fn()
+            torch.cuda.synchronize()
+            ts.append(time.perf_counter() - t0)
+        out[name + "_GBps"] = round(nbytes / statistics.median(ts) / 1e9, 1)
+    return out
+
+
+def measure_workload(args, w, dev, rank, world, local_rank, steps, primary):
+    """One workload: the timed rounds (one CUDA graph each), a second pass of
+    the same rounds as three graphs for the segments, the attention roofline,
+    the logits segments, the end-to-end round through the host API, the
+    oracle's flags and (primary, rank 0, one process) the CPU baseline."""
     import torch
 
     from paper_2608_08721_gb300 import binding as lr
-    from paper_2608_08721_gb300 import build as cuda_build
     from paper_2608_08721_gb300 import dist as pdist
     from paper_2608_08721_gb300 import workloads
-    from paper_2608_08721_gb300.api import VerifyRound
 
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if rank == 0 or not os.path.exists(lr.LIB_PATH):
-        cuda_build.build()
-    pdist.barrier()
-    w = workloads.WORKLOADS[args.config]
     kv = workloads.kv_lengths(w)
     seq_offset = rank * w.B  # weak scaling: each rank verifies its own B sequences
     inp = workloads.logits(w, device=dev)
@@ -432,24 +506,36 @@ def run_ours(args, rank, world, local_rank):
                             inp["temperature"], w.philox_seed, ws, seq_offset=seq_offset, n_accepted=n_acc,
                             bonus_token=bonus)
 
+    # the plain chain round is the library's one-call round (the acceptance plan runs before the
+    # attention layers); the variants chain their step calls
+    one_call = not (N or P or head is not None or args.selector != "gain")
+    outs = lr.RoundOutputs(conf, dstat, L, n_acc, bonus, Os, None) if one_call else None
+
+    def seg_round():
+        if one_call:
+            lr.libraspec_verify_round(inp["draft_logits"], inp["draft_tokens"], inp["temperature"], cost,
+                                      inp["target_logits"], layers, kv_t, w.philox_seed, ws, seq_offset=seq_offset,
+                                      outputs=outs)
+        else:
+            seg_select()
+            seg_attn()
+            seg_accept()
+
     def device_status():
         st = lr.libraspec_get_status(ws) | (lr.libraspec_get_status(head["ws"]) if head is not None else 0)
         return st | (lr.libraspec_get_status(tree["ws"]) if N else 0)
 
-    # eager warm-up (also configures kernels), then capture three graphs
+    # eager warm-up (also configures kernels), then capture the graphs
     for _ in range(3):
+        seg_round()
         seg_select(); seg_attn(); seg_accept()
     torch.cuda.synchronize()
     if device_status() != 0:
         raise RuntimeError("device status set during warm-up")
-    # the timed step: the whole round in one CUDA graph; the same round split
-    # into three graphs (events between) times the segments in a second pass
     side = torch.cuda.Stream(device=dev)
     round_graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(round_graph, stream=side):
-        seg_select()
-        seg_attn()
-        seg_accept()
+        seg_round()
     graphs = []
     for seg in (seg_select, seg_attn, seg_accept):
         gr = torch.cuda.CUDAGraph()
@@ -457,9 +543,6 @@ def run_ours(args, rank, world, local_rank):
             seg()
         graphs.append(gr)
     stream = torch.cuda.current_stream()
-
-    def step():
-        round_graph.replay()
 
     def step_split(ev_a, ev_b, ev_0, ev_c):
         ev_0.record(stream)
@@ -471,36 +554,33 @@ def run_ours(args, rank, world, local_rank):
         ev_c.record(stream)
 
     for _ in range(max(3, args.warmup)):
-        step()
+        round_graph.replay()
         for gr in graphs:
             gr.replay()
     torch.cuda.synchronize()
-    # steps: enough for ~2 s of timed work unless given
-    if args.steps > 0:
-        K_steps = args.steps
-    else:
+    if steps <= 0:  # enough for ~2 s of timed work
         t0 = time.perf_counter()
         for _ in range(20):
-            step()
+            round_graph.replay()
         torch.cuda.synchronize()
         per = (time.perf_counter() - t0) / 20
-        K_steps = int(min(20000, max(50, 2.0 / max(per, 1e-6))))
-    ev_0 = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
-    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
-    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
-    ev_c = [torch.cuda.Event(enable_timing=True) for _ in range(K_steps)]
+        steps = int(min(20000, max(50, 2.0 / max(per, 1e-6))))
+    ev_0 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ev_c = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     pdist.barrier()
     torch.cuda.synchronize()
     with ClockSampler(physical_gpu(local_rank)) as clocks:
         start.record(stream)
-        for i in range(K_steps):
-            step()
+        for _ in range(steps):
+            round_graph.replay()
         end.record(stream)
         torch.cuda.synchronize()
         pdist.barrier()
-        # second pass: the same K rounds as three graphs, for the kernels' launch durations
-        for i in range(K_steps):
+        # second pass: the same rounds as three graphs, for the kernels' launch durations
+        for i in range(steps):
             step_split(ev_a[i], ev_b[i], ev_0[i], ev_c[i])
         torch.cuda.synchronize()
     pdist.barrier()
@@ -514,24 +594,26 @@ def run_ours(args, rank, world, local_rank):
 
     Lh = L.cpu().numpy()
     nh = n_acc.cpu().numpy()
+    bh = bonus.cpu().numpy()
     temp = inp["temperature"].cpu().numpy()
     L_tree = np.full(w.B, N, np.int64) if N else None
     by = round_bytes(w, kv, Lh, temp, nh, logit_bytes=2 if args.logits == "bf16" else 4, L_tree=L_tree)
-    us_per_round = elapsed_ms * 1000.0 / K_steps
+    us_per_round = elapsed_ms * 1000.0 / steps
     # one persistent attention launch runs up to ATTN_LAYERS_PER_LAUNCH layers
     attn_launches = -(-w.n_layers // ATTN_LAYERS_PER_LAUNCH)
-    attn_launch_s = attn_ms / 1000.0 / (K_steps * attn_launches)
+    attn_launch_s = attn_ms / 1000.0 / (steps * attn_launches)
     attn_bytes_launch = by["attn_per_launch"] * w.n_layers / attn_launches
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks["hbm_gbs"])
     tensor_peak = float(peaks.get("bf16_tflops_sustained") or peaks.get("bf16_tflops") or 1700.0)
     achieved = attn_bytes_launch / attn_launch_s / 1e9
-    trec = None
+    prof = None
     if not N and not P:
-        trec = traffic_record(os.path.join(ROOT, "paper_2608_08721_gb300", "csrc", "attn.cu"))
+        prof = attn_profile_record(os.path.join(ROOT, "paper_2608_08721_gb300", "csrc", "attn.cu"), w.name)
     roof = {"kernel": "verify_attn", "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
             "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
-            "traffic": None if trec is None else trec.get("traffic_bytes_per_launch"),
+            "traffic": None if prof is None else prof.get("traffic_bytes_per_launch"),
+            "tensor_pipe_pct": None if prof is None else prof.get("tensor_pipe_pct"),
             "algorithmic_bytes_per_launch": attn_bytes_launch,
             "layers_per_launch": round(w.n_layers / attn_launches, 2),
             "launch_us": round(attn_launch_s * 1e6, 3),
@@ -550,15 +632,26 @@ def run_ours(args, rank, world, local_rank):
     # end to end through the public API with host buffers (the chain round on dense caches)
     e2e = None
     if args.e2e_steps > 0 and not N and not P:
-        e2e = run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset)
+        e2e = run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset, steps=args.e2e_steps if primary else 5)
+        if primary:
+            e2e["host_link"] = host_link(e2e["h2d_bytes_per_step"], dev)
+            best = max(e2e["host_link"]["single_copy_GBps"], e2e["host_link"]["three_streams_GBps"])
+            e2e["host_link"]["copy_us_at_best_rate"] = round(e2e["h2d_bytes_per_step"] / best / 1e3, 1)
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        import oracle
-
+    host = None
+    if rank == 0 and world == 1 and (not args.no_cpu_baseline or not (N or head is not None)):
         # bf16 logits widen exactly to f32 for the oracle
         host = {k: (v.float() if v.dtype == torch.bfloat16 else v).cpu().numpy() for k, v in inp.items()}
         host["cost_table"] = workloads.cost_table(w, kv)
+
+    flags = None
+    if host is not None and not N and head is None and args.selector == "gain":
+        flags = oracle_flags(w, host, Lh, nh, bh)
+
+    cpu = None
+    if primary and host is not None and not args.no_cpu_baseline:
+        import oracle
+
         conf_fn = attn_fn = None
         if P:
             table_np = table.cpu().numpy()
@@ -583,19 +676,25 @@ def run_ours(args, rank, world, local_rank):
                 lay0 = {"Q": lay0["Q"], "Kc": oracle.gather_pages(lay0["Kp"], table_np, S_all),
                         "Vc": oracle.gather_pages(lay0["Vp"], table_np, S_all)}
             us, cores, sample = oracle_tree_round_time(w, host, th, lay0, kv, args.cpu_seconds)
+            cpu = {"value": round(us, 1), "unit": "us", "cores": cores, "kind": "oracle", "sample": sample}
         else:
             variant = "".join([
                 "; the confidence from the hidden states and the LM head" if head is not None else "",
                 "; attention on the cache gathered from its pages" if P else ""])
-            us, cores, sample = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds, conf_fn=conf_fn,
+            us, cores, sample = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds * 0.6, conf_fn=conf_fn,
                                                   attn_fn=attn_fn, variant=variant)
-        cpu = {"value": round(us, 1), "unit": "us", "cores": cores, "kind": "oracle", "sample": sample}
+            cpu = {"value": round(us, 1), "unit": "us", "cores": cores, "kind": "oracle", "sample": sample}
+            if conf_fn is None and attn_fn is None:
+                # single-threaded, on a subset of the batch (about 1/16 of its sequences), scaled
+                us1, _, sample1 = oracle_round_time(w, host, lay_host, kv, args.cpu_seconds * 0.4, threads=1,
+                                                    seqs=max(1, w.B // 16))
+                cpu["single_thread"] = {"value": round(us1, 1), "unit": "us", "cores": 1, "sample": sample1}
 
     lm = None
     if head is not None:
         # the conf+select graph is the head's GEMM plus a selection of a few microseconds
         head_bytes = (w.V + w.B * w.K) * w.hidden * 2
-        lm_s = select_ms / 1000.0 / K_steps
+        lm_s = select_ms / 1000.0 / steps
         lm = {"kernel": "lm_head_stats (tcgen05 GEMM, statistics in the epilogue)", "us": round(lm_s * 1e6, 3),
               "bytes": head_bytes, "GBps": round(head_bytes / lm_s / 1e9, 1),
               "frac_of_measured_hbm": round(head_bytes / lm_s / 1e9 / hbm_peak, 4),
@@ -607,57 +706,108 @@ def run_ours(args, rank, world, local_rank):
         logits = {}
         for name, nbytes, ms in (("conf_select", by["conf"] + by["select"], select_ms),
                                  ("accept", by["accept"], accept_ms)):
-            sec = ms / 1000.0 / K_steps
+            sec = ms / 1000.0 / steps
             logits[name] = {"us": round(sec * 1e6, 3), "bytes": int(nbytes), "GBps": round(nbytes / sec / 1e9, 1),
                             "frac_of_measured_hbm": round(nbytes / sec / 1e9 / hbm_peak, 4)}
+    # kernels launched per round: confidence + selection (one fused launch for the Thm. 4 selector, the LM
+    # head's GEMM + merge + selection, or confidence + selection), the attention launches (+ the tree-mask
+    # kernel per launch), and the acceptance: plan + rows + draws (the tree: statistics + walk)
+    conf_launches = 3 if args.lm_head else (1 if args.selector == "gain" else 2)
+    accept_launches = 2 if N else 3
+    launches_per_round = attn_launches * (2 if N else 1) + conf_launches + accept_launches
+    return {
+        "w": w, "steps": steps, "elapsed_max_ms": elapsed_max, "us_per_round": us_per_round, "by": by,
+        "Lh": Lh, "kv": kv, "n_res": n_res, "block_size": block_size, "hbm_peak": hbm_peak,
+        "roofline": roof, "lm_head": lm, "logits_segments": logits,
+        "segments_us": {"conf_select": round(select_ms * 1000.0 / steps, 3),
+                        "attention": round(attn_ms * 1000.0 / steps, 3),
+                        "accept": round(accept_ms * 1000.0 / steps, 3)},
+        "clocks": clocks.summary(), "launches": launches_per_round * steps, "e2e": e2e, "cpu": cpu, "flags": flags,
+        "one_call": one_call,
+    }
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+
+    from paper_2608_08721_gb300 import binding as lr
+    from paper_2608_08721_gb300 import build as cuda_build
+    from paper_2608_08721_gb300 import dist as pdist
+    from paper_2608_08721_gb300 import workloads
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if rank == 0 or not os.path.exists(lr.LIB_PATH):
+        cuda_build.build()
+    pdist.barrier()
+    w = workloads.WORKLOADS[args.config]
+    m = measure_workload(args, w, dev, rank, world, local_rank, args.steps, primary=True)
+    also = {}
+    variant = args.tree or args.page_size or args.lm_head or args.selector != "gain" or args.logits != "f32"
+    if not variant:
+        for name in [x for x in args.also.split(",") if x and x != args.config]:
+            torch.cuda.empty_cache()
+            a = measure_workload(args, workloads.WORKLOADS[name], dev, rank, world, local_rank, args.also_steps,
+                                 primary=False)
+            also[name] = {
+                "value_us": round(a["elapsed_max_ms"] * 1000.0 / (a["steps"] * world), 3), "steps": a["steps"],
+                "config": {"B": a["w"].B, "K": a["w"].K, "V": a["w"].V, "layers": a["w"].n_layers,
+                           "gqa": "%d/%d" % (a["w"].Hq, a["w"].Hkv), "kv_len": [int(a["kv"].min()), int(a["kv"].max())],
+                           "selected_L": [int(a["Lh"].min()), int(a["Lh"].max())]},
+                "hbm_tbs": round(a["by"]["total"] / (a["us_per_round"] * 1e-6) / 1e12, 3),
+                "roofline": a["roofline"], "logits_segments": a["logits_segments"],
+                "segments_us": a["segments_us"], "flags": a["flags"], "e2e": a["e2e"],
+                "gpu_launches": a["launches"]}
     if rank != 0:
         return
-    clk = clocks.summary()
-    value = elapsed_max * 1000.0 / (K_steps * world)
-    # attention (+ the tree-mask kernel per launch); confidence and selection (one fused launch for the
-    # Thm. 4 selector, the LM head's GEMM + merge + selection, or confidence + selection); 2 for acceptance
-    conf_launches = 3 if args.lm_head else (1 if args.selector == "gain" else 2)
-    launches = K_steps * (attn_launches * (2 if N else 1) + conf_launches + 2)
+    w, by, Lh, kv, K_steps = m["w"], m["by"], m["Lh"], m["kv"], m["steps"]
+    clk = m["clocks"]
+    us_per_round = m["us_per_round"]
+    value = m["elapsed_max_ms"] * 1000.0 / (K_steps * world)
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "us", "n_gpus": world, "steps": K_steps,
-        "warmup": max(3, args.warmup), "ms_per_step": round(elapsed_max / K_steps, 6), "higher_is_better": False,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16+f32",
+        "warmup": max(3, args.warmup), "ms_per_step": round(m["elapsed_max_ms"] / K_steps, 6),
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "bf16+f32",
         "data": "synthetic (seeded; shapes of the paper's 8B-70B-class targets, random values)",
         "config": {"workload": w.name, "B": w.B, "K": w.K, "V": w.V, "layers": w.n_layers,
-                   "resident_kv_layers": n_res, "gqa": "%d/%d" % (w.Hq, w.Hkv), "head_dim": w.d,
+                   "resident_kv_layers": m["n_res"], "gqa": "%d/%d" % (w.Hq, w.Hkv), "head_dim": w.d,
                    "kv_len": [int(kv.min()), int(kv.max())], "selected_L": [int(Lh.min()), int(Lh.max())],
-                   "selector": ("alpha (Algorithm 1, alpha %g, first block %d)" % (args.alpha, block_size)
+                   "selected_L_mean": round(float(Lh.mean()), 3),
+                   "cost_table": w.cost[0] if w.cost[0] != "measured" else "measured (%s)" % w.cost[1],
+                   "selector": ("alpha (Algorithm 1, alpha %g, first block %d)" % (args.alpha, m["block_size"])
                                 if args.selector == "alpha" else "marginal gain (Thm. 4)"),
                    "logits": args.logits,
-                   "draft": ("DDTree-shaped tree of %d nodes (best-first, depth <= %d), tree walk" % (N, w.K)
-                             if N else "chain"),
-                   "kv_cache": "paged, %d keys per page" % P if P else "dense",
+                   "draft": ("DDTree-shaped tree of %d nodes (best-first, depth <= %d), tree walk" %
+                             (args.tree, w.K) if args.tree else "chain"),
+                   "kv_cache": "paged, %d keys per page" % args.page_size if args.page_size else "dense",
                    "confidence": ("from hidden states [%d, %d] and a %d x %d LM head (fused epilogue)" %
                                   (w.B * w.K, w.hidden, w.V, w.hidden) if args.lm_head else "from drafter logits"),
                    "parallelism": "dp%d (independent sequences)" % world,
                    "l2": "no flush: %.0f MB of distinct inputs per step > 129 MB L2" % (by["total"] / 1e6),
-                   "timing": ("value: K rounds, each one CUDA graph replay, events around the loop; segments and "
-                              "roofline: a second pass of the same K rounds as three graphs (conf+select | "
-                              "attention layers | accept) with events between")},
+                   "timing": ("value: K rounds, each one CUDA graph replay of %s, events around the loop; "
+                              "segments and roofline: a second pass of the same K rounds as three graphs "
+                              "(conf+select | attention layers | accept, the acceptance plan included) with "
+                              "events between" % ("libraspec_verify_round" if m["one_call"] else
+                                                  "the round's step calls"))},
         "hbm_tbs": round(by["total"] / (us_per_round * 1e-6) / 1e12, 3),
-        "hbm_frac_of_measured": round(by["total"] / (us_per_round * 1e-6) / 1e9 / hbm_peak, 4),
+        "hbm_frac_of_measured": round(by["total"] / (us_per_round * 1e-6) / 1e9 / m["hbm_peak"], 4),
         "hbm_frac_of_nominal_8tbs": round(by["total"] / (us_per_round * 1e-6) / 1e9 / NOMINAL_HBM_GBS, 4),
-        "roofline": roof,
-        "lm_head": lm,
-        "logits_segments": logits,
-        "segments_us": {"conf_select": round(select_ms * 1000.0 / K_steps, 3),
-                        "attention": round(attn_ms * 1000.0 / K_steps, 3),
-                        "accept": round(accept_ms * 1000.0 / K_steps, 3)},
+        "roofline": m["roofline"],
+        "lm_head": m["lm_head"],
+        "logits_segments": m["logits_segments"],
+        "segments_us": m["segments_us"],
+        "flags": m["flags"],
         "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
                    "samples": clk["samples"]},
-        "gpu_launches": launches,
-        "e2e": e2e,
-        "cpu_baseline": cpu,
+        "gpu_launches": m["launches"],
+        "e2e": m["e2e"],
+        "cpu_baseline": m["cpu"],
+        "also": also or None,
     }
     print(json.dumps(line), flush=True)
 
 
-def run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset):
+def run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset, steps):
     """Same metric through the public host-buffer API: per round, the round's
     inputs (one pinned buffer) are copied in, the block's keys and values
     appended to the caches, and the results read back."""
@@ -682,11 +832,11 @@ def run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset):
         runner.run_staged(w.philox_seed, seq_offset=seq_offset)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
-    for _ in range(args.e2e_steps):
+    for _ in range(steps):
         runner.run_staged(w.philox_seed, seq_offset=seq_offset)
     dt = time.perf_counter() - t0
-    return {"value": round(dt * 1e6 / args.e2e_steps, 3), "unit": "us", "h2d_bytes_per_step": runner.h2d_bytes(),
-            "d2h_bytes_per_step": runner.d2h_bytes(), "steps": args.e2e_steps,
+    return {"value": round(dt * 1e6 / steps, 3), "unit": "us", "h2d_bytes_per_step": runner.h2d_bytes(),
+            "d2h_bytes_per_step": runner.d2h_bytes(), "steps": steps,
             "api": "paper_2608_08721_gb300.api.VerifyRound.run_staged (one pinned H2D copy, libraspec_kv_append, "
                    "libraspec_verify_round)"}
 

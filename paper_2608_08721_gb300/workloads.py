@@ -14,7 +14,9 @@ and the CPU oracle in tests and benchmarks.
 from __future__ import annotations
 
 import dataclasses
+import json
 import math
+import os
 from typing import List, Optional
 
 import numpy as np
@@ -35,7 +37,7 @@ class Workload:
     temperature: tuple     # ("const", T) | ("alternate", T_even, T_odd)
     target: tuple          # ("normal", sigma) | ("normal_peak", sigma, peak) | ("normal_sigma_u", lo, hi)
     draft_noise: tuple     # ("const", s) | ("uniform", lo, hi)
-    cost: tuple            # ("poly", c0, c1, c2) | ("attn_bytes",)
+    cost: tuple            # ("poly", c0, c1, c2) | ("measured", file) | ("attn_bytes",)
     philox_seed: int
     data_seed: int
     resident_layers: int = 0   # >0: distinct KV buffers kept on the device (rest reuse them)
@@ -65,7 +67,7 @@ WORKLOADS = {
     "ragged": Workload("ragged", B=64, K=32, V=128256, Hq=32, Hkv=8, d=128, n_layers=1,
                        kv=("loguniform", 512, 32768), temperature=("alternate", 0.0, 0.8),
                        target=("normal_sigma_u", 1.0, 8.0), draft_noise=("const", 1.0),
-                       cost=("attn_bytes",), philox_seed=3, data_seed=3),
+                       cost=("measured", "ragged_verify_attn_cost.json"), philox_seed=3, data_seed=3),
     "70b": Workload("70b", B=8, K=16, V=128256, Hq=64, Hkv=8, d=128, n_layers=80,
                     kv=("const", 131072), temperature=("const", 0.7), target=("normal", 4.0),
                     draft_noise=("const", 1.0), cost=("poly", 1.0, 0.008, 0.0),
@@ -121,21 +123,35 @@ def attn_bytes(w: Workload, kv: np.ndarray, L) -> float:
 # Fixed per-launch latency folded into the byte-count cost model, expressed
 # in bytes at the measured copy bandwidth (about 3 us at 6.76 TB/s).
 _LAUNCH_BYTES = 3e-6 * 6.756e12
+_DATA = os.path.join(os.path.dirname(os.path.abspath(__file__)), "data")
 
 
 def cost_table(w: Workload, kv: Optional[np.ndarray] = None) -> np.ndarray:
     """T_verify(L) for L = 0..K, float32 [K+1], positive.
 
-    Polynomial tables are the workloads' stated ones. The ragged workload's
-    table models one verify-attention launch with every sequence at length L:
-    the launch latency plus the bytes it must move at a fixed bandwidth,
-    normalised so that T(0) = 1 (the kernel is bandwidth bound, so its time is
-    proportional to these bytes)."""
+    Polynomial tables are the workloads' stated ones. A measured table (the
+    ragged workload's) is the verify-attention kernel's own latency with
+    every sequence at length L, frozen to JSON by ``measure_cost_table``
+    (normalised to T(0) = 1, running maximum). ``attn_bytes`` models one
+    launch as a fixed latency plus the bytes it must move at a fixed
+    bandwidth (normalised, running maximum); it is also the fallback of a
+    measured table whose file is missing."""
     Ls = np.arange(w.K + 1)
-    if w.cost[0] == "poly":
+    kind = w.cost[0]
+    if kind == "measured":
+        path = os.path.join(_DATA, w.cost[1])
+        if os.path.exists(path):
+            with open(path) as f:
+                rec = json.load(f)
+            t = np.asarray(rec["T"], np.float64)
+            if t.shape != (w.K + 1,):
+                raise ValueError("%s holds %d entries, the workload needs %d" % (path, t.size, w.K + 1))
+            return t.astype(np.float32)
+        kind = "attn_bytes"
+    if kind == "poly":
         c0, c1, c2 = w.cost[1:]
         t = c0 + c1 * Ls + c2 * Ls * Ls
-    elif w.cost[0] == "attn_bytes":
+    elif kind == "attn_bytes":
         kv = kv_lengths(w) if kv is None else kv
         t = np.array([_LAUNCH_BYTES + attn_bytes(w, kv, L) for L in Ls])
         t = t / t[0]

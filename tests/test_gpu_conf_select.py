@@ -98,8 +98,11 @@ def test_round_selection_matches_oracle_chain(orc, name):
     L_ref, flag = orc.select_lengths(q_ref, cost.astype(np.float64))
     assert_exact_unless_flagged(L, L_ref, flag, "L")
     if name == "ragged":
-        # the per-sequence peakedness spreads the selected lengths widely
-        assert L_ref.min() == 0 and L_ref.max() >= 8, "ragged lengths: %s" % L_ref
+        # the per-sequence peakedness spreads the selected lengths: the measured cost table is a
+        # staircase (flat between the latency steps at L = 1, 5, 8, ...), so the scan stops just
+        # below a step, at several different lengths
+        assert L_ref.min() == 0 and L_ref.max() >= 4 and len(set(L_ref.tolist())) >= 3, \
+            "ragged lengths: %s" % L_ref
 
 
 def test_select_edge_cases(orc):
