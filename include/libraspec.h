@@ -429,6 +429,21 @@ int libraspec_kv_append_paged(const uint16_t* kv_new, uint16_t* const* Kp, uint1
                               size_t ws_bytes, void* stream);
 
 /*
+ * Failure-detection self-test (no counterpart in the paper: it checks the
+ * library's own bounded waits). One CTA waits, with the bounded wait that
+ * acceptance's draws use for their sequence's decision, until the device
+ * word *flag is non-zero, giving up after limit_ns nanoseconds
+ * (1 <= limit_ns <= 2e9; the kernels' own waits give up after 2 s). On
+ * expiry it raises LIBRASPEC_ST_TIMEOUT in the workspace's status word and
+ * returns: the CUDA context stays usable. *observed (device i32) receives 1
+ * if the flag was seen, 0 if the wait gave up. flag and observed are
+ * caller-owned device pointers (4-byte aligned); the workspace needs only
+ * its status word (>= 256 bytes, 256-byte aligned). Enqueues one launch.
+ */
+int libraspec_selftest_wait(const uint32_t* flag, uint64_t limit_ns, int32_t* observed, void* workspace,
+                            size_t ws_bytes, void* stream);
+
+/*
  * Step 4 — acceptance (paper Sec. 3.1; the standard speculative-sampling
  * rule of Leviathan et al. that the paper cites, lossless with respect to
  * the target distribution).

@@ -31,6 +31,7 @@ SIGNATURES = {
     "libraspec_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I, _I]),
     "libraspec_workspace_init": (_I, [_P, _SZ, _P]),
     "libraspec_get_status": (_I, [_P, _P, _P]),
+    "libraspec_selftest_wait": (_I, [_P, _U64, _P, _P, _SZ, _P]),
     "libraspec_confidence": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "libraspec_confidence_bf16": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _SZ, _P]),
     "libraspec_confidence_noalloc": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P]),
@@ -159,6 +160,19 @@ def libraspec_get_status(ws: Workspace, stream=None) -> int:
     if rc not in (OK, EDEVICE):
         _check(rc, "libraspec_get_status")
     return int(out.value)
+
+
+def libraspec_selftest_wait(flag, limit_ns: int, ws: Workspace, observed=None, stream=None) -> torch.Tensor:
+    """The library's bounded wait on the device word ``flag`` (uint32 stored as int32 [1]) with a limit of
+    limit_ns; returns ``observed`` (int32 [1] on the device): 1 if the flag was seen, 0 if the wait gave up
+    (LIBRASPEC_ST_TIMEOUT is then set in the workspace's status)."""
+    _req(flag, torch.int32, "flag", (1,))
+    observed = torch.empty((1,), dtype=torch.int32, device=flag.device) if observed is None else _req(
+        observed, torch.int32, "observed", (1,))
+    rc = load().libraspec_selftest_wait(_ptr(flag), int(limit_ns), _ptr(observed), ws.ptr, ws.nbytes,
+                                        _stream(stream))
+    _check(rc, "libraspec_selftest_wait")
+    return observed
 
 
 def libraspec_confidence(draft_logits, draft_tokens, temperature, ws: Workspace, conf=None, dstat=None,

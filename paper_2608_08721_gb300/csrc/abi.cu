@@ -37,6 +37,7 @@ template <typename T>
 cudaError_t launch_accept(const T*, const T*, const int32_t*, const float*, const float*, const int32_t*,
                           const float*, int, int, int, uint64_t, uint64_t, uint32_t, int32_t*, int32_t*, char*,
                           const WsLayout&, cudaStream_t, const uint64_t*, bool);
+cudaError_t launch_selftest_wait(const uint32_t*, uint64_t, int32_t*, int*, cudaStream_t);
 template <typename T>
 cudaError_t launch_accept_plan(const T*, const T*, const float*, const float*, const int32_t*, const float*, int,
                                int, int, int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
@@ -107,6 +108,15 @@ size_t libraspec_workspace_size(int B, int K, int V, int Hq, int Hkv, int head_d
 int libraspec_workspace_init(void* workspace, size_t bytes, void* stream) {
   if (!workspace || !aligned(workspace, 256)) return LIBRASPEC_EINVAL;
   return from_cuda(cudaMemsetAsync(workspace, 0, bytes, static_cast<cudaStream_t>(stream)));
+}
+
+int libraspec_selftest_wait(const uint32_t* flag, uint64_t limit_ns, int32_t* observed, void* workspace,
+                            size_t ws_bytes, void* stream) {
+  if (!flag || !observed || !workspace || !aligned(workspace, 256) || ws_bytes < 256 || !aligned(flag, 4) ||
+      !aligned(observed, 4) || limit_ns < 1 || limit_ns > 2000000000ull)
+    return LIBRASPEC_EINVAL;
+  return from_cuda(launch_selftest_wait(flag, limit_ns, observed, static_cast<int*>(workspace),
+                                        static_cast<cudaStream_t>(stream)));
 }
 
 int libraspec_get_status(void* workspace, void* stream, int32_t* host_status) {

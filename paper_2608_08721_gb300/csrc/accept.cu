@@ -347,8 +347,8 @@ __device__ __forceinline__ void publish_draw(ResEntry* res, uint32_t* ready, int
   asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(ready + b), "r"(1u) : "memory");
 }
 
-// Bounded wait for a published flag: false after 2 s (LIBRASPEC_ST_TIMEOUT).
-__device__ bool wait_published(const uint32_t* flag, int* status) {
+// Bounded wait for a published flag: false after limit_ns (LIBRASPEC_ST_TIMEOUT).
+__device__ bool wait_published(const uint32_t* flag, int* status, uint64_t limit_ns = 2000000000ull) {
   uint64_t t0 = 0;
   for (uint32_t it = 0;; ++it) {
     if (ld_acquire_u32(flag) != 0u) return true;
@@ -357,7 +357,7 @@ __device__ bool wait_published(const uint32_t* flag, int* status) {
     } else if ((it & 7u) == 0u) {
       uint64_t t;
       asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
-      if (t - t0 > 2000000000ull) {
+      if (t - t0 > limit_ns) {
         raise_status(status, LIBRASPEC_ST_TIMEOUT);
         return false;
       }
@@ -734,6 +734,14 @@ __global__ void __launch_bounds__(kRowThreads, 4) accept_race_kernel(const Accep
   }
 }
 
+// Failure-detection self-test: the draws' bounded wait on a device flag with
+// a caller-given limit; observed = 1 if the flag was seen, 0 if the wait
+// gave up (and raised LIBRASPEC_ST_TIMEOUT).
+__global__ void selftest_wait_kernel(const uint32_t* __restrict__ flag, uint64_t limit_ns,
+                                     int32_t* __restrict__ observed, int* __restrict__ status) {
+  if (threadIdx.x == 0) *observed = wait_published(flag, status, limit_ns) ? 1 : 0;
+}
+
 // ---------------------------------------------------------------------------
 // Per-node draws of a draft tree. Grid (nsplit, N+1, B); nodes t > L_b exit
 // at once. A greedy sequence (temperature 0) takes the argmax of the node's
@@ -1082,6 +1090,12 @@ template cudaError_t launch_accept_plan<float>(const float*, const float*, const
 template cudaError_t launch_accept_plan<uint16_t>(const uint16_t*, const uint16_t*, const float*, const float*,
                                                   const int32_t*, const float*, int, int, int, int32_t*, int32_t*,
                                                   char*, const WsLayout&, cudaStream_t);
+cudaError_t launch_selftest_wait(const uint32_t* flag, uint64_t limit_ns, int32_t* observed, int* status,
+                                 cudaStream_t stream) {
+  selftest_wait_kernel<<<1, 32, 0, stream>>>(flag, limit_ns, observed, status);
+  return cudaGetLastError();
+}
+
 template cudaError_t launch_accept<uint16_t>(const uint16_t*, const uint16_t*, const int32_t*, const float*,
                                              const float*, const int32_t*, const float*, int, int, int, uint64_t,
                                              uint64_t, uint32_t, int32_t*, int32_t*, char*, const WsLayout&,

@@ -56,3 +56,12 @@ def assert_exact_unless_flagged(gpu, ref, flag, what):
     assert not bad.any(), "%s differs on unflagged sequences %s: gpu %s oracle %s" % (
         what, np.nonzero(bad)[0].tolist(), gpu[bad].tolist(), ref[bad].tolist())
     return int((flag != 0).sum())
+
+
+def assert_flag_budget(n_flagged, B, what, per=16):
+    """Flagged sequences are left out of the exact comparison; keep them few
+    (at most max(1, B / per)) so that a flag rule too wide to test anything
+    shows up. The count is printed for the record."""
+    budget = max(1, B // per)
+    print("%s: %d of %d sequences flagged (budget %d)" % (what, n_flagged, B, budget))
+    assert n_flagged <= budget, "%s: %d of %d sequences flagged, budget %d" % (what, n_flagged, B, budget)

@@ -114,3 +114,9 @@ def test_newer_entry_points_reject_bad_arguments_before_any_launch(lib):
     # the staged round without its parts
     args = [None] * 18 + [1, fake] + [1, 4, 64, 8, 2, 64, 64] + [0.1, 0, 0, 0] + [fake] * 6 + [1 << 30, None]
     assert lib.libraspec_verify_round_staged(*args) == lr.EINVAL
+    # the bounded-wait self-test: a limit of 0 or above 2 s, a missing flag, a small workspace
+    fake256 = P(0x1000)
+    assert lib.libraspec_selftest_wait(fake, 0, fake, fake256, 256, None) == lr.EINVAL
+    assert lib.libraspec_selftest_wait(fake, 3_000_000_000, fake, fake256, 256, None) == lr.EINVAL
+    assert lib.libraspec_selftest_wait(None, 1000, fake, fake256, 256, None) == lr.EINVAL
+    assert lib.libraspec_selftest_wait(fake, 1000, fake, fake256, 16, None) == lr.EINVAL

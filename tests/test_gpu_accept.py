@@ -3,7 +3,7 @@ import numpy as np
 import pytest
 import torch
 
-from helpers import assert_exact_unless_flagged, cuda
+from helpers import assert_exact_unless_flagged, assert_flag_budget, cuda
 from paper_2608_08721_gb300 import binding as lr
 from paper_2608_08721_gb300 import workloads
 
@@ -39,8 +39,9 @@ def test_accept_full_size_selected_lengths(orc, name):
     L = lr.libraspec_select_lengths(conf, torch.tensor(workloads.cost_table(w), device=cuda()), ws).cpu().numpy()
     n, bonus = _gpu_accept(inp, L, w.philox_seed)
     n_ref, b_ref, flag = _oracle_accept(orc, inp, L, w.philox_seed)
-    assert_exact_unless_flagged(n, n_ref, flag, "n_accepted")
+    nf = assert_exact_unless_flagged(n, n_ref, flag, "n_accepted")
     assert_exact_unless_flagged(bonus, b_ref, flag, "bonus_token")
+    assert_flag_budget(nf, w.B, "%s acceptance" % name)
     greedy = inp["temperature"].cpu().numpy() == 0
     assert not flag[greedy].any(), "greedy decisions are exact and never flagged"
 

@@ -141,7 +141,14 @@ def test_attn_full_size_sampled_rows(orc, name):
         for h in rng.choice(w.Hq, size=min(3, w.Hq), replace=False):
             rows.append((b, int(h), int(L[b])))
             rows.append((b, int(h), int(rng.integers(0, L[b] + 1))))
-    rows = np.array(rows, np.int32)
+    # complete (sequence, kv head) row groups: every head of the kv head at every verified
+    # position, the rows the kernel's split-KV merge writes together (sequence 0 at L = K,
+    # so (K + 1) g rows: one full 128-row tile or more; and the last sequence)
+    g = w.Hq // w.Hkv
+    for b in sorted({0, w.B - 1}):
+        kvh = int(rng.integers(0, w.Hkv))
+        rows += [(b, kvh * g + i, t) for i in range(g) for t in range(int(L[b]) + 1)]
+    rows = np.array(sorted(set(rows)), np.int32)
     O_ref, lse_ref = orc.verify_attn(lay["Q"], lay["Kc"], lay["Vc"], kv, L, rows=rows)
     check_attn(O, lse, O_ref, lse_ref, L, rows=[tuple(r) for r in rows])
 

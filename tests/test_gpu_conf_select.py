@@ -3,7 +3,7 @@ import numpy as np
 import pytest
 import torch
 
-from helpers import PROB_ATOL, assert_exact_unless_flagged, cuda
+from helpers import PROB_ATOL, assert_exact_unless_flagged, assert_flag_budget, cuda
 from paper_2608_08721_gb300 import binding as lr
 from paper_2608_08721_gb300 import workloads
 
@@ -96,7 +96,8 @@ def test_round_selection_matches_oracle_chain(orc, name):
     q_ref, _ = orc.confidence(inp["draft_logits"].cpu().numpy(), inp["draft_tokens"].cpu().numpy(),
                               inp["temperature"].cpu().numpy())
     L_ref, flag = orc.select_lengths(q_ref, cost.astype(np.float64))
-    assert_exact_unless_flagged(L, L_ref, flag, "L")
+    nf = assert_exact_unless_flagged(L, L_ref, flag, "L")
+    assert_flag_budget(nf, w.B, "%s selection" % name, per=32)
     if name == "ragged":
         # the per-sequence peakedness spreads the selected lengths: the measured cost table is a
         # staircase (flat between the latency steps at L = 1, 5, 8, ...), so the scan stops just

@@ -45,11 +45,14 @@ def test_select_alpha_random(orc, K, kind, alpha):
     rng = np.random.default_rng(K * 131 + int(alpha * 10))
     B = 700
     q = _conf(kind, B, K, rng)
+    # flags come from bounds alpha * S_i + i that are exact integers: runs of q = 1.0 (float32) in the
+    # "confident" drafts at an integral alpha flag up to 99 of the 700 sequences (the oracle's count on
+    # these seeds), every other case at most 6
+    budget = 120 if (kind == "confident" and alpha in (2.0, 4.0)) else 8
     for n in sorted({1, max(1, K // 3), min(16, K), K}):
         nf = _check(orc, q, n, alpha)
-        # flags come from bounds that are exact integers (q = 1.0 in float32
-        # runs, alpha = 2); most sequences must still be compared
-        assert nf <= B // 4, "too many flagged sequences (%d)" % nf
+        print("K=%d %s alpha=%g n=%d: %d of %d sequences flagged (budget %d)" % (K, kind, alpha, n, nf, B, budget))
+        assert nf <= budget, "%d of %d sequences flagged, budget %d" % (nf, B, budget)
 
 
 @pytest.mark.parametrize("K,n", [(24, 16), (16, 10), (32, 16), (64, 7)])
