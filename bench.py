@@ -833,12 +833,18 @@ def run_e2e(args, w, kv, inp, layers, cost, dev, seq_offset, steps):
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(steps):
-        runner.run_staged(w.philox_seed, seq_offset=seq_offset)
+        n_acc, _ = runner.run_staged(w.philox_seed, seq_offset=seq_offset)
     dt = time.perf_counter() - t0
-    return {"value": round(dt * 1e6 / steps, 3), "unit": "us", "h2d_bytes_per_step": runner.h2d_bytes(),
+    L = runner.out.L.cpu().numpy()
+    return {"value": round(dt * 1e6 / steps, 3), "unit": "us",
+            "h2d_bytes_per_step": runner.h2d_bytes(L, n_acc, inp["temperature"].cpu().numpy()),
             "d2h_bytes_per_step": runner.d2h_bytes(), "steps": steps,
-            "api": "paper_2608_08721_gb300.api.VerifyRound.run_staged (one pinned H2D copy, libraspec_kv_append, "
-                   "libraspec_verify_round)"}
+            "inputs": ("read in place from pinned host memory by the kernels (the queries copied); the bytes "
+                       "counted are those the round reads over the host link" if runner.in_place else
+                       "the pinned buffer copied to the device in three parts"),
+            "pinned_input_buffer_bytes": runner._host_stage.numel(),
+            "api": "paper_2608_08721_gb300.api.VerifyRound.run_staged (libraspec_verify_round_staged: the "
+                   "block's keys and values appended, then the round; the results read back)"}
 
 
 def main():

@@ -4,13 +4,20 @@
 whole round through ``libraspec_verify_round``. The KV caches are model state
 and stay on the device. Every per-round input (drafter and target logits,
 draft tokens, temperatures, the cost table, each layer's queries and the
-verified block's new keys and values) lives in ONE pinned host buffer and its
-device mirror, laid out in the order the round needs them: the drafter block
-(confidence and selection), the layers' queries and new keys/values
-(``libraspec_kv_append``, then attention), the target rows (acceptance). A
-round copies the three parts in on a side stream while the round's kernels
-start as soon as their part has landed, then reads the accepted counts and
-bonus tokens back (8 bytes per sequence).
+verified block's new keys and values) lives in ONE pinned host buffer, laid
+out in the order the round needs them: the drafter block (confidence and
+selection), the layers' queries and new keys/values (``libraspec_kv_append``,
+then attention), the target rows (acceptance).
+
+By default the kernels read the inputs in place, over the host link: a
+pinned allocation's address is valid on the device (unified addressing), and
+a verify round reads most of its inputs once, or not at all (acceptance reads
+only the verified target rows), so only the bytes the round uses cross the
+link. The layers' queries, which the attention kernel's TMA loads, are copied
+in on a side stream while the confidence streams the drafter block. With
+``inputs_in_place=False`` the three parts are copied to a device mirror
+instead, each step starting once its part has landed. Either way the accepted
+counts and bonus tokens come back into pinned memory (8 bytes per sequence).
 """
 from __future__ import annotations
 
@@ -36,9 +43,10 @@ def _layout(regions):
 class VerifyRound:
     def __init__(self, B: int, K: int, V: int, Hq: int, Hkv: int, head_dim: int, S_cap: int,
                  caches: List[Dict[str, torch.Tensor]], kv_len: torch.Tensor, device=None,
-                 logits_dtype=torch.float32):
+                 logits_dtype=torch.float32, inputs_in_place: bool = True):
         """caches: per layer {"Kc", "Vc"} bf16 [B,Hkv,S_cap,d] on the device;
-        logits_dtype: float32 or bfloat16 drafter and target logits."""
+        logits_dtype: float32 or bfloat16 drafter and target logits; inputs_in_place: the kernels read
+        the pinned inputs over the host link (only the queries are copied), else every part is copied."""
         if logits_dtype not in (torch.float32, torch.bfloat16):
             raise ValueError("logits_dtype must be torch.float32 or torch.bfloat16")
         self.B, self.K, self.V, self.Hq, self.Hkv, self.d, self.S_cap = B, K, V, Hq, Hkv, head_dim, S_cap
@@ -71,10 +79,21 @@ class VerifyRound:
 
         self._host = views(self._host_stage)
         self._dev = views(self._dev_stage)
-        d = self._dev
+        self.in_place = bool(inputs_in_place)
+        # in place: everything but the queries is read from the pinned buffer (part 1 is copied up to
+        # the new keys and values, i.e. the queries only)
+        d = dict(self._dev)
+        copy_parts = (True, True, True)
+        if self.in_place:
+            for name in ("draft_logits", "draft_tokens", "temperature", "cost_table", "kv_new", "target_logits",
+                         "rng"):
+                d[name] = self._host[name]
+            self._parts[1] = (offs["Q"], offs["kv_new"])
+            copy_parts = (False, True, False)
+        self._copied = sum(b - a for (a, b), c in zip(self._parts, copy_parts) if c)
         self.draft_logits, self.target_logits = d["draft_logits"], d["target_logits"]
         self.draft_tokens, self.temperature, self.cost_table = d["draft_tokens"], d["temperature"], d["cost_table"]
-        self.layers = [{"Q": d["Q"][l], "Kc": c["Kc"], "Vc": c["Vc"]} for l, c in enumerate(caches)]
+        self.layers = [{"Q": self._dev["Q"][l], "Kc": c["Kc"], "Vc": c["Vc"]} for l, c in enumerate(caches)]
         self.out = binding.RoundOutputs(
             torch.empty((B, K), dtype=f32, device=dev), torch.empty((B, K, 2), dtype=f32, device=dev),
             torch.empty((B,), dtype=i32, device=dev), torch.empty((B,), dtype=i32, device=dev),
@@ -87,7 +106,8 @@ class VerifyRound:
             [self._host_stage[a:b] for a, b in self._parts], [self._dev_stage[a:b] for a, b in self._parts],
             d["kv_new"], self.result_host[0], self.result_host[1], self.draft_logits, self.draft_tokens,
             self.temperature, self.cost_table, self.target_logits, self.layers, self.kv_len, self.out, self.ws,
-            self._host["rng"], d["rng"])
+            self._host["rng"], d["rng"], copy_parts=copy_parts)
+        self._dims = (B, K, V, n, Hq, Hkv, head_dim, torch.empty((), dtype=logits_dtype).element_size())
 
     def host_inputs(self) -> Dict[str, torch.Tensor]:
         """Pinned host views to fill before ``run_staged``: draft_logits [B,K,V], target_logits [B,K+1,V],
@@ -96,15 +116,40 @@ class VerifyRound:
         return {k: v for k, v in self._host.items() if k != "rng"}
 
     def run_device(self, seed: int, round_offset: int = 0, seq_offset: int = 0, stream=None):
-        """The round on inputs already resident in this object's device buffers
-        (the new keys and values already in the caches)."""
+        """The round on inputs resident in this object's device buffers (the new keys and values already
+        in the caches). Reading in place, the host buffer is first copied to the device buffers."""
+        if self.in_place:
+            self._dev_stage.copy_(self._host_stage, non_blocking=True)
+        d = self._dev
         return binding.libraspec_verify_round(
-            self.draft_logits, self.draft_tokens, self.temperature, self.cost_table, self.target_logits,
-            self.layers, self.kv_len, seed, self.ws, round_offset=round_offset, seq_offset=seq_offset,
-            outputs=self.out, stream=stream)
+            d["draft_logits"], d["draft_tokens"], d["temperature"], d["cost_table"], d["target_logits"],
+            [{"Q": d["Q"][l], "Kc": c["Kc"], "Vc": c["Vc"]} for l, c in enumerate(self.caches)], self.kv_len, seed,
+            self.ws, round_offset=round_offset, seq_offset=seq_offset, outputs=self.out, stream=stream)
 
-    def h2d_bytes(self) -> int:
-        return self._host_stage.numel()
+    def h2d_bytes(self, L=None, n_accepted=None, temperature=None) -> int:
+        """Bytes that move host -> device per round. Copying every part: the whole pinned buffer. In
+        place: the copied queries, plus what the kernels read over the link: the drafter block, the
+        new keys and values, and the target rows acceptance reads given the round's lengths L,
+        accepted counts and temperatures (rows 0..L_b, and a rejected sampling sequence's target and
+        drafter rows at the rejection once more); without them, every target row."""
+        if not self.in_place:
+            return self._host_stage.numel()
+        B, K, V, n, Hq, Hkv, d, eb = self._dims
+        h = self._host
+        small = sum(h[k].numel() * h[k].element_size() for k in ("draft_tokens", "temperature", "cost_table", "rng"))
+        drafter = B * K * V * eb
+        kv_new = h["kv_new"].numel() * h["kv_new"].element_size()
+        if L is None:
+            target = B * (K + 1) * V * eb
+        else:
+            import numpy as np
+
+            L = np.asarray(L)
+            rows = int(np.sum(L + 1))
+            if n_accepted is not None and temperature is not None:
+                rows += 2 * int(np.sum((np.asarray(n_accepted) < L) & (np.asarray(temperature) > 0)))
+            target = rows * V * eb
+        return self._copied + drafter + small + kv_new + target
 
     def d2h_bytes(self) -> int:
         return self.result_host.numel() * 4

@@ -113,6 +113,17 @@ def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
     return None if t is None else t.data_ptr()
 
 
+def _req_dev_or_pinned(t: torch.Tensor, dtype, name: str, shape=None) -> torch.Tensor:
+    """_req, or the same checks on a pinned host tensor (read in place by the kernels)."""
+    if isinstance(t, torch.Tensor) and not t.is_cuda:
+        if not t.is_pinned():
+            raise ValueError("%s must be on a CUDA device or in pinned host memory" % name)
+        if t.dtype != dtype or not t.is_contiguous() or (shape is not None and tuple(t.shape) != tuple(shape)):
+            raise ValueError("%s: dtype %s, contiguous, shape %s required" % (name, dtype, shape))
+        return t
+    return _req(t, dtype, name, shape)
+
+
 def _req(t: torch.Tensor, dtype, name: str, shape=None) -> torch.Tensor:
     if not isinstance(t, torch.Tensor):
         raise TypeError("%s must be a torch tensor" % name)
@@ -604,15 +615,19 @@ class StagedRound:
 
     def __init__(self, host_parts, dev_parts, kv_new, n_host, bonus_host, draft_logits, draft_tokens, temperature,
                  cost_table, target_logits, layers, kv_len, outputs: "RoundOutputs", ws: Workspace,
-                 rng_host, rng_dev, softmax_scale=None, copy_stream=None):
+                 rng_host, rng_dev, softmax_scale=None, copy_stream=None, copy_parts=(True, True, True)):
+        """copy_parts[i] False: part i is not copied; its typed inputs (and kv_new / rng_dev when they
+        lie in it) are then pinned host tensors that the kernels read in place (a pinned allocation's
+        address is valid on the device under unified addressing)."""
         B, K, V = draft_logits.shape
         bf16 = draft_logits.dtype == torch.bfloat16
         ldt = torch.bfloat16 if bf16 else torch.float32
-        _req(draft_logits, ldt, "draft_logits")
-        _req(target_logits, ldt, "target_logits", (B, K + 1, V))
-        _req(draft_tokens, torch.int32, "draft_tokens", (B, K))
-        _req(temperature, torch.float32, "temperature", (B,))
-        _req(cost_table, torch.float32, "cost_table", (K + 1,))
+        req = _req_dev_or_pinned
+        req(draft_logits, ldt, "draft_logits")
+        req(target_logits, ldt, "target_logits", (B, K + 1, V))
+        req(draft_tokens, torch.int32, "draft_tokens", (B, K))
+        req(temperature, torch.float32, "temperature", (B,))
+        req(cost_table, torch.float32, "cost_table", (K + 1,))
         _req(kv_len, torch.int32, "kv_len", (B,))
         n_layers = len(layers)
         Hq, D = layers[0]["Q"].shape[2], layers[0]["Q"].shape[3]
@@ -621,13 +636,13 @@ class StagedRound:
             _req(lay["Q"], torch.bfloat16, "Q[%d]" % i, (B, K + 1, Hq, D))
             _req(lay["Kc"], torch.bfloat16, "Kc[%d]" % i, (B, Hkv, S_cap, D))
             _req(lay["Vc"], torch.bfloat16, "Vc[%d]" % i, (B, Hkv, S_cap, D))
-        _req(kv_new, torch.bfloat16, "kv_new", (n_layers, 2, B, Hkv, K + 1, D))
+        req(kv_new, torch.bfloat16, "kv_new", (n_layers, 2, B, Hkv, K + 1, D))
         if len(host_parts) != 3 or len(dev_parts) != 3:
             raise ValueError("three host and three device parts")
         for h, d in zip(host_parts, dev_parts):
             if not h.is_pinned() or h.numel() != d.numel() or not d.is_cuda:
                 raise ValueError("each part: a pinned host tensor and a device tensor of the same size")
-        _req(rng_dev, torch.int64, "rng_dev", (3,))
+        req(rng_dev, torch.int64, "rng_dev", (3,))
         if (not isinstance(rng_host, torch.Tensor) or rng_host.dtype != torch.int64 or rng_host.numel() != 3
                 or not rng_host.is_pinned()):
             raise ValueError("rng_host must be 3 int64 of pinned host memory inside host part 2")
@@ -636,8 +651,9 @@ class StagedRound:
         self._keep = (host_parts, dev_parts, layers, outputs, n_host, bonus_host, rng_host, rng_dev)
         self._hp = (ctypes.c_void_p * 3)(*[h.data_ptr() for h in host_parts])
         self._dp = (ctypes.c_void_p * 3)(*[d.data_ptr() for d in dev_parts])
-        self._nb = (ctypes.c_size_t * 3)(*[h.numel() * h.element_size() for h in host_parts])
-        self._copy = copy_stream if copy_stream is not None else torch.cuda.Stream(device=draft_logits.device)
+        self._nb = (ctypes.c_size_t * 3)(*[h.numel() * h.element_size() if c else 0
+                                           for h, c in zip(host_parts, copy_parts)])
+        self._copy = copy_stream if copy_stream is not None else torch.cuda.Stream(device=kv_len.device)
         self._qa = _ptr_array([l["Q"] for l in layers])
         self._ka = _ptr_array([l["Kc"] for l in layers])
         self._va = _ptr_array([l["Vc"] for l in layers])

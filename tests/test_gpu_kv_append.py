@@ -79,16 +79,19 @@ def test_kv_append_paged_matches_dense(P):
                 assert torch.equal(pools[l]["Vp"][perm[b, j]], dense[l]["Vc"][b, :, j * P:(j + 1) * P])
 
 
-def test_staged_round_appends_and_matches_device_round():
+@pytest.mark.parametrize("in_place", [True, False])
+def test_staged_round_appends_and_matches_device_round(in_place):
     """run_staged: the block rows land in the caches, and the round's outputs
-    equal run_device on the same (already appended) inputs."""
+    equal run_device on the same (already appended) inputs; the kernels read
+    the pinned inputs in place, or the parts are copied to the device."""
     w = workloads.WORKLOADS["tiny"]
     kv = workloads.kv_lengths(w)
     lay = workloads.layer(w, 0, kv, device=cuda())
     inp = workloads.logits(w)
     K1 = w.K + 1
     caches = [{"Kc": lay["Kc"].clone(), "Vc": lay["Vc"].clone()}]
-    runner = api.VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, lay["Kc"].shape[2], caches, torch.tensor(kv))
+    runner = api.VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, lay["Kc"].shape[2], caches, torch.tensor(kv),
+                             inputs_in_place=in_place)
     h = runner.host_inputs()
     for name in ("draft_logits", "target_logits", "draft_tokens", "temperature"):
         h[name].copy_(inp[name])
@@ -109,6 +112,9 @@ def test_staged_round_appends_and_matches_device_round():
     np.testing.assert_array_equal(runner.out.n_accepted.cpu().numpy(), n2)
     np.testing.assert_array_equal(runner.out.bonus_token.cpu().numpy(), b2)
     assert runner.h2d_bytes() >= h["draft_logits"].numel() * 4 + h["target_logits"].numel() * 4
+    if in_place:  # given the round's lengths, only the verified target rows count
+        L = runner.out.L.cpu().numpy()
+        assert runner.h2d_bytes(L) == runner.h2d_bytes() - (w.K - int(L.sum())) * w.V * 4 * w.B
 
 
 def test_staged_round_bf16_logits_matches_device_round():

@@ -69,14 +69,16 @@ def test_verify_round_matches_oracle(orc, name, n_layers, logits):
                    rows=None if rows is None else [tuple(r) for r in rows])
 
 
-def test_host_buffer_api_round_trip(orc):
+@pytest.mark.parametrize("in_place", [True, False])
+def test_host_buffer_api_round_trip(orc, in_place):
     w = workloads.WORKLOADS["tiny"]
     kv = workloads.kv_lengths(w)
     lay = workloads.layer(w, 0, kv, device=cuda())
     inp = workloads.logits(w)
     K1 = w.K + 1
     caches = [{"Kc": lay["Kc"].clone(), "Vc": lay["Vc"].clone()}]
-    runner = api.VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, lay["Kc"].shape[2], caches, torch.tensor(kv))
+    runner = api.VerifyRound(w.B, w.K, w.V, w.Hq, w.Hkv, w.d, lay["Kc"].shape[2], caches, torch.tensor(kv),
+                             inputs_in_place=in_place)
     host = {k: v.pin_memory() for k, v in inp.items()}
     host["cost_table"] = torch.tensor(workloads.cost_table(w)).pin_memory()
     kvb = int(kv[0])
