@@ -136,7 +136,10 @@ int libraspec_confidence_bf16(const uint16_t* draft_logits, const int32_t* draft
  * larger calls return LIBRASPEC_EUNSUPPORTED and launch nothing. The call
  * allocates nothing. The first call on a device looks the array's address up
  * (cudaGetSymbolAddress, with that device current, which may load the
- * module): make it before any stream capture. Each call clears the status
+ * module): make it before any stream capture. The address is kept per device
+ * and CUDA context; a call in a new context on the device (after a
+ * cudaDeviceReset, say) looks it up again, and is then a first call too.
+ * Each call clears the status
  * word and its row tickets in the array (cudaMemsetAsync on `stream`).
  * Calls share the one array per device, so calls whose executions overlap
  * (other streams, other host threads) race and give undefined results: order

@@ -25,26 +25,59 @@ constexpr size_t kScratchBytes = kPartOff + kNoAllocRows * kConfMaxSplits * size
 __device__ __align__(256) char g_noalloc_scratch[kScratchBytes];
 
 constexpr int kMaxDevices = 64;
-std::atomic<char*> g_scratch_addr[kMaxDevices];
+// per device: the CUDA context the address was looked up in, and the address
+struct ScratchAddr {
+  std::atomic<void*> ctx{nullptr};
+  std::atomic<char*> addr{nullptr};
+};
+ScratchAddr g_scratch_addr[kMaxDevices];
 std::mutex g_setup_mu;
 
+// The driver's cuCtxGetCurrent, resolved once.
+typedef int (*CtxGetCurrentFn)(void**);
+CtxGetCurrentFn ctx_get_current() {
+  static std::atomic<CtxGetCurrentFn> fn{nullptr};
+  CtxGetCurrentFn f = fn.load(std::memory_order_acquire);
+  if (!f) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess) {
+      f = reinterpret_cast<CtxGetCurrentFn>(p);
+      fn.store(f, std::memory_order_release);
+    }
+  }
+  return f;
+}
+
 // Address of the scratch array on the current device, looked up once per
-// device (cudaGetSymbolAddress, with that device current).
+// device and context (cudaGetSymbolAddress, with that device current). A new
+// context on the device (after cudaDeviceReset, say) reloads the module, so
+// the address is looked up again.
 cudaError_t scratch_on_current_device(char** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  char* p = g_scratch_addr[dev].load(std::memory_order_acquire);
-  if (!p) {
+  CtxGetCurrentFn get = ctx_get_current();
+  if (!get) return cudaErrorDeviceUninitialized;
+  void* ctx = nullptr;
+  if (get(&ctx) != 0) return cudaErrorDeviceUninitialized;  // null: no context current yet
+  ScratchAddr& slot = g_scratch_addr[dev];
+  char* p = slot.addr.load(std::memory_order_acquire);
+  if (!p || !ctx || slot.ctx.load(std::memory_order_acquire) != ctx) {
     std::lock_guard<std::mutex> lock(g_setup_mu);
-    p = g_scratch_addr[dev].load(std::memory_order_relaxed);
-    if (!p) {
+    p = slot.addr.load(std::memory_order_relaxed);
+    if (!p || !ctx || slot.ctx.load(std::memory_order_relaxed) != ctx) {
+      // the lookup makes the device's primary context current if none was
       void* a = nullptr;
       e = cudaGetSymbolAddress(&a, g_noalloc_scratch);
       if (e != cudaSuccess) return e;
+      if (get(&ctx) != 0 || !ctx) return cudaErrorDeviceUninitialized;
       p = static_cast<char*>(a);
-      g_scratch_addr[dev].store(p, std::memory_order_release);
+      slot.addr.store(nullptr, std::memory_order_release);
+      slot.ctx.store(ctx, std::memory_order_release);
+      slot.addr.store(p, std::memory_order_release);
     }
   }
   *out = p;

@@ -96,4 +96,6 @@ def test_noalloc_calls_no_allocator():
         None, ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
     torch.cuda.synchronize()
     assert torch.cuda.memory_stats().get("allocation.all.allocated", 0) == n0
-    assert torch.cuda.mem_get_info()[0] == free0
+    # device-wide free memory can move for reasons outside the call (the driver, other processes);
+    # an allocation of the call's scratch (4.2 MB, in 2 MB pages) would take more than this
+    assert free0 - torch.cuda.mem_get_info()[0] < (1 << 20)
