@@ -185,11 +185,18 @@ __device__ TileLoc locate_tile(long long pos, int B, const int32_t* kv_len, cons
   return loc;
 }
 
-__device__ __forceinline__ long long range_lo(int c, long long T, int G) { return (long long)c * T / G; }
+// a / b for a >= 0, b > 0: 32-bit when both fit (a 64-bit division is a
+// long software sequence, and the plan runs on one warp before any copy)
+__device__ __forceinline__ long long div_nn(long long a, long long b) {
+  if ((((unsigned long long)a | (unsigned long long)b) >> 32) == 0) return (long long)((uint32_t)a / (uint32_t)b);
+  return a / b;
+}
+
+__device__ __forceinline__ long long range_lo(int c, long long T, int G) { return div_nn((long long)c * T, G); }
 
 // CTA whose range holds tile t: the largest c with c*T/G <= t.
 __device__ __forceinline__ int cta_of(long long t, long long T, int G) {
-  return (int)(((t + 1) * (long long)G - 1) / T);
+  return (int)div_nn((t + 1) * (long long)G - 1, T);
 }
 
 // Bounded poll of a grid-barrier counter (acquire).
@@ -250,16 +257,21 @@ struct AttnSmem {
   static constexpr int kK = kQ + kQSlots * kQSlot;
   static constexpr int kV = kK + STAGES * kTileBytes;
   // mbarriers: full[S], empty[S], qfull[2], qempty[2], sfull[2], sfree[2],
-  // pfull[4], pvdone[4], ofree[2], drain, merged
+  // pfull[4], pvdone[4], ofree[2], drain
   static constexpr int kBar = kV + STAGES * kTileBytes;
-  static constexpr int kNumBars = 2 * STAGES + 2 * 4 + 2 * kPBufs + 2 + 2;
+  static constexpr int kNumBars = 2 * STAGES + 2 * 4 + 2 * kPBufs + 2 + 1;
   static constexpr int kInfo = kBar + ((8 * kNumBars + 63) / 64) * 64;
   static constexpr int kTasks = kInfo + 2 * 64;
   static constexpr int kTmem = kTasks + 64;
   // [0] abort, [1] merge tasks, [2] items per layer, [3] merge chunks per
   // layer, [4] chunks claimed, [5] chunks done
   static constexpr int kMisc = kTmem + 16;
-  static constexpr int kBytes = kMisc + 32;
+  // kv_len and L of up to kPlanCap sequences, read once from global memory
+  // for the CTA's tile plan (a larger batch plans from global memory)
+  static constexpr int kPlanCap = 1024;
+  static constexpr int kRange = kMisc + 32;  // the CTA's tile range [lo, hi)
+  static constexpr int kPlan = kRange + 16;
+  static constexpr int kBytes = kPlan + 2 * 4 * kPlanCap;
   static constexpr int kAlloc = kBytes + 1024;           // room to align the base to 1024
   // tensor-memory columns
   static constexpr int kColS = 0;                        // S[2]: 64 fp32 columns each
@@ -399,17 +411,17 @@ __device__ __forceinline__ void merge_chunk(const MergeTask& t, int u0, int nr, 
   }
 }
 
-// Claims and merges chunks of layer `layer` until none is left; the warp
-// that completes the layer's last chunk arrives on `merged`. Chunks are
-// numbered [layer * C, (layer + 1) * C) on the CTA's monotonic counters.
+// Claims and merges chunks of layers up to `last_layer` until none is left,
+// oldest first. Chunks are numbered [l * C, (l + 1) * C) for layer l on the
+// CTA's monotonic counters; ctr_done counts the chunks merged (stores done).
 template <int D>
-__device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int C, int* ctr_claim, int* ctr_done,
-                             uint32_t merged, int K, int Hq, int Hkv, int R, const float* __restrict__ part_o,
-                             const float* __restrict__ part_ml, __nv_bfloat16* __restrict__ O,
-                             float* __restrict__ lse) {
+__device__ void merge_chunks(int last_layer, const LayerSet& set, const MergeTask* tasks, int n_tasks, int C,
+                             int* ctr_claim, int* ctr_done, int K, int Hq, int Hkv, int R,
+                             const float* __restrict__ part_buf_o, const float* __restrict__ part_buf_ml,
+                             size_t part_o_stride, size_t part_ml_stride) {
   const int lane = threadIdx.x & 31;
   const int g = Hq / Hkv;
-  const int hi = (layer + 1) * C;
+  const int hi = (last_layer + 1) * C;
   for (;;) {
     int u = 0;
     if (lane == 0) {
@@ -422,7 +434,12 @@ __device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int
     }
     u = __shfl_sync(0xffffffffu, u, 0);
     if (u >= hi) return;
-    // the chunk's task and its index within the task
+    // the chunk's layer, task and index within the task
+    const int layer = u / C;
+    const float* part_o = part_buf_o + (layer % kAttnPartBufs) * part_o_stride;
+    const float* part_ml = part_buf_ml + (layer % kAttnPartBufs) * part_ml_stride;
+    __nv_bfloat16* O = set.p[layer].O;
+    float* lse = set.p[layer].lse;
     int lc = u - layer * C, ti = 0, u0 = 0, nr = 0;
     for (; ti < n_tasks; ++ti) {
       nr = merge_share(tasks[ti], u0);
@@ -437,7 +454,7 @@ __device__ void merge_chunks(int layer, const MergeTask* tasks, int n_tasks, int
       else merge_chunk<4, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
     }
     __syncwarp();
-    if (lane == 0 && atomicAdd(ctr_done, 1) + 1 == hi) mbar_arrive(merged);
+    if (lane == 0) atomicAdd(ctr_done, 1);
   }
 }
 
@@ -472,7 +489,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   const uint32_t bPVDone = bPFull + 8 * kPBufs;
   const uint32_t bOFree = bPVDone + 8 * kPBufs;
   const uint32_t bDrain = bOFree + 16;
-  const uint32_t bMerged = bDrain + 8;  // the merge warp finished a layer's merge
   ItemInfo* info = reinterpret_cast<ItemInfo*>(smem + SM::kInfo);
   MergeTask* tasks = reinterpret_cast<MergeTask*>(smem + SM::kTasks);
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + SM::kTmem);
@@ -484,6 +500,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   const int R = g * (kAttnRows / g);  // rows per group: whole block positions
   const int n_layers = set.n;
   const uint32_t n_ctas = gridDim.x;
+  // the tensor maps' first use then finds them on chip
+  if (warp == kProducerWarp)
+    for (int l = lane; l < n_layers; l += 32) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&set.Q[l])) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&set.K[l])) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&set.V[l])) : "memory");
+    }
+  // the plan reads kv_len and L from shared memory when the batch fits
+  const bool plan_cached = B <= SM::kPlanCap;
+  int32_t* plan_kv = reinterpret_cast<int32_t*>(smem + SM::kPlan);
+  int32_t* plan_L = plan_kv + SM::kPlanCap;
+  const int32_t* kvs = plan_cached ? plan_kv : kv_len;
+  const int32_t* Lss = plan_cached ? plan_L : Ls;
 
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -502,7 +531,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       mbar_init(bPVDone + 8 * p, 1);
     }
     mbar_init(bDrain, 1);
-    mbar_init(bMerged, 1);
     misc[0] = 0;
     misc[4] = 0;
     misc[5] = 0;
@@ -519,22 +547,48 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   // The plan (identical for every layer): this CTA's tile range, its item
   // count and the split groups it helps merge.
   if (warp == 0) {
-    const long long T = total_tiles(B, kv_len, Ls, K, g, R, Hkv, S_cap, status, blockIdx.x == 0);
+    if (plan_cached) {
+      // one round trip: four sequences per lane in flight
+      for (int b0 = 0; b0 < B; b0 += 128) {
+        int kv4[4], L4[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int b = b0 + u * 32 + lane;
+          kv4[u] = b < B ? kv_len[b] : 0;
+          L4[u] = b < B ? Ls[b] : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int b = b0 + u * 32 + lane;
+          if (b < B) {
+            plan_kv[b] = kv4[u];
+            plan_L[b] = L4[u];
+          }
+        }
+      }
+      __syncwarp();
+    }
+    const long long T = total_tiles(B, kvs, Lss, K, g, R, Hkv, S_cap, status, blockIdx.x == 0);
     int G = (int)n_ctas;
     if (T > 0) {
-      const long long g_cap = (T + min_tiles - 1) / min_tiles;
+      const long long g_cap = div_nn(T + min_tiles - 1, min_tiles);
       if ((long long)G > g_cap) G = (int)g_cap;
     }
     const int c = blockIdx.x;
     int n_items = 0, n_tasks = 0;
+    long long* range = reinterpret_cast<long long*>(smem + SM::kRange);
+    if (lane == 0) {
+      range[0] = (T > 0 && c < G) ? range_lo(c, T, G) : 0;
+      range[1] = (T > 0 && c < G) ? range_lo(c + 1, T, G) : 0;
+    }
     if (T > 0 && c < G) {
       const long long lo = range_lo(c, T, G), hi = range_lo(c + 1, T, G);
       int group_lo = 0;
       for (int e = 0; e < 2; ++e) {
         const long long pos = e == 0 ? lo : hi - 1;
-        const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, R, Hkv, S_cap);
+        const TileLoc loc = locate_tile(pos, B, kvs, Lss, K, g, R, Hkv, S_cap);
         const int nt = loc.p.n_tiles;
-        const int gib = (int)((pos - loc.seq_start) / nt);
+        const int gib = (int)div_nn(pos - loc.seq_start, nt);
         const long long gstart = loc.seq_start + (long long)gib * nt, gend = gstart + nt;
         const int group = loc.group0 + gib;
         if (e == 0) group_lo = group;
@@ -572,19 +626,22 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     if ((threadIdx.x & 31) == 0) ok = wait_counter(bar_cnt + layer, n_ctas) && !misc[0];
     return __shfl_sync(0xffffffffu, ok, 0) != 0;
   };
+  // bounded wait (one lane) until the CTA has merged n chunks
+  auto merged_upto = [&](int n) {
+    for (int i = 0; i < kMaxWaitIters; ++i) {
+      if (*reinterpret_cast<volatile int*>(merge_done) >= n) return true;
+      if (misc[0]) return false;
+      __nanosleep(64);
+    }
+    return false;
+  };
   const uint32_t tmem = *tmem_slot;
 
   if (warp == kProducerWarp) {
     // ======================= producer =======================
-    const long long T = total_tiles(B, kv_len, Ls, K, g, R, Hkv, S_cap, status, false);
-    int G = (int)n_ctas;
-    if (T > 0) {
-      const long long g_cap = (T + min_tiles - 1) / min_tiles;
-      if ((long long)G > g_cap) G = (int)g_cap;
-    }
     const int c = blockIdx.x;
-    const long long lo = (T > 0 && c < G) ? range_lo(c, T, G) : 0;
-    const long long hi = (T > 0 && c < G) ? range_lo(c + 1, T, G) : 0;
+    const long long lo = reinterpret_cast<const long long*>(smem + SM::kRange)[0];
+    const long long hi = reinterpret_cast<const long long*>(smem + SM::kRange)[1];
     uint32_t item_ctr = 0, tile_ctr = 0;
     // lane 0 reads the abort flag for the whole warp (the loop body has warp-wide steps)
     auto aborted = [&]() { return __shfl_sync(0xffffffffu, misc[0], 0) != 0; };
@@ -603,9 +660,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     };
     if (pages_cached) {
       for (long long pos = lo; pos < hi;) {
-        const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, R, Hkv, S_cap);
+        const TileLoc loc = locate_tile(pos, B, kvs, Lss, K, g, R, Hkv, S_cap);
         const int nt = loc.p.n_tiles;
-        const long long gstart = loc.seq_start + (pos - loc.seq_start) / nt * nt;
+        const long long gstart = loc.seq_start + div_nn(pos - loc.seq_start, nt) * nt;
         const long long iend = gstart + nt < hi ? gstart + nt : hi;
         const int key0 = (int)(pos - gstart) * kAttnTileKeys;
         for (int i = lane; i < (int)(iend - pos); i += 32)
@@ -620,9 +677,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       bool ready = layer == 0;
       for (long long pos = lo; pos < hi && !aborted();) {
         ItemInfo it{};
-        const TileLoc loc = locate_tile(pos, B, kv_len, Ls, K, g, R, Hkv, S_cap);
+        const TileLoc loc = locate_tile(pos, B, kvs, Lss, K, g, R, Hkv, S_cap);
         const int nt = loc.p.n_tiles;
-        const int gib = (int)((pos - loc.seq_start) / nt);
+        const int gib = (int)div_nn(pos - loc.seq_start, nt);
         const long long gstart = loc.seq_start + (long long)gib * nt;
         const long long gend = gstart + nt;
         const long long iend = gend < hi ? gend : hi;
@@ -630,7 +687,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         it.kvh = gib / loc.p.n_mg;
         it.mg = gib % loc.p.n_mg;
         it.rows = min(R, loc.p.M - it.mg * R);
-        it.kv = kv_len[loc.b];
+        it.kv = kvs[loc.b];
         it.key0 = (int)(pos - gstart) * kAttnTileKeys;
         it.key1 = min(loc.p.N, (int)(iend - gstart) * kAttnTileKeys);
         it.partial = ((pos == gstart) && (gend <= hi)) ? 0 : 1;
@@ -641,7 +698,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         pos = iend;
         const uint32_t q = item_ctr % SM::kQSlots;
         if (lane == 0) {
-          bool ok = mbar_wait(bQEmpty + 8 * q, ((item_ctr / SM::kQSlots) & 1) ^ 1);
+          bool ok = true;
           int issued = 0;
           auto issue_tile = [&](int i) {
             const uint32_t s = tile_ctr % STAGES;
@@ -660,21 +717,44 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             }
             ++tile_ctr;
           };
-          // tiles whose stage is free go out first; before the barrier only
-          // tiles that lie wholly in the cache prefix, issued as stages free
-          // while the barrier is polled
-          const int n_pre = ready ? n_tiles : min(n_tiles, max(0, (it.kv - it.key0) / kAttnTileKeys));
-          for (int spin = 0; ok; ++spin) {
+          // Tiles go out as their stages free, before the item's Q slot is
+          // free (the previous item's last S), so the ring does not drain
+          // between items; before the layer barrier only tiles that lie
+          // wholly in the cache prefix (the block's keys are the previous
+          // layer's output).
+          // (a free Q slot at once: Q goes first, the item's first S needs it)
+          if (!ready) {
+            // Q is read once the layer barrier passes; bring it into L2 now
+#pragma unroll
+            for (int hb = 0; hb < SM::kBoxes; ++hb)
+              tma_prefetch_3d(&set.Q[layer], hb * 64, it.kvh * g, it.b * (K + 1) + it.mg * (R / g));
+          }
+          int n_pre = ready ? n_tiles : min(n_tiles, max(0, (it.kv - it.key0) / kAttnTileKeys));
+          // a layer's first item: its prefix tiles go out once the previous
+          // layer's last S has read its Q slot (earlier copies only slow the
+          // previous layer, whose barrier this layer waits for)
+          bool q_free = !ready && mbar_wait(bQEmpty + 8 * q, ((item_ctr / SM::kQSlots) & 1) ^ 1);
+          for (int spin = 0;; ++spin) {
+            if (!q_free) q_free = mbar_test_wait(bQEmpty + 8 * q, ((item_ctr / SM::kQSlots) & 1) ^ 1);
+            if (ready && q_free) break;
             while (issued < n_pre &&
                    mbar_test_wait(bEmpty + 8 * (tile_ctr % STAGES), ((tile_ctr / STAGES) & 1) ^ 1)) {
               issue_tile(issued);
               ++issued;
             }
-            if (ready) break;
-            uint32_t v;
-            asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(bar_cnt + (layer - 1)) : "memory");
-            if (v >= n_ctas) break;
-            if (spin >= kMaxWaitIters) ok = false;
+            if (!ready) {
+              uint32_t v;
+              asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(bar_cnt + (layer - 1)) : "memory");
+              if (v >= n_ctas) {
+                ready = true;
+                n_pre = n_tiles;
+                continue;
+              }
+            }
+            if (spin >= kMaxWaitIters) {
+              ok = false;
+              break;
+            }
             __nanosleep(32);
           }
           if (ok) {
@@ -783,8 +863,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     // layer n_layers has no items: it only helps with the last layer's merge
     for (int layer = 0; layer <= n_layers && ok; ++layer) {
       const bool has_items = layer < n_layers;
-      float* part_o = part_buf_o + (layer & 1) * part_o_stride;
-      float* part_ml = part_buf_ml + (layer & 1) * part_ml_stride;
+      float* part_o = part_buf_o + (layer % kAttnPartBufs) * part_o_stride;
+      float* part_ml = part_buf_ml + (layer % kAttnPartBufs) * part_ml_stride;
       if (layer > 0 && has_items) {
         // layer's inputs are ready once every CTA is done with the previous layer
         if (tid == 0 && !wait_counter(bar_cnt + (layer - 1), n_ctas)) {
@@ -959,21 +1039,21 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         ++item_ctr;
       }
       if (!ok) break;
-      // this CTA is done with the layer's items; the previous layer's partials
-      // (the other parity buffer) must be merged before any CTA may start the
-      // next layer and overwrite them: help with what the merge warp has left
-      // if that is much; after the last layer, help with its merge (the tail
-      // of the launch) once its grid barrier has passed
-      if (layer > 0 && merge_n > 0 && (has_items ? merge_n >= kMergeHelpChunks : layer_done(layer - 1)))
-        merge_chunks<D>(layer - 1, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv, R,
-                        part_buf_o + ((layer - 1) & 1) * part_o_stride, part_buf_ml + ((layer - 1) & 1) * part_ml_stride,
-                        set.p[layer - 1].O, set.p[layer - 1].lse);
+      // This CTA is done with the layer's items. Once its grid barrier
+      // passes, CTAs write layer + 1's partials into the buffer of layer - 2,
+      // whose merge must be done first. Help with the merge warp's backlog
+      // (layers up to layer - 1) if it is large; after the last layer, help
+      // with its merge (the tail of the launch) once its barrier has passed.
+      if (layer > 0 && merge_n > 0 &&
+          (has_items ? layer * merge_n - *reinterpret_cast<volatile int*>(merge_claimed) >= kMergeHelpChunks
+                     : layer_done(layer - 1)))
+        merge_chunks<D>(layer - 1, set, tasks, n_tasks, merge_n, merge_claimed, merge_done, K, Hq, Hkv, R, part_buf_o,
+                        part_buf_ml, part_o_stride, part_ml_stride);
       if (!has_items) break;
-      if (layer > 0 && merge_n > 0) {
-        if (warp == 0 && !warp_wait(bMerged, (layer - 1) & 1) && tid == 0) {
-          raise_status(status, LIBRASPEC_ST_TIMEOUT);
-          misc[0] = 1;
-        }
+      if (layer >= kAttnPartBufs - 1 && merge_n > 0 && tid == 0 &&
+          !merged_upto((layer - (kAttnPartBufs - 2)) * merge_n)) {
+        raise_status(status, LIBRASPEC_ST_TIMEOUT);
+        misc[0] = 1;
       }
       softmax_sync();
       if (misc[0]) {
@@ -990,20 +1070,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   } else if (warp == kMergeWarp) {
     // ======================= merge warp =======================
     // Layer l's split groups, once every CTA has finished layer l (its grid
-    // barrier), while the softmax warps already run layer l+1.
+    // barrier), while the softmax warps already run the next layers.
     bool ok = true;
     for (int layer = 0; layer < n_layers && ok; ++layer) {
       ok = layer_done(layer);
       if (!ok) break;
       if (merge_n > 0)
-        merge_chunks<D>(layer, tasks, n_tasks, merge_n, merge_claimed, merge_done, bMerged, K, Hq, Hkv, R,
-                        part_buf_o + (layer & 1) * part_o_stride, part_buf_ml + (layer & 1) * part_ml_stride,
-                        set.p[layer].O, set.p[layer].lse);
+        merge_chunks<D>(layer, set, tasks, n_tasks, merge_n, merge_claimed, merge_done, K, Hq, Hkv, R, part_buf_o,
+                        part_buf_ml, part_o_stride, part_ml_stride);
     }
-    // every chunk of the last layer is merged (by whichever warp) before the exit count
+    // every chunk of every layer is merged (by whichever warp) before the exit count
     if (ok && merge_n > 0 && n_layers > 0) {
-      if (lane == 0) ok = mbar_wait(bMerged, (n_layers - 1) & 1);
-      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (lane == 0) ok = merged_upto(n_layers * merge_n);
+      ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
     }
     if (!ok) {
       if (lane == 0 && !misc[0]) {
@@ -1256,7 +1335,9 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
         c->valid = true;
       }
     }
-    const size_t o_half = (lay.attn_ml - lay.attn_o) / 2, ml_half = (lay.attn_cnt - lay.attn_ml) / 2;
+    // one partial buffer's share, kept 256-byte aligned
+    const size_t o_part = ((lay.attn_ml - lay.attn_o) / kAttnPartBufs) & ~size_t(255);
+    const size_t ml_part = ((lay.attn_cnt - lay.attn_ml) / kAttnPartBufs) & ~size_t(255);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(kAttnThreads);
@@ -1271,8 +1352,8 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     cudaError_t e = cudaLaunchKernelEx(
         &cfg, kern, set, kv_len, L, tree_vis, tree_words(K), block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
         Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(),
-        reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_half / sizeof(float),
-        ml_half / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
+        reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_part / sizeof(float),
+        ml_part / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

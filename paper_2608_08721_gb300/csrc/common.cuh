@@ -22,6 +22,9 @@ constexpr int kConfMaxSplits = 64;    // CTAs per drafter row
 constexpr int kRowMaxSplits = 64;     // CTAs per target row (acceptance)
 constexpr int kRaceMaxSplits = 128;   // CTAs per sequence for a vocabulary draw
 constexpr int kAttnMaxCtas = 192;     // persistent attention grid cap (one CTA per SM)
+// Buffers of split-group partials: layer l writes buffer l % 3, so layer l's
+// merge may run until layer l + 2 starts, a layer after the one it overlaps.
+constexpr int kAttnPartBufs = 3;
 constexpr int kAttnRows = 128;        // query rows per attention row group (at most)
 constexpr int kAttnTileKeys = 64;     // keys per KV tile
 constexpr int kAttnMaxLayers = LIBRASPEC_ATTN_LAYERS_PER_LAUNCH;  // layers per attention launch
@@ -103,10 +106,10 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.acc_ready = take(size_t(B) * sizeof(uint32_t));  // res[b] published
   // the acceptance plan: a header, then one 8-byte descriptor per unit
   w.acc_plan = take(16 + 8 * std::max(size_t(kAccMaxGrid), rows_t));
-  // two partial slots per attention CTA (its first and its last item), in two
-  // buffers that alternate with the layer parity
-  w.attn_o = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * d * sizeof(float));
-  w.attn_ml = take(2 * size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
+  // two partial slots per attention CTA (its first and its last item), in
+  // kAttnPartBufs buffers that rotate with the layer (layer % kAttnPartBufs)
+  w.attn_o = take(kAttnPartBufs * size_t(2 * kAttnMaxCtas) * kAttnRows * d * sizeof(float));
+  w.attn_ml = take(kAttnPartBufs * size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
   // grid-barrier counters, one per layer of a launch, then the exit counter
   w.attn_cnt = take((kAttnMaxLayers + 1) * sizeof(uint32_t));
   // ancestor masks of a draft tree, ceil(K / 64) words per block position

@@ -177,10 +177,13 @@ def test_attn_deterministic():
             assert torch.equal(lse[b, rows], outs[0][1][b, rows])
 
 
-@pytest.mark.parametrize("B,kv_hi,d,seed", [(300, 200, 64, 1), (40, 9000, 128, 2), (129, 64, 128, 3)])
+@pytest.mark.parametrize("B,kv_hi,d,seed", [(300, 200, 64, 1), (40, 9000, 128, 2), (129, 64, 128, 3),
+                                             (1500, 40, 128, 4)])
 def test_attn_many_sequences_stream_k_ranges(orc, B, kv_hi, d, seed):
     """Many ragged sequences: CTA tile ranges start and end inside row groups,
-    one CTA covers several whole groups, and groups spread over many CTAs."""
+    one CTA covers several whole groups, and groups spread over many CTAs.
+    B = 1500 is past the 1024 sequences whose lengths the kernel keeps in
+    shared memory for its plan: that batch plans from global memory."""
     rng = np.random.default_rng(seed)
     K, Hq, Hkv = 12, 16, 4
     kv = rng.integers(0, kv_hi + 1, size=B).astype(np.int32)
