@@ -548,6 +548,16 @@ __global__ void __launch_bounds__(kRowThreads, 6) accept_rows_kernel(const Accep
     // ---- decision for sequence b (this CTA completed its last slice) ----
     __threadfence();
     const size_t row0 = (size_t)b * (K + 1);
+    // the first 32 decisions' inputs, loaded beside the merges
+    int xj = 0;
+    float yj = 0.f, qj = 0.f;
+    if (warp == 0 && lane < Lb) {
+      xj = a.tokens[(size_t)b * K + lane];
+      if (sampling) {
+        yj = __ldcg(&a.yx[row0 + lane]);
+        qj = a.conf[(size_t)b * K + lane];
+      }
+    }
     for (int jj = warp; jj < rows_b; jj += kRowThreads / 32) {
       const RowPartial* p = a.part + (row0 + jj) * kRowMaxSplits;
       float M;
@@ -575,16 +585,16 @@ __global__ void __launch_bounds__(kRowThreads, 6) accept_rows_kernel(const Accep
         const int jj = base + lane;
         bool reject = false;
         if (jj < Lb) {
-          const int x = a.tokens[(size_t)b * K + jj];
+          const int x = base == 0 ? xj : a.tokens[(size_t)b * K + jj];
           if (x < 0 || x >= V) {
             raise_status(a.status, LIBRASPEC_ST_BAD_TOKEN);
             reject = true;
           } else if (!sampling) {
             reject = s_arg[jj] != x;
           } else {
-            const float y = __ldcg(&a.yx[row0 + jj]);
+            const float y = base == 0 ? yj : __ldcg(&a.yx[row0 + jj]);
             const double p = (double)exp2f((y - s_m[jj]) * c) / s_Z[jj];
-            const double q = (double)a.conf[(size_t)b * K + jj];
+            const double q = (double)(base == 0 ? qj : a.conf[(size_t)b * K + jj]);
             const double ratio = (q <= p) ? 1.0 : p / q;
             const uint4 w = philox_block(seed, 0u, (uint32_t)jj, seq_offset + (uint32_t)b, 0u, round_offset);
             reject = !((double)word_to_uniform(w.x) < ratio);

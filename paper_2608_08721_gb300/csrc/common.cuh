@@ -35,6 +35,7 @@ struct RowPartial {      // one CTA's share of a logit row
   int arg;               // argmax (lowest index among maxima)
   double s;              // sum of exp((x - m) / T)
 };
+static_assert(sizeof(RowPartial) == 16, "a partial is read as one 16-byte load");
 
 struct RowStat {         // merged statistics of a target row
   float m;

@@ -172,13 +172,34 @@ __device__ __forceinline__ void cta_reduce_arg(float& m, int& arg, float* smf /*
 // s_i was summed relative to its own max m_i; it is rescaled to the row max M
 // by 2^((m_i - M) c), c = log2(e)/T, and the shares are added in binary64
 // (additions only: GB300 runs binary64 at a small fraction of the fp32 rate).
+// A lane reads each of its partials whole (one 16-byte load) and keeps up to
+// kMergeHeld of them, so up to 32 * kMergeHeld partials cost one memory round
+// trip; the sums are taken in the same order either way.
+constexpr int kMergeHeld = 2;
 __device__ __forceinline__ void warp_merge_partials(const RowPartial* __restrict__ p, int nsplit, float c,
                                                     bool want_arg, float& m_out, int& arg_out,
                                                     double& s_out) {
   const int lane = threadIdx.x & 31;
+  float mh[kMergeHeld];
+  double sh[kMergeHeld];
   float m = -INFINITY;
   int arg = 0x7fffffff;
-  for (int i = lane; i < nsplit; i += 32) {
+#pragma unroll
+  for (int k = 0; k < kMergeHeld; ++k) {
+    const int i = lane + 32 * k;
+    mh[k] = -INFINITY;
+    sh[k] = 0.0;
+    if (i < nsplit) {
+      const double2 raw = __ldcg(reinterpret_cast<const double2*>(p + i));
+      const long long mw = __double_as_longlong(raw.x);
+      mh[k] = __int_as_float((int)(mw & 0xffffffffll));
+      const int ai = (int)(mw >> 32);
+      sh[k] = raw.y;
+      if (want_arg) argmax_combine(m, arg, mh[k], ai);
+      else m = fmaxf(m, mh[k]);
+    }
+  }
+  for (int i = lane + 32 * kMergeHeld; i < nsplit; i += 32) {
     const float mi = __ldcg(&p[i].m);
     const int ai = __ldcg(&p[i].arg);
     if (want_arg) argmax_combine(m, arg, mi, ai);
@@ -193,7 +214,10 @@ __device__ __forceinline__ void warp_merge_partials(const RowPartial* __restrict
   }
   double s = 0.0;
   if (m != -INFINITY) {
-    for (int i = lane; i < nsplit; i += 32) {
+#pragma unroll
+    for (int k = 0; k < kMergeHeld; ++k)
+      if (mh[k] != -INFINITY) s += sh[k] * (double)ex2_approx((mh[k] - m) * c);
+    for (int i = lane + 32 * kMergeHeld; i < nsplit; i += 32) {
       const float mi = __ldcg(&p[i].m);
       const double si = __ldcg(&p[i].s);
       if (mi != -INFINITY) s += si * (double)ex2_approx((mi - m) * c);
