@@ -116,19 +116,27 @@ __device__ __forceinline__ SeqPlan seq_plan(int b, int B, const int32_t* kv_len,
   return p;
 }
 
-// Warp-wide: total tiles T of the batch; flags invalid sequences.
+// Warp-wide: total tiles T of the batch and its row groups (*groups);
+// flags invalid sequences.
 __device__ long long total_tiles(int B, const int32_t* kv_len, const int32_t* Ls, int K, int g, int R, int Hkv,
-                                 int S_cap, int* status, bool report) {
+                                 int S_cap, int* status, bool report, long long* groups) {
   const int lane = threadIdx.x & 31;
-  long long tot = 0;
+  long long tot = 0, ng = 0;
   bool bad = false;
   for (int b = lane; b < B; b += 32) {
     const SeqPlan p = seq_plan(b, B, kv_len, Ls, K, g, R, S_cap);
     if (!p.ok) bad = true;
-    else tot += (long long)Hkv * p.n_mg * p.n_tiles;
+    else {
+      tot += (long long)Hkv * p.n_mg * p.n_tiles;
+      ng += (long long)Hkv * p.n_mg;
+    }
   }
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, off);
+  for (int off = 16; off > 0; off >>= 1) {
+    tot += __shfl_xor_sync(0xffffffffu, tot, off);
+    ng += __shfl_xor_sync(0xffffffffu, ng, off);
+  }
+  *groups = ng;
   if (report && __any_sync(0xffffffffu, bad) && lane == 0) {
     int bits = 0;
     for (int b = 0; b < B; ++b) {
@@ -197,6 +205,55 @@ __device__ __forceinline__ long long range_lo(int c, long long T, int G) { retur
 // CTA whose range holds tile t: the largest c with c*T/G <= t.
 __device__ __forceinline__ int cta_of(long long t, long long T, int G) {
   return (int)div_nn((t + 1) * (long long)G - 1, T);
+}
+
+// Cost-weighted Stream-K. A row group costs its key tiles plus C (an item's
+// fixed cost: the Q load the first S waits for, the epilogue, a partial's
+// merge, in tile-equivalents), placed before its tiles; the batch weighs
+// W = T + C * groups, and CTA c takes the tiles of the weighted range
+// [c W / G, (c+1) W / G). A boundary inside a group's C falls on the
+// group's first tile. C = 0 is the plain split by tiles.
+__device__ long long tile_of_weighted(long long x, long long W, long long T, int C, int B, const int32_t* kv_len,
+                                      const int32_t* Ls, int K, int g, int R, int Hkv, int S_cap) {
+  if (x >= W) return T;
+  const int lane = threadIdx.x & 31;
+  long long carry_w = 0, carry_t = 0;
+  for (int base = 0; base < B; base += 32) {
+    const int b = base + lane;
+    const SeqPlan p = seq_plan(b, B, kv_len, Ls, K, g, R, S_cap);
+    const long long nt = p.ok ? (long long)Hkv * p.n_mg * p.n_tiles : 0;
+    const long long nw = p.ok ? nt + (long long)C * Hkv * p.n_mg : 0;
+    long long inc_w = nw, inc_t = nt;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const long long a = __shfl_up_sync(0xffffffffu, inc_w, off);
+      const long long t = __shfl_up_sync(0xffffffffu, inc_t, off);
+      if (lane >= off) { inc_w += a; inc_t += t; }
+    }
+    const long long sw = carry_w + inc_w - nw;
+    const bool mine = nw > 0 && x >= sw && x < sw + nw;
+    const unsigned ball = __ballot_sync(0xffffffffu, mine);
+    if (ball) {
+      const int src = __ffs(ball) - 1;
+      const long long wstart = __shfl_sync(0xffffffffu, sw, src);
+      const long long tstart = __shfl_sync(0xffffffffu, carry_t + inc_t - nt, src);
+      const SeqPlan q = seq_plan(base + src, B, kv_len, Ls, K, g, R, S_cap);
+      const long long per = q.n_tiles + C;
+      const long long o = x - wstart;
+      const long long gib = div_nn(o, per);
+      const long long r = o - gib * per;
+      return tstart + gib * q.n_tiles + (r > C ? r - C : 0);
+    }
+    carry_w += __shfl_sync(0xffffffffu, inc_w, 31);
+    carry_t += __shfl_sync(0xffffffffu, inc_t, 31);
+  }
+  return T;
+}
+
+// Weighted position of tile t of global row group `group` (the groups up to
+// and including it each put C before their tiles).
+__device__ __forceinline__ long long weighted_pos(long long t, long long group, int C) {
+  return t + (long long)C * (group + 1);
 }
 
 // Bounded poll of a grid-barrier counter (acquire).
@@ -470,7 +527,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     const __grid_constant__ LayerSet set, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
     const uint64_t* __restrict__ tree_vis, int tree_words,
     const int32_t* __restrict__ block_table, int max_pages, int page_size, int n_pages, int page_cache,
-    int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, float* __restrict__ part_buf_o,
+    int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, int item_tiles,
+    float* __restrict__ part_buf_o,
     float* __restrict__ part_buf_ml, size_t part_o_stride, size_t part_ml_stride, uint32_t* __restrict__ bar_cnt,
     int* __restrict__ status) {
   using SM = AttnSmem<D, STAGES>;
@@ -568,21 +626,32 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       }
       __syncwarp();
     }
-    const long long T = total_tiles(B, kvs, Lss, K, g, R, Hkv, S_cap, status, blockIdx.x == 0);
+    long long NG = 0;
+    const long long T = total_tiles(B, kvs, Lss, K, g, R, Hkv, S_cap, status, blockIdx.x == 0, &NG);
     int G = (int)n_ctas;
     if (T > 0) {
       const long long g_cap = div_nn(T + min_tiles - 1, min_tiles);
       if ((long long)G > g_cap) G = (int)g_cap;
     }
     const int c = blockIdx.x;
+    const long long W = T + (long long)item_tiles * NG;  // weighted length
+    long long lo = 0, hi = 0;
+    if (T > 0 && c < G) {
+      if (item_tiles == 0) {
+        lo = range_lo(c, T, G);
+        hi = range_lo(c + 1, T, G);
+      } else {
+        lo = tile_of_weighted(range_lo(c, W, G), W, T, item_tiles, B, kvs, Lss, K, g, R, Hkv, S_cap);
+        hi = tile_of_weighted(range_lo(c + 1, W, G), W, T, item_tiles, B, kvs, Lss, K, g, R, Hkv, S_cap);
+      }
+    }
     int n_items = 0, n_tasks = 0;
     long long* range = reinterpret_cast<long long*>(smem + SM::kRange);
     if (lane == 0) {
-      range[0] = (T > 0 && c < G) ? range_lo(c, T, G) : 0;
-      range[1] = (T > 0 && c < G) ? range_lo(c + 1, T, G) : 0;
+      range[0] = lo;
+      range[1] = hi;
     }
-    if (T > 0 && c < G) {
-      const long long lo = range_lo(c, T, G), hi = range_lo(c + 1, T, G);
+    if (lo < hi) {
       int group_lo = 0;
       for (int e = 0; e < 2; ++e) {
         const long long pos = e == 0 ? lo : hi - 1;
@@ -600,8 +669,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             t.kvh = gib / loc.p.n_mg;
             t.mg = gib % loc.p.n_mg;
             t.rows = min(R, loc.p.M - t.mg * R);
-            t.c0 = cta_of(gstart, T, G);
-            t.np = cta_of(gend - 1, T, G) - t.c0 + 1;
+            t.c0 = cta_of(weighted_pos(gstart, group, item_tiles), W, G);
+            t.np = cta_of(weighted_pos(gend - 1, group, item_tiles), W, G) - t.c0 + 1;
             tasks[n_tasks] = t;
           }
           ++n_tasks;
@@ -1156,6 +1225,21 @@ static int attn_min_tiles() {
   return t;
 }
 
+// Tile-equivalents an item costs in the Stream-K split (see
+// tile_of_weighted); the LIBRASPEC_ATTN_ITEM_TILES environment variable
+// overrides the default, read once per process.
+static int attn_item_tiles() {
+  static int t = [] {
+    int v = 3;
+    if (const char* e = getenv("LIBRASPEC_ATTN_ITEM_TILES")) {
+      int a = 0;
+      if (sscanf(e, "%d", &a) == 1 && a >= 0 && a <= 64) v = a;
+    }
+    return v;
+  }();
+  return t;
+}
+
 // Ancestor sets of a draft tree, one CTA per sequence, by pointer jumping:
 // after round r, m[t] holds the nodes on the path from t up to (not
 // including) up[t], the ancestor at distance 2^r (the root absorbs: m[0] =
@@ -1351,7 +1435,7 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(
         &cfg, kern, set, kv_len, L, tree_vis, tree_words(K), block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
-        Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(),
+        Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(), attn_item_tiles(),
         reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_part / sizeof(float),
         ml_part / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
     if (e != cudaSuccess) return e;
