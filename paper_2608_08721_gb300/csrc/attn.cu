@@ -273,13 +273,16 @@ struct ItemInfo {
   int key0, key1;     // keys [key0, key1)
   int partial;        // 1: write a partial, else write O
   int slot;           // partial slot
-  int pad[7];
+  int grp;            // global row group index
+  int pad[6];
 };
 
 // A split row group this CTA helps merge (the same for every layer).
 struct MergeTask {
   int b, kvh, mg, rows, c0, np;
+  int grp;  // global row group index
 };
+static_assert(2 * sizeof(MergeTask) <= 64, "two merge tasks fit their shared-memory slot");
 
 constexpr int kMaxLayers = kAttnMaxLayers;
 
@@ -530,7 +533,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     int B, int K, int Hq, int Hkv, int S_cap, float scale_log2, int min_tiles, int item_tiles,
     float* __restrict__ part_buf_o,
     float* __restrict__ part_buf_ml, size_t part_o_stride, size_t part_ml_stride, uint32_t* __restrict__ bar_cnt,
-    int* __restrict__ status) {
+    uint32_t* __restrict__ grp_cnt, int* __restrict__ status) {
   using SM = AttnSmem<D, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -592,6 +595,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     misc[0] = 0;
     misc[4] = 0;
     misc[5] = 0;
+    misc[6] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == kMmaWarp) {
@@ -671,6 +675,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             t.rows = min(R, loc.p.M - t.mg * R);
             t.c0 = cta_of(weighted_pos(gstart, group, item_tiles), W, G);
             t.np = cta_of(weighted_pos(gend - 1, group, item_tiles), W, G) - t.c0 + 1;
+            t.grp = group;
             tasks[n_tasks] = t;
           }
           ++n_tasks;
@@ -693,6 +698,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   auto layer_done = [&](int layer) {
     bool ok = false;
     if ((threadIdx.x & 31) == 0) ok = wait_counter(bar_cnt + layer, n_ctas) && !misc[0];
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+  };
+  // bounded wait (warp-wide) until the merge warp has seen every split group
+  // of the last layer complete
+  auto last_groups_ready = [&]() {
+    bool ok = false;
+    if ((threadIdx.x & 31) == 0) {
+      for (int i = 0; i < kMaxWaitIters; ++i) {
+        if (misc[6]) { ok = true; break; }
+        if (misc[0]) break;
+        __nanosleep(64);
+      }
+    }
     return __shfl_sync(0xffffffffu, ok, 0) != 0;
   };
   // bounded wait (one lane) until the CTA has merged n chunks
@@ -761,6 +779,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         it.key1 = min(loc.p.N, (int)(iend - gstart) * kAttnTileKeys);
         it.partial = ((pos == gstart) && (gend <= hi)) ? 0 : 1;
         it.slot = (pos == gstart) ? 2 * c + 1 : 2 * c;
+        it.grp = loc.group0 + gib;
         const int n_tiles = (int)(iend - pos);
         const int zc = loc.b * Hkv + it.kvh;
         const long long item_pos = pos;  // the item's first tile in the tile sequence
@@ -1104,6 +1123,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(bOFree + 8 * ob);
+          if (it.partial && layer == n_layers - 1) {
+            // the last layer's split groups are merged as soon as their
+            // parts are written (no grid barrier): count this part in (the
+            // barrier orders the warpgroup's writes before the release)
+            softmax_sync();
+            if (tid == 0)
+              asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(grp_cnt + 2 * it.grp), "r"(1u) : "memory");
+          }
         }
         ++item_ctr;
       }
@@ -1115,7 +1142,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       // with its merge (the tail of the launch) once its barrier has passed.
       if (layer > 0 && merge_n > 0 &&
           (has_items ? layer * merge_n - *reinterpret_cast<volatile int*>(merge_claimed) >= kMergeHelpChunks
-                     : layer_done(layer - 1)))
+                     : last_groups_ready()))
         merge_chunks<D>(layer - 1, set, tasks, n_tasks, merge_n, merge_claimed, merge_done, K, Hq, Hkv, R, part_buf_o,
                         part_buf_ml, part_o_stride, part_ml_stride);
       if (!has_items) break;
@@ -1142,7 +1169,27 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     // barrier), while the softmax warps already run the next layers.
     bool ok = true;
     for (int layer = 0; layer < n_layers && ok; ++layer) {
-      ok = layer_done(layer);
+      if (layer < n_layers - 1) {
+        ok = layer_done(layer);
+      } else {
+        // the last layer: each split group once its np parts are counted in
+        // (no grid barrier); the last CTA past a group's wait resets its
+        // counters for the next launch
+        if (lane == 0) {
+          for (int ti = 0; ti < n_tasks && ok; ++ti) ok = wait_counter(grp_cnt + 2 * tasks[ti].grp, tasks[ti].np);
+          if (ok) {
+            misc[6] = 1;  // the softmax warps may help now
+            for (int ti = 0; ti < n_tasks; ++ti) {
+              uint32_t* gc = grp_cnt + 2 * tasks[ti].grp;
+              if (atomicAdd(gc + 1, 1u) == (uint32_t)tasks[ti].np - 1) {
+                gc[0] = 0u;
+                gc[1] = 0u;
+              }
+            }
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0) != 0 && !misc[0];
+      }
       if (!ok) break;
       if (merge_n > 0)
         merge_chunks<D>(layer, set, tasks, n_tasks, merge_n, merge_claimed, merge_done, K, Hq, Hkv, R, part_buf_o,
@@ -1153,20 +1200,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       if (lane == 0) ok = merged_upto(n_layers * merge_n);
       ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
     }
-    if (!ok) {
-      if (lane == 0 && !misc[0]) {
-        raise_status(status, LIBRASPEC_ST_TIMEOUT);
-        misc[0] = 1;
-      }
-    } else if (lane == 0 && n_layers > 0) {
-      // the last CTA out resets the barrier counters for the next launch
-      __threadfence();
-      const uint32_t done = atomicAdd(exit_cnt, 1u);
-      if (done == n_ctas - 1) {
-        for (int l = 0; l < n_layers; ++l) bar_cnt[l] = 0u;
-        *exit_cnt = 0u;
-        __threadfence();
-      }
+    if (!ok && lane == 0 && !misc[0]) {
+      raise_status(status, LIBRASPEC_ST_TIMEOUT);
+      misc[0] = 1;
     }
     __syncwarp();
   }
@@ -1174,6 +1210,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (tid == 0 && !misc[0] && n_layers > 0) {
+    // the last CTA out resets the barrier counters for the next launch (each
+    // CTA has arrived at every layer's barrier by now)
+    __threadfence();
+    const uint32_t done = atomicAdd(exit_cnt, 1u);
+    if (done == n_ctas - 1) {
+      for (int l = 0; l < n_layers; ++l) bar_cnt[l] = 0u;
+      *exit_cnt = 0u;
+      __threadfence();
+    }
+  }
   if (warp == kMmaWarp)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(kTmemCols) : "memory");
 }
@@ -1437,7 +1484,8 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
         &cfg, kern, set, kv_len, L, tree_vis, tree_words(K), block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
         Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(), attn_item_tiles(),
         reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_part / sizeof(float),
-        ml_part / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt), reinterpret_cast<int*>(ws + lay.status));
+        ml_part / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt),
+        reinterpret_cast<uint32_t*>(ws + lay.attn_grp), reinterpret_cast<int*>(ws + lay.status));
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

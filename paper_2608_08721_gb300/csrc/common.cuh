@@ -72,7 +72,7 @@ struct ResEntry {
 struct WsLayout {
   size_t status, conf_part, conf_cnt, seq_cnt, row_part, row_cnt, row_stat, race_part, race_cnt;
   size_t acc_seq, acc_yx, acc_res, acc_ready, acc_plan;
-  size_t attn_o, attn_ml, attn_cnt, tree_vis, total;
+  size_t attn_o, attn_ml, attn_cnt, attn_grp, tree_vis, total;
   int max_items, max_groups;
 };
 
@@ -113,6 +113,8 @@ inline WsLayout ws_layout(int B, int K, int V, int Hq, int Hkv, int d, int S_cap
   w.attn_ml = take(kAttnPartBufs * size_t(2 * kAttnMaxCtas) * kAttnRows * 2 * sizeof(float));
   // grid-barrier counters, one per layer of a launch, then the exit counter
   w.attn_cnt = take((kAttnMaxLayers + 1) * sizeof(uint32_t));
+  // per row group: parts of the last layer counted in, CTAs past its wait
+  w.attn_grp = take(2 * size_t(w.max_groups) * sizeof(uint32_t));
   // ancestor masks of a draft tree, ceil(K / 64) words per block position
   w.tree_vis = take(rows_t * size_t(K <= 64 ? 1 : (K + 63) / 64) * sizeof(uint64_t));
   w.total = off;
