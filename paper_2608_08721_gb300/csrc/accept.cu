@@ -978,7 +978,8 @@ template cudaError_t launch_accept_tree<uint16_t>(const uint16_t*, const int32_t
                                                   int32_t*, int32_t*, char*, const WsLayout&, cudaStream_t);
 
 // CTAs of the acceptance rows kernel resident at once on the current device;
-// its grid is four waves of them (at most kAccMaxGrid).
+// its grid is two waves of them (at most kAccMaxGrid; measured on the ragged
+// batch: 51.5 us back to back against 54.3 with four waves, 53.0 with three).
 template <bool VEC, typename T>
 int accept_grid() {
   static int cached[64];
@@ -991,7 +992,7 @@ int accept_grid() {
             cudaSuccess ||
         per_sm < 1)
       per_sm = 1;
-    g = std::min(4 * per_sm * num_sms_current(), kAccMaxGrid);
+    g = std::min(2 * per_sm * num_sms_current(), kAccMaxGrid);
     cached[dev] = g;
   }
   return g;
