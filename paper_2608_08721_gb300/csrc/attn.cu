@@ -281,7 +281,14 @@ struct ItemInfo {
 struct MergeTask {
   int b, kvh, mg, rows, c0, np;
   int grp;  // global row group index
+  int epi;  // in the last layer, merged whole by the CTA completing it (small groups)
 };
+// A split group whose merge reads at most this many (row, 4-column) items
+// over all its parts (rows x d/4 x parts) is merged, in a launch's last
+// layer, by the CTA whose part completes it, in that part's epilogue (a few
+// memory round trips, and no wait); a larger one (a long group spread over
+// many CTAs) is merged share by share by all its CTAs.
+constexpr int kEpiMaxItems = 8192;
 static_assert(2 * sizeof(MergeTask) <= 64, "two merge tasks fit their shared-memory slot");
 
 constexpr int kMaxLayers = kAttnMaxLayers;
@@ -324,7 +331,8 @@ struct AttnSmem {
   static constexpr int kTasks = kInfo + 2 * 64;
   static constexpr int kTmem = kTasks + 64;
   // [0] abort, [1] merge tasks, [2] items per layer, [3] merge chunks per
-  // layer, [4] chunks claimed, [5] chunks done
+  // layer, [4] chunks claimed, [5] chunks done, [6] the last layer's shared
+  // merges may start, [7] this item's epilogue merges its group
   static constexpr int kMisc = kTmem + 16;
   // kv_len and L of up to kPlanCap sequences, read once from global memory
   // for the CTA's tile plan (a larger batch plans from global memory)
@@ -357,6 +365,7 @@ struct AttnSmem {
 // round trip per batch and no weights are staged in shared memory.
 
 // This CTA's share [u0, u0 + nr) of task t's rows.
+__device__ __forceinline__ int merge_share(const MergeTask& t, int& u0);
 __device__ __forceinline__ int merge_share(const MergeTask& t, int& u0) {
   const int k_me = (int)blockIdx.x - t.c0;
   u0 = (int)((long long)t.rows * k_me / t.np);
@@ -380,6 +389,35 @@ __device__ __forceinline__ int merge_j(int np, int items) {
   const int trips1 = ((items + 31) / 32) * ((np + 15) / 16);
   const int trips4 = ((items + 127) / 128) * ((np + 3) / 4);
   return trips4 < trips1 ? 4 : 1;
+}
+
+template <int J, int D>
+__device__ __forceinline__ void merge_chunk(const MergeTask& t, int u0, int nr, int lc, const float* __restrict__ part_o,
+                                            const float* __restrict__ part_ml, int K, int Hq, int g, int R,
+                                            __nv_bfloat16* __restrict__ O, float* __restrict__ lse);
+
+// The whole of group t by the softmax warpgroup (warp w of 4 takes every
+// fourth chunk), share by share with each share's chunk shape, so the result
+// has the bits the group's CTAs would each give for their share. Out of line:
+// it runs once per small split group of a launch's last layer, and keeps its
+// code out of the item loop's instruction stream.
+template <int D>
+__device__ __noinline__ void merge_group_whole(const MergeTask t, int warp, const float* __restrict__ part_o,
+                                               const float* __restrict__ part_ml, int K, int Hq, int g, int R,
+                                               __nv_bfloat16* __restrict__ O, float* __restrict__ lse) {
+  int gi = 0;
+  for (int k = 0; k < t.np; ++k) {
+    const int u0 = (int)((long long)t.rows * k / t.np);
+    const int nr = (int)((long long)t.rows * (k + 1) / t.np) - u0;
+    const int items = nr * (D / 4);
+    const int J = merge_j(t.np, items);
+    const int nc = (items + 32 * J - 1) / (32 * J);
+    for (int lc = 0; lc < nc; ++lc, ++gi) {
+      if (gi % kSoftmaxWarps != warp) continue;
+      if (J == 1) merge_chunk<1, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
+      else merge_chunk<4, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
+    }
+  }
 }
 
 template <int D>
@@ -478,7 +516,7 @@ template <int D>
 __device__ void merge_chunks(int last_layer, const LayerSet& set, const MergeTask* tasks, int n_tasks, int C,
                              int* ctr_claim, int* ctr_done, int K, int Hq, int Hkv, int R,
                              const float* __restrict__ part_buf_o, const float* __restrict__ part_buf_ml,
-                             size_t part_o_stride, size_t part_ml_stride) {
+                             size_t part_o_stride, size_t part_ml_stride, int epi_layer) {
   const int lane = threadIdx.x & 31;
   const int g = Hq / Hkv;
   const int hi = (last_layer + 1) * C;
@@ -508,7 +546,7 @@ __device__ void merge_chunks(int last_layer, const LayerSet& set, const MergeTas
       if (lc < nc) break;
       lc -= nc;
     }
-    if (ti < n_tasks) {
+    if (ti < n_tasks && !(layer == epi_layer && tasks[ti].epi)) {  // (an epilogue merge: counted, no work)
       const MergeTask& t = tasks[ti];
       if (merge_j(t.np, nr * (D / 4)) == 1) merge_chunk<1, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
       else merge_chunk<4, D>(t, u0, nr, lc, part_o, part_ml, K, Hq, g, R, O, lse);
@@ -676,6 +714,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             t.c0 = cta_of(weighted_pos(gstart, group, item_tiles), W, G);
             t.np = cta_of(weighted_pos(gend - 1, group, item_tiles), W, G) - t.c0 + 1;
             t.grp = group;
+            t.epi = (long long)t.rows * (D / 4) * t.np <= kEpiMaxItems ? 1 : 0;
             tasks[n_tasks] = t;
           }
           ++n_tasks;
@@ -1124,12 +1163,35 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           __syncwarp();
           if (lane == 0) mbar_arrive(bOFree + 8 * ob);
           if (it.partial && layer == n_layers - 1) {
-            // the last layer's split groups are merged as soon as their
-            // parts are written (no grid barrier): count this part in (the
-            // barrier orders the warpgroup's writes before the release)
+            // The last layer's split groups need no grid barrier: each part is
+            // counted in as written (the barrier orders the warpgroup's writes
+            // before the release). A small group is merged at once, whole, by
+            // the CTA whose part completes it (the acquire makes the other
+            // parts visible), share by share as its CTAs would merge it, so
+            // the result is the same bits; a larger one by the merge warps of
+            // all its CTAs once its count is complete.
+            int ti = 0;
+            while (ti + 1 < n_tasks && tasks[ti].grp != it.grp) ++ti;
+            const MergeTask t = tasks[ti];
             softmax_sync();
-            if (tid == 0)
-              asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(grp_cnt + 2 * it.grp), "r"(1u) : "memory");
+            if (tid == 0) {
+              bool last = false;
+              if (t.epi) {
+                uint32_t old;
+                asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;"
+                             : "=r"(old)
+                             : "l"(grp_cnt + 2 * it.grp), "r"(1u)
+                             : "memory");
+                last = old == (uint32_t)t.np - 1;
+                if (last) grp_cnt[2 * it.grp] = 0u;  // every part is in: ready for the next launch
+              } else {
+                asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(grp_cnt + 2 * it.grp), "r"(1u)
+                             : "memory");
+              }
+              misc[7] = last ? 1 : 0;
+            }
+            softmax_sync();
+            if (misc[7]) merge_group_whole<D>(t, warp, part_o, part_ml, K, Hq, g, R, O, lse);
           }
         }
         ++item_ctr;
@@ -1144,7 +1206,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           (has_items ? layer * merge_n - *reinterpret_cast<volatile int*>(merge_claimed) >= kMergeHelpChunks
                      : last_groups_ready()))
         merge_chunks<D>(layer - 1, set, tasks, n_tasks, merge_n, merge_claimed, merge_done, K, Hq, Hkv, R, part_buf_o,
-                        part_buf_ml, part_o_stride, part_ml_stride);
+                        part_buf_ml, part_o_stride, part_ml_stride, n_layers - 1);
       if (!has_items) break;
       if (layer >= kAttnPartBufs - 1 && merge_n > 0 && tid == 0 &&
           !merged_upto((layer - (kAttnPartBufs - 2)) * merge_n)) {
@@ -1176,10 +1238,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
         // (no grid barrier); the last CTA past a group's wait resets its
         // counters for the next launch
         if (lane == 0) {
-          for (int ti = 0; ti < n_tasks && ok; ++ti) ok = wait_counter(grp_cnt + 2 * tasks[ti].grp, tasks[ti].np);
+          for (int ti = 0; ti < n_tasks && ok; ++ti)
+            if (!tasks[ti].epi) ok = wait_counter(grp_cnt + 2 * tasks[ti].grp, tasks[ti].np);
           if (ok) {
             misc[6] = 1;  // the softmax warps may help now
             for (int ti = 0; ti < n_tasks; ++ti) {
+              if (tasks[ti].epi) continue;
               uint32_t* gc = grp_cnt + 2 * tasks[ti].grp;
               if (atomicAdd(gc + 1, 1u) == (uint32_t)tasks[ti].np - 1) {
                 gc[0] = 0u;
@@ -1193,7 +1257,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       if (!ok) break;
       if (merge_n > 0)
         merge_chunks<D>(layer, set, tasks, n_tasks, merge_n, merge_claimed, merge_done, K, Hq, Hkv, R, part_buf_o,
-                        part_buf_ml, part_o_stride, part_ml_stride);
+                        part_buf_ml, part_o_stride, part_ml_stride, n_layers - 1);
     }
     // every chunk of every layer is merged (by whichever warp) before the exit count
     if (ok && merge_n > 0 && n_layers > 0) {
