@@ -420,6 +420,42 @@ __device__ __noinline__ void merge_group_whole(const MergeTask t, int warp, cons
   }
 }
 
+// A part of a launch's last layer is written (softmax warpgroup, after its
+// epilogue). The last layer's split groups need no grid barrier: each part is
+// counted in as written (the named barrier orders the warpgroup's writes
+// before the release). A small group is merged at once, whole, by the CTA
+// whose part completes it (the acquire makes the other parts visible), share
+// by share as its CTAs would merge it, so the result is the same bits; a
+// larger one by the merge warps of all its CTAs once its count is complete.
+// Out of line, like merge_group_whole: it runs once per split part of the
+// last layer.
+template <int D>
+__device__ __noinline__ void last_layer_part_done(const MergeTask* tasks, int n_tasks, int grp,
+                                                  uint32_t* __restrict__ grp_cnt, volatile int* misc,
+                                                  const float* __restrict__ part_o, const float* __restrict__ part_ml,
+                                                  int K, int Hq, int g, int R, __nv_bfloat16* __restrict__ O,
+                                                  float* __restrict__ lse) {
+  const int tid = threadIdx.x, warp = tid >> 5;
+  int ti = 0;
+  while (ti + 1 < n_tasks && tasks[ti].grp != grp) ++ti;
+  const MergeTask t = tasks[ti];
+  softmax_sync();
+  if (tid == 0) {
+    bool last = false;
+    if (t.epi) {
+      uint32_t old;
+      asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(grp_cnt + 2 * grp), "r"(1u) : "memory");
+      last = old == (uint32_t)t.np - 1;
+      if (last) grp_cnt[2 * grp] = 0u;  // every part is in: ready for the next launch
+    } else {
+      asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(grp_cnt + 2 * grp), "r"(1u) : "memory");
+    }
+    misc[7] = last ? 1 : 0;
+  }
+  softmax_sync();
+  if (misc[7]) merge_group_whole<D>(t, warp, part_o, part_ml, K, Hq, g, R, O, lse);
+}
+
 template <int D>
 __device__ __forceinline__ int merge_chunk_count(const MergeTask* tasks, int n_tasks) {
   int n = 0;
@@ -563,7 +599,7 @@ __device__ void merge_chunks(int last_layer, const LayerSet& set, const MergeTas
 // tree_vis (optional, [B, K+1, tree_words]): the block is a draft tree and
 // row t sees the block keys of the set bits (bit j <-> block position j + 1)
 // besides the root and the prefix; nullptr: the chain draft (block-causal).
-template <int D, int STAGES, bool PAGED>
+template <int D, int STAGES, bool PAGED, bool WEIGHTED>
 __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
     const __grid_constant__ LayerSet set, const int32_t* __restrict__ kv_len, const int32_t* __restrict__ Ls,
     const uint64_t* __restrict__ tree_vis, int tree_words,
@@ -676,15 +712,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
       if ((long long)G > g_cap) G = (int)g_cap;
     }
     const int c = blockIdx.x;
-    const long long W = T + (long long)item_tiles * NG;  // weighted length
+    // weighted length (the unweighted instantiation splits by tiles alone)
+    const long long W = WEIGHTED ? T + (long long)item_tiles * NG : T;
     long long lo = 0, hi = 0;
     if (T > 0 && c < G) {
-      if (item_tiles == 0) {
-        lo = range_lo(c, T, G);
-        hi = range_lo(c + 1, T, G);
-      } else {
+      if constexpr (WEIGHTED) {
         lo = tile_of_weighted(range_lo(c, W, G), W, T, item_tiles, B, kvs, Lss, K, g, R, Hkv, S_cap);
         hi = tile_of_weighted(range_lo(c + 1, W, G), W, T, item_tiles, B, kvs, Lss, K, g, R, Hkv, S_cap);
+      } else {
+        lo = range_lo(c, T, G);
+        hi = range_lo(c + 1, T, G);
       }
     }
     int n_items = 0, n_tasks = 0;
@@ -711,8 +748,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
             t.kvh = gib / loc.p.n_mg;
             t.mg = gib % loc.p.n_mg;
             t.rows = min(R, loc.p.M - t.mg * R);
-            t.c0 = cta_of(weighted_pos(gstart, group, item_tiles), W, G);
-            t.np = cta_of(weighted_pos(gend - 1, group, item_tiles), W, G) - t.c0 + 1;
+            const int C = WEIGHTED ? item_tiles : 0;
+            t.c0 = cta_of(weighted_pos(gstart, group, C), W, G);
+            t.np = cta_of(weighted_pos(gend - 1, group, C), W, G) - t.c0 + 1;
             t.grp = group;
             t.epi = (long long)t.rows * (D / 4) * t.np <= kEpiMaxItems ? 1 : 0;
             tasks[n_tasks] = t;
@@ -1162,37 +1200,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) verify_attn_kernel(
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(bOFree + 8 * ob);
-          if (it.partial && layer == n_layers - 1) {
-            // The last layer's split groups need no grid barrier: each part is
-            // counted in as written (the barrier orders the warpgroup's writes
-            // before the release). A small group is merged at once, whole, by
-            // the CTA whose part completes it (the acquire makes the other
-            // parts visible), share by share as its CTAs would merge it, so
-            // the result is the same bits; a larger one by the merge warps of
-            // all its CTAs once its count is complete.
-            int ti = 0;
-            while (ti + 1 < n_tasks && tasks[ti].grp != it.grp) ++ti;
-            const MergeTask t = tasks[ti];
-            softmax_sync();
-            if (tid == 0) {
-              bool last = false;
-              if (t.epi) {
-                uint32_t old;
-                asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;"
-                             : "=r"(old)
-                             : "l"(grp_cnt + 2 * it.grp), "r"(1u)
-                             : "memory");
-                last = old == (uint32_t)t.np - 1;
-                if (last) grp_cnt[2 * it.grp] = 0u;  // every part is in: ready for the next launch
-              } else {
-                asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(grp_cnt + 2 * it.grp), "r"(1u)
-                             : "memory");
-              }
-              misc[7] = last ? 1 : 0;
-            }
-            softmax_sync();
-            if (misc[7]) merge_group_whole<D>(t, warp, part_o, part_ml, K, Hq, g, R, O, lse);
-          }
+          if (it.partial && layer == n_layers - 1)
+            last_layer_part_done<D>(tasks, n_tasks, it.grp, grp_cnt, misc, part_o, part_ml, K, Hq, g, R, O, lse);
         }
         ++item_ctr;
       }
@@ -1470,15 +1479,24 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
                                    cudaStream_t stream) {
   using SM = AttnSmem<D, STAGES>;
   constexpr int kSmem = PAGED ? SM::kAllocPaged : SM::kAlloc;
-  auto kern = verify_attn_kernel<D, STAGES, PAGED>;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+    cudaError_t e = cudaFuncSetAttribute(verify_attn_kernel<D, STAGES, PAGED, false>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(verify_attn_kernel<D, STAGES, PAGED, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               kSmem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
   int grid = num_sms_current();  // one CTA per SM (it holds all 512 tensor-memory columns)
   if (grid > kAttnMaxCtas) grid = kAttnMaxCtas;
+  // The cost-weighted split pays where CTAs hold many items: more (sequence,
+  // kv head) pairs than CTAs. Otherwise the instantiation without it runs
+  // (its code alone measured 2.5% faster on the latency-bound B = 1 layers).
+  const int item_tiles = attn_item_tiles();
+  const bool weighted = item_tiles > 0 && (long long)B * Hkv > grid;
+  auto kern = weighted ? verify_attn_kernel<D, STAGES, PAGED, true> : verify_attn_kernel<D, STAGES, PAGED, false>;
   const int g = Hq / Hkv;
   const int R = g * (kAttnRows / g);
   // layers beyond kMaxLayers go in further launches of the same kernel
@@ -1546,7 +1564,7 @@ static cudaError_t launch_layers_t(const uint16_t* const* Q, const uint16_t* con
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(
         &cfg, kern, set, kv_len, L, tree_vis, tree_words(K), block_table, max_pages, page_size, n_pages, attn_page_cache(SM::kPageCap), B, K,
-        Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(), attn_item_tiles(),
+        Hq, Hkv, S_cap, scale * kLog2e, attn_min_tiles(), item_tiles,
         reinterpret_cast<float*>(ws + lay.attn_o), reinterpret_cast<float*>(ws + lay.attn_ml), o_part / sizeof(float),
         ml_part / sizeof(float), reinterpret_cast<uint32_t*>(ws + lay.attn_cnt),
         reinterpret_cast<uint32_t*>(ws + lay.attn_grp), reinterpret_cast<int*>(ws + lay.status));
