@@ -252,7 +252,7 @@ cudaError_t launch_confidence(const T* x, const int32_t* tokens, const float* te
                               const float* cost, int32_t* L) {
   const long rows = (long)B * K;
   if (rows == 0) return cudaSuccess;
-  const int nsplit0 = row_splits(rows, V, num_sms_current(), kConfMaxSplits, 4096);
+  const int nsplit0 = conf_row_splits(rows, V, num_sms_current(), kConfMaxSplits, 4096);
   const int chunk = row_chunk(V, nsplit0);
   const int nsplit = (V + chunk - 1) / chunk;
   const bool vec = rows_vectorizable(x, V);

@@ -243,6 +243,23 @@ inline int row_splits(long rows, int V, int num_sms, int max_splits, int min_ele
   return (int)ns;
 }
 
+// Splits per drafter row for the confidence pass: the fewest that give about
+// 0.6 of one wave of resident CTAs (8 per SM), each of at least min_elems
+// elements. Long CTAs amortise each CTA's reduction and ticket, and a count
+// below a whole wave leaves no straggling wave (measured: sampling's 256
+// rows 37.2 us at 10 splits, 33.1 at 3; ragged's 2048 rows 156.7 us at 2,
+// 152.2 at 1).
+inline int conf_row_splits(long rows, int V, int num_sms, int max_splits, int min_elems) {
+  if (rows <= 0) return 1;
+  const long target = (6L * 8 * num_sms + 9) / 10;
+  long ns = (target + rows - 1) / rows;
+  const long cap = (V + min_elems - 1) / min_elems;
+  if (ns > cap) ns = cap;
+  if (ns > max_splits) ns = max_splits;
+  if (ns < 1) ns = 1;
+  return (int)ns;
+}
+
 // Split length: a multiple of 8 elements (whole 128-bit loads of fp32 or bf16).
 constexpr int kRowAlign = 8;
 inline int row_chunk(int V, int nsplit) {
