@@ -307,6 +307,38 @@ def host_inputs(w, kv, n_layer_samples=1):
     return host, layers
 
 
+def workload_config(args, w, kv, Lh, world, block_size):
+    """The workload a line measures (shapes, the lengths selected, the
+    variant); the same dict in both arms for the same arguments."""
+    return {"workload": w.name, "B": w.B, "K": w.K, "V": w.V, "layers": w.n_layers,
+            "resident_kv_layers": w.resident_layers if w.resident_layers else w.n_layers,
+            "gqa": "%d/%d" % (w.Hq, w.Hkv), "head_dim": w.d,
+            "kv_len": [int(kv.min()), int(kv.max())], "selected_L": [int(Lh.min()), int(Lh.max())],
+            "selected_L_mean": round(float(Lh.mean()), 3),
+            "cost_table": w.cost[0] if w.cost[0] != "measured" else "measured (%s)" % w.cost[1],
+            "selector": ("alpha (Algorithm 1, alpha %g, first block %d)" % (args.alpha, block_size)
+                         if args.selector == "alpha" else "marginal gain (Thm. 4)"),
+            "logits": args.logits,
+            "draft": ("DDTree-shaped tree of %d nodes (best-first, depth <= %d), tree walk" %
+                      (args.tree, w.K) if args.tree else "chain"),
+            "kv_cache": "paged, %d keys per page" % args.page_size if args.page_size else "dense",
+            "confidence": ("from hidden states [%d, %d] and a %d x %d LM head (fused epilogue)" %
+                           (w.B * w.K, w.hidden, w.V, w.hidden) if args.lm_head else "from drafter logits"),
+            "parallelism": "dp%d (independent sequences)" % world,
+            "l2": l2_note(w, kv)}
+
+
+def l2_note(w, kv):
+    """Whether a step's distinct inputs (both logit blocks and the resident
+    KV caches) exceed the 129 MB L2; timed steps are not separated by a flush."""
+    n_res = w.resident_layers if w.resident_layers else w.n_layers
+    mb = (w.B * w.K * w.V * 4 + w.B * (w.K + 1) * w.V * 4 +
+          n_res * float(np.sum(kv.astype(np.float64))) * w.Hkv * w.d * 2 * 2) / 1e6
+    if mb > 129:
+        return "no flush: about %d MB of distinct inputs per step exceed the 129 MB L2" % (int(mb) // 10 * 10)
+    return "no flush: about %d MB of inputs per step fit the 129 MB L2 (timed warm)" % max(1, int(mb))
+
+
 def run_reference(args, rank, world):
     """The reference arm: the oracle as it stands, on this host's cores."""
     from paper_2608_08721_gb300 import workloads
@@ -326,12 +358,18 @@ def run_reference(args, rank, world):
         us, cores, sample = oracle_round_time(w, host, layers, kv, budget / steps)
         per.append(us)
     value = statistics.median(per)
+    # the lengths the round selects (the oracle's; the GPU selects the same unless a sequence is flagged)
+    import oracle
+
+    q, _ = oracle.confidence(host["draft_logits"], host["draft_tokens"], host["temperature"])
+    Lh, _ = oracle.select_lengths(q, np.asarray(host["cost_table"], np.float64))
+    block_size = args.block_size if args.block_size > 0 else max(1, (2 * w.K) // 3)
     line = {"metric": METRIC, "value": round(value, 3), "unit": "us", "n_gpus": args.gpus, "steps": steps,
             "warmup": args.warmup, "ms_per_step": round(value / 1000, 6), "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "impl": "reference",
-            "config": {"workload": w.name, "B": w.B, "K": w.K, "V": w.V, "layers": w.n_layers,
-                       "gqa": "%d/%d" % (w.Hq, w.Hkv), "head_dim": w.d, "parallelism": "replicas"},
+            "config": workload_config(args, w, kv, np.asarray(Lh), world, block_size),
+            "timing": "the fp64 C oracle's round on the host cores, a bounded sample per step (cpu_baseline)",
             "cpu_baseline": {"value": round(value, 3), "unit": "us", "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": round(value, 3), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -769,26 +807,12 @@ def run_ours(args, rank, world, local_rank):
         "warmup": max(3, args.warmup), "ms_per_step": round(m["elapsed_max_ms"] / K_steps, 6),
         "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "bf16+f32",
         "data": "synthetic (seeded; shapes of the paper's 8B-70B-class targets, random values)",
-        "config": {"workload": w.name, "B": w.B, "K": w.K, "V": w.V, "layers": w.n_layers,
-                   "resident_kv_layers": m["n_res"], "gqa": "%d/%d" % (w.Hq, w.Hkv), "head_dim": w.d,
-                   "kv_len": [int(kv.min()), int(kv.max())], "selected_L": [int(Lh.min()), int(Lh.max())],
-                   "selected_L_mean": round(float(Lh.mean()), 3),
-                   "cost_table": w.cost[0] if w.cost[0] != "measured" else "measured (%s)" % w.cost[1],
-                   "selector": ("alpha (Algorithm 1, alpha %g, first block %d)" % (args.alpha, m["block_size"])
-                                if args.selector == "alpha" else "marginal gain (Thm. 4)"),
-                   "logits": args.logits,
-                   "draft": ("DDTree-shaped tree of %d nodes (best-first, depth <= %d), tree walk" %
-                             (args.tree, w.K) if args.tree else "chain"),
-                   "kv_cache": "paged, %d keys per page" % args.page_size if args.page_size else "dense",
-                   "confidence": ("from hidden states [%d, %d] and a %d x %d LM head (fused epilogue)" %
-                                  (w.B * w.K, w.hidden, w.V, w.hidden) if args.lm_head else "from drafter logits"),
-                   "parallelism": "dp%d (independent sequences)" % world,
-                   "l2": "no flush: %.0f MB of distinct inputs per step > 129 MB L2" % (by["total"] / 1e6),
-                   "timing": ("value: K rounds, each one CUDA graph replay of %s, events around the loop; "
-                              "segments and roofline: a second pass of the same K rounds as three graphs "
-                              "(conf+select | attention layers | accept, the acceptance plan included) with "
-                              "events between" % ("libraspec_verify_round" if m["one_call"] else
-                                                  "the round's step calls"))},
+        "config": workload_config(args, w, kv, Lh, world, m["block_size"]),
+        "timing": ("value: K rounds, each one CUDA graph replay of %s, events around the loop; "
+                   "segments and roofline: a second pass of the same K rounds as three graphs "
+                   "(conf+select | attention layers | accept, the acceptance plan included) with "
+                   "events between" % ("libraspec_verify_round" if m["one_call"] else "the round's step calls")),
+        "l2_bytes_per_step": int(by["total"]),
         "hbm_tbs": round(by["total"] / (us_per_round * 1e-6) / 1e12, 3),
         "hbm_frac_of_measured": round(by["total"] / (us_per_round * 1e-6) / 1e9 / m["hbm_peak"], 4),
         "hbm_frac_of_nominal_8tbs": round(by["total"] / (us_per_round * 1e-6) / 1e9 / NOMINAL_HBM_GBS, 4),
