@@ -173,7 +173,13 @@ def logits(w: Workload, device="cpu") -> dict:
     to the target). Greedy sequences draft the drafter's argmax; sampling
     sequences draft a token sampled from the drafter's softmax at their
     temperature (Gumbel-max with the torch generator), so that the rejection
-    sampler sees drafts distributed as q."""
+    sampler sees drafts distributed as q.
+
+    The values are drawn on the host with torch's CPU generator whatever the
+    device, then moved there, so every consumer (the GPU path, the oracle, the
+    reference arm of the benchmark) sees the same tensors for a workload."""
+    out_device = device
+    device = "cpu"
     g = torch.Generator(device=device)
     g.manual_seed(w.data_seed * 1000003 + 17)
     B, K, V = w.B, w.K, w.V
@@ -208,8 +214,8 @@ def logits(w: Workload, device="cpu") -> dict:
             u = torch.rand((K, V), generator=g, device=device).clamp_(1e-30, 1.0 - 1e-7)
             gumbel = -torch.log(-torch.log(u))
             tokens[b] = torch.argmax(draft[b] / T + gumbel, dim=-1).to(torch.int32)
-    return {"target_logits": target.contiguous(), "draft_logits": draft.contiguous(),
-            "draft_tokens": tokens.contiguous(), "temperature": temp.contiguous()}
+    out = {"target_logits": target, "draft_logits": draft, "draft_tokens": tokens, "temperature": temp}
+    return {k: v.contiguous().to(out_device) for k, v in out.items()}
 
 
 def layer(w: Workload, l: int, kv: np.ndarray, device="cpu", peaky: bool = False,

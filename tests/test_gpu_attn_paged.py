@@ -137,3 +137,31 @@ print("status", status)
             assert "status 0" in out.stdout
             res[cache] = np.load(path)
         np.testing.assert_array_equal(res["0"], res["4096"])
+
+
+def test_paged_cost_weighted_split(orc):
+    """More (sequence, kv head) pairs than CTAs: the launch takes the kernel
+    whose Stream-K ranges are cut by cost (tiles plus each item's fixed
+    cost). Paged against the oracle and bit for bit against the dense kernel
+    (the same split, tiles and arithmetic)."""
+    K, Hq, Hkv, d, P = 12, 32, 8, 128, 128
+    rng = np.random.default_rng(21)
+    B = 40  # 320 (sequence, kv head) pairs
+    kv = rng.integers(0, 1500, size=B).tolist()
+    L = rng.integers(0, K + 1, size=B).tolist()
+    layers, dense, table, S_cap = _paged_inputs(B, K, Hq, Hkv, d, kv, L, P, seed=21, n_layers=2)
+    outs, lses, status = _run_paged(layers, table, kv, L, K, S_cap)
+    assert status == 0
+    for l in range(2):
+        O_ref, lse_ref = orc.verify_attn_paged(layers[l]["Q"], layers[l]["Kp"], layers[l]["Vp"],
+                                               table.cpu().numpy(), np.array(kv), np.array(L))
+        check_attn(outs[l], lses[l], O_ref, lse_ref, L)
+    ws = lr.Workspace(B, K, 1, Hq, Hkv, d, S_cap, device=cuda())
+    O_d, lse_d = lr.libraspec_verify_attn_layers(dense, torch.tensor(kv, dtype=torch.int32, device=cuda()),
+                                                 torch.tensor(L, dtype=torch.int32, device=cuda()), ws,
+                                                 want_lse=True)
+    torch.cuda.synchronize()
+    for l in range(2):
+        for b in range(B):
+            assert torch.equal(outs[l][b, : L[b] + 1], O_d[l][b, : L[b] + 1])
+            assert torch.equal(lses[l][b, : L[b] + 1], lse_d[l][b, : L[b] + 1])

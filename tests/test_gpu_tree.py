@@ -410,3 +410,23 @@ def test_tree_edge_cases_empty_trees_and_fresh_caches(orc):
     np.testing.assert_array_equal(n.cpu().numpy(), rn)
     np.testing.assert_array_equal(bonus.cpu().numpy(), rbonus)
     assert n[0].item() == 0 and bonus[0].item() == int(x[0, 0].argmax())
+
+
+def test_tree_attn_cost_weighted_split(orc):
+    """Draft trees on a batch with more (sequence, kv head) pairs than CTAs
+    (the kernel whose Stream-K ranges are cut by cost), two layers in one
+    launch, against the oracle."""
+    K, Hq, Hkv, d = 16, 32, 8, 128
+    rng = np.random.default_rng(31)
+    B = 24  # 192 (sequence, kv head) pairs
+    kv = rng.integers(0, 1200, size=B).tolist()
+    L = rng.integers(0, K + 1, size=B).tolist()
+    S = (max(k + l + 1 for k, l in zip(kv, L)) + 63) // 64 * 64
+    parent = workloads.draft_tree(B, K, L, seed=31, shape="random")
+    layers = _layers(B, K, Hq, Hkv, d, S, seed=31, n_layers=2)
+    outs, lses, status = _run_tree(layers, parent, kv, L, K)
+    assert status == 0
+    for l in range(2):
+        O_ref, lse_ref = orc.verify_attn_tree(layers[l]["Q"], layers[l]["Kc"], layers[l]["Vc"], np.array(kv),
+                                              np.array(L), parent)
+        check_attn(outs[l], lses[l], O_ref, lse_ref, L)
