@@ -1350,7 +1350,7 @@ static int attn_min_tiles() {
 // overrides the default, read once per process.
 static int attn_item_tiles() {
   static int t = [] {
-    int v = 3;
+    int v = 2;
     if (const char* e = getenv("LIBRASPEC_ATTN_ITEM_TILES")) {
       int a = 0;
       if (sscanf(e, "%d", &a) == 1 && a >= 0 && a <= 64) v = a;
