@@ -402,7 +402,7 @@ __global__ void __launch_bounds__(kPlanThreads) accept_plan_kernel(const int32_t
     if (bad_len || (sampling && !have_q)) {
       n_accepted[b] = 0;
       bonus[b] = 0;
-      publish_draw(res, ready, b, en);
+      if (sampling) publish_draw(res, ready, b, en);  // its draw CTAs wait for a draw (none)
       raise_status(status, bad_len ? LIBRASPEC_ST_BAD_LENGTH : LIBRASPEC_ST_MISSING_INPUT);
     } else if (!sampling) {
       r = Lb + 1;
@@ -617,14 +617,16 @@ __global__ void __launch_bounds__(kRowThreads, 6) accept_rows_kernel(const Accep
           const int w = s_arg[n];
           a.n_accepted[b] = n;
           a.bonus[b] = w == 0x7fffffff ? 0 : w;  // a row without a finite logit
-        } else if (n == Lb) {
-          en.mode = 1;  // all drafts accepted: the bonus draw from row L_b
         } else {
-          en.mode = 2;  // rejected at n: the residual draw
-          en.mp = s_m[n];
-          en.invZp = (float)(1.0 / s_Z[n]);
+          if (n == Lb) {
+            en.mode = 1;  // all drafts accepted: the bonus draw from row L_b
+          } else {
+            en.mode = 2;  // rejected at n: the residual draw
+            en.mp = s_m[n];
+            en.invZp = (float)(1.0 / s_Z[n]);
+          }
+          publish_draw(a.res, a.ready, b, en);
         }
-        publish_draw(a.res, a.ready, b, en);
       }
     }
     __syncthreads();
@@ -645,6 +647,9 @@ __global__ void __launch_bounds__(kRowThreads, 4) accept_race_kernel(const Accep
   __shared__ int sh[2];
   __shared__ ResEntry s_en;
   const int s = blockIdx.x, b = blockIdx.y;
+  // a greedy sequence has no draw (and publishes none): its CTAs leave at
+  // once, so they hold no slot while the sampling races wait and run
+  if (!(a.temperature[b] > 0.f)) return;
   if (threadIdx.x == 0) {
     sh[0] = wait_published(a.ready + b, a.status);
     s_en = a.res[b];

@@ -61,7 +61,8 @@ struct RaceCand {
 // The draw that ends a sampling sequence's acceptance: mode 1, the bonus
 // draw from target row n = L_b (all drafts accepted); mode 2, the residual
 // draw max(0, p_n - q_n) after a rejection at n (with row n's max and
-// normaliser); mode 0, none (a greedy sequence, or one without units).
+// normaliser); mode 0, none (a sampling sequence without units: a length
+// out of range, or no drafter statistics). A greedy sequence publishes none.
 struct ResEntry {
   int n;
   int mode;
