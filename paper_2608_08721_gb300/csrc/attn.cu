@@ -10,9 +10,11 @@
 // key tile) pairs of the batch form one tile sequence (sequence-major, then kv
 // head, row group, key tile); CTA c of the persistent grid (one CTA per SM)
 // takes the contiguous range [c*T/G, (c+1)*T/G) of it, so every CTA streams
-// the same number of tiles whatever the ragged lengths. The plan is derived
-// on the device from L[] and kv_len[] by every CTA, and it is the same for
-// every layer (all layers share L and kv_len).
+// the same number of tiles whatever the ragged lengths; with more (sequence,
+// kv head) pairs than CTAs the ranges are cut by cost instead (each row
+// group weighs its tiles plus an item's fixed cost; tile_of_weighted). The
+// plan is derived on the device from L[] and kv_len[] by every CTA, and it
+// is the same for every layer (all layers share L and kv_len).
 //
 // Roles in a CTA (192 threads):
 //  * producer warp: walks the CTA's range layer after layer in items (runs of
@@ -44,10 +46,12 @@
 // Split groups. A row group covered by one CTA is written directly. A group
 // spread over CTAs c0..c1 leaves one fp32 partial (O, m, l) per CTA, in slot
 // 2c+1 for c0 (its last item) and 2c for the others (their first item), in a
-// buffer chosen by the layer parity. After the barrier that ends layer l,
-// each of those CTAs merges its share of the group's rows from all parts in
-// CTA order (deterministic, spread over every contributing SM); the merge of
-// layer l runs after the CTA's items of layer l+1.
+// buffer chosen by the layer (l mod 3). After the barrier that ends layer
+// l, each of those CTAs merges its share of the group's rows from all parts
+// in CTA order (deterministic, spread over every contributing SM); the merge
+// of layer l runs beside the CTA's items of layer l+1. The last layer waits
+// for no grid barrier: a group's parts are counted in as they are written,
+// and a small group is merged whole by the CTA whose part completes it.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -365,7 +369,6 @@ struct AttnSmem {
 // round trip per batch and no weights are staged in shared memory.
 
 // This CTA's share [u0, u0 + nr) of task t's rows.
-__device__ __forceinline__ int merge_share(const MergeTask& t, int& u0);
 __device__ __forceinline__ int merge_share(const MergeTask& t, int& u0) {
   const int k_me = (int)blockIdx.x - t.c0;
   u0 = (int)((long long)t.rows * k_me / t.np);
