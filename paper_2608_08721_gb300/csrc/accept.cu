@@ -174,40 +174,62 @@ __device__ __forceinline__ void race_combine(float& E, float& y, int& i, float E
   }
 }
 
-// One group of four logits y (tokens v0 .. v0+3, those >= c1 skipped) in
-// the bonus race: uniforms from the Philox block w4 (word v & 3).
-__device__ __forceinline__ void bonus_race_group(const float (&y)[4], int v0, int c1, uint4 w4, float c, float& bE,
-                                                 float& by, int& bi) {
-  const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
+// The best candidate that any lane of the warp holds, (bEw, byw); bEw = inf
+// when no lane has one. Lanes rank their candidates by the log2 key
+// log2(bE) - by c with the fast logarithm: a slightly wrong pick only makes
+// the screen below a little looser, never unsafe, since the picked
+// candidate is a token some lane has drawn. All 32 lanes take part.
+__device__ __forceinline__ void warp_best_candidate(float bE, float by, float c, float& bEw, float& byw) {
+  const bool has = bE < INFINITY;
+  const float lk = has ? __log2f(bE) - by * c : INFINITY;
+  float mn = lk;
 #pragma unroll
-  for (int t = 0; t < 4; ++t) {
-    const int v = v0 + t;
-    if (v >= c1 || !(y[t] > -INFINITY)) continue;
-    const float u = word_to_uniform(ws[t]);
-    if (!(bE < INFINITY)) {
-      bE = -logf(u); by = y[t]; bi = v;
-      continue;
-    }
-    // v wins iff E_v = -ln u < X = bE 2^((y - by) c), i.e. u > exp(-X): a
-    // margin of 2^-12 above the fast exponentials' error keeps every possible
-    // winner, whose E is then compared exactly
-    const float X = bE * ex2_approx((y[t] - by) * c);
-    if (u > ex2_approx(-X * kLog2e) * 0.999755859375f) {
-      const float Ev = -logf(u);
-      if (Ev < X) { bE = Ev; by = y[t]; bi = v; }
-    }
+  for (int off = 16; off > 0; off >>= 1) mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
+  const unsigned ball = __ballot_sync(0xffffffffu, has && lk == mn);
+  const int src = ball ? __ffs(ball) - 1 : 0;
+  const float e = __shfl_sync(0xffffffffu, bE, src);
+  byw = __shfl_sync(0xffffffffu, by, src);
+  bEw = ball ? e : INFINITY;
+}
+
+// Token v (logit y, Philox word w) in the bonus race. v beats a candidate
+// (E, y') iff E_v = -ln u_v < X = E 2^((y - y') c), i.e. u_v > exp(-X). The
+// screen tests that against the warp's best candidate (bEw, byw), a token
+// already drawn, with a margin of 2^-12 above the fast exponentials' error,
+// so every token that can still win the race passes it; a token that
+// passes takes the exact logarithm and is compared with the lane's own
+// candidate (bE, by, bi). Screening against the warp's candidate rather
+// than the lane's own skips the logarithm for most of the slice: a warp
+// runs the exact step whenever any of its lanes needs it.
+__device__ __forceinline__ void bonus_race_token(float y, uint32_t w, int v, float c, float bEw, float byw, float& bE,
+                                                 float& by, int& bi) {
+  const float u = word_to_uniform(w);
+  if (bEw < INFINITY) {
+    const float Xw = bEw * ex2_approx((y - byw) * c);
+    if (!(u > ex2_approx(-Xw * kLog2e) * 0.999755859375f)) return;
+  }
+  const float Ev = -logf(u);
+  if (!(bE < INFINITY) || Ev < bE * ex2_approx((y - by) * c)) {
+    bE = Ev; by = y; bi = v;
   }
 }
 
 // The bonus race over logits [c0, c1) of row j (sampling at c = log2(e)/T):
 // uniforms from Philox at (v >> 2, j, seq, purpose 1), word v & 3. Four
-// groups of four logits are loaded before any is used.
+// groups of four logits are loaded before any is used. The trip counts are
+// the warp's (lanes past the slice's end idle), so that every lane joins
+// the refreshes of the warp's candidate: after the first token, then
+// before every later group.
 template <bool VEC, typename E>
 __device__ __forceinline__ void bonus_race_slice(const E* __restrict__ yr, int c0, int c1, int V, float c,
                                                  uint64_t seed, uint32_t j, uint32_t seq, uint64_t round_offset,
                                                  float& bE, float& by, int& bi) {
   const int g1 = (c1 + 3) >> 2;
-  for (int g = (c0 >> 2) + threadIdx.x; g < g1; g += 4 * kRowThreads) {
+  const int lane = threadIdx.x & 31;
+  float bEw = INFINITY, byw = 0.f;
+  bool first = true;
+  for (int gw = (c0 >> 2) + (int)(threadIdx.x & ~31u); gw < g1; gw += 4 * kRowThreads) {
+    const int g = gw + lane;
     float yv[4][4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -219,14 +241,26 @@ __device__ __forceinline__ void bonus_race_slice(const E* __restrict__ yr, int c
 #pragma unroll
           for (int t = 0; t < 4; ++t) yv[k][t] = 4 * gg + t < V ? Logit<E>::at(yr, 4 * gg + t) : -INFINITY;
         }
+      } else {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) yv[k][t] = -INFINITY;
       }
     }
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
+      if (gw + k * kRowThreads >= g1) break;  // the same for the whole warp
+      if (!first) warp_best_candidate(bE, by, c, bEw, byw);
       const int gg = g + k * kRowThreads;
-      if (gg >= g1) break;
-      bonus_race_group(yv[k], 4 * gg, c1, philox_block(seed, (uint32_t)gg, j, seq, 1u, round_offset), c, bE, by,
-                       bi);
+      uint4 w4 = make_uint4(0u, 0u, 0u, 0u);
+      if (gg < g1) w4 = philox_block(seed, (uint32_t)gg, j, seq, 1u, round_offset);
+      const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int v = 4 * gg + t;
+        if (v < c1 && yv[k][t] > -INFINITY) bonus_race_token(yv[k][t], ws[t], v, c, bEw, byw, bE, by, bi);
+        if (t == 0 && first) warp_best_candidate(bE, by, c, bEw, byw);
+      }
+      first = false;
     }
   }
 }
@@ -261,15 +295,29 @@ __device__ __forceinline__ int seq_of_row(const int* start, int B, int r) {
   return lo;
 }
 
+// The smallest key any lane of the warp holds (all 32 lanes take part).
+__device__ __forceinline__ float warp_min_key(float k) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) k = fminf(k, __shfl_xor_sync(0xffffffffu, k, off));
+  return k;
+}
+
 // Residual race of queued entry e over slice s: w_v = max(0, p_v - q_v),
-// key E_v / w_v, uniforms at (v >> 2, n, seq, purpose 1).
+// key E_v / w_v, uniforms at (v >> 2, n, seq, purpose 1). The screen tests
+// each token against the smaller of the lane's best key and the warp's best
+// at its last refresh (a key some lane has drawn); the trip counts are the
+// warp's, so every lane joins the refreshes.
 template <bool VEC, typename E>
 __device__ __forceinline__ void residual_race_slice(const E* __restrict__ yr, const E* __restrict__ dr, int c0,
                                                     int c1, int V, float c, float mp, float invZp, float mq,
                                                     float invZq, uint64_t seed, uint32_t n, uint32_t seq,
                                                     uint64_t round_offset, float& best, int& besti) {
   const int g1 = (c1 + 3) >> 2;
-  for (int g = (c0 >> 2) + threadIdx.x; g < g1; g += 2 * kRowThreads) {
+  const int lane = threadIdx.x & 31;
+  float bw = INFINITY;
+  bool first = true;
+  for (int gw = (c0 >> 2) + (int)(threadIdx.x & ~31u); gw < g1; gw += 2 * kRowThreads) {
+    const int g = gw + lane;
     float yv[2][4], dv[2][4];
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
@@ -286,32 +334,44 @@ __device__ __forceinline__ void residual_race_slice(const E* __restrict__ yr, co
             dv[k][t] = v < V ? Logit<E>::at(dr, v) : 0.f;
           }
         }
+      } else {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          yv[k][t] = -INFINITY;
+          dv[k][t] = 0.f;
+        }
       }
     }
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
+      if (gw + k * kRowThreads >= g1) break;  // the same for the whole warp
+      if (!first) bw = warp_min_key(best);
       const int gg = g + k * kRowThreads;
-      if (gg >= g1) break;
-      const uint4 w4 = philox_block(seed, (uint32_t)gg, n, seq, 1u, round_offset);
+      uint4 w4 = make_uint4(0u, 0u, 0u, 0u);
+      if (gg < g1) w4 = philox_block(seed, (uint32_t)gg, n, seq, 1u, round_offset);
       const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
         const int v = 4 * gg + t;
-        if (v >= c1) break;
-        // exponents are <= 0 (below the row maxima), so the fast base-2
-        // exponential is exact to a few ulp
-        const float wv = ex2_approx((yv[k][t] - mp) * c) * invZp - ex2_approx((dv[k][t] - mq) * c) * invZq;
-        if (wv > 0.f) {
-          // E / w < best  <=>  u > exp(-best * w): a candidate whose uniform is
-          // below that (with a margin far above the rounding of the test)
-          // cannot win, and skips the logarithm
-          const float u = word_to_uniform(ws[t]);
-          if (best == INFINITY || u > ex2_approx(-best * wv * kLog2e) * (1.f - 9.5367431640625e-7f)) {
-            const float Ev = -logf(u);
-            argmin_combine(best, besti, __fdividef(Ev, wv), v);
+        if (v < c1 && gg < g1) {
+          // exponents are <= 0 (below the row maxima), so the fast base-2
+          // exponential is exact to a few ulp
+          const float wv = ex2_approx((yv[k][t] - mp) * c) * invZp - ex2_approx((dv[k][t] - mq) * c) * invZq;
+          if (wv > 0.f) {
+            // E / w < thr  <=>  u > exp(-thr * w): a candidate whose uniform is
+            // below that (with a margin far above the rounding of the test)
+            // cannot win, and skips the logarithm
+            const float u = word_to_uniform(ws[t]);
+            const float thr = fminf(best, bw);
+            if (thr == INFINITY || u > ex2_approx(-thr * wv * kLog2e) * (1.f - 9.5367431640625e-7f)) {
+              const float Ev = -logf(u);
+              argmin_combine(best, besti, __fdividef(Ev, wv), v);
+            }
           }
         }
+        if (t == 0 && first) bw = warp_min_key(best);
       }
+      first = false;
     }
   }
 }
@@ -803,31 +863,46 @@ __global__ void __launch_bounds__(kRowThreads) tree_rows_kernel(
     const uint32_t seq = seq_offset + (uint32_t)b;
     float best = INFINITY;
     int besti = 0x7fffffff;
-    for (int g = (c0 >> 2) + threadIdx.x; 4 * g < c1; g += kRowThreads) {
-      const uint4 w4 = philox_block(seed, (uint32_t)g, (uint32_t)j, seq, 2u, round_offset);
-      const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
-      float yv[4];
-      if (VEC) {
-        Logit<E>::stream4(xr + 4 * g, yv);
-      } else {
+    // the screen's threshold: the smaller of the lane's best key and the
+    // warp's best at its last refresh (a key some lane has drawn), refreshed
+    // after the first token and then before groups 1, 2, 3 and every fourth;
+    // the trip counts are the warp's, so every lane joins the refreshes
+    float bw = INFINITY;
+    const int lane = threadIdx.x & 31;
+    int it = 0;
+    for (int gw = (c0 >> 2) + (int)(threadIdx.x & ~31u); 4 * gw < c1; gw += kRowThreads, ++it) {
+      if (it > 0 && (it < 4 || (it & 3) == 0)) bw = warp_min_key(best);
+      const int g = gw + lane;
+      const bool live = 4 * g < c1;
+      uint4 w4 = make_uint4(0u, 0u, 0u, 0u);
+      float yv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      if (live) {
+        w4 = philox_block(seed, (uint32_t)g, (uint32_t)j, seq, 2u, round_offset);
+        if (VEC) {
+          Logit<E>::stream4(xr + 4 * g, yv);
+        } else {
 #pragma unroll
-        for (int t = 0; t < 4; ++t) yv[t] = 4 * g + t < V ? Logit<E>::at(xr, 4 * g + t) : -INFINITY;
+          for (int t = 0; t < 4; ++t) yv[t] = 4 * g + t < V ? Logit<E>::at(xr, 4 * g + t) : -INFINITY;
+        }
       }
+      const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
         const int v = 4 * g + t;
-        if (v >= c1) break;
         const float yc = yv[t] * c;
-        if (!(yc > -INFINITY)) continue;
-        const float u = word_to_uniform(ws[t]);
-        // key < best  <=>  u > exp(-2^(best + yc)) =: h. The fast exponentials
-        // give h to a relative 2e-4 while h is a normal float (exponent above
-        // -150; below, h flushes to 0 and every candidate passes): a margin of
-        // 2^-12 keeps every possible winner, whose key is then compared exactly.
-        if (best == INFINITY || u > ex2_approx(-ex2_approx(best + yc) * kLog2e) * 0.999755859375f) {
-          const float key = log2f(-logf(u)) - yc;
-          argmin_combine(best, besti, key, v);
+        if (v < c1 && yc > -INFINITY) {
+          const float u = word_to_uniform(ws[t]);
+          // key < thr  <=>  u > exp(-2^(thr + yc)) =: h. The fast exponentials
+          // give h to a relative 2e-4 while h is a normal float (exponent above
+          // -150; below, h flushes to 0 and every candidate passes): a margin of
+          // 2^-12 keeps every possible winner, whose key is then compared exactly.
+          const float thr = fminf(best, bw);
+          if (thr == INFINITY || u > ex2_approx(-ex2_approx(thr + yc) * kLog2e) * 0.999755859375f) {
+            const float key = log2f(-logf(u)) - yc;
+            argmin_combine(best, besti, key, v);
+          }
         }
+        if (t == 0 && it == 0) bw = warp_min_key(best);
       }
     }
     m = -best;

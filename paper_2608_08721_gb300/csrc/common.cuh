@@ -155,8 +155,12 @@ __device__ __forceinline__ uint4 philox_block(uint64_t seed, uint32_t idx, uint3
 }
 
 // u = ((w >> 9) + 1/2) * 2^-23: strictly inside (0,1), exact in binary32.
+// Formed without an integer-to-float conversion: the word's top 23 bits as
+// the mantissa of a = 1 + (w >> 9) 2^-23 in [1, 2), then a - (1 - 2^-24),
+// which is exact (Sterbenz: the operands are within a factor of two), so u
+// has the same bits as the conversion-and-scale form.
 __device__ __forceinline__ float word_to_uniform(uint32_t w) {
-  return (__uint2float_rn(w >> 9) + 0.5f) * 1.1920928955078125e-07f;
+  return __fsub_rn(__uint_as_float(0x3F800000u | (w >> 9)), 0.999999940395355224609375f);
 }
 
 // ---------------------------------------------------------------------------
