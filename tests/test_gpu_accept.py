@@ -119,3 +119,56 @@ def test_accept_missing_confidence_for_sampling_sets_status():
                         torch.zeros((B, K), dtype=torch.int32, device=cuda()), None, None,
                         torch.ones(B, dtype=torch.int32, device=cuda()), torch.ones(B, device=cuda()), 0, ws)
     assert lr.libraspec_get_status(ws) & lr.ST_MISSING_INPUT
+
+
+def _race_rows(V, seed):
+    """Ten sampling sequences (T = 1, K = 2) whose draws stress the races'
+    screens: bonus draws (L = 0) from a flat row, a flat row with every other
+    token at -inf, a row with one dominant token, a very peaked row, a row
+    with three finite tokens and a plain row; residual draws (L = 2, the
+    drafted token's target logit lowered so that it is rejected) from plain
+    rows, and one (the last) where the drafter only raises its drafted token,
+    so that every other token's residual max(0, p - q) is a small difference
+    of nearly equal probabilities."""
+    g = torch.Generator().manual_seed(seed)
+    B, K = 10, 2
+    tgt = torch.randn((B, K + 1, V), generator=g)
+    tgt[0] = 0.0
+    tgt[1] = 0.0
+    tgt[1, :, ::2] = -float("inf")
+    tgt[2, :, 17] += 25.0
+    tgt[3] *= 8.0
+    tgt[4] = -float("inf")
+    tgt[4, :, 3], tgt[4, :, V // 2], tgt[4, :, V - 1] = 0.0, 0.5, 1.0
+    tgt[6:] *= 2.0
+    dr = tgt[:, :K] + torch.randn((B, K, V), generator=g) * 3.0
+    dr[9] = tgt[9, :K]
+    tok = dr.argmax(-1).int()
+    for b in range(6, 9):
+        for j in range(K):
+            tgt[b, j, int(tok[b, j])] -= 8.0
+    for j in range(K):
+        dr[9, j, int(tok[9, j])] += 6.0
+    L = np.array([0] * 6 + [2] * 4, np.int32)
+    inp = {"target_logits": tgt.contiguous().to(cuda()), "draft_logits": dr.contiguous().to(cuda()),
+           "draft_tokens": tok.to(cuda()), "temperature": torch.ones(B, device=cuda())}
+    return inp, L
+
+
+@pytest.mark.parametrize("V", [50000, 50001])
+def test_accept_race_degenerate_rows(orc, V):
+    """The exponential races on flat, masked, dominated and peaked rows and on
+    residuals obtained by cancellation, in both vector paths, against the
+    oracle (exact unless flagged)."""
+    inp, L = _race_rows(V, seed=V)
+    unflagged = 0
+    for round_offset in (0, 3):
+        n, bonus = _gpu_accept(inp, L, seed=11, round_offset=round_offset)
+        n_ref, b_ref, flag = _oracle_accept(orc, inp, L, 11, round_offset=round_offset)
+        assert_exact_unless_flagged(n, n_ref, flag, "n_accepted")
+        assert_exact_unless_flagged(bonus, b_ref, flag, "bonus_token")
+        unflagged += int((flag == 0).sum())
+        assert n_ref[6:9].tolist() == [0, 0, 0], "the lowered drafted tokens are rejected at once"
+        assert bonus[2] == 17 or flag[2], "the dominant token wins the bonus draw"
+        assert bonus[4] in (3, V // 2, V - 1) and bonus[1] % 2 == 1, "only finite logits can be drawn"
+    assert unflagged >= 16, "%d of 20 draws unflagged" % unflagged
