@@ -706,6 +706,7 @@ __global__ void __launch_bounds__(kRowThreads, 4) accept_race_kernel(const Accep
   __shared__ int smi[32];
   __shared__ int sh[2];
   __shared__ ResEntry s_en;
+  __shared__ float s_c;
   const int s = blockIdx.x, b = blockIdx.y;
   // a greedy sequence has no draw (and publishes none): its CTAs leave at
   // once, so they hold no slot while the sampling races wait and run
@@ -713,6 +714,7 @@ __global__ void __launch_bounds__(kRowThreads, 4) accept_race_kernel(const Accep
   if (threadIdx.x == 0) {
     sh[0] = wait_published(a.ready + b, a.status);
     s_en = a.res[b];
+    s_c = log2e_over(a.temperature[b]);  // once per CTA: a binary32 division and reciprocal
   }
   __syncthreads();
   if (!sh[0]) return;
@@ -734,7 +736,7 @@ __global__ void __launch_bounds__(kRowThreads, 4) accept_race_kernel(const Accep
   }
   const int K = a.K, V = a.V;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const float c = log2e_over(a.temperature[b]);
+  const float c = s_c;
   const E* yr = a.target + ((size_t)b * (K + 1) + n) * V;
   const uint32_t seq = seq_offset + (uint32_t)b;
   const int c0 = s * a.chunkB, c1 = min(V, c0 + a.chunkB);
